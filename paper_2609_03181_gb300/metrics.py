@@ -1,0 +1,50 @@
+"""Speculative-decoding statistics with the definitions of the paper's efficiency table
+(Sec. 7.3, Table "Decoding efficiency ... with FastMTP"):
+
+* tau: mean number of tokens committed per speculative step, bonus token included;
+* acceptance rate: the position-averaged (tau - 1) / k;
+* a_d: probability that draft depth d is accepted given that all shallower depths were;
+* c = tau / S: cost of one speculative step in units of one autoregressive step;
+* the fixed per-step overhead implied by c: t_AR * (c - 1).
+"""
+from __future__ import annotations
+
+from typing import Dict, Sequence
+
+
+def tau_from_conditional(a: Sequence[float]) -> float:
+    """tau = 1 + a_1 + a_1 a_2 + ... (depth d is reached only if depths < d were accepted)."""
+    tau, run = 1.0, 1.0
+    for ad in a:
+        run *= ad
+        tau += run
+    return tau
+
+
+def acceptance_rate(tau: float, k: int) -> float:
+    return (tau - 1.0) / k
+
+
+def step_cost(tau: float, speedup: float) -> float:
+    return tau / speedup
+
+
+def fixed_overhead(t_ar: float, c: float) -> float:
+    """Extra time of one speculative step over one autoregressive step."""
+    return t_ar * (c - 1.0)
+
+
+def from_accept_hist(hist: Sequence[int]) -> Dict[str, object]:
+    """Statistics from a histogram of accepted draft lengths m = 0..K (one entry per verified
+    sequence-step).  Committed tokens per step are m + 1."""
+    K = len(hist) - 1
+    n = sum(hist)
+    if n == 0:
+        return {"steps": 0, "tau": 0.0, "acceptance_rate": 0.0, "a_d": [0.0] * K}
+    tau = sum((m + 1) * c for m, c in enumerate(hist)) / n
+    a_d = []
+    for d in range(1, K + 1):
+        reached = sum(hist[d - 1:])          # depths < d all accepted: m >= d-1
+        acc = sum(hist[d:])                  # depth d accepted: m >= d
+        a_d.append(acc / reached if reached else 0.0)
+    return {"steps": n, "tau": tau, "acceptance_rate": acceptance_rate(tau, K) if K else 0.0, "a_d": a_d}

@@ -1,0 +1,204 @@
+"""Seeded synthetic inputs for the FastMTP speculative decode step.
+
+This module only draws random numbers: the shape contract of the compact MoE decoder
+(Table "Model specification": 12 layers, d=1280, 64 routed + 2 shared experts, top-6,
+vocabulary 129,280, RoPE theta 1e6, position limit 32,768) with the shapes the paper leaves
+open (10 heads x 128, expert intermediate 896, draft-block intermediate 3584, RMSNorm eps
+1e-6), random bf16 weights ~N(0, 0.02), synthetic committed KV prefixes ~N(0, 1), context
+lengths, token ids and coin flips.  It holds none of the method's arithmetic, so both the
+fp64 oracle and the CUDA path can take their inputs from it without sharing any compute code.
+
+Every tensor is drawn from its own Philox stream keyed by (seed, name, chunk), so any single
+tensor (one expert's matrices, one sequence's KV prefix) can be regenerated on its own and
+large tensors are filled by several threads at once.
+"""
+from __future__ import annotations
+
+import math
+import zlib
+from concurrent.futures import ThreadPoolExecutor
+from dataclasses import dataclass, field
+from typing import List, Optional
+
+import numpy as np
+import torch
+
+_CHUNK = 1 << 22  # elements per Philox stream
+
+
+@dataclass(frozen=True)
+class ModelShape:
+    hidden: int = 1280
+    n_heads: int = 10
+    head_dim: int = 128
+    n_layers: int = 12
+    n_experts: int = 64
+    top_k: int = 6
+    n_shared: int = 2
+    expert_inter: int = 896
+    draft_inter: int = 3584
+    vocab: int = 129280
+    rms_eps: float = 1e-6
+    rope_theta: float = 1.0e6
+    max_position: int = 32768
+
+    def replace(self, **kw) -> "ModelShape":
+        d = dict(self.__dict__)
+        d.update(kw)
+        return ModelShape(**d)
+
+
+def _stream(seed: int, name: str, chunk: int) -> np.random.Generator:
+    ss = np.random.SeedSequence([int(seed) & 0xFFFFFFFF, zlib.crc32(name.encode()), int(chunk)])
+    return np.random.Generator(np.random.Philox(ss))
+
+
+_POOL: Optional[ThreadPoolExecutor] = None
+
+
+def _pool() -> ThreadPoolExecutor:
+    global _POOL
+    if _POOL is None:
+        import os
+        _POOL = ThreadPoolExecutor(max_workers=max(1, min(32, os.cpu_count() or 1)))
+    return _POOL
+
+
+def normal(seed: int, name: str, shape, std: float = 1.0, dtype=torch.bfloat16) -> torch.Tensor:
+    """N(0, std^2) samples of the given shape, rounded to `dtype` (bf16 by default)."""
+    n = int(np.prod(shape)) if len(shape) else 1
+    out = np.empty(n, dtype=np.float32)
+    nchunks = (n + _CHUNK - 1) // _CHUNK
+
+    def fill(c):
+        lo, hi = c * _CHUNK, min(n, (c + 1) * _CHUNK)
+        g = _stream(seed, name, c)
+        g.standard_normal(hi - lo, dtype=np.float32, out=out[lo:hi])
+        if std != 1.0:
+            out[lo:hi] *= np.float32(std)
+
+    if nchunks > 1:
+        list(_pool().map(fill, range(nchunks)))
+    elif n:
+        fill(0)
+    return torch.from_numpy(out).reshape(tuple(shape)).to(dtype)
+
+
+def integers(seed: int, name: str, n: int, lo: int, hi: int) -> np.ndarray:
+    """n integers uniform in [lo, hi] (inclusive), int64."""
+    return _stream(seed, name, 0).integers(lo, hi + 1, size=n, dtype=np.int64)
+
+
+def uniforms(seed: int, name: str, n: int) -> np.ndarray:
+    """n floats uniform in [0, 1), float64."""
+    return _stream(seed, name, 0).random(n)
+
+
+def permutation(seed: int, name: str, n: int) -> np.ndarray:
+    return _stream(seed, name, 0).permutation(n)
+
+
+def _gain(seed: int, name: str, d: int, gain_std: float) -> torch.Tensor:
+    """RMSNorm gain: exactly 1 (the workloads' initialisation) or 1 + N(0, gain_std^2)."""
+    if gain_std == 0.0:
+        return torch.ones(d, dtype=torch.bfloat16)
+    return (1.0 + normal(seed, name, (d,), gain_std, torch.float32)).to(torch.bfloat16)
+
+
+@dataclass
+class LayerWeights:
+    attn_norm: torch.Tensor        # [d]
+    wqkv: torch.Tensor             # [3d][d]  rows: q (H*hd), k (H*hd), v (H*hd)
+    wo: torch.Tensor               # [d][H*hd]
+    moe_norm: torch.Tensor         # [d]
+    router: torch.Tensor           # [E][d]
+    w_gate_up: torch.Tensor        # [E][2I][d]  rows 0..I-1 gate, I..2I-1 up
+    w_down: torch.Tensor           # [E][d][I]
+    shared_gate_up: torch.Tensor   # [S][2I][d]
+    shared_down: torch.Tensor      # [S][d][I]
+    router_bias: Optional[torch.Tensor] = None  # fp32 [E] or None
+
+
+@dataclass
+class VerifierWeights:
+    shape: ModelShape
+    embed: torch.Tensor        # [V][d]
+    lm_head: torch.Tensor      # [V][d]
+    final_norm: torch.Tensor   # [d]
+    layers: List[LayerWeights] = field(default_factory=list)
+
+
+@dataclass
+class DraftWeights:
+    enorm: torch.Tensor        # [d]
+    hnorm: torch.Tensor        # [d]
+    eh_proj: torch.Tensor      # [d][2d]  input = [N_e(e); N_h(a)]
+    attn_norm: torch.Tensor    # [d]
+    wqkv: torch.Tensor         # [3d][d]
+    wo: torch.Tensor           # [d][d]
+    ffn_norm: torch.Tensor     # [d]
+    w_gate_up: torch.Tensor    # [2*Id][d] rows 0..Id-1 gate, Id..2Id-1 up
+    w_down: torch.Tensor       # [d][Id]
+
+
+def zipf_router_bias(seed: int, layer: int, n_experts: int, s: float = 1.2) -> torch.Tensor:
+    """Per-expert router-logit bias -s*ln(rank) over a seeded permutation of the experts.
+
+    Added to the router logits it makes P(select expert of rank r) fall off like r^-s, the
+    skewed-load case of the throughput sweep."""
+    rank = permutation(seed, f"zipf.{layer}", n_experts) + 1
+    return torch.tensor([-s * math.log(r) for r in rank], dtype=torch.float32)
+
+
+def verifier_weights(shape: ModelShape, seed: int, std: float = 0.02, gain_std: float = 0.0,
+                     zipf_s: Optional[float] = None) -> VerifierWeights:
+    d, H, hd, E, I, S = (shape.hidden, shape.n_heads, shape.head_dim, shape.n_experts,
+                         shape.expert_inter, shape.n_shared)
+    w = VerifierWeights(
+        shape=shape,
+        embed=normal(seed, "embed", (shape.vocab, d), std),
+        lm_head=normal(seed, "lm_head", (shape.vocab, d), std),
+        final_norm=_gain(seed, "final_norm", d, gain_std),
+    )
+    for l in range(shape.n_layers):
+        w.layers.append(LayerWeights(
+            attn_norm=_gain(seed, f"l{l}.attn_norm", d, gain_std),
+            wqkv=normal(seed, f"l{l}.wqkv", (3 * H * hd, d), std),
+            wo=normal(seed, f"l{l}.wo", (d, H * hd), std),
+            moe_norm=_gain(seed, f"l{l}.moe_norm", d, gain_std),
+            router=normal(seed, f"l{l}.router", (E, d), std),
+            w_gate_up=normal(seed, f"l{l}.w_gate_up", (E, 2 * I, d), std),
+            w_down=normal(seed, f"l{l}.w_down", (E, d, I), std),
+            shared_gate_up=normal(seed, f"l{l}.shared_gate_up", (S, 2 * I, d), std),
+            shared_down=normal(seed, f"l{l}.shared_down", (S, d, I), std),
+            router_bias=(zipf_router_bias(seed, l, E, zipf_s) if zipf_s else None),
+        ))
+    return w
+
+
+def draft_weights(shape: ModelShape, seed: int, std: float = 0.02, gain_std: float = 0.0) -> DraftWeights:
+    d, H, hd, Id = shape.hidden, shape.n_heads, shape.head_dim, shape.draft_inter
+    return DraftWeights(
+        enorm=_gain(seed, "mtp.enorm", d, gain_std),
+        hnorm=_gain(seed, "mtp.hnorm", d, gain_std),
+        eh_proj=normal(seed, "mtp.eh_proj", (d, 2 * d), std),
+        attn_norm=_gain(seed, "mtp.attn_norm", d, gain_std),
+        wqkv=normal(seed, "mtp.wqkv", (3 * H * hd, d), std),
+        wo=normal(seed, "mtp.wo", (d, H * hd), std),
+        ffn_norm=_gain(seed, "mtp.ffn_norm", d, gain_std),
+        w_gate_up=normal(seed, "mtp.w_gate_up", (2 * Id, d), std),
+        w_down=normal(seed, "mtp.w_down", (d, Id), std),
+    )
+
+
+def kv_prefix(seed: int, seq: int, n_layers: int, ctx: int, n_heads: int, head_dim: int) -> torch.Tensor:
+    """Committed verifier KV for positions 0..ctx-1 of one sequence, bf16 [L][2][ctx][H][hd] ~N(0,1).
+
+    It stands in for the prefill of the 256 + 100n visual tokens and the prompt; keys are taken
+    as already rotated (the cache stores post-RoPE keys)."""
+    return normal(seed, f"kv.{seq}", (n_layers, 2, ctx, n_heads, head_dim), 1.0)
+
+
+def draft_kv_prefix(seed: int, seq: int, ctx: int, n_heads: int, head_dim: int) -> torch.Tensor:
+    """Committed draft-block KV for rows 0..ctx-1 of one sequence, bf16 [2][ctx][H][hd] ~N(0,1)."""
+    return normal(seed, f"dkv.{seq}", (2, ctx, n_heads, head_dim), 1.0)
