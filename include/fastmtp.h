@@ -1,0 +1,200 @@
+/*
+ * fastmtp.h -- C ABI of the GB300 (sm_103a) FastMTP speculative decode step.
+ *
+ * The operation is the speculative greedy decode step of arXiv 2609.03181 ("Jina-OCR-v1"),
+ * Sec. 3 "Model Architecture" and Sec. 3.1 "Draft-head architecture":
+ *   draft_step   -- the FastMTP draft head (draft-head equation of Sec. 3.1): one shared
+ *                   dense block B_theta applied recursively K times along the diagonal
+ *                   p = j+k-1 (Fig. "FastMTP state-shift alignment"), with the embedding E,
+ *                   output norm N_o and LM head W_lm tied to the verifier;
+ *   verify_step  -- the verifier forward of the DeepSeekMoE decoder (Table "Model
+ *                   specification": 12 layers, d=1280, 64 routed + 2 shared experts, top-6,
+ *                   vocabulary 129,280, RoPE theta=1e6) over the K+1 candidates of every
+ *                   sequence against its paged bf16 KV cache, then greedy acceptance: per-row
+ *                   argmax v_r and the longest equality prefix m (acceptance equation of
+ *                   Sec. 3.1);
+ *   accept_commit-- commit x^_{1:m} then v_{m+1} (the bonus token when m = K), append the
+ *                   K/V of the accepted candidates to the cache, drop the rejected tail.
+ * The committed stream equals plain greedy decoding (K = 0) for any drafts (Sec. 3.1).
+ *
+ * Conventions (all entry points):
+ *  - Pointers marked "dev" are CUDA device pointers on the device that was current at
+ *    spec_init; "host" pointers are host memory.  Sizes are element counts.
+ *  - Weights and KV pools are owned by the caller and borrowed for the context's lifetime.
+ *    The context owns only its workspace (allocated once in spec_init, freed in
+ *    spec_destroy); no step allocates memory.
+ *  - Every step is asynchronous on the stream given to spec_init.  Arguments are validated
+ *    on the host before any launch; a rejected call launches nothing and leaves the state
+ *    unchanged.  Data-dependent faults found on the device (a token id out of range, a page
+ *    index outside the pool, a candidate 0 that is not the pending token, a wait that ran
+ *    out) set a device guard flag instead of trapping; spec_sync() reports it as
+ *    SPEC_EDEVICE.  Kernels never trap and never spin without a time limit.
+ *  - bf16 tensors are row-major with the last dimension contiguous; matrices are stored
+ *    [out_features][in_features].
+ *  - Layout of the verifier KV pool (bf16): [n_layers][n_pages_total][2 (K,V)][n_heads]
+ *    [page_size][head_dim]; keys are stored after RoPE.  The draft-block pool has the same
+ *    layout with one layer.  Both caches of a sequence use the same block table.
+ */
+#ifndef FASTMTP_H
+#define FASTMTP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct spec_ctx spec_ctx;  /* opaque */
+
+typedef enum {
+  SPEC_OK = 0,
+  SPEC_EINVAL = 1,   /* bad argument (host-side check); nothing launched */
+  SPEC_ENOMEM = 2,   /* workspace allocation failed in spec_init */
+  SPEC_ECUDA = 3,    /* a CUDA runtime call failed; message in spec_last_error */
+  SPEC_ESTATE = 4,   /* call out of order (e.g. accept_commit without a verify_step) */
+  SPEC_EDEVICE = 5   /* the device guard flag is set (see spec_sync) */
+} spec_status;
+
+/* Shape contract.  The kernels are built for hidden = 1280, n_heads = 10, head_dim = 128,
+ * n_experts = 64, top_k = 6, n_shared = 2, expert_inter = 896, draft_inter = 3584 (the
+ * paper's decoder with the widths the paper leaves open); spec_init rejects other values of
+ * those fields.  vocab, n_layers, page_size and the capacity fields are free. */
+typedef struct spec_config {
+  int32_t hidden, n_heads, head_dim, n_layers;
+  int32_t n_experts, top_k, n_shared, expert_inter, draft_inter, vocab;
+  int32_t page_size;          /* tokens per KV page, a multiple of 16 */
+  int32_t max_batch;          /* largest B of any step; also the number of sequence slots */
+  int32_t max_pages_per_seq;  /* block-table width */
+  int32_t n_pages_total;      /* pages in each pool */
+  int32_t K_max;              /* largest draft depth K, 0..7 */
+  int32_t max_position;       /* RoPE table length (position limit, e.g. 32768) */
+  float rms_eps, rope_theta;  /* 1e-6, 1e6 */
+} spec_config;
+
+/* One verifier layer (all dev, bf16 unless noted). */
+typedef struct spec_layer_weights {
+  const void* attn_norm;       /* [d] */
+  const void* wqkv;            /* [3*H*hd][d]: q rows, then k rows, then v rows */
+  const void* wo;              /* [d][H*hd] */
+  const void* moe_norm;        /* [d] */
+  const void* router;          /* [E][d] */
+  const void* w_gate_up;       /* [E][2I][d]: gate rows 0..I-1, up rows I..2I-1 */
+  const void* w_down;          /* [E][d][I] */
+  const void* shared_gate_up;  /* [n_shared][2I][d] */
+  const void* shared_down;     /* [n_shared][d][I] */
+  const float* router_bias;    /* fp32 [E] added to the router logits, or NULL */
+} spec_layer_weights;
+
+/* All weights (dev, bf16).  E, N_o and W_lm are shared by the verifier and the draft head
+ * (Sec. 3.1: tied); the mtp_* block is B_theta, enorm/hnorm are N_e/N_h, eh_proj is P. */
+typedef struct spec_weights {
+  const void* embed;            /* [V][d] */
+  const void* lm_head;          /* [V][d] */
+  const void* final_norm;       /* [d] (N_o) */
+  const spec_layer_weights* layers;  /* host array of n_layers */
+  const void* enorm;            /* [d] */
+  const void* hnorm;            /* [d] */
+  const void* eh_proj;          /* [d][2d]: input [N_e(e); N_h(a)] */
+  const void* mtp_attn_norm;    /* [d] */
+  const void* mtp_wqkv;         /* [3*H*hd][d] */
+  const void* mtp_wo;           /* [d][H*hd] */
+  const void* mtp_ffn_norm;     /* [d] */
+  const void* mtp_w_gate_up;    /* [2*Id][d]: gate rows, then up rows */
+  const void* mtp_w_down;       /* [d][Id] */
+} spec_weights;
+
+/* Creates a context on the current device.  kv_pool / draft_kv_pool: dev, layouts above,
+ * n_pages_total pages each.  stream: a cudaStream_t (NULL = legacy default stream).  Builds
+ * the TMA descriptors of every weight matrix and the RoPE table, allocates the workspace
+ * (sized for max_batch x (K_max+1) rows) and zeroes all sequence slots.
+ * Errors: SPEC_EINVAL (shape contract, null pointer, misaligned matrix), SPEC_ENOMEM,
+ * SPEC_ECUDA.  On error *out is NULL. */
+spec_status spec_init(const spec_config* cfg, const spec_weights* w, void* kv_pool,
+                      void* draft_kv_pool, void* stream, spec_ctx** out);
+
+/* Sets sequence slot `slot` to a committed prefix: ctx_len KV positions already in both
+ * pools (positions 0..ctx_len-1 of the verifier cache and rows 0..ctx_len-1 of the draft
+ * cache), pending token `pending` (committed, not yet consumed, at position ctx_len), and
+ * its block table (host int32 [max_pages_per_seq], page ids into both pools; entries the
+ * sequence will never reach may be -1).  The slot has no queued draft rows: the first step
+ * on it must be verify_step with K = 0.  Synchronous with the stream.  Errors: SPEC_EINVAL
+ * (slot, ctx_len, token or page id out of range). */
+spec_status spec_seq_reset(spec_ctx* ctx, int32_t slot, int32_t ctx_len,
+                           const int32_t* block_table, int32_t pending);
+
+/* Queues n_rows (1..K_max+1) draft rows on slot `slot` as if a commit had just made them:
+ * base states b_p (dev bf16 [n_rows][d]) of rows p = ctx_len-n_rows .. ctx_len-1 and the
+ * tokens x_{p+1} that follow them (host int32 [n_rows]; the last one must equal the
+ * pending token).  Lets a caller start the draft head from states computed elsewhere.
+ * Synchronous.  Errors: SPEC_EINVAL. */
+spec_status spec_seq_set_draft_rows(spec_ctx* ctx, int32_t slot, int32_t n_rows,
+                                    const void* b_rows, const int32_t* next_tokens);
+
+/* FastMTP draft step (Sec. 3.1) for B sequences (dev int32 slots[B], distinct).  For each
+ * sequence the rows queued by the last commit enter the draft cache at depth 1 (committed,
+ * base states), then the chain from the last of them drafts x^_1..x^_K.  Writes
+ * cand (dev int32 [B][K+1]) = [pending token, x^_1, .., x^_K], the candidate layout
+ * verify_step takes.  1 <= K <= K_max.  Errors: SPEC_EINVAL, SPEC_ESTATE (a verify is
+ * waiting for its accept_commit). */
+spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int32_t* slots,
+                       int32_t* cand);
+
+/* Verifier forward + greedy acceptance for B sequences.  cand: dev int32 [B][K+1] with
+ * cand[b][0] the pending token of slots[b] and cand[b][1..K] its drafts; candidate r sits at
+ * position ctx_len + r.  Writes verifier_tokens (dev int32 [B][K+1], v_{r+1} = argmax of row
+ * r, lowest id on ties) and accept_len (dev int32 [B], m in 0..K).  The K/V of the
+ * candidates are staged in the workspace, not yet in the pools.  0 <= K <= K_max; K = 0 is
+ * one step of plain greedy decoding.  Errors: SPEC_EINVAL, SPEC_ESTATE (previous verify not
+ * committed). */
+spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const int32_t* slots,
+                        const int32_t* cand, int32_t* verifier_tokens, int32_t* accept_len);
+
+/* Commits the last verify_step (same B and slots): copies the staged K/V of candidates
+ * 0..m into the verifier pool, advances ctx_len by m+1, makes v_{m+1} the pending token and
+ * queues the m+1 new rows for the next draft_step.  Writes committed (dev int32 [B][K+1]:
+ * x^_1..x^_m, v_{m+1}; entries past m+1 are -1) and n_committed (dev int32 [B] = m+1).
+ * Errors: SPEC_EINVAL, SPEC_ESTATE (no verify to commit). */
+spec_status accept_commit(spec_ctx* ctx, int32_t B, const int32_t* slots, int32_t* committed,
+                          int32_t* n_committed);
+
+/* Waits for the context's stream and reports the device guard flag: SPEC_OK, or
+ * SPEC_EDEVICE with the flag bits in spec_last_error (the flag is then cleared).  Also
+ * SPEC_ECUDA if the stream reports an error. */
+spec_status spec_sync(spec_ctx* ctx);
+
+/* Reads one slot's state (synchronous): committed KV length and pending token. */
+spec_status spec_seq_state(spec_ctx* ctx, int32_t slot, int32_t* ctx_len, int32_t* pending);
+
+/* Workspace views for tests and statistics.  Copies (synchronously) `bytes` bytes of the
+ * named workspace tensor into host memory `dst`.  Valid after the step that writes it:
+ *   SPEC_WS_B          bf16 [B][K+1][d]    post-norm verifier states b = N_o(h_L)
+ *   SPEC_WS_ROUTE_IDX  int32 [L][B*(K+1)][top_k] selected experts per layer (row b*(K+1)+r)
+ *   SPEC_WS_ROUTE_GATE fp32 [L][B*(K+1)][top_k] their router probabilities
+ *   SPEC_WS_EXPERT_CNT int32 [L][n_experts] tokens routed to each expert
+ *   SPEC_WS_DRAFT_U    bf16 [K][B][d]      draft states u^(k) of the last draft_step
+ *   SPEC_WS_HIDDEN     fp32 [B*(K+1)][d]   residual stream after the last layer
+ * Errors: SPEC_EINVAL (unknown id or bytes larger than the tensor). */
+enum { SPEC_WS_B = 0, SPEC_WS_ROUTE_IDX = 1, SPEC_WS_ROUTE_GATE = 2, SPEC_WS_EXPERT_CNT = 3,
+       SPEC_WS_DRAFT_U = 4, SPEC_WS_HIDDEN = 5 };
+spec_status spec_read_workspace(spec_ctx* ctx, int32_t id, void* dst, size_t bytes);
+
+/* Dense projection Y = X W^T on the tcgen05 GEMM engine every projection of the step runs
+ * on (X dev bf16 [M][Kdim], W dev bf16 [N][Kdim], Y dev fp32 [M][N]); M >= 1, N a multiple
+ * of 128 or any N >= 1 (a ragged last tile is masked), Kdim a multiple of 64, both base
+ * pointers 16-byte aligned.  Asynchronous on `stream`; needs no context.  Errors:
+ * SPEC_EINVAL, SPEC_ECUDA. */
+spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, int32_t N,
+                           int32_t Kdim, void* stream);
+
+/* Frees the workspace.  Borrowed weights and pools are untouched.  NULL is ignored. */
+void spec_destroy(spec_ctx* ctx);
+
+/* Last error message of the context ("" if none); NULL ctx gives the last error of
+ * spec_init / spec_gemm_bf16 in this thread. */
+const char* spec_last_error(const spec_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FASTMTP_H */

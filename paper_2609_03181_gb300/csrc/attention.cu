@@ -1,0 +1,196 @@
+// Split-KV decode attention over a paged bf16 KV cache plus staged candidate rows.
+//
+// Each sequence has R queries at consecutive positions p0..p0+R-1 (the K+1 verify
+// candidates, or one draft row).  Keys at positions < ctx_len live in the sequence's pages,
+// keys at positions >= ctx_len in a staging buffer (candidates not yet committed).  The key
+// range is cut into chunks of 128 positions fixed by absolute position; one CTA per
+// (chunk, head, sequence) stages the chunk's K and V in shared memory with 16-byte
+// cp.async copies, scores every (query, key) pair in fp32, and writes the chunk's
+// (max, sum, unnormalised output) per query.  A second kernel merges the chunks of each query
+// in chunk order.  Masked keys contribute exact zeros, so a query's result is the same
+// whether its key sits in a page or in staging and however many other queries share the
+// chunk: greedy decoding (K = 0) and speculative verification see identical rows.
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace fm {
+
+constexpr int kCH = kAttnChunk;
+constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 4 + kMaxR * kCH * 4;
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
+  extern __shared__ __align__(16) uint8_t asmem[];
+  bf16* sK = reinterpret_cast<bf16*>(asmem);               // [kCH][kHD], 16-byte chunks swizzled by row
+  bf16* sV = sK + kCH * kHD;
+  float* sq = reinterpret_cast<float*>(sV + kCH * kHD);    // [R][kHD]
+  float* sp = sq + kMaxR * kHD;                           // [R][kCH] scores, then probabilities
+
+  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int R = a.R;
+  const int slot = a.slots[b];
+  const int sl = a.seq_len[slot];
+  const int p0 = sl + a.qoff;
+  const int last = p0 + R - 1;
+  const int start = c * kCH;
+  if (start > last || p0 < 0) return;
+  const int nk = min(kCH, last + 1 - start);
+  const int tid = threadIdx.x;
+
+  // K and V rows of the chunk -> shared memory (zero-filled past the last key)
+  for (int v = tid; v < kCH * 16; v += 128) {
+    const int j = v >> 4, ch = v & 15;
+    const int pos = start + j;
+    const bf16* srck = a.pool;
+    const bf16* srcv = a.pool;
+    int bytes = 0;
+    if (j < nk) {
+      if (pos < sl) {
+        const int pi = pos / a.page_size;
+        const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+        if (page >= 0 && page < a.n_pages) {
+          const size_t base = ((static_cast<size_t>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
+          srck = a.pool + base;
+          srcv = a.pool + base + static_cast<size_t>(kH) * a.page_size * kHD;
+          bytes = 16;
+        } else if (ch == 0) {
+          atomicOr(a.err, ERR_PAGE_RANGE);
+        }
+      } else {
+        const size_t base = b * a.stage_seq_stride + static_cast<size_t>(pos - sl) * a.stage_row_stride +
+                            static_cast<size_t>(h) * kHD;
+        srck = a.stage + base;
+        srcv = a.stage + base + a.stage_kv_stride;
+        bytes = 16;
+      }
+    }
+    const int sw = ((ch ^ (j & 7)) * 8);
+    cp_async16(sK + j * kHD + sw, srck + ch * 8 * (bytes ? 1 : 0), bytes);
+    cp_async16(sV + j * kHD + sw, srcv + ch * 8 * (bytes ? 1 : 0), bytes);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+
+  // queries, pre-scaled by log2(e) / sqrt(hd) so that softmax uses exp2
+  const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));
+  const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
+  for (int v = tid; v < R * kHD; v += 128) {
+    const int r = v / kHD, d = v % kHD;
+    sq[v] = a.q[(static_cast<size_t>(qrow0 + r) * kH + h) * kHD + d] * qscale;
+  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
+
+  // scores: thread j owns key j of the chunk
+  {
+    const int j = tid;
+    float s[kMaxR];
+#pragma unroll
+    for (int r = 0; r < kMaxR; ++r) s[r] = 0.f;
+#pragma unroll 4
+    for (int ch = 0; ch < 16; ++ch) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(sK + j * kHD + ((ch ^ (j & 7)) * 8));
+      const bf16* kv = reinterpret_cast<const bf16*>(&raw);
+      float kf[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) kf[u] = __bfloat162float(kv[u]);
+#pragma unroll
+      for (int r = 0; r < kMaxR; ++r) {
+        if (r < R) {
+          const float* qr = sq + r * kHD + ch * 8;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) s[r] += qr[u] * kf[u];
+        }
+      }
+    }
+    const int pos = start + j;
+#pragma unroll
+    for (int r = 0; r < kMaxR; ++r)
+      if (r < R) sp[r * kCH + j] = (j < nk && pos <= p0 + r) ? s[r] : -INFINITY;
+  }
+  __syncthreads();
+
+  // per query: chunk max, probabilities (exact zeros where masked), sum
+  const int warp = tid >> 5, lane = tid & 31;
+  float* part = a.part + ((static_cast<size_t>(b) * kH + h) * a.n_chunks + c) * R * (kHD + 2);
+  for (int r = warp; r < R; r += 4) {
+    float x[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) x[i] = sp[r * kCH + lane + 32 * i];
+    const float m = warp_max(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])));
+    float l = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float p = (m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m);
+      sp[r * kCH + lane + 32 * i] = p;
+      l += p;
+    }
+    l = warp_sum(l);
+    if (lane == 0) {
+      part[r * (kHD + 2) + kHD] = m;
+      part[r * (kHD + 2) + kHD + 1] = l;
+    }
+  }
+  __syncthreads();
+
+  // P V: thread d owns output dim d
+  {
+    const int d = tid;
+    float acc[kMaxR];
+#pragma unroll
+    for (int r = 0; r < kMaxR; ++r) acc[r] = 0.f;
+    for (int j = 0; j < nk; ++j) {
+      const float vv = __bfloat162float(sV[j * kHD + (((d >> 3) ^ (j & 7)) * 8) + (d & 7)]);
+#pragma unroll
+      for (int r = 0; r < kMaxR; ++r)
+        if (r < R) acc[r] += sp[r * kCH + j] * vv;
+    }
+#pragma unroll
+    for (int r = 0; r < kMaxR; ++r)
+      if (r < R) part[r * (kHD + 2) + d] = acc[r];
+  }
+}
+
+// Merges the chunks 0..floor(p/128) of each query in chunk order: softmax-weighted combination.
+__global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
+  const int R = a.R;
+  const int b = blockIdx.x / R, r = blockIdx.x % R, h = blockIdx.y;
+  const int slot = a.slots[b];
+  const int p = a.seq_len[slot] + a.qoff + r;
+  if (p < 0) return;
+  const int lastc = p / kCH;
+  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * a.n_chunks * R * (kHD + 2);
+  float M = -INFINITY;
+  for (int c = 0; c <= lastc; ++c) M = fmaxf(M, part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + kHD]);
+  float L = 0.f, O = 0.f;
+  for (int c = 0; c <= lastc; ++c) {
+    const float* pc = part + (static_cast<size_t>(c) * R + r) * (kHD + 2);
+    const float mc = pc[kHD];
+    const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
+    L += pc[kHD + 1] * w;
+    O += pc[threadIdx.x] * w;
+  }
+  a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + threadIdx.x] =
+      __float2bfloat16(O / L);
+}
+
+cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(attn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  attn_chunk_kernel<<<dim3(a.n_chunks, kH, B), 128, kAttnSmem, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  attn_merge_kernel<<<dim3(B * a.R, kH), 128, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace fm

@@ -1,0 +1,538 @@
+// Persistent tcgen05 GEMM engine for the decode regime (few activation rows, weight bytes
+// dominate).  Every projection of the verify and draft steps runs here: QKV (+RoPE, KV
+// staging), O-proj (+residual), the grouped routed/shared expert SwiGLU FFNs, the draft
+// block's projections and the LM head (+argmax, logits never written).
+//
+// Swap-AB tiling: the weight matrix W [N][K] is the MMA's A operand (M = 128 weight rows
+// per tile), the activations X [rows][K] are the B operand (N = 16..256 rows), so a tile
+// D^T[128][rows] = W_tile X^T accumulates in TMEM.  Both operands are K-major bf16 tiles of
+// 64 columns loaded by TMA with the 128-byte swizzle.  One CTA per SM; warp 0 issues TMA,
+// warp 1 owns TMEM and issues tcgen05.mma from one thread, warps 2-5 drain the
+// double-buffered accumulator through tcgen05.ld and run the fused epilogue.
+//
+// Determinism: each output element is the fp32 sum of its K range in the fixed k-chunk
+// order; split-K partials are reduced by the last-arriving CTA of a tile in split order (an
+// atomic ticket, no spin-wait).  Split counts depend on the matrix shape only, so a row's
+// result never depends on how many other rows share the launch.
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace fm {
+
+template <int NMAX>
+struct Cfg {
+  static constexpr int A_BYTES = 128 * 128;            // 128 rows x 64 bf16
+  static constexpr int B_BYTES = NMAX * 128;           // NMAX rows x 64 bf16
+  static constexpr int STAGES = (NMAX <= 64) ? 8 : 4;
+  static constexpr int TMEM_COLS = 2 * NMAX;           // two accumulator buffers
+  static constexpr int XCHG_FLOATS = 128 * 17;
+  static constexpr int SMEM_BYTES = 1024 + STAGES * (A_BYTES + B_BYTES) + 256 + XCHG_FLOATS * 4 + 4 * 16 * 8;
+};
+
+struct Item {
+  int e, n_tile, b_row, out_row, rows, split, box_log;
+};
+
+__device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it) {
+  if (a.items != nullptr) {
+    const int4 v = a.items[i];
+    it.e = v.x & 0xFFFF;
+    it.n_tile = v.x >> 16;
+    it.b_row = v.y;
+    it.out_row = v.z;
+    it.rows = v.w;
+    it.split = 0;
+    int bl = 0;
+    while ((16 << bl) < it.rows) ++bl;
+    it.box_log = bl;
+  } else {
+    const int mt = i % a.m_tiles;
+    const int t = i / a.m_tiles;
+    it.split = t % a.split_k;
+    it.n_tile = t / a.split_k;
+    it.e = 0;
+    const int box = 16 << a.box_log;
+    it.out_row = mt * box;
+    it.b_row = a.b_row_off + it.out_row;
+    it.rows = min(box, a.M - it.out_row);
+    it.box_log = a.box_log;
+  }
+}
+
+// ------------------------------------------------------------------ epilogues
+// v: 16 accumulator columns (activation rows j0..j0+15 of the item) of tile row `row`.
+template <int EPI>
+__device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int row, int j0, float (&v)[16],
+                                          float* xchg, float* am_s_val, int* am_s_idx) {
+  const int lane = threadIdx.x & 31;
+  if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
+    const int n = it.n_tile * 128 + row;
+    if (n < a.N) {
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) {
+        const int r = j0 + jj;
+        if (r < it.rows) {
+          float* p = a.out + static_cast<size_t>(it.out_row + r) * a.ldo + n;
+          if constexpr (EPI == EPI_RESID) *p += v[jj];
+          else *p = v[jj];
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_SCATTER) {
+    const int n = it.n_tile * 128 + row;
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      const int r = j0 + jj;
+      if (r < it.rows) {
+        const int m = it.out_row + r;
+        const int t = a.sorted_tok[m], s = a.sorted_slot[m];
+        a.y[(static_cast<size_t>(t) * kSlots + s) * kD + n] = v[jj];
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
+    named_bar_sync(1, 128);
+    if (row < 64) {
+      const int f = it.n_tile * 64 + row;
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) {
+        const int r = j0 + jj;
+        if (r < it.rows) {
+          const float u = xchg[(row + 64) * 17 + jj];
+          a.act[static_cast<size_t>(it.out_row + r) * a.ld_act + f] = __float2bfloat16(silu_f(v[jj]) * u);
+        }
+      }
+    }
+    named_bar_sync(1, 128);
+  } else if constexpr (EPI == EPI_QKV) {
+    const int which = it.n_tile / kH;   // 0 q, 1 k, 2 v
+    const int head = it.n_tile % kH;
+    float partner[16];
+    if (which < 2) {
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
+      named_bar_sync(1, 128);
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) partner[jj] = xchg[(row ^ 64) * 17 + jj];
+      named_bar_sync(1, 128);
+    }
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      const int r = j0 + jj;
+      if (r >= it.rows) continue;
+      const int m = it.out_row + r;
+      float val = v[jj];
+      if (which < 2) {
+        int p = a.pos[m];
+        if (p < 0 || p >= a.max_pos) {
+          atomicOr(a.err, ERR_POSITION);
+          p = 0;
+        }
+        const float2 cs = a.rope[static_cast<size_t>(p) * (kHD / 2) + (row & 63)];
+        val = (row < 64) ? (v[jj] * cs.x - partner[jj] * cs.y) : (v[jj] * cs.x + partner[jj] * cs.y);
+      }
+      if (which == 0) {
+        a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + row] = val;
+      } else {
+        const long long off = a.kv_rowoff[m];
+        if (off >= 0)
+          a.kv_base[off + (which == 2 ? a.v_off : 0) + head * a.head_stride + row] = __float2bfloat16(val);
+      }
+    }
+  } else if constexpr (EPI == EPI_ARGMAX) {
+    const int q = (threadIdx.x >> 5) & 3;
+    const int n = it.n_tile * 128 + row;
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      float bv = (n < a.N) ? v[jj] : -INFINITY;
+      int bi = n;
+      warp_argmax(bv, bi);
+      if (lane == 0) {
+        am_s_val[q * 16 + jj] = bv;
+        am_s_idx[q * 16 + jj] = bi;
+      }
+    }
+    named_bar_sync(1, 128);
+    if (row < 16) {
+      const int r = j0 + row;
+      if (r < it.rows) {
+        float bv = am_s_val[row];
+        int bi = am_s_idx[row];
+#pragma unroll
+        for (int w = 1; w < 4; ++w)
+          if (better(am_s_val[w * 16 + row], am_s_idx[w * 16 + row], bv, bi)) {
+            bv = am_s_val[w * 16 + row];
+            bi = am_s_idx[w * 16 + row];
+          }
+        const size_t o = static_cast<size_t>(it.n_tile) * a.am_ld + it.out_row + r;
+        a.am_val[o] = bv;
+        a.am_idx[o] = bi;
+      }
+    }
+    named_bar_sync(1, 128);
+  }
+}
+
+// ------------------------------------------------------------------ kernel
+template <int NMAX, int EPI>
+__global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
+  using C = Cfg<NMAX>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t base_u32 = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
+  uint8_t* smA = smem;
+  uint8_t* smB = smA + C::STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smB + C::STAGES * C::B_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + C::STAGES;
+  uint64_t* tfull = bars + 2 * C::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* fin = tempty + 2;
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(fin + 1);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+  int* s_vote = const_cast<int*>(s_abort) + 1;   // [4]
+  int* s_last = s_vote + 4;
+  float* xchg = reinterpret_cast<float*>(smem + C::STAGES * (C::A_BYTES + C::B_BYTES) + 256);
+  float* am_s_val = xchg + C::XCHG_FLOATS;
+  int* am_s_idx = reinterpret_cast<int*>(am_s_val + 64);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&tfull[s], 1);
+      mbar_init(&tempty[s], 4);
+    }
+    mbar_init(fin, 1);
+    *s_abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&a.a_map[0]);
+    tma_prefetch_desc(&a.a_map[1]);
+  }
+  if (warp == 1) {
+    tmem_alloc(s_tmem, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+
+  const int n_items = (a.items != nullptr) ? *a.n_items_dev : a.n_items;
+  const int kc_total = a.K / 64;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_x = l2_policy_evict_last();
+      uint32_t g = 0;   // loads issued
+      bool failed = false;
+      for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x) {
+        Item it;
+        get_item(a, i, it);
+        const int src = (a.items != nullptr && it.e >= a.n_routed) ? 1 : 0;
+        const int el = it.e - (src ? a.n_routed : 0);
+        const CUtensorMap* amap = &a.a_map[src];
+        const CUtensorMap* bmap = &a.b_map[src][it.box_log];
+        const uint32_t bytes = C::A_BYTES + (16u << it.box_log) * 128u;
+        const int kc0 = it.split * kc_total / a.split_k, kc1 = (it.split + 1) * kc_total / a.split_k;
+        for (int kc = kc0; kc < kc1; ++kc, ++g) {
+          const int st = g % C::STAGES;
+          const uint32_t ph = (g / C::STAGES) & 1u;
+          if (!mbar_wait(&empty[st], ph ^ 1u, s_abort)) {
+            failed = true;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[st], bytes);
+          uint8_t* sa = smA + st * C::A_BYTES;
+          const int k = kc * 64;
+          if (a.paired) {
+            const int r0 = it.n_tile * 64;
+            if (a.a3d) {
+              tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
+              tma_load_3d(sa + 8192, amap, &full[st], k, a.half_rows + r0, el, pol_w);
+            } else {
+              tma_load_2d(sa, amap, &full[st], k, r0, pol_w);
+              tma_load_2d(sa + 8192, amap, &full[st], k, a.half_rows + r0, pol_w);
+            }
+          } else {
+            const int r0 = it.n_tile * 128;
+            if (a.a3d) tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
+            else tma_load_2d(sa, amap, &full[st], k, r0, pol_w);
+          }
+          tma_load_2d(smB + st * C::B_BYTES, bmap, &full[st], k, it.b_row, pol_x);
+        }
+      }
+      if (failed) {
+        *s_abort = 1;
+        atomicOr(a.err, ERR_WAIT_TIMEOUT);
+        // let the copies still in flight land before the CTA's shared memory is released
+        volatile int never = 0;
+        const uint32_t back = g < C::STAGES ? g : C::STAGES;
+        for (uint32_t b = 1; b <= back; ++b) {
+          const uint32_t gg = g - b;
+          mbar_wait(&full[gg % C::STAGES], (gg / C::STAGES) & 1u, &never, 100000000ull);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      uint32_t g = 0;
+      int local = 0;
+      bool failed = false;
+      for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x, ++local) {
+        Item it;
+        get_item(a, i, it);
+        const int acc = local & 1;
+        const uint32_t acc_ph = (local >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, s_abort)) {
+          failed = true;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * NMAX;
+        const uint32_t idesc = idesc_bf16(128, 16 << it.box_log);
+        const int kc0 = it.split * kc_total / a.split_k, kc1 = (it.split + 1) * kc_total / a.split_k;
+        for (int kc = kc0; kc < kc1; ++kc, ++g) {
+          const int st = g % C::STAGES;
+          const uint32_t ph = (g / C::STAGES) & 1u;
+          if (!mbar_wait(&full[st], ph, s_abort)) {
+            failed = true;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = sw128_kmajor_desc(smem_u32(smA + st * C::A_BYTES));
+          const uint64_t bd = sw128_kmajor_desc(smem_u32(smB + st * C::B_BYTES));
+#pragma unroll
+          for (int s = 0; s < 4; ++s)   // 4 x K=16 per 64-column chunk: +32 B in the swizzled row
+            tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > kc0 || s > 0) ? 1u : 0u);
+          tc_commit(&empty[st]);
+        }
+        if (failed) break;
+        tc_commit(&tfull[acc]);
+      }
+      if (failed) {
+        *s_abort = 1;
+        atomicOr(a.err, ERR_WAIT_TIMEOUT);
+        if (g > 0) {
+          // every MMA issued so far has completed once `fin` flips
+          tc_commit(fin);
+          volatile int never = 0;
+          mbar_wait(fin, 0, &never, 100000000ull);
+        }
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue (warps 2..5)
+    const int q = warp & 3;                // TMEM lane quadrant of this warp
+    const int row = q * 32 + lane;         // tile row = weight row within the tile
+    const int ew = warp - 2;
+    int local = 0;
+    for (int i = blockIdx.x; i < n_items; i += gridDim.x, ++local) {
+      Item it;
+      get_item(a, i, it);
+      const int acc = local & 1;
+      const uint32_t acc_ph = (local >> 1) & 1;
+      bool ok = mbar_wait(&tfull[acc], acc_ph, s_abort);
+      ok = __all_sync(0xffffffffu, ok);
+      if (lane == 0) s_vote[ew] = ok ? 1 : 0;
+      named_bar_sync(1, 128);
+      const bool all_ok = s_vote[0] && s_vote[1] && s_vote[2] && s_vote[3];
+      named_bar_sync(1, 128);
+      if (!all_ok) {
+        *s_abort = 1;
+        atomicOr(a.err, ERR_WAIT_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * NMAX;
+      const int nchunks = (it.rows + 15) >> 4;
+      float v[16];
+      if (a.split_k == 1) {
+        for (int c = 0; c < nchunks; ++c) {
+          tc_ld16(tb + c * 16, v);
+          epi_chunk<EPI>(a, it, row, c * 16, v, xchg, am_s_val, am_s_idx);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+      } else {
+        const int n = it.n_tile * 128 + row;
+        for (int c = 0; c < nchunks; ++c) {
+          tc_ld16(tb + c * 16, v);
+#pragma unroll
+          for (int jj = 0; jj < 16; ++jj) {
+            const int r = c * 16 + jj;
+            if (r < it.rows && n < a.N)
+              a.sk_ws[(static_cast<size_t>(it.split) * a.sk_rows + it.out_row + r) * a.N + n] = v[jj];
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (threadIdx.x == 64) {
+          const int tile = it.n_tile * a.m_tiles + it.out_row / (16 << it.box_log);
+          const int old = atomicAdd(&a.sk_tickets[tile], 1);
+          *s_last = (old == a.split_k - 1) ? 1 : 0;
+          if (old == a.split_k - 1) a.sk_tickets[tile] = 0;
+        }
+        named_bar_sync(1, 128);
+        if (*s_last) {
+          __threadfence();
+          for (int c = 0; c < nchunks; ++c) {
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) {
+              const int r = c * 16 + jj;
+              float s = 0.f;
+              if (r < it.rows && n < a.N)
+                for (int sp = 0; sp < a.split_k; ++sp)
+                  s += __ldcg(&a.sk_ws[(static_cast<size_t>(sp) * a.sk_rows + it.out_row + r) * a.N + n]);
+              v[jj] = s;
+            }
+            epi_chunk<EPI>(a, it, row, c * 16, v, xchg, am_s_val, am_s_idx);
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+namespace {
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+template <int NMAX, int EPI>
+cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s) {
+  static bool attr = false;
+  auto k = gemm_tc_kernel<NMAX, EPI>;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<NMAX>::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  k<<<grid, 192, Cfg<NMAX>::SMEM_BYTES, s>>>(a);
+  return cudaGetLastError();
+}
+}  // namespace
+
+bool encode_map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
+                   std::string* err) {
+  auto fn = get_encode();
+  if (fn == nullptr) {
+    *err = "cuTensorMapEncodeTiled not available from the driver";
+    return false;
+  }
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *err = "cuTensorMapEncodeTiled (2-D) failed with code " + std::to_string(static_cast<int>(r));
+    return false;
+  }
+  return true;
+}
+
+bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t depth,
+                   uint32_t box_rows, std::string* err) {
+  auto fn = get_encode();
+  if (fn == nullptr) {
+    *err = "cuTensorMapEncodeTiled not available from the driver";
+    return false;
+  }
+  cuuint64_t dims[3] = {inner, rows, depth};
+  cuuint64_t strides[2] = {inner * 2, inner * rows * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    *err = "cuTensorMapEncodeTiled (3-D) failed with code " + std::to_string(static_cast<int>(r));
+    return false;
+  }
+  return true;
+}
+
+bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err) {
+  for (int b = 0; b < 5; ++b)
+    if (!encode_map_2d(&maps[b], base, inner, rows, 16u << b, err)) return false;
+  return true;
+}
+
+int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+int dense_split_k(int N, int K) {
+  const int n_tiles = (N + 127) / 128;
+  const int kc = K / 64;
+  int s = (148 + n_tiles - 1) / n_tiles;
+  if (s > kc) s = kc;
+  if (s < 1) s = 1;
+  return s;
+}
+
+cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s) {
+  if (grid <= 0) return cudaSuccess;
+#define FM_CASE(E)                                                                      \
+  case E:                                                                               \
+    return nmax <= 64 ? launch_one<64, E>(a, grid, s) : launch_one<256, E>(a, grid, s);
+  switch (epi) {
+    FM_CASE(EPI_F32)
+    FM_CASE(EPI_RESID)
+    FM_CASE(EPI_QKV)
+    FM_CASE(EPI_SWIGLU)
+    FM_CASE(EPI_SCATTER)
+    FM_CASE(EPI_ARGMAX)
+    default:
+      return cudaErrorInvalidValue;
+  }
+#undef FM_CASE
+}
+
+}  // namespace fm

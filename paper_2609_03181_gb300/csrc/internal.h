@@ -1,0 +1,137 @@
+// Host-side interfaces between the FastMTP translation units: the GEMM engine's argument
+// block and the launchers of every kernel.  Not part of the public ABI (include/fastmtp.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+namespace fm {
+
+typedef __nv_bfloat16 bf16;
+
+// Fixed widths of the decoder the kernels are built for.
+constexpr int kD = 1280;        // hidden
+constexpr int kH = 10;          // heads
+constexpr int kHD = 128;        // head dim
+constexpr int kE = 64;          // routed experts
+constexpr int kTopK = 6;
+constexpr int kShared = 2;
+constexpr int kI = 896;         // expert intermediate
+constexpr int kId = 3584;       // draft-block intermediate
+constexpr int kSlots = kTopK + kShared;   // per-token expert outputs combined
+constexpr int kAttnChunk = 128;           // split-KV chunk (keys), fixed by absolute position
+constexpr int kMaxR = 8;                  // K_max + 1 <= 8 candidate rows per sequence
+
+// ------------------------------------------------------------------------- GEMM engine
+enum EpiKind : int {
+  EPI_F32 = 0,      // out[row][n] = acc
+  EPI_RESID = 1,    // out[row][n] += acc (fp32 residual stream)
+  EPI_QKV = 2,      // RoPE on q/k, q -> fp32 buffer, k/v -> bf16 cache rows
+  EPI_SWIGLU = 3,   // tile = 64 gate rows + 64 up rows -> bf16 silu(g)*u
+  EPI_SCATTER = 4,  // expert down: out row (token, slot) from the sorted index
+  EPI_ARGMAX = 5    // per-tile (max, argmax) of each column (LM head)
+};
+
+// One work item: weight tile x activation rows.  x = expert | n_tile << 16, y = TMA row of
+// the activation source, z = output row (row index of the epilogue), w = number of rows.
+// Dense launches generate items implicitly; grouped launches read them from a device list.
+struct GemmArgs {
+  CUtensorMap a_map[2];        // weights: [0] main / routed experts, [1] shared experts
+  CUtensorMap b_map[2][5];     // activations: [source][box height 16,32,64,128,256]
+  int N;                       // output features of the weight matrix (bounds of the last tile)
+  int K;                       // reduction length, multiple of 64
+  int a3d;                     // weight maps are 3-D [experts][rows][K]
+  int paired;                  // SwiGLU: tile rows 0..63 gate, 64..127 up (offset half_rows)
+  int half_rows;
+  int n_routed;                // experts with id >= n_routed read a_map[1] and source 1
+  int split_k;                 // >= 1, fixed per matrix shape
+  const int4* items;           // grouped: device item list
+  const int* n_items_dev;      //          and its length
+  int n_items;                 // dense: number of items
+  int M;                       // dense: activation rows
+  int m_tiles, box_log;        // dense: row tiles of 16 << box_log rows
+  int b_row_off;               // dense: first activation row read by TMA
+  int n_tiles;                 // dense: weight tiles
+  // epilogue operands
+  float* out; int ldo;                                        // F32 / RESID
+  float* q_out; bf16* kv_base; const long long* kv_rowoff;   // QKV
+  long long head_stride, v_off; const int* pos; const float2* rope; int max_pos;
+  bf16* act; int ld_act;                                      // SWIGLU
+  float* y; const int* sorted_tok; const int* sorted_slot;    // SCATTER
+  float* am_val; int* am_idx; int am_ld;                      // ARGMAX partials [n_tile][am_ld]
+  float* sk_ws; int* sk_tickets; int sk_rows;                 // split-K partials / tickets
+  int* err;
+};
+
+// Encodes a 2-D or 3-D bf16 tensor map with the 128-byte swizzle (box inner dim 64).
+bool encode_map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
+                   std::string* err);
+bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t depth,
+                   uint32_t box_rows, std::string* err);
+// Fills b_map[src][*] for an activation buffer of `rows` x `inner` bf16.
+bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err);
+
+// Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).
+cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s);
+int num_sms();
+
+// Split-K count of a dense matrix: depends on (N, K) only, never on M, so every row's sum
+// order is the same at any batch size.
+int dense_split_k(int N, int K);
+
+// ------------------------------------------------------------------------- other kernels
+struct AttnArgs {
+  const float* q;              // [rows][H][hd] fp32
+  const int* q_row0;           // per sequence first query row (NULL: b * R)
+  int R;                       // queries per sequence
+  int qoff;                    // query r of sequence b sits at seq_len[slot] + qoff + r
+  const int* slots; const int* seq_len;   // keys at positions < seq_len[slot] are in pages
+  const bf16* pool; int page_size; int n_pages; const int* block_table; int max_pages;
+  const bf16* stage;           // keys at positions >= seq_len[slot]: staged row (pos - seq_len)
+  long long stage_seq_stride, stage_row_stride, stage_kv_stride;
+  float* part;                 // [B][H][n_chunks][R][kHD + 2]
+  int n_chunks;
+  bf16* out;                   // [B*R][H*hd]
+  int out_row_stride_seq;      // rows of out per sequence (R)
+  int* err;
+};
+cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s);
+
+cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
+                              const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
+                              float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int* err,
+                              cudaStream_t s);
+cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
+cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
+                          const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s);
+cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
+                           int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
+                           cudaStream_t s);
+cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
+                           bf16* out, cudaStream_t s);
+cudaError_t argmax_final_launch(int mode, const float* am_val, const int* am_idx, int n_tiles, int am_ld,
+                                int B, int R, const int* cand, int* vtok_out, int* accept_out,
+                                int* m_ws, int* vtok_ws, cudaStream_t s);
+cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots, const int* m_ws, const int* vtok_ws,
+                          const int* cand_ws, const bf16* stage, bf16* pool, int L, int n_pages,
+                          int page_size, const int* block_table, int max_pages, int* seq_len, int* pending,
+                          const bf16* b_ws, bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
+                          int* n_committed, int* err, cudaStream_t s);
+cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len, const int* pending,
+                              const int* draft_n, const bf16* draft_b, const int* draft_tok,
+                              const bf16* embed, int vocab, const bf16* enorm, const bf16* hnorm, float eps,
+                              bf16* dcat, int* pos, long long* kv_rowoff, int* last_row, int page_size,
+                              const int* block_table, int max_pages, int n_pages, int* cand, int cand_ld,
+                              int* err, cudaStream_t s);
+cudaError_t gather_rows_launch(const float* src, const int* rows, int B, float* dst, cudaStream_t s);
+cudaError_t draft_next_launch(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int B, int k,
+                              int K, const int* slots, const int* seq_len, const bf16* u, const bf16* embed,
+                              const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
+                              long long* kv_rowoff, long long dstage_seq_stride, int* cand, int cand_ld,
+                              cudaStream_t s);
+
+}  // namespace fm

@@ -1,0 +1,559 @@
+// Latency-bound kernels of the FastMTP step: embedding + RMSNorm, RMSNorm, router
+// (norm, logits, softmax, top-6), token permute/scatter by expert, MoE combine (+ the next
+// RMSNorm), the argmax reduction with the greedy-accept epilogue, the KV commit, and the
+// glue of the draft chain.  Every reduction runs in a fixed order, so a row's result never
+// depends on the other rows of the batch.
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace fm {
+
+// Sum over a 128-thread block in a fixed order (warp trees, then warps 0..3).
+__device__ __forceinline__ float block128_sum(float v, float* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  __syncthreads();
+  const float s = ((red[0] + red[1]) + red[2]) + red[3];
+  __syncthreads();
+  return s;
+}
+
+// x (10 values per thread, element i = tid + 128*k) -> bf16 x * rsqrt(mean(x^2) + eps) * gain
+__device__ __forceinline__ void norm_row_store(const float (&x)[10], const bf16* gain, float eps, bf16* out,
+                                               float* red) {
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < 10; ++k) ss += x[k] * x[k];
+  ss = block128_sum(ss, red);
+  const float inv = rsqrtf(ss / kD + eps);
+#pragma unroll
+  for (int k = 0; k < 10; ++k) {
+    const int i = threadIdx.x + 128 * k;
+    out[i] = __float2bfloat16(x[k] * inv * __bfloat162float(gain[i]));
+  }
+}
+
+// ---------------------------------------------------------------- embedding + norm
+__global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R, const int* slots, const int* pending,
+                                                         const int* seq_len, const bf16* embed, int vocab,
+                                                         const bf16* gain, float eps, float* h, bf16* xn, int* pos,
+                                                         long long* kv_rowoff, int stage_R, int* err) {
+  __shared__ float red[4];
+  const int row = blockIdx.x, b = row / R, r = row % R;
+  const int slot = slots[b];
+  int tok = cand[row];
+  if (tok < 0 || tok >= vocab) {
+    if (threadIdx.x == 0) atomicOr(err, ERR_TOKEN_RANGE);
+    tok = 0;
+  }
+  if (r == 0 && tok != pending[slot] && threadIdx.x == 0) atomicOr(err, ERR_PENDING);
+  const bf16* e = embed + static_cast<size_t>(tok) * kD;
+  float x[10];
+#pragma unroll
+  for (int k = 0; k < 10; ++k) {
+    const int i = threadIdx.x + 128 * k;
+    x[k] = __bfloat162float(e[i]);
+    h[static_cast<size_t>(row) * kD + i] = x[k];
+  }
+  norm_row_store(x, gain, eps, xn + static_cast<size_t>(row) * kD, red);
+  if (threadIdx.x == 0) {
+    pos[row] = seq_len[slot] + r;
+    kv_rowoff[row] = static_cast<long long>(b * stage_R + r) * 2 * kH * kHD;
+  }
+}
+
+cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
+                              const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
+                              float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int* err,
+                              cudaStream_t s) {
+  embed_norm_kernel<<<B * R, 128, 0, s>>>(cand, R, slots, pending, seq_len, embed, vocab, gain, eps, h, xn, pos,
+                                           kv_rowoff, stage_R, err);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- RMSNorm
+__global__ void __launch_bounds__(128) rmsnorm_kernel(const float* x, const bf16* gain, float eps, bf16* out) {
+  __shared__ float red[4];
+  const size_t row = blockIdx.x;
+  float v[10];
+#pragma unroll
+  for (int k = 0; k < 10; ++k) v[k] = x[row * kD + threadIdx.x + 128 * k];
+  norm_row_store(v, gain, eps, out + row * kD, red);
+}
+
+cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  rmsnorm_kernel<<<rows, 128, 0, s>>>(x, gain, eps, out);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- router
+// RMSNorm of the residual row -> xn (bf16, also the experts' input); logits of the 64
+// experts from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).
+__global__ void __launch_bounds__(128) router_kernel(const float* h, const bf16* gain, float eps, const bf16* wr,
+                                                     const float* bias, bf16* xn, int* idx, float* gate) {
+  __shared__ float red[4];
+  __shared__ __align__(16) float xs[kD];
+  __shared__ float lg[kE];
+  const size_t t = blockIdx.x;
+  float v[10];
+#pragma unroll
+  for (int k = 0; k < 10; ++k) v[k] = h[t * kD + threadIdx.x + 128 * k];
+  bf16* xo = xn + t * kD;
+  norm_row_store(v, gain, eps, xo, red);
+#pragma unroll
+  for (int k = 0; k < 10; ++k) {
+    const int i = threadIdx.x + 128 * k;
+    xs[i] = __bfloat162float(xo[i]);   // the rounded row, as the experts see it
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int e = warp * 16; e < warp * 16 + 16; ++e) {
+    const bf16* w = wr + static_cast<size_t>(e) * kD;
+    float acc = 0.f;
+#pragma unroll
+    for (int c = 0; c < 5; ++c) {
+      const int i0 = c * 256 + lane * 8;
+      const uint4 raw = *reinterpret_cast<const uint4*>(w + i0);
+      const bf16* wv = reinterpret_cast<const bf16*>(&raw);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) acc += __bfloat162float(wv[u]) * xs[i0 + u];
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) lg[e] = acc + (bias ? bias[e] : 0.f);
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const float l0 = lg[lane], l1 = lg[lane + 32];
+    const float m = warp_max(fmaxf(l0, l1));
+    const float e0 = expf(l0 - m), e1 = expf(l1 - m);
+    const float sum = warp_sum(e0 + e1);
+    float p0 = e0 / sum, p1 = e1 / sum;
+    bool taken0 = false, taken1 = false;
+    for (int k = 0; k < kTopK; ++k) {
+      float bv = -1.f;
+      int bi = 1 << 30;
+      if (!taken0) { bv = p0; bi = lane; }
+      if (!taken1 && better(p1, lane + 32, bv, bi)) { bv = p1; bi = lane + 32; }
+      warp_argmax(bv, bi);
+      if (bi == lane) taken0 = true;
+      if (bi == lane + 32) taken1 = true;
+      if (lane == 0) {
+        idx[t * kTopK + k] = bi;
+        gate[t * kTopK + k] = bv;
+      }
+    }
+  }
+}
+
+cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
+                          const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s) {
+  router_kernel<<<T, 128, 0, s>>>(h, gain, eps, w_router, bias, xn, idx, gate);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- permute / scatter
+// Groups the (token, slot) pairs of this layer by expert.  Routed rows of expert e take
+// act rows offs[e] .. offs[e+1]-1 in token order; the two shared experts follow with all T
+// tokens each.  Every CTA builds the ranking in shared memory (a per-expert token bitmap and
+// its prefix popcounts); the copies of the selected activation rows are spread over the
+// grid; CTA 0 writes the sorted index and the GEMM work lists.
+constexpr int kPermThreads = 256;
+constexpr int kMaxT = 2048;
+constexpr int kMaxW = kMaxT / 32;
+
+__global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, int T, const bf16* xn, bf16* xs,
+                                                               int* sorted_tok, int* sorted_slot, int4* items_gu,
+                                                               int4* items_dn, int* n_items, int* counts) {
+  extern __shared__ int psm[];
+  const int W = (T + 31) / 32;
+  int* s_idx = psm;                       // [T*6]
+  unsigned* bits = reinterpret_cast<unsigned*>(s_idx + T * kTopK);   // [64][W]
+  int* pre = reinterpret_cast<int*>(bits + kE * W);                // [64][W]
+  int* cnt = pre + kE * W;                // [66]
+  int* offs = cnt + kE + kShared;         // [67]
+  int* ibase = offs + kE + kShared + 1;   // [67] gate_up item offsets
+  int* dbase = ibase + kE + kShared + 1;  // [67]
+  const int tid = threadIdx.x;
+  const int T6 = T * kTopK;
+  for (int p = tid; p < T6; p += kPermThreads) s_idx[p] = idx[p];
+  for (int p = tid; p < kE * W; p += kPermThreads) bits[p] = 0u;
+  for (int p = tid; p < kE + kShared; p += kPermThreads) cnt[p] = 0;
+  __syncthreads();
+  for (int p = tid; p < T6; p += kPermThreads) {
+    const int t = p / kTopK, e = s_idx[p];
+    atomicOr(&bits[e * W + (t >> 5)], 1u << (t & 31));
+  }
+  __syncthreads();
+  if (tid < kE) {
+    int run = 0;
+    for (int w = 0; w < W; ++w) {
+      pre[tid * W + w] = run;
+      run += __popc(bits[tid * W + w]);
+    }
+    cnt[tid] = run;
+  } else if (tid < kE + kShared) {
+    cnt[tid] = T;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    offs[0] = 0;
+    ibase[0] = 0;
+    dbase[0] = 0;
+    for (int e = 0; e < kE + kShared; ++e) {
+      offs[e + 1] = offs[e] + cnt[e];
+      const int mt = (cnt[e] + 255) / 256;
+      ibase[e + 1] = ibase[e] + mt * (kI / 64);
+      dbase[e + 1] = dbase[e] + mt * (kD / 128);
+    }
+    if (blockIdx.x == 0) {
+      n_items[0] = ibase[kE + kShared];
+      n_items[1] = dbase[kE + kShared];
+    }
+  }
+  __syncthreads();
+  // copies of the routed activation rows, one warp per pair, spread over the grid
+  const int warp = tid >> 5, lane = tid & 31;
+  const int gw = blockIdx.x * (kPermThreads / 32) + warp, nw = gridDim.x * (kPermThreads / 32);
+  for (int p = gw; p < T6; p += nw) {
+    const int t = p / kTopK, e = s_idx[p];
+    const int rank = pre[e * W + (t >> 5)] + __popc(bits[e * W + (t >> 5)] & ((1u << (t & 31)) - 1u));
+    const int dst = offs[e] + rank;
+    const uint4* src = reinterpret_cast<const uint4*>(xn + static_cast<size_t>(t) * kD);
+    uint4* d = reinterpret_cast<uint4*>(xs + static_cast<size_t>(dst) * kD);
+    for (int c = lane; c < kD / 8; c += 32) d[c] = src[c];
+  }
+  if (blockIdx.x != 0) return;
+  for (int p = tid; p < T6; p += kPermThreads) {
+    const int t = p / kTopK, s = p % kTopK, e = s_idx[p];
+    const int rank = pre[e * W + (t >> 5)] + __popc(bits[e * W + (t >> 5)] & ((1u << (t & 31)) - 1u));
+    sorted_tok[offs[e] + rank] = t;
+    sorted_slot[offs[e] + rank] = s;
+  }
+  for (int p = tid; p < kShared * T; p += kPermThreads) {
+    const int j = p / T, t = p % T;
+    sorted_tok[offs[kE + j] + t] = t;
+    sorted_slot[offs[kE + j] + t] = kTopK + j;
+  }
+  if (tid < kE + kShared) {
+    const int e = tid, n = cnt[e];
+    if (e < kE) counts[e] = n;
+    const int mt = (n + 255) / 256;
+    for (int m = 0; m < mt; ++m) {
+      const int rows = min(256, n - 256 * m);
+      const int out_row = offs[e] + 256 * m;
+      const int b_row_gu = (e < kE) ? out_row : 256 * m;   // shared experts read xn rows directly
+      for (int nt = 0; nt < kI / 64; ++nt)
+        items_gu[ibase[e] + m * (kI / 64) + nt] = make_int4(e | (nt << 16), b_row_gu, out_row, rows);
+      for (int nt = 0; nt < kD / 128; ++nt)
+        items_dn[dbase[e] + m * (kD / 128) + nt] = make_int4(e | (nt << 16), out_row, out_row, rows);
+    }
+  }
+}
+
+cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
+                           int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
+                           cudaStream_t s) {
+  if (T > kMaxT) return cudaErrorInvalidValue;
+  const int W = (T + 31) / 32;
+  const size_t smem = sizeof(int) * (static_cast<size_t>(T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(permute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(sizeof(int) * (kMaxT * kTopK + 2 * kE * kMaxW + 4 * 67)));
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int pairs = T * kTopK;
+  int grid = (pairs + 63) / 64;   // ~64 row copies per CTA
+  if (grid > 64) grid = 64;
+  if (grid < 1) grid = 1;
+  permute_kernel<<<grid, kPermThreads, smem, s>>>(idx, T, xn, x_sorted, sorted_tok, sorted_slot, items_gu, items_dn,
+                                                  n_items, counts);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- combine
+// h += sum_{s<6} gate_s * y_s + y_shared0 + y_shared1 (fixed slot order), then RMSNorm -> out.
+__global__ void __launch_bounds__(128) combine_kernel(float* h, const float* y, const float* gate, const bf16* gain,
+                                                      float eps, bf16* out) {
+  __shared__ float red[4];
+  const size_t t = blockIdx.x;
+  float g[kTopK];
+#pragma unroll
+  for (int s = 0; s < kTopK; ++s) g[s] = gate[t * kTopK + s];
+  float x[10];
+#pragma unroll
+  for (int k = 0; k < 10; ++k) {
+    const int i = threadIdx.x + 128 * k;
+    const float* yt = y + t * kSlots * kD + i;
+    float acc = 0.f;
+#pragma unroll
+    for (int s = 0; s < kTopK; ++s) acc += g[s] * yt[s * kD];
+    acc += yt[kTopK * kD];
+    acc += yt[(kTopK + 1) * kD];
+    x[k] = h[t * kD + i] + acc;
+    h[t * kD + i] = x[k];
+  }
+  norm_row_store(x, gain, eps, out + t * kD, red);
+}
+
+cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
+                           bf16* out, cudaStream_t s) {
+  combine_kernel<<<T, 128, 0, s>>>(h, y, gate, gain, eps, out);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- argmax + greedy accept
+// Row (b, r) of the verify batch: v = argmax over the LM-head tile partials (value, lower
+// id on ties).  Then m = longest prefix r with cand[b][r+1] == v[b][r] (acceptance equation
+// of Sec. 3.1).
+__device__ __forceinline__ void reduce_partials(const float* am_val, const int* am_idx, int n_tiles, int am_ld,
+                                                int row, float& bv, int& bi) {
+  const int lane = threadIdx.x & 31;
+  bv = -INFINITY;
+  bi = 0x7fffffff;
+  for (int t = lane; t < n_tiles; t += 32) {
+    const float v = am_val[static_cast<size_t>(t) * am_ld + row];
+    const int i = am_idx[static_cast<size_t>(t) * am_ld + row];
+    if (better(v, i, bv, bi)) { bv = v; bi = i; }
+  }
+  warp_argmax(bv, bi);
+}
+
+__global__ void argmax_accept_kernel(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int R,
+                                     const int* cand, int* vtok_out, int* accept_out, int* m_ws, int* vtok_ws) {
+  __shared__ int sv[kMaxR];
+  const int b = blockIdx.x, r = threadIdx.x >> 5;
+  float bv;
+  int bi;
+  reduce_partials(am_val, am_idx, n_tiles, am_ld, b * R + r, bv, bi);
+  if ((threadIdx.x & 31) == 0) {
+    sv[r] = bi;
+    vtok_out[b * R + r] = bi;
+    vtok_ws[b * R + r] = bi;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int m = 0;
+    for (int s = 1; s < R; ++s) {
+      if (cand[b * R + s] == sv[s - 1]) m = s;
+      else break;
+    }
+    accept_out[b] = m;
+    m_ws[b] = m;
+  }
+}
+
+cudaError_t argmax_final_launch(int mode, const float* am_val, const int* am_idx, int n_tiles, int am_ld, int B,
+                                int R, const int* cand, int* vtok_out, int* accept_out, int* m_ws, int* vtok_ws,
+                                cudaStream_t s) {
+  (void)mode;
+  argmax_accept_kernel<<<B, 32 * R, 0, s>>>(am_val, am_idx, n_tiles, am_ld, R, cand, vtok_out, accept_out, m_ws,
+                                             vtok_ws);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- KV commit
+// Appends the staged K/V of candidates 0..m of each sequence to its pages (16-byte
+// vectors), advances the slot, writes the committed tokens and queues the m+1 new rows
+// (base states b and next tokens) for the draft head.  The rejected tail stays in the
+// staging buffer and is overwritten by the next verify.
+__global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bmax, const int* slots, const int* m_ws,
+                                                     const int* vtok, const int* cand, const bf16* stage, bf16* pool,
+                                                     int L, int n_pages, int page_size, const int* block_table,
+                                                     int max_pages, int* seq_len, int* pending, const bf16* b_ws,
+                                                     bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
+                                                     int* n_committed, int* err) {
+  const int b = blockIdx.x, slot = slots[b];
+  const int m = m_ws[b];
+  const int c = seq_len[slot];
+  constexpr int kVec = kHD / 8;   // 16-byte vectors per head row
+  const int total = (m + 1) * L * 2 * kH * kVec;
+  for (int v = threadIdx.x; v < total; v += blockDim.x) {
+    int t = v;
+    const int vec = t % kVec; t /= kVec;
+    const int h = t % kH; t /= kH;
+    const int kv = t % 2; t /= 2;
+    const int l = t % L;
+    const int r = t / L;
+    const int pos = c + r;
+    const int pi = pos / page_size;
+    const int page = (pi < max_pages) ? block_table[slot * max_pages + pi] : -1;
+    if (page < 0 || page >= n_pages) {
+      atomicOr(err, ERR_PAGE_RANGE);
+      continue;
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(
+        stage + ((((static_cast<size_t>(l) * Bmax + b) * stage_R + r) * 2 + kv) * kH + h) * kHD) + vec;
+    uint4* dst = reinterpret_cast<uint4*>(
+        pool + ((((static_cast<size_t>(l) * n_pages + page) * 2 + kv) * kH + h) * page_size + pos % page_size) * kHD) +
+        vec;
+    *dst = *src;
+  }
+  // queue the new rows for the draft head: b_p and x_{p+1}
+  for (int v = threadIdx.x; v < (m + 1) * (kD / 8); v += blockDim.x) {
+    const int r = v / (kD / 8), c8 = v % (kD / 8);
+    reinterpret_cast<uint4*>(draft_b + (static_cast<size_t>(slot) * kMaxR + r) * kD)[c8] =
+        reinterpret_cast<const uint4*>(b_ws + static_cast<size_t>(b * R + r) * kD)[c8];
+  }
+  __syncthreads();
+  if (threadIdx.x < R) {
+    const int r = threadIdx.x;
+    const int tok = (r < m) ? cand[b * R + r + 1] : (r == m ? vtok[b * R + m] : -1);
+    committed[b * R + r] = tok;
+    if (r <= m) draft_tok[slot * kMaxR + r] = tok;
+  }
+  if (threadIdx.x == 0) {
+    n_committed[b] = m + 1;
+    pending[slot] = vtok[b * R + m];
+    seq_len[slot] = c + m + 1;
+    draft_n[slot] = m + 1;
+  }
+}
+
+cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots, const int* m_ws,
+                          const int* vtok_ws, const int* cand_ws, const bf16* stage, bf16* pool, int L, int n_pages,
+                          int page_size, const int* block_table, int max_pages, int* seq_len, int* pending,
+                          const bf16* b_ws, bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
+                          int* n_committed, int* err, cudaStream_t s) {
+  commit_kernel<<<B, 256, 0, s>>>(R, stage_R, Bmax, slots, m_ws, vtok_ws, cand_ws, stage, pool, L,
+                                   n_pages, page_size, block_table, max_pages, seq_len, pending, b_ws, draft_b,
+                                   draft_tok, draft_n, committed, n_committed, err);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- draft glue
+// Depth-1 rows of the draft step: for the rows queued by the last commit, dcat =
+// [N_e(E x_{p+1}); N_h(b_p)] (bf16), positions p and page offsets of their committed draft
+// K/V; padding rows are zero and write no K/V.  Also cand[b][0] = pending token.
+__global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots, const int* seq_len,
+                                                         const int* pending, const int* draft_n, const bf16* draft_b,
+                                                         const int* draft_tok, const bf16* embed, int vocab,
+                                                         const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat,
+                                                         int* pos, long long* kv_rowoff, int* last_row, int page_size,
+                                                         const int* block_table, int max_pages, int n_pages, int* cand,
+                                                         int cand_ld, int* err) {
+  __shared__ float red[4];
+  const int b = blockIdx.x / R, i = blockIdx.x % R, row = blockIdx.x;
+  const int slot = slots[b];
+  int n = draft_n[slot];
+  if (n < 1 || n > kMaxR) {
+    if (threadIdx.x == 0 && i == 0) atomicOr(err, ERR_NO_DRAFT_ROWS);
+    n = 0;
+  }
+  if (i == 0 && threadIdx.x == 0) {
+    cand[b * cand_ld] = pending[slot];
+    last_row[b] = b * R + (n > 0 ? n - 1 : 0);
+  }
+  bf16* out = dcat + static_cast<size_t>(row) * 2 * kD;
+  if (i >= n) {
+    for (int k = threadIdx.x; k < 2 * kD; k += 128) out[k] = __float2bfloat16(0.f);
+    if (threadIdx.x == 0) {
+      pos[row] = 0;
+      kv_rowoff[row] = -1;
+    }
+    return;
+  }
+  int tok = draft_tok[slot * kMaxR + i];
+  if (tok < 0 || tok >= vocab) {
+    if (threadIdx.x == 0) atomicOr(err, ERR_TOKEN_RANGE);
+    tok = 0;
+  }
+  float x[10];
+#pragma unroll
+  for (int k = 0; k < 10; ++k) x[k] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * k]);
+  norm_row_store(x, enorm, eps, out, red);
+#pragma unroll
+  for (int k = 0; k < 10; ++k)
+    x[k] = __bfloat162float(draft_b[(static_cast<size_t>(slot) * kMaxR + i) * kD + threadIdx.x + 128 * k]);
+  norm_row_store(x, hnorm, eps, out + kD, red);
+  if (threadIdx.x == 0) {
+    const int p = seq_len[slot] - n + i;
+    pos[row] = p;
+    const int pi = p / page_size;
+    const int page = (p >= 0 && pi < max_pages) ? block_table[slot * max_pages + pi] : -1;
+    if (page < 0 || page >= n_pages) {
+      atomicOr(err, ERR_PAGE_RANGE);
+      kv_rowoff[row] = -1;
+    } else {
+      kv_rowoff[row] = (static_cast<long long>(page) * 2 * kH * page_size + (p % page_size)) * kHD;
+    }
+  }
+}
+
+cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len, const int* pending,
+                              const int* draft_n, const bf16* draft_b, const int* draft_tok, const bf16* embed,
+                              int vocab, const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
+                              long long* kv_rowoff, int* last_row, int page_size, const int* block_table,
+                              int max_pages, int n_pages, int* cand, int cand_ld, int* err, cudaStream_t s) {
+  draft_prep_kernel<<<B * R, 128, 0, s>>>(R, slots, seq_len, pending, draft_n, draft_b, draft_tok, embed, vocab,
+                                           enorm, hnorm, eps, dcat, pos, kv_rowoff, last_row, page_size, block_table,
+                                           max_pages, n_pages, cand, cand_ld, err);
+  return cudaGetLastError();
+}
+
+__global__ void gather_rows_kernel(const float* src, const int* rows, float* dst) {
+  const int b = blockIdx.x;
+  const float4* s = reinterpret_cast<const float4*>(src + static_cast<size_t>(rows[b]) * kD);
+  float4* d = reinterpret_cast<float4*>(dst + static_cast<size_t>(b) * kD);
+  for (int i = threadIdx.x; i < kD / 4; i += blockDim.x) d[i] = s[i];
+}
+
+cudaError_t gather_rows_launch(const float* src, const int* rows, int B, float* dst, cudaStream_t s) {
+  gather_rows_kernel<<<B, 128, 0, s>>>(src, rows, dst);
+  return cudaGetLastError();
+}
+
+// After the LM head of depth k: x^_k = argmax; for k < K the inputs of depth k+1:
+// dcat = [N_e(E x^_k); N_h(u^(k))], position p = j + k (j = ctx_len - 1) and the staging
+// row k-1 of its tentative draft K/V.
+__global__ void __launch_bounds__(128) draft_next_kernel(const float* am_val, const int* am_idx, int n_tiles, int am_ld,
+                                                         int k, int K, const int* slots, const int* seq_len,
+                                                         const bf16* u, const bf16* embed, const bf16* enorm,
+                                                         const bf16* hnorm, float eps, bf16* dcat, int* pos,
+                                                         long long* kv_rowoff, long long dstage_seq_stride, int* cand,
+                                                         int cand_ld) {
+  __shared__ float red[4];
+  __shared__ int s_tok;
+  const int b = blockIdx.x;
+  if (threadIdx.x < 32) {
+    float bv;
+    int bi;
+    reduce_partials(am_val, am_idx, n_tiles, am_ld, b, bv, bi);
+    if (threadIdx.x == 0) {
+      s_tok = bi;
+      cand[b * cand_ld + k] = bi;
+    }
+  }
+  __syncthreads();
+  if (k >= K) return;
+  const int tok = s_tok;
+  bf16* out = dcat + static_cast<size_t>(b) * 2 * kD;
+  float x[10];
+#pragma unroll
+  for (int q = 0; q < 10; ++q) x[q] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * q]);
+  norm_row_store(x, enorm, eps, out, red);
+#pragma unroll
+  for (int q = 0; q < 10; ++q) x[q] = __bfloat162float(u[static_cast<size_t>(b) * kD + threadIdx.x + 128 * q]);
+  norm_row_store(x, hnorm, eps, out + kD, red);
+  if (threadIdx.x == 0) {
+    pos[b] = seq_len[slots[b]] + k - 1;
+    kv_rowoff[b] = b * dstage_seq_stride + static_cast<long long>(k - 1) * 2 * kH * kHD;
+  }
+}
+
+cudaError_t draft_next_launch(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int B, int k, int K,
+                              const int* slots, const int* seq_len, const bf16* u, const bf16* embed,
+                              const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
+                              long long* kv_rowoff, long long dstage_seq_stride, int* cand, int cand_ld,
+                              cudaStream_t s) {
+  draft_next_kernel<<<B, 128, 0, s>>>(am_val, am_idx, n_tiles, am_ld, k, K, slots, seq_len, u, embed, enorm, hnorm,
+                                       eps, dcat, pos, kv_rowoff, dstage_seq_stride, cand, cand_ld);
+  return cudaGetLastError();
+}
+
+}  // namespace fm

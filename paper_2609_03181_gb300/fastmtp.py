@@ -1,0 +1,249 @@
+"""Python binding of libfastmtp.so, the C ABI in include/fastmtp.h.
+
+Argument marshalling only: every step of the decode path runs in the library's CUDA kernels.
+PyTorch provides device memory (weights, KV pools, inputs and outputs) and the stream.  There
+is no fallback: if the library cannot be built or loaded, or no GPU is present, the calls
+raise."""
+from __future__ import annotations
+
+import ctypes
+from typing import List, Optional, Sequence
+
+import torch
+
+from . import build as _build
+
+SPEC_OK, SPEC_EINVAL, SPEC_ENOMEM, SPEC_ECUDA, SPEC_ESTATE, SPEC_EDEVICE = range(6)
+STATUS = {0: "SPEC_OK", 1: "SPEC_EINVAL", 2: "SPEC_ENOMEM", 3: "SPEC_ECUDA", 4: "SPEC_ESTATE", 5: "SPEC_EDEVICE"}
+WS_B, WS_ROUTE_IDX, WS_ROUTE_GATE, WS_EXPERT_CNT, WS_DRAFT_U, WS_HIDDEN = range(6)
+
+# Public entry points, in the order include/fastmtp.h declares them.
+ENTRY_POINTS = ["spec_init", "spec_seq_reset", "spec_seq_set_draft_rows", "draft_step", "verify_step",
+                "accept_commit", "spec_sync", "spec_seq_state", "spec_read_workspace", "spec_gemm_bf16",
+                "spec_destroy", "spec_last_error"]
+
+
+class SpecConfig(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "hidden", "n_heads", "head_dim", "n_layers", "n_experts", "top_k", "n_shared", "expert_inter",
+        "draft_inter", "vocab", "page_size", "max_batch", "max_pages_per_seq", "n_pages_total", "K_max",
+        "max_position")] + [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+
+
+class SpecLayerWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in (
+        "attn_norm", "wqkv", "wo", "moe_norm", "router", "w_gate_up", "w_down", "shared_gate_up",
+        "shared_down", "router_bias")]
+
+
+class SpecWeights(ctypes.Structure):
+    _fields_ = [("embed", ctypes.c_void_p), ("lm_head", ctypes.c_void_p), ("final_norm", ctypes.c_void_p),
+                ("layers", ctypes.POINTER(SpecLayerWeights))] + [(n, ctypes.c_void_p) for n in (
+                    "enorm", "hnorm", "eh_proj", "mtp_attn_norm", "mtp_wqkv", "mtp_wo", "mtp_ffn_norm",
+                    "mtp_w_gate_up", "mtp_w_down")]
+
+
+class FastMTPError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+_LIB: Optional[ctypes.CDLL] = None
+
+
+def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
+    """Loads libfastmtp.so (building it with nvcc first when needed)."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = _build.build() if build_if_needed else _build.LIB
+    lib = ctypes.CDLL(path)
+    P, I32 = ctypes.c_void_p, ctypes.c_int32
+    sig = {
+        "spec_init": (ctypes.c_int, [ctypes.POINTER(SpecConfig), ctypes.POINTER(SpecWeights), P, P, P,
+                                     ctypes.POINTER(P)]),
+        "spec_seq_reset": (ctypes.c_int, [P, I32, I32, ctypes.POINTER(I32), I32]),
+        "spec_seq_set_draft_rows": (ctypes.c_int, [P, I32, I32, P, ctypes.POINTER(I32)]),
+        "draft_step": (ctypes.c_int, [P, I32, I32, P, P]),
+        "verify_step": (ctypes.c_int, [P, I32, I32, P, P, P, P]),
+        "accept_commit": (ctypes.c_int, [P, I32, P, P, P]),
+        "spec_sync": (ctypes.c_int, [P]),
+        "spec_seq_state": (ctypes.c_int, [P, I32, ctypes.POINTER(I32), ctypes.POINTER(I32)]),
+        "spec_read_workspace": (ctypes.c_int, [P, I32, P, ctypes.c_size_t]),
+        "spec_gemm_bf16": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
+        "spec_destroy": (None, [P]),
+        "spec_last_error": (ctypes.c_char_p, [P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _LIB = lib
+    return lib
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream_handle(stream: Optional[torch.cuda.Stream]) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def gemm_bf16(X: torch.Tensor, W: torch.Tensor, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Y = X W^T through spec_gemm_bf16 (X [M][K], W [N][K] bf16 CUDA tensors) -> fp32 [M][N]."""
+    lib = load_library()
+    assert X.is_cuda and W.is_cuda and X.dtype == torch.bfloat16 and W.dtype == torch.bfloat16
+    X, W = X.contiguous(), W.contiguous()
+    M, K = X.shape
+    N = W.shape[0]
+    Y = torch.empty(M, N, dtype=torch.float32, device=X.device)
+    st = lib.spec_gemm_bf16(X.data_ptr(), W.data_ptr(), Y.data_ptr(), M, N, K, _stream_handle(stream))
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+    return Y
+
+
+class Engine:
+    """A spec_ctx with device copies of the verifier and draft weights and the two KV pools.
+
+    vw / dw: synth_inputs.VerifierWeights / DraftWeights (bf16 CPU tensors).  Slot b owns pages
+    b*max_pages_per_seq .. (b+1)*max_pages_per_seq-1 of both pools."""
+
+    def __init__(self, vw, dw, max_batch: int, K_max: int, max_ctx: int, page_size: int = 64,
+                 device: str = "cuda", stream: Optional[torch.cuda.Stream] = None, max_position: int = 32768):
+        self.lib = load_library()
+        if not torch.cuda.is_available():
+            raise RuntimeError("FastMTP needs a CUDA GPU")
+        s = vw.shape
+        self.shape = s
+        self.device = torch.device(device)
+        self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
+        self.page_size = page_size
+        self.max_batch = max_batch
+        self.K_max = K_max
+        self.max_pages = (max_ctx + K_max + 1 + page_size - 1) // page_size
+        self.n_pages = max_batch * self.max_pages
+        dev = lambda t: t.to(self.device).contiguous()
+        self._keep: List[torch.Tensor] = []
+
+        def keep(t):
+            t = dev(t)
+            self._keep.append(t)
+            return t
+
+        self.embed = keep(vw.embed)
+        self.lm_head = keep(vw.lm_head)
+        final_norm = keep(vw.final_norm)
+        self._layers = (SpecLayerWeights * s.n_layers)()
+        for l, lw in enumerate(vw.layers[:s.n_layers]):
+            L = self._layers[l]
+            L.attn_norm = keep(lw.attn_norm).data_ptr()
+            L.wqkv = keep(lw.wqkv).data_ptr()
+            L.wo = keep(lw.wo).data_ptr()
+            L.moe_norm = keep(lw.moe_norm).data_ptr()
+            L.router = keep(lw.router).data_ptr()
+            L.w_gate_up = keep(lw.w_gate_up).data_ptr()
+            L.w_down = keep(lw.w_down).data_ptr()
+            L.shared_gate_up = keep(lw.shared_gate_up).data_ptr()
+            L.shared_down = keep(lw.shared_down).data_ptr()
+            L.router_bias = keep(lw.router_bias.float()).data_ptr() if lw.router_bias is not None else None
+        w = SpecWeights()
+        w.embed, w.lm_head, w.final_norm = self.embed.data_ptr(), self.lm_head.data_ptr(), final_norm.data_ptr()
+        w.layers = self._layers
+        for name in ("enorm", "hnorm", "eh_proj"):
+            setattr(w, name, keep(getattr(dw, name)).data_ptr())
+        for name in ("attn_norm", "wqkv", "wo", "ffn_norm", "w_gate_up", "w_down"):
+            setattr(w, "mtp_" + name, keep(getattr(dw, name)).data_ptr())
+        self._w = w
+        H, hd = s.n_heads, s.head_dim
+        self.kv_pool = torch.zeros(s.n_layers, self.n_pages, 2, H, page_size, hd, dtype=torch.bfloat16,
+                                   device=self.device)
+        self.dkv_pool = torch.zeros(self.n_pages, 2, H, page_size, hd, dtype=torch.bfloat16, device=self.device)
+        cfg = SpecConfig(hidden=s.hidden, n_heads=H, head_dim=hd, n_layers=s.n_layers, n_experts=s.n_experts,
+                         top_k=s.top_k, n_shared=s.n_shared, expert_inter=s.expert_inter,
+                         draft_inter=s.draft_inter, vocab=s.vocab, page_size=page_size, max_batch=max_batch,
+                         max_pages_per_seq=self.max_pages, n_pages_total=self.n_pages, K_max=K_max,
+                         max_position=max_position, rms_eps=s.rms_eps, rope_theta=s.rope_theta)
+        self._cfg = cfg
+        ctx = ctypes.c_void_p()
+        torch.cuda.synchronize(self.device)
+        st = self.lib.spec_init(ctypes.byref(cfg), ctypes.byref(w), self.kv_pool.data_ptr(), self.dkv_pool.data_ptr(),
+                                self.stream.cuda_stream, ctypes.byref(ctx))
+        if st != SPEC_OK:
+            raise FastMTPError(st, self.lib.spec_last_error(None).decode())
+        self.ctx = ctx
+
+    # ------------------------------------------------------------------ helpers
+    def _check(self, st: int):
+        if st != SPEC_OK:
+            raise FastMTPError(st, self.lib.spec_last_error(self.ctx).decode())
+
+    def block_table(self, slot: int) -> List[int]:
+        return [slot * self.max_pages + i for i in range(self.max_pages)]
+
+    def load_prefix(self, slot: int, kv: torch.Tensor, dkv: torch.Tensor, pending: int):
+        """Places a synthetic committed prefix in slot `slot`'s pages and resets the slot.
+        kv: bf16 [L][2][ctx][H][hd]; dkv: bf16 [2][ctx][H][hd]."""
+        ctx = kv.shape[2]
+        ps = self.page_size
+        bt = self.block_table(slot)
+        n = (ctx + ps - 1) // ps
+        if n:
+            pad = n * ps - ctx
+            src = torch.nn.functional.pad(kv.to(self.device), (0, 0, 0, 0, 0, pad))
+            src = src.reshape(kv.shape[0], 2, n, ps, kv.shape[3], kv.shape[4]).permute(0, 2, 1, 4, 3, 5)
+            self.kv_pool[:, bt[0]:bt[0] + n] = src
+            dsrc = torch.nn.functional.pad(dkv.to(self.device), (0, 0, 0, 0, 0, pad))
+            dsrc = dsrc.reshape(2, n, ps, dkv.shape[2], dkv.shape[3]).permute(1, 0, 3, 2, 4)
+            self.dkv_pool[bt[0]:bt[0] + n] = dsrc
+        torch.cuda.synchronize(self.device)
+        self.reset_seq(slot, ctx, bt, pending)
+
+    def reset_seq(self, slot: int, ctx_len: int, block_table: Sequence[int], pending: int):
+        arr = (ctypes.c_int32 * self.max_pages)(*list(block_table))
+        self._check(self.lib.spec_seq_reset(self.ctx, slot, ctx_len, arr, pending))
+
+    def set_draft_rows(self, slot: int, b_rows: torch.Tensor, next_tokens: Sequence[int]):
+        b_rows = b_rows.to(self.device, torch.bfloat16).contiguous()
+        arr = (ctypes.c_int32 * len(next_tokens))(*[int(t) for t in next_tokens])
+        self._check(self.lib.spec_seq_set_draft_rows(self.ctx, slot, len(next_tokens), b_rows.data_ptr(), arr))
+
+    def seq_state(self, slot: int):
+        a, b = ctypes.c_int32(), ctypes.c_int32()
+        self._check(self.lib.spec_seq_state(self.ctx, slot, ctypes.byref(a), ctypes.byref(b)))
+        return a.value, b.value
+
+    # ------------------------------------------------------------------ the step
+    def draft_step(self, slots: torch.Tensor, K: int, cand: torch.Tensor):
+        self._check(self.lib.draft_step(self.ctx, slots.numel(), K, slots.data_ptr(), cand.data_ptr()))
+
+    def verify_step(self, slots: torch.Tensor, cand: torch.Tensor, vtok: torch.Tensor, accept: torch.Tensor):
+        K = cand.shape[1] - 1
+        self._check(self.lib.verify_step(self.ctx, slots.numel(), K, slots.data_ptr(), cand.data_ptr(),
+                                         vtok.data_ptr(), accept.data_ptr()))
+
+    def accept_commit(self, slots: torch.Tensor, committed: torch.Tensor, n_committed: torch.Tensor):
+        self._check(self.lib.accept_commit(self.ctx, slots.numel(), slots.data_ptr(), committed.data_ptr(),
+                                           n_committed.data_ptr()))
+
+    def sync(self):
+        self._check(self.lib.spec_sync(self.ctx))
+
+    def read_workspace(self, which: int, shape, dtype) -> torch.Tensor:
+        out = torch.empty(*shape, dtype=dtype)
+        self._check(self.lib.spec_read_workspace(self.ctx, which, out.data_ptr(), out.numel() * out.element_size()))
+        return out
+
+    def close(self):
+        if getattr(self, "ctx", None):
+            self.lib.spec_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,98 @@
+"""verify_step + accept_commit through the C ABI against the fp64 oracle (storage-rounding
+mode): one decoder layer at the paper's widths (B=1, K=3, context 512, full vocabulary), then
+the 12-layer decoder (B=8, K=3, contexts U[768,1024] with a 256-token synthetic visual prefix).
+
+Rules: b = N_o(h_L) and the committed K/V within max relative error 2e-2; router experts,
+verifier tokens and accept lengths bit-exact where the oracle's fp64 top-2 margin exceeds 1e-3."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import synth_inputs as S
+from paper_2609_03181_gb300 import fastmtp as F
+from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, index_parity
+
+pytestmark = pytest.mark.gpu
+
+
+def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
+    B = len(ctx_lens)
+    vw = S.verifier_weights(shape, seed, gain_std=gain_std)
+    dw = S.draft_weights(shape, seed, gain_std=gain_std)
+    model = O.Verifier(vw)
+    kvs, dkvs = seq_prefixes(shape, seed, ctx_lens)
+    pend = S.integers(seed, "pending", B, 0, shape.vocab - 1)
+    caches = [O.SeqCache.from_prefix(kvs[b], int(pend[b])) for b in range(B)]
+    cand = make_drafts(model, caches, K, seed)
+    ref = O.verify(model, caches, cand, rb=True)
+
+    eng = F.Engine(vw, dw, max_batch=B, K_max=max(K, 3), max_ctx=max(ctx_lens) + 8, page_size=64)
+    for b in range(B):
+        eng.load_prefix(b, kvs[b], dkvs[b], int(pend[b]))
+    dev = torch.device("cuda")
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    cand_d = torch.tensor(cand, dtype=torch.int32, device=dev)
+    vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    acc = torch.empty(B, dtype=torch.int32, device=dev)
+    eng.verify_step(slots, cand_d, vt, acc)
+    eng.sync()
+    T = B * (K + 1)
+    b_gpu = eng.read_workspace(F.WS_B, (T, shape.hidden), torch.bfloat16)
+    assert rel_err(b_gpu, ref.b.reshape(T, -1)) < REL_TOL
+
+    ridx = eng.read_workspace(F.WS_ROUTE_IDX, (shape.n_layers, eng.max_batch * (eng.K_max + 1), shape.top_k),
+                              torch.int32)
+    for l in range(shape.n_layers):
+        g = ridx[l, :T].numpy()
+        r = ref.route_idx[l].numpy()
+        n_ok, n_skip, n_bad = index_parity(np.sort(g, -1), np.sort(r, -1), ref.route_gap[l].numpy())
+        assert n_bad == 0, f"layer {l}: {n_bad} router mismatches over {n_ok} rows"
+
+    v_ok, v_skip, v_bad = index_parity(vt.cpu().numpy().reshape(-1), ref.v.numpy().reshape(-1),
+                                       ref.v_gap.numpy().reshape(-1))
+    assert v_bad == 0
+    for b in range(B):
+        if all(ref.v_gap[b, : K].numpy() > GAP):
+            assert int(acc[b]) == ref.m[b]
+
+    committed = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    ncom = torch.empty(B, dtype=torch.int32, device=dev)
+    eng.accept_commit(slots, committed, ncom)
+    eng.sync()
+    ps = eng.page_size
+    for b in range(B):
+        m = int(acc[b])
+        assert int(ncom[b]) == m + 1
+        toks = committed[b].tolist()
+        assert toks[:m + 1] == cand[b][1:m + 1] + [int(vt[b, m])] and all(t == -1 for t in toks[m + 1:])
+        ln, pending = eng.seq_state(b)
+        assert ln == ctx_lens[b] + m + 1 and pending == int(vt[b, m])
+        bt = eng.block_table(b)
+        for l in range(shape.n_layers):
+            for r in range(m + 1):
+                p = ctx_lens[b] + r
+                page, off = bt[p // ps], p % ps
+                k_gpu = eng.kv_pool[l, page, 0, :, off, :].cpu()
+                v_gpu = eng.kv_pool[l, page, 1, :, off, :].cpu()
+                assert rel_err(k_gpu, ref.new_k[b][l][r]) < REL_TOL
+                assert rel_err(v_gpu, ref.new_v[b][l][r]) < REL_TOL
+    eng.close()
+    return v_ok, v_skip
+
+
+def test_verify_one_layer_cfg0():
+    shape = S.ModelShape(n_layers=1)
+    run_verify_case(shape, 0, [512], K=3)
+
+
+def test_verify_ragged_small_contexts():
+    """Empty committed context, contexts inside the first chunk and across page boundaries."""
+    shape = S.ModelShape(n_layers=2, vocab=4096)
+    run_verify_case(shape, 5, [0, 1, 63, 64, 129, 200], K=2)
+
+
+def test_verify_twelve_layers_cfg1():
+    shape = S.ModelShape()
+    ctx = [int(c) for c in S.integers(1, "ctx", 8, 768, 1024)]
+    run_verify_case(shape, 1, ctx, K=3, gain_std=0.0)
