@@ -187,6 +187,27 @@ spec_status spec_read_workspace(spec_ctx* ctx, int32_t id, void* dst, size_t byt
 spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, int32_t N,
                            int32_t Kdim, void* stream);
 
+/* Kernel-class timing for measurement.  spec_profile(ctx, 1) zeroes the counters and starts
+ * recording a CUDA event pair around every kernel the context launches (on its stream);
+ * spec_profile(ctx, 0) stops.  Launch counts and the expert counter are kept whether or not
+ * events are recorded.  spec_profile_read waits for the stream and fills *out:
+ *   launches[c], ms[c]  kernel launches and summed event time of class c (SPEC_K_*);
+ *   experts_touched     routed + shared experts with at least one row, summed over the
+ *                       grouped-GEMM launches (the expert weight bytes actually read);
+ *   expert_rows         (token, expert) rows processed by those launches. */
+enum { SPEC_K_EMBED = 0, SPEC_K_QKV = 1, SPEC_K_ATTN = 2, SPEC_K_OPROJ = 3, SPEC_K_ROUTER = 4,
+       SPEC_K_PERMUTE = 5, SPEC_K_EXPERT_GU = 6, SPEC_K_EXPERT_DN = 7, SPEC_K_COMBINE = 8,
+       SPEC_K_LMHEAD = 9, SPEC_K_ARGMAX = 10, SPEC_K_COMMIT = 11, SPEC_K_DRAFT_GEMM = 12,
+       SPEC_K_DRAFT_MISC = 13, SPEC_K_COUNT = 14 };
+typedef struct spec_profile_t {
+  int64_t launches[SPEC_K_COUNT];
+  double ms[SPEC_K_COUNT];
+  int64_t experts_touched;
+  int64_t expert_rows;
+} spec_profile_t;
+spec_status spec_profile(spec_ctx* ctx, int32_t enable);
+spec_status spec_profile_read(spec_ctx* ctx, spec_profile_t* out);
+
 /* Frees the workspace.  Borrowed weights and pools are untouched.  NULL is ignored. */
 void spec_destroy(spec_ctx* ctx);
 

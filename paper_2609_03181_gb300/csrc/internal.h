@@ -110,7 +110,7 @@ cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, co
                           const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s);
 cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
                            int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
-                           cudaStream_t s);
+                           unsigned long long* expert_ctr, cudaStream_t s);
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
                            bf16* out, cudaStream_t s);
 cudaError_t argmax_final_launch(int mode, const float* am_val, const int* am_idx, int n_tiles, int am_ld,

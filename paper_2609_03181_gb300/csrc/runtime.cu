@@ -92,6 +92,14 @@ struct spec_ctx {
   float2* rope = nullptr;
   int* d_err = nullptr;
 
+  // measurement: event pairs per kernel class, launch counts, expert counters (device int64[2])
+  bool prof_on = false;
+  std::vector<cudaEvent_t> ev_free;
+  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> marks;
+  int64_t launches[SPEC_K_COUNT] = {};
+  double prof_ms[SPEC_K_COUNT] = {};
+  unsigned long long* d_expert_ctr = nullptr;
+
   // host-side state machine
   bool verified = false;
   int last_B = 0, last_K = 0;
@@ -160,7 +168,47 @@ cudaError_t run_dense(spec_ctx* ctx, GemmArgs g, int epi, const CUtensorMap& wma
 
 size_t align_up(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
+cudaEvent_t take_event(spec_ctx* ctx) {
+  if (!ctx->ev_free.empty()) {
+    cudaEvent_t e = ctx->ev_free.back();
+    ctx->ev_free.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Brackets one launch group of kernel class `cls` (n_kernels kernels) with an event pair
+// when profiling is on, and counts its launches always.
+struct ProfScope {
+  spec_ctx* ctx;
+  int cls;
+  cudaEvent_t e0 = nullptr;
+  ProfScope(spec_ctx* c, int k) : ctx(c), cls(k) {
+    if (ctx->prof_on) {
+      e0 = take_event(ctx);
+      cudaEventRecord(e0, ctx->stream);
+    }
+  }
+  void done(int n_kernels) {
+    ctx->launches[cls] += n_kernels;
+    if (ctx->prof_on) {
+      cudaEvent_t e1 = take_event(ctx);
+      cudaEventRecord(e1, ctx->stream);
+      ctx->marks.push_back({cls, {e0, e1}});
+    }
+  }
+};
+
 }  // namespace
+
+#define LAUNCH(cls, nk, call)          \
+  do {                                 \
+    ProfScope ps_(ctx, cls);           \
+    CK(call);                          \
+    ps_.done(nk);                      \
+  } while (0)
 
 // ============================================================================ init / destroy
 extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, void* kv_pool, void* draft_kv_pool,
@@ -280,6 +328,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->sk_tickets, sizeof(int) * 16384);
   add(&ctx->rope, sizeof(float2) * static_cast<size_t>(c.max_position) * (kHD / 2));
   add(&ctx->d_err, sizeof(int) * 4);
+  add(&ctx->d_expert_ctr, sizeof(unsigned long long) * 2);
   size_t total = 0;
   for (auto& s : subs) total += align_up(s.bytes);
   if (cudaMalloc(&ctx->ws, total) != cudaSuccess) {
@@ -355,6 +404,11 @@ extern "C" void spec_destroy(spec_ctx* ctx) {
   if (ctx == nullptr) return;
   if (ctx->stream != nullptr) cudaStreamSynchronize(ctx->stream);
   else cudaDeviceSynchronize();
+  for (auto& m : ctx->marks) {
+    cudaEventDestroy(m.second.first);
+    cudaEventDestroy(m.second.second);
+  }
+  for (cudaEvent_t e : ctx->ev_free) cudaEventDestroy(e);
   cudaFree(ctx->ws);
   delete ctx;
 }
@@ -439,7 +493,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   const size_t pool_layer = static_cast<size_t>(c.n_pages_total) * 2 * kH * c.page_size * kHD;
 
   CK(cudaMemcpyAsync(ctx->cand_ws, cand, sizeof(int) * T, cudaMemcpyDeviceToDevice, s));
-  CK(embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
+  LAUNCH(SPEC_K_EMBED, 1, embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
                        c.vocab, static_cast<const bf16*>(ctx->layers[0].attn_norm), eps, ctx->h, ctx->xn, ctx->pos,
                        ctx->kv_rowoff, ctx->Rmax, ctx->d_err, s));
   const int nmax_grouped = T <= 64 ? 64 : 256;
@@ -455,7 +509,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.head_stride = kHD;
       g.v_off = static_cast<long long>(kH) * kHD;
       g.pos = ctx->pos;
-      CK(run_dense(ctx, g, EPI_QKV, M.wqkv, ctx->a_xn, 3 * kD, kD, T, true));
+      LAUNCH(SPEC_K_QKV, 1, run_dense(ctx, g, EPI_QKV, M.wqkv, ctx->a_xn, 3 * kD, kD, T, true));
     }
     // attention over committed pages + staged candidates
     {
@@ -480,21 +534,22 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       a.out = ctx->attn_out;
       a.out_row_stride_seq = R;
       a.err = ctx->d_err;
-      CK(attention_launch(a, B, s));
+      LAUNCH(SPEC_K_ATTN, 2, attention_launch(a, B, s));
     }
     // O-proj + residual
     {
       GemmArgs g = base_args(ctx);
       g.out = ctx->h;
       g.ldo = kD;
-      CK(run_dense(ctx, g, EPI_RESID, M.wo, ctx->a_attn, kD, kD, T, true));
+      LAUNCH(SPEC_K_OPROJ, 1, run_dense(ctx, g, EPI_RESID, M.wo, ctx->a_attn, kD, kD, T, true));
     }
     int* ridx = ctx->route_idx + static_cast<size_t>(l) * ctx->Tmax * kTopK;
     float* rgate = ctx->route_gate + static_cast<size_t>(l) * ctx->Tmax * kTopK;
-    CK(router_launch(ctx->h, T, static_cast<const bf16*>(W.moe_norm), eps, static_cast<const bf16*>(W.router),
+    LAUNCH(SPEC_K_ROUTER, 1, router_launch(ctx->h, T, static_cast<const bf16*>(W.moe_norm), eps, static_cast<const bf16*>(W.router),
                      W.router_bias, ctx->xn, ridx, rgate, s));
-    CK(permute_launch(ridx, T, ctx->xn, ctx->x_sorted, ctx->sorted_tok, ctx->sorted_slot, ctx->items_gu,
-                      ctx->items_dn, ctx->n_items, ctx->counts + l * kE, s));
+    LAUNCH(SPEC_K_PERMUTE, 1, permute_launch(ridx, T, ctx->xn, ctx->x_sorted, ctx->sorted_tok, ctx->sorted_slot,
+                                              ctx->items_gu, ctx->items_dn, ctx->n_items, ctx->counts + l * kE,
+                                              ctx->d_expert_ctr, s));
     // routed + shared experts: gate/up + SwiGLU
     {
       GemmArgs g = base_args(ctx);
@@ -514,7 +569,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.n_items_dev = ctx->n_items;
       g.act = ctx->act;
       g.ld_act = kI;
-      CK(gemm_launch(EPI_SWIGLU, nmax_grouped, g, num_sms(), s));
+      LAUNCH(SPEC_K_EXPERT_GU, 1, gemm_launch(EPI_SWIGLU, nmax_grouped, g, num_sms(), s));
     }
     // routed + shared experts: down, scattered to (token, slot)
     {
@@ -534,19 +589,19 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.y = ctx->y;
       g.sorted_tok = ctx->sorted_tok;
       g.sorted_slot = ctx->sorted_slot;
-      CK(gemm_launch(EPI_SCATTER, nmax_grouped, g, num_sms(), s));
+      LAUNCH(SPEC_K_EXPERT_DN, 1, gemm_launch(EPI_SCATTER, nmax_grouped, g, num_sms(), s));
     }
     const bf16* next_gain =
         static_cast<const bf16*>(l + 1 < L ? ctx->layers[l + 1].attn_norm : ctx->w.final_norm);
-    CK(combine_launch(ctx->h, ctx->y, rgate, T, next_gain, eps, l + 1 < L ? ctx->xn : ctx->b_ws, s));
+    LAUNCH(SPEC_K_COMBINE, 1, combine_launch(ctx->h, ctx->y, rgate, T, next_gain, eps, l + 1 < L ? ctx->xn : ctx->b_ws, s));
   }
   // LM head + argmax (logits never leave the SM) + greedy accept
   {
     GemmArgs g = base_args(ctx);
     g.am_val = ctx->am_val;
     g.am_idx = ctx->am_idx;
-    CK(run_dense(ctx, g, EPI_ARGMAX, ctx->lm, ctx->a_b, c.vocab, kD, T, false));
-    CK(argmax_final_launch(0, ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, R, ctx->cand_ws,
+    LAUNCH(SPEC_K_LMHEAD, 1, run_dense(ctx, g, EPI_ARGMAX, ctx->lm, ctx->a_b, c.vocab, kD, T, false));
+    LAUNCH(SPEC_K_ARGMAX, 1, argmax_final_launch(0, ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, R, ctx->cand_ws,
                            verifier_tokens, accept_len, ctx->m_ws, ctx->vtok, s));
   }
   ctx->verified = true;
@@ -565,7 +620,7 @@ extern "C" spec_status accept_commit(spec_ctx* ctx, int32_t B, const int32_t* sl
     return fail(ctx, SPEC_EINVAL, "B and slots must be those of the last verify_step");
   if (committed == nullptr || n_committed == nullptr) return fail(ctx, SPEC_EINVAL, "null argument");
   const spec_config& c = ctx->cfg;
-  CK(commit_launch(B, ctx->last_K + 1, ctx->Rmax, ctx->Bmax, slots, ctx->m_ws, ctx->vtok, ctx->cand_ws, ctx->stage,
+  LAUNCH(SPEC_K_COMMIT, 1, commit_launch(B, ctx->last_K + 1, ctx->Rmax, ctx->Bmax, slots, ctx->m_ws, ctx->vtok, ctx->cand_ws, ctx->stage,
                    ctx->kv_pool, c.n_layers, c.n_pages_total, c.page_size, ctx->block_table, c.max_pages_per_seq,
                    ctx->seq_len, ctx->pending, ctx->b_ws, ctx->draft_b, ctx->draft_tok, ctx->draft_n, committed,
                    n_committed, ctx->d_err, ctx->stream));
@@ -587,7 +642,7 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
   const long long dstage_seq = static_cast<long long>(ctx->dstage_rows) * 2 * kD;
 
   // depth 1: the rows committed by the last step enter the draft cache with their base states
-  CK(draft_prep_launch(B, Rm, slots, ctx->seq_len, ctx->pending, ctx->draft_n, ctx->draft_b, ctx->draft_tok,
+  LAUNCH(SPEC_K_DRAFT_MISC, 1, draft_prep_launch(B, Rm, slots, ctx->seq_len, ctx->pending, ctx->draft_n, ctx->draft_b, ctx->draft_tok,
                        static_cast<const bf16*>(ctx->w.embed), c.vocab, static_cast<const bf16*>(ctx->w.enorm),
                        static_cast<const bf16*>(ctx->w.hnorm), eps, ctx->dcat, ctx->pos, ctx->kv_rowoff, ctx->last_row,
                        c.page_size, ctx->block_table, c.max_pages_per_seq, c.n_pages_total, cand, ld, ctx->d_err, s));
@@ -595,9 +650,9 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
     GemmArgs g = base_args(ctx);
     g.out = ctx->z;
     g.ldo = kD;
-    CK(run_dense(ctx, g, EPI_F32, ctx->eh, ctx->a_dcat, kD, 2 * kD, T1, true));
+    LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_F32, ctx->eh, ctx->a_dcat, kD, 2 * kD, T1, true));
   }
-  CK(rmsnorm_launch(ctx->z, T1, static_cast<const bf16*>(ctx->w.mtp_attn_norm), eps, ctx->dxn, s));
+  LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->z, T1, static_cast<const bf16*>(ctx->w.mtp_attn_norm), eps, ctx->dxn, s));
   {
     GemmArgs g = base_args(ctx);
     g.q_out = ctx->q;
@@ -606,17 +661,17 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
     g.head_stride = static_cast<long long>(c.page_size) * kHD;
     g.v_off = static_cast<long long>(kH) * c.page_size * kHD;
     g.pos = ctx->pos;
-    CK(run_dense(ctx, g, EPI_QKV, ctx->mqkv, ctx->a_dxn, 3 * kD, kD, T1, true));
+    LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_QKV, ctx->mqkv, ctx->a_dxn, 3 * kD, kD, T1, true));
   }
-  CK(gather_rows_launch(ctx->z, ctx->last_row, B, ctx->dres, s));
+  LAUNCH(SPEC_K_DRAFT_MISC, 1, gather_rows_launch(ctx->z, ctx->last_row, B, ctx->dres, s));
 
   for (int k = 1; k <= K; ++k) {
     if (k > 1) {
       GemmArgs g = base_args(ctx);
       g.out = ctx->dres;
       g.ldo = kD;
-      CK(run_dense(ctx, g, EPI_F32, ctx->eh, ctx->a_dcat, kD, 2 * kD, B, true));
-      CK(rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.mtp_attn_norm), eps, ctx->dxn, s));
+      LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_F32, ctx->eh, ctx->a_dcat, kD, 2 * kD, B, true));
+      LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.mtp_attn_norm), eps, ctx->dxn, s));
       GemmArgs q = base_args(ctx);
       q.q_out = ctx->q;
       q.kv_base = ctx->dstage;
@@ -624,7 +679,7 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       q.head_stride = kHD;
       q.v_off = static_cast<long long>(kH) * kHD;
       q.pos = ctx->pos;
-      CK(run_dense(ctx, q, EPI_QKV, ctx->mqkv, ctx->a_dxn, 3 * kD, kD, B, true));
+      LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, q, EPI_QKV, ctx->mqkv, ctx->a_dxn, 3 * kD, kD, B, true));
     }
     {
       AttnArgs a{};
@@ -648,29 +703,29 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       a.out = ctx->dattn;
       a.out_row_stride_seq = 1;
       a.err = ctx->d_err;
-      CK(attention_launch(a, B, s));
+      LAUNCH(SPEC_K_ATTN, 2, attention_launch(a, B, s));
     }
     {
       GemmArgs g = base_args(ctx);
       g.out = ctx->dres;
       g.ldo = kD;
-      CK(run_dense(ctx, g, EPI_RESID, ctx->mwo, ctx->a_dattn, kD, kD, B, true));
+      LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_RESID, ctx->mwo, ctx->a_dattn, kD, kD, B, true));
     }
-    CK(rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.mtp_ffn_norm), eps, ctx->dxn, s));
+    LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.mtp_ffn_norm), eps, ctx->dxn, s));
     {
       GemmArgs g = base_args(ctx);
       g.act = ctx->dact;
       g.ld_act = kId;
-      CK(run_dense(ctx, g, EPI_SWIGLU, ctx->mgu, ctx->a_dxn, 2 * kId, kD, B, true, true, kId));
+      LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_SWIGLU, ctx->mgu, ctx->a_dxn, 2 * kId, kD, B, true, true, kId));
     }
     {
       GemmArgs g = base_args(ctx);
       g.out = ctx->dres;
       g.ldo = kD;
-      CK(run_dense(ctx, g, EPI_RESID, ctx->mdn, ctx->a_dact, kD, kId, B, true));
+      LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_RESID, ctx->mdn, ctx->a_dact, kD, kId, B, true));
     }
     bf16* uk = ctx->u + static_cast<size_t>(k - 1) * ctx->Bmax * kD;
-    CK(rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.final_norm), eps, uk, s));
+    LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.final_norm), eps, uk, s));
     {
       GemmArgs g = base_args(ctx);
       g.am_val = ctx->am_val;
@@ -689,9 +744,9 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       g.n_items = g.n_tiles * g.m_tiles;
       g.b_row_off = (k - 1) * ctx->Bmax;
       const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
-      CK(gemm_launch(EPI_ARGMAX, box <= 64 ? 64 : 256, g, grid, s));
+      LAUNCH(SPEC_K_LMHEAD, 1, gemm_launch(EPI_ARGMAX, box <= 64 ? 64 : 256, g, grid, s));
     }
-    CK(draft_next_launch(ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, k, K, slots, ctx->seq_len, uk,
+    LAUNCH(SPEC_K_ARGMAX, 1, draft_next_launch(ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, k, K, slots, ctx->seq_len, uk,
                          static_cast<const bf16*>(ctx->w.embed), static_cast<const bf16*>(ctx->w.enorm),
                          static_cast<const bf16*>(ctx->w.hnorm), eps, ctx->dcat, ctx->pos, ctx->kv_rowoff, dstage_seq,
                          cand, ld, s));
@@ -715,6 +770,48 @@ extern "C" spec_status spec_sync(spec_ctx* ctx) {
              "mismatch, 16 no draft rows, 32 position)", flag);
     return fail(ctx, SPEC_EDEVICE, buf);
   }
+  return SPEC_OK;
+}
+
+extern "C" spec_status spec_profile(spec_ctx* ctx, int32_t enable) {
+  if (ctx == nullptr) return fail(nullptr, SPEC_EINVAL, "ctx is NULL");
+  if (enable) {
+    CK(cudaStreamSynchronize(ctx->stream));
+    for (auto& m : ctx->marks) {
+      ctx->ev_free.push_back(m.second.first);
+      ctx->ev_free.push_back(m.second.second);
+    }
+    ctx->marks.clear();
+    for (int i = 0; i < SPEC_K_COUNT; ++i) {
+      ctx->launches[i] = 0;
+      ctx->prof_ms[i] = 0.0;
+    }
+    CK(cudaMemsetAsync(ctx->d_expert_ctr, 0, 2 * sizeof(unsigned long long), ctx->stream));
+  }
+  ctx->prof_on = enable != 0;
+  return SPEC_OK;
+}
+
+extern "C" spec_status spec_profile_read(spec_ctx* ctx, spec_profile_t* out) {
+  if (ctx == nullptr) return fail(nullptr, SPEC_EINVAL, "ctx is NULL");
+  if (out == nullptr) return fail(ctx, SPEC_EINVAL, "out is NULL");
+  CK(cudaStreamSynchronize(ctx->stream));
+  for (auto& m : ctx->marks) {
+    float ms = 0.f;
+    CK(cudaEventElapsedTime(&ms, m.second.first, m.second.second));
+    ctx->prof_ms[m.first] += ms;
+    ctx->ev_free.push_back(m.second.first);
+    ctx->ev_free.push_back(m.second.second);
+  }
+  ctx->marks.clear();
+  unsigned long long ctr[2] = {0, 0};
+  CK(cudaMemcpy(ctr, ctx->d_expert_ctr, sizeof(ctr), cudaMemcpyDeviceToHost));
+  for (int i = 0; i < SPEC_K_COUNT; ++i) {
+    out->launches[i] = ctx->launches[i];
+    out->ms[i] = ctx->prof_ms[i];
+  }
+  out->experts_touched = static_cast<int64_t>(ctr[0]);
+  out->expert_rows = static_cast<int64_t>(ctr[1]);
   return SPEC_OK;
 }
 

@@ -167,7 +167,8 @@ constexpr int kMaxW = kMaxT / 32;
 
 __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, int T, const bf16* xn, bf16* xs,
                                                                int* sorted_tok, int* sorted_slot, int4* items_gu,
-                                                               int4* items_dn, int* n_items, int* counts) {
+                                                               int4* items_dn, int* n_items, int* counts,
+                                                               unsigned long long* expert_ctr) {
   extern __shared__ int psm[];
   const int W = (T + 31) / 32;
   int* s_idx = psm;                       // [T*6]
@@ -241,6 +242,10 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, i
   if (tid < kE + kShared) {
     const int e = tid, n = cnt[e];
     if (e < kE) counts[e] = n;
+    if (n > 0) {
+      atomicAdd(&expert_ctr[0], 1ull);
+      atomicAdd(&expert_ctr[1], static_cast<unsigned long long>(n));
+    }
     const int mt = (n + 255) / 256;
     for (int m = 0; m < mt; ++m) {
       const int rows = min(256, n - 256 * m);
@@ -256,7 +261,7 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, i
 
 cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
                            int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
-                           cudaStream_t s) {
+                           unsigned long long* expert_ctr, cudaStream_t s) {
   if (T > kMaxT) return cudaErrorInvalidValue;
   const int W = (T + 31) / 32;
   const size_t smem = sizeof(int) * (static_cast<size_t>(T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
@@ -272,7 +277,7 @@ cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted
   if (grid > 64) grid = 64;
   if (grid < 1) grid = 1;
   permute_kernel<<<grid, kPermThreads, smem, s>>>(idx, T, xn, x_sorted, sorted_tok, sorted_slot, items_gu, items_dn,
-                                                  n_items, counts);
+                                                  n_items, counts, expert_ctr);
   return cudaGetLastError();
 }
 

@@ -20,7 +20,9 @@ WS_B, WS_ROUTE_IDX, WS_ROUTE_GATE, WS_EXPERT_CNT, WS_DRAFT_U, WS_HIDDEN = range(
 # Public entry points, in the order include/fastmtp.h declares them.
 ENTRY_POINTS = ["spec_init", "spec_seq_reset", "spec_seq_set_draft_rows", "draft_step", "verify_step",
                 "accept_commit", "spec_sync", "spec_seq_state", "spec_read_workspace", "spec_gemm_bf16",
-                "spec_destroy", "spec_last_error"]
+                "spec_profile", "spec_profile_read", "spec_destroy", "spec_last_error"]
+KERNEL_CLASSES = ["embed", "qkv", "attention", "oproj", "router", "permute", "expert_gate_up", "expert_down",
+                  "combine", "lm_head", "argmax", "commit", "draft_gemm", "draft_misc"]
 
 
 class SpecConfig(ctypes.Structure):
@@ -41,6 +43,11 @@ class SpecWeights(ctypes.Structure):
                 ("layers", ctypes.POINTER(SpecLayerWeights))] + [(n, ctypes.c_void_p) for n in (
                     "enorm", "hnorm", "eh_proj", "mtp_attn_norm", "mtp_wqkv", "mtp_wo", "mtp_ffn_norm",
                     "mtp_w_gate_up", "mtp_w_down")]
+
+
+class SpecProfile(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_int64 * len(KERNEL_CLASSES)), ("ms", ctypes.c_double * len(KERNEL_CLASSES)),
+                ("experts_touched", ctypes.c_int64), ("expert_rows", ctypes.c_int64)]
 
 
 class FastMTPError(RuntimeError):
@@ -72,6 +79,8 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
         "spec_seq_state": (ctypes.c_int, [P, I32, ctypes.POINTER(I32), ctypes.POINTER(I32)]),
         "spec_read_workspace": (ctypes.c_int, [P, I32, P, ctypes.c_size_t]),
         "spec_gemm_bf16": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
+        "spec_profile": (ctypes.c_int, [P, I32]),
+        "spec_profile_read": (ctypes.c_int, [P, ctypes.POINTER(SpecProfile)]),
         "spec_destroy": (None, [P]),
         "spec_last_error": (ctypes.c_char_p, [P]),
     }
@@ -184,23 +193,31 @@ class Engine:
     def block_table(self, slot: int) -> List[int]:
         return [slot * self.max_pages + i for i in range(self.max_pages)]
 
-    def load_prefix(self, slot: int, kv: torch.Tensor, dkv: torch.Tensor, pending: int):
+    def load_prefix(self, slot: int, kv: Optional[torch.Tensor], dkv: Optional[torch.Tensor], pending: int,
+                    ctx_len: Optional[int] = None):
         """Places a synthetic committed prefix in slot `slot`'s pages and resets the slot.
-        kv: bf16 [L][2][ctx][H][hd]; dkv: bf16 [2][ctx][H][hd]."""
-        ctx = kv.shape[2]
+        kv: bf16 [L][2][ctx][H][hd] (verifier rows) or None; dkv: bf16 [2][ctx'][H][hd] (draft rows)
+        or None; ctx_len defaults to the verifier prefix length."""
         ps = self.page_size
         bt = self.block_table(slot)
-        n = (ctx + ps - 1) // ps
-        if n:
-            pad = n * ps - ctx
-            src = torch.nn.functional.pad(kv.to(self.device), (0, 0, 0, 0, 0, pad))
-            src = src.reshape(kv.shape[0], 2, n, ps, kv.shape[3], kv.shape[4]).permute(0, 2, 1, 4, 3, 5)
-            self.kv_pool[:, bt[0]:bt[0] + n] = src
-            dsrc = torch.nn.functional.pad(dkv.to(self.device), (0, 0, 0, 0, 0, pad))
-            dsrc = dsrc.reshape(2, n, ps, dkv.shape[2], dkv.shape[3]).permute(1, 0, 3, 2, 4)
-            self.dkv_pool[bt[0]:bt[0] + n] = dsrc
+        if kv is not None:
+            ctx = kv.shape[2]
+            n = (ctx + ps - 1) // ps
+            if n:
+                src = torch.nn.functional.pad(kv.to(self.device), (0, 0, 0, 0, 0, n * ps - ctx))
+                src = src.reshape(kv.shape[0], 2, n, ps, kv.shape[3], kv.shape[4]).permute(0, 2, 1, 4, 3, 5)
+                self.kv_pool[:, bt[0]:bt[0] + n] = src
+        if dkv is not None:
+            ctx = dkv.shape[1]
+            n = (ctx + ps - 1) // ps
+            if n:
+                dsrc = torch.nn.functional.pad(dkv.to(self.device), (0, 0, 0, 0, 0, n * ps - ctx))
+                dsrc = dsrc.reshape(2, n, ps, dkv.shape[2], dkv.shape[3]).permute(1, 0, 3, 2, 4)
+                self.dkv_pool[bt[0]:bt[0] + n] = dsrc
+        if ctx_len is None:
+            ctx_len = kv.shape[2] if kv is not None else dkv.shape[1]
         torch.cuda.synchronize(self.device)
-        self.reset_seq(slot, ctx, bt, pending)
+        self.reset_seq(slot, ctx_len, bt, pending)
 
     def reset_seq(self, slot: int, ctx_len: int, block_table: Sequence[int], pending: int):
         arr = (ctypes.c_int32 * self.max_pages)(*list(block_table))
@@ -236,6 +253,16 @@ class Engine:
         out = torch.empty(*shape, dtype=dtype)
         self._check(self.lib.spec_read_workspace(self.ctx, which, out.data_ptr(), out.numel() * out.element_size()))
         return out
+
+    def profile(self, enable: bool):
+        self._check(self.lib.spec_profile(self.ctx, 1 if enable else 0))
+
+    def profile_read(self) -> dict:
+        p = SpecProfile()
+        self._check(self.lib.spec_profile_read(self.ctx, ctypes.byref(p)))
+        return {"launches": {k: int(p.launches[i]) for i, k in enumerate(KERNEL_CLASSES)},
+                "ms": {k: float(p.ms[i]) for i, k in enumerate(KERNEL_CLASSES)},
+                "experts_touched": int(p.experts_touched), "expert_rows": int(p.expert_rows)}
 
     def close(self):
         if getattr(self, "ctx", None):

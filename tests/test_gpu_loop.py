@@ -1,0 +1,135 @@
+"""The speculative loop on the GPU: committed streams equal plain greedy decoding (K = 0)
+token for token, for injected drafts that are all right, all wrong or random and for the
+FastMTP head's own drafts (Sec. 3.1: greedy verification is lossless); a sequence verified
+alone and inside a batch gives bit-identical rows; the greedy stream agrees with the oracle's
+greedy decoding wherever the oracle's top-2 margin exceeds 1e-3."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import synth_inputs as S
+from paper_2609_03181_gb300 import fastmtp as F
+from tests.gpu_util import GAP
+
+pytestmark = pytest.mark.gpu
+
+SHAPE = S.ModelShape(n_layers=2, vocab=4096)
+B, K, N_TOK = 4, 3, 24
+
+
+@pytest.fixture(scope="module")
+def setup():
+    seed = 3
+    vw = S.verifier_weights(SHAPE, seed, gain_std=0.1)
+    dw = S.draft_weights(SHAPE, seed, gain_std=0.1)
+    ctx = [int(c) for c in S.integers(seed, "ctx", B, 100, 300)]
+    kvs = [S.kv_prefix(seed, b, SHAPE.n_layers, ctx[b], SHAPE.n_heads, SHAPE.head_dim) for b in range(B)]
+    dkvs = [S.draft_kv_prefix(seed, b, ctx[b], SHAPE.n_heads, SHAPE.head_dim) for b in range(B)]
+    pend = [int(x) for x in S.integers(seed, "pending", B, 0, SHAPE.vocab - 1)]
+    eng = F.Engine(vw, dw, max_batch=8, K_max=K, max_ctx=max(ctx) + 2 * N_TOK + 16, page_size=64)
+    yield dict(vw=vw, dw=dw, ctx=ctx, kvs=kvs, dkvs=dkvs, pend=pend, eng=eng)
+    eng.close()
+
+
+def reset(st):
+    for b in range(B):
+        st["eng"].load_prefix(b, st["kvs"][b], st["dkvs"][b], st["pend"][b])
+
+
+def run_loop(st, n_tok, K_step, draft_source=None):
+    """Returns per sequence the committed tokens (first n_tok) and the accept lengths."""
+    eng = st["eng"]
+    dev = torch.device("cuda")
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    out = [[] for _ in range(B)]
+    ms = []
+    first = True
+    while min(len(o) for o in out) < n_tok:
+        if first or K_step == 0:
+            cand = torch.tensor([[eng.seq_state(b)[1]] for b in range(B)], dtype=torch.int32, device=dev)
+        elif draft_source == "head":
+            cand = torch.empty(B, K_step + 1, dtype=torch.int32, device=dev)
+            eng.draft_step(slots, K_step, cand)
+        else:
+            pend = [eng.seq_state(b)[1] for b in range(B)]
+            cand = torch.tensor([[pend[b]] + draft_source(b, out[b]) for b in range(B)], dtype=torch.int32,
+                                device=dev)
+        Kc = cand.shape[1] - 1
+        vt = torch.empty(B, Kc + 1, dtype=torch.int32, device=dev)
+        acc = torch.empty(B, dtype=torch.int32, device=dev)
+        eng.verify_step(slots, cand, vt, acc)
+        com = torch.empty(B, Kc + 1, dtype=torch.int32, device=dev)
+        nc = torch.empty(B, dtype=torch.int32, device=dev)
+        eng.accept_commit(slots, com, nc)
+        eng.sync()
+        for b in range(B):
+            out[b].extend(com[b, : int(nc[b])].tolist())
+        ms.extend(acc.tolist() if Kc > 0 else [])
+        first = False
+    return [o[:n_tok] for o in out], ms
+
+
+def test_speculative_equals_greedy_injected_drafts(setup):
+    reset(setup)
+    greedy, _ = run_loop(setup, N_TOK + K + 2, 0)
+    rng = np.random.default_rng(0)
+    sources = {
+        "right": lambda b, done: greedy[b][len(done):len(done) + K],
+        "wrong": lambda b, done: [(t + 1) % SHAPE.vocab for t in greedy[b][len(done):len(done) + K]],
+        "random": lambda b, done: [int(x) for x in rng.integers(0, SHAPE.vocab, K)],
+    }
+    for name, fn in sources.items():
+        reset(setup)
+        got, ms = run_loop(setup, N_TOK, K, fn)
+        assert got == [g[:N_TOK] for g in greedy], name
+        if name == "right":
+            assert all(m == K for m in ms)
+        if name == "wrong":
+            assert all(m == 0 for m in ms)
+
+
+def test_speculative_with_draft_head_equals_greedy(setup):
+    reset(setup)
+    greedy, _ = run_loop(setup, N_TOK, 0)
+    reset(setup)
+    got, ms = run_loop(setup, N_TOK, K, "head")
+    assert got == greedy
+    assert all(0 <= m <= K for m in ms)
+
+
+def test_greedy_matches_oracle_greedy(setup):
+    reset(setup)
+    n = 6
+    greedy, _ = run_loop(setup, n, 0)
+    model = O.Verifier(setup["vw"])
+    for b in range(2):
+        cache = O.SeqCache.from_prefix(setup["kvs"][b], setup["pend"][b])
+        for i in range(n):
+            vo = O.verify(model, [cache], [[cache.pending]], rb=True)
+            if float(vo.v_gap[0, 0]) <= GAP:
+                break
+            assert greedy[b][i] == int(vo.v[0, 0]), (b, i)
+            O.commit([cache], vo, [[cache.pending]])
+
+
+def test_batch_invariance_alone_vs_in_batch(setup):
+    """Sequence 0 verified alone (B=1) and as row 0 of the batch of 4: identical b rows."""
+    eng = setup["eng"]
+    dev = torch.device("cuda")
+    res = []
+    for bsz in (1, B):
+        reset(setup)
+        slots = torch.arange(bsz, dtype=torch.int32, device=dev)
+        pend = [eng.seq_state(b)[1] for b in range(bsz)]
+        cand = torch.tensor([[pend[b], 11, 12, 13] for b in range(bsz)], dtype=torch.int32, device=dev)
+        vt = torch.empty(bsz, K + 1, dtype=torch.int32, device=dev)
+        acc = torch.empty(bsz, dtype=torch.int32, device=dev)
+        eng.verify_step(slots, cand, vt, acc)
+        bst = eng.read_workspace(F.WS_B, (bsz * (K + 1), SHAPE.hidden), torch.bfloat16)
+        com = torch.empty(bsz, K + 1, dtype=torch.int32, device=dev)
+        nc = torch.empty(bsz, dtype=torch.int32, device=dev)
+        eng.accept_commit(slots, com, nc)
+        eng.sync()
+        res.append((bst[: K + 1].clone(), vt[0].cpu().clone()))
+    assert torch.equal(res[0][0], res[1][0]) and torch.equal(res[0][1], res[1][1])
