@@ -187,10 +187,12 @@ spec_status spec_read_workspace(spec_ctx* ctx, int32_t id, void* dst, size_t byt
 spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, int32_t N,
                            int32_t Kdim, void* stream);
 
-/* Kernel-class timing for measurement.  spec_profile(ctx, 1) zeroes the counters and starts
- * recording a CUDA event pair around every kernel the context launches (on its stream);
- * spec_profile(ctx, 0) stops.  Launch counts and the expert counter are kept whether or not
- * events are recorded.  spec_profile_read waits for the stream and fills *out:
+/* Kernel-class timing for measurement.  spec_profile(ctx, mode): mode 1 zeroes the counters
+ * and starts recording a CUDA event pair around every launch group (inside the captured CUDA
+ * graph of each call, as external event nodes; a profiled call then waits for its graph to
+ * finish); mode 2 zeroes the counters without recording events; mode 0 stops recording.
+ * Launch counts and the expert counters are kept in every mode.  spec_profile_read waits for
+ * the stream and fills *out:
  *   launches[c], ms[c]  kernel launches and summed event time of class c (SPEC_K_*);
  *   experts_touched     routed + shared experts with at least one row, summed over the
  *                       grouped-GEMM launches (the expert weight bytes actually read);
@@ -205,7 +207,7 @@ typedef struct spec_profile_t {
   int64_t experts_touched;
   int64_t expert_rows;
 } spec_profile_t;
-spec_status spec_profile(spec_ctx* ctx, int32_t enable);
+spec_status spec_profile(spec_ctx* ctx, int32_t mode);
 spec_status spec_profile_read(spec_ctx* ctx, spec_profile_t* out);
 
 /* Frees the workspace.  Borrowed weights and pools are untouched.  NULL is ignored. */

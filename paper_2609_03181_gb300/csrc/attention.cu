@@ -179,13 +179,11 @@ __global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
       __float2bfloat16(O / L);
 }
 
+cudaError_t attention_prepare() {
+  return cudaFuncSetAttribute(attn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+}
+
 cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(attn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
   attn_chunk_kernel<<<dim3(a.n_chunks, kH, B), 128, kAttnSmem, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;

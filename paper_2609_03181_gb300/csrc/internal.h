@@ -63,7 +63,7 @@ struct GemmArgs {
   bf16* act; int ld_act;                                      // SWIGLU
   float* y; const int* sorted_tok; const int* sorted_slot;    // SCATTER
   float* am_val; int* am_idx; int am_ld;                      // ARGMAX partials [n_tile][am_ld]
-  float* sk_ws; int* sk_tickets; int sk_rows;                 // split-K partials / tickets
+  float* sk_ws; int sk_rows;                                  // split-K partials [split][sk_rows][N]
   int* err;
 };
 
@@ -75,9 +75,14 @@ bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t ro
 // Fills b_map[src][*] for an activation buffer of `rows` x `inner` bf16.
 bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err);
 
-// Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).
+// Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).  With
+// split_k > 1 (dense only) it writes partials and a reduction kernel applies the epilogue.
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s);
 int num_sms();
+// Kernel attributes (dynamic shared memory limits) set once, before any launch or capture.
+cudaError_t gemm_prepare();
+cudaError_t attention_prepare();
+cudaError_t permute_prepare();
 
 // Split-K count of a dense matrix: depends on (N, K) only, never on M, so every row's sum
 // order is the same at any batch size.

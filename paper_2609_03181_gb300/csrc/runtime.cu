@@ -2,6 +2,7 @@
 // TMA descriptors and the launch sequence of draft_step / verify_step / accept_commit.
 #include <math.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <string>
@@ -22,6 +23,26 @@ struct LayerMaps {
 
 struct ActMaps {
   CUtensorMap m[5];
+};
+
+typedef std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>> Mark;
+
+// One captured call: the key of everything its kernels bake in (sizes and caller pointers),
+// the instantiated graph, its launch counts per kernel class and, for profiled graphs, the
+// event pairs recorded around each launch group.
+struct GraphKey {
+  int kind, B, K, prof;
+  const void* p[4];
+  bool operator==(const GraphKey& o) const {
+    return kind == o.kind && B == o.B && K == o.K && prof == o.prof && p[0] == o.p[0] && p[1] == o.p[1] &&
+           p[2] == o.p[2] && p[3] == o.p[3];
+  }
+};
+struct CallGraph {
+  GraphKey key;
+  cudaGraphExec_t exec = nullptr;
+  std::vector<std::pair<int, int>> counts;
+  std::vector<Mark> marks;
 };
 
 }  // namespace
@@ -88,14 +109,17 @@ struct spec_ctx {
   bf16* dstage = nullptr;
   int* last_row = nullptr;
   float* sk_ws = nullptr;
-  int* sk_tickets = nullptr;
   float2* rope = nullptr;
   int* d_err = nullptr;
 
   // measurement: event pairs per kernel class, launch counts, expert counters (device int64[2])
   bool prof_on = false;
   std::vector<cudaEvent_t> ev_free;
-  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> marks;
+  std::vector<Mark> marks;
+  // CUDA graphs: one per distinct call key, replayed on later calls with the same key
+  bool use_graphs = true;
+  std::vector<CallGraph*> graphs;
+  CallGraph* capturing = nullptr;
   int64_t launches[SPEC_K_COUNT] = {};
   double prof_ms[SPEC_K_COUNT] = {};
   unsigned long long* d_expert_ctr = nullptr;
@@ -133,7 +157,6 @@ GemmArgs base_args(spec_ctx* ctx) {
   g.rope = ctx->rope;
   g.max_pos = ctx->cfg.max_position;
   g.sk_ws = ctx->sk_ws;
-  g.sk_tickets = ctx->sk_tickets;
   g.sk_rows = ctx->Tmax;
   g.am_ld = ctx->Tmax;
   g.err = ctx->d_err;
@@ -179,19 +202,35 @@ cudaEvent_t take_event(spec_ctx* ctx) {
   return e;
 }
 
-// Brackets one launch group of kernel class `cls` (n_kernels kernels) with an event pair
-// when profiling is on, and counts its launches always.
+// Brackets one launch group of kernel class `cls` (n_kernels kernels): counts its launches
+// and, when profiling, records an event pair around it (as external event nodes while a
+// profiled graph is being captured).
 struct ProfScope {
   spec_ctx* ctx;
   int cls;
   cudaEvent_t e0 = nullptr;
   ProfScope(spec_ctx* c, int k) : ctx(c), cls(k) {
-    if (ctx->prof_on) {
+    if (ctx->capturing != nullptr) {
+      if (ctx->capturing->key.prof) {
+        cudaEventCreate(&e0);
+        cudaEventRecordWithFlags(e0, ctx->stream, cudaEventRecordExternal);
+      }
+    } else if (ctx->prof_on) {
       e0 = take_event(ctx);
       cudaEventRecord(e0, ctx->stream);
     }
   }
   void done(int n_kernels) {
+    if (ctx->capturing != nullptr) {
+      ctx->capturing->counts.push_back({cls, n_kernels});
+      if (ctx->capturing->key.prof) {
+        cudaEvent_t e1 = nullptr;
+        cudaEventCreate(&e1);
+        cudaEventRecordWithFlags(e1, ctx->stream, cudaEventRecordExternal);
+        ctx->capturing->marks.push_back({cls, {e0, e1}});
+      }
+      return;
+    }
     ctx->launches[cls] += n_kernels;
     if (ctx->prof_on) {
       cudaEvent_t e1 = take_event(ctx);
@@ -200,6 +239,66 @@ struct ProfScope {
     }
   }
 };
+
+void destroy_graph(CallGraph* g) {
+  if (g->exec) cudaGraphExecDestroy(g->exec);
+  for (auto& m : g->marks) {
+    cudaEventDestroy(m.second.first);
+    cudaEventDestroy(m.second.second);
+  }
+  delete g;
+}
+
+// Runs `body` (the launch sequence of one call) through a CUDA graph: captured the first
+// time a key is seen, replayed afterwards.  Profiled graphs are synchronised after each replay
+// so that their event pairs can be read before the next replay records them again.
+template <class F>
+spec_status run_graphed(spec_ctx* ctx, GraphKey key, F body) {
+  key.prof = ctx->prof_on ? 1 : 0;
+  if (!ctx->use_graphs || ctx->stream == nullptr) return body();
+  CallGraph* g = nullptr;
+  for (CallGraph* c : ctx->graphs)
+    if (c->key == key) g = c;
+  if (g == nullptr) {
+    g = new CallGraph();
+    g->key = key;
+    cudaError_t e = cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) {
+      delete g;
+      return fail(ctx, SPEC_ECUDA, std::string("cudaStreamBeginCapture: ") + cudaGetErrorString(e));
+    }
+    ctx->capturing = g;
+    spec_status st = body();
+    ctx->capturing = nullptr;
+    cudaGraph_t graph = nullptr;
+    e = cudaStreamEndCapture(ctx->stream, &graph);
+    if (st != SPEC_OK || e != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      destroy_graph(g);
+      if (st != SPEC_OK) return st;
+      return fail(ctx, SPEC_ECUDA, std::string("cudaStreamEndCapture: ") + cudaGetErrorString(e));
+    }
+    e = cudaGraphInstantiate(&g->exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+      destroy_graph(g);
+      return fail(ctx, SPEC_ECUDA, std::string("cudaGraphInstantiate: ") + cudaGetErrorString(e));
+    }
+    ctx->graphs.push_back(g);
+  }
+  cudaError_t e = cudaGraphLaunch(g->exec, ctx->stream);
+  if (e != cudaSuccess) return fail(ctx, SPEC_ECUDA, std::string("cudaGraphLaunch: ") + cudaGetErrorString(e));
+  for (auto& c : g->counts) ctx->launches[c.first] += c.second;
+  if (key.prof) {
+    e = cudaStreamSynchronize(ctx->stream);
+    if (e != cudaSuccess) return fail(ctx, SPEC_ECUDA, std::string("profiled graph: ") + cudaGetErrorString(e));
+    for (auto& m : g->marks) {
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, m.second.first, m.second.second) == cudaSuccess) ctx->prof_ms[m.first] += ms;
+    }
+  }
+  return SPEC_OK;
+}
 
 }  // namespace
 
@@ -246,6 +345,12 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   for (const void* p : top)
     if (!aligned16(p)) return fail(nullptr, SPEC_EINVAL, "matrix or pool not 16-byte aligned");
 
+  {
+    cudaError_t e = gemm_prepare();
+    if (e == cudaSuccess) e = attention_prepare();
+    if (e == cudaSuccess) e = permute_prepare();
+    if (e != cudaSuccess) return fail(nullptr, SPEC_ECUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
+  }
   ctx = new spec_ctx();
   ctx->cfg = c;
   ctx->stream = static_cast<cudaStream_t>(stream);
@@ -255,6 +360,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ctx->w.layers = ctx->layers.data();
   ctx->kv_pool = static_cast<bf16*>(kv_pool);
   ctx->dkv_pool = static_cast<bf16*>(draft_kv_pool);
+  ctx->use_graphs = getenv("FASTMTP_NO_GRAPHS") == nullptr;
 
   const int L = c.n_layers;
   ctx->Bmax = c.max_batch;
@@ -325,7 +431,6 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->dstage, sizeof(bf16) * Bmax * ctx->dstage_rows * 2 * d);
   add(&ctx->last_row, sizeof(int) * Bmax);
   add(&ctx->sk_ws, sizeof(float) * ctx->sk_floats);
-  add(&ctx->sk_tickets, sizeof(int) * 16384);
   add(&ctx->rope, sizeof(float2) * static_cast<size_t>(c.max_position) * (kHD / 2));
   add(&ctx->d_err, sizeof(int) * 4);
   add(&ctx->d_expert_ctr, sizeof(unsigned long long) * 2);
@@ -409,6 +514,7 @@ extern "C" void spec_destroy(spec_ctx* ctx) {
     cudaEventDestroy(m.second.second);
   }
   for (cudaEvent_t e : ctx->ev_free) cudaEventDestroy(e);
+  for (CallGraph* g : ctx->graphs) destroy_graph(g);
   cudaFree(ctx->ws);
   delete ctx;
 }
@@ -492,6 +598,8 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   const size_t stage_layer = static_cast<size_t>(ctx->Bmax) * ctx->Rmax * 2 * kD;
   const size_t pool_layer = static_cast<size_t>(c.n_pages_total) * 2 * kH * c.page_size * kHD;
 
+  GraphKey key{1, B, K, 0, {slots, cand, verifier_tokens, accept_len}};
+  spec_status st = run_graphed(ctx, key, [&]() -> spec_status {
   CK(cudaMemcpyAsync(ctx->cand_ws, cand, sizeof(int) * T, cudaMemcpyDeviceToDevice, s));
   LAUNCH(SPEC_K_EMBED, 1, embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
                        c.vocab, static_cast<const bf16*>(ctx->layers[0].attn_norm), eps, ctx->h, ctx->xn, ctx->pos,
@@ -604,6 +712,9 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
     LAUNCH(SPEC_K_ARGMAX, 1, argmax_final_launch(0, ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, R, ctx->cand_ws,
                            verifier_tokens, accept_len, ctx->m_ws, ctx->vtok, s));
   }
+    return SPEC_OK;
+  });
+  if (st != SPEC_OK) return st;
   ctx->verified = true;
   ctx->last_B = B;
   ctx->last_K = K;
@@ -620,10 +731,15 @@ extern "C" spec_status accept_commit(spec_ctx* ctx, int32_t B, const int32_t* sl
     return fail(ctx, SPEC_EINVAL, "B and slots must be those of the last verify_step");
   if (committed == nullptr || n_committed == nullptr) return fail(ctx, SPEC_EINVAL, "null argument");
   const spec_config& c = ctx->cfg;
+  GraphKey key{2, B, ctx->last_K, 0, {slots, committed, n_committed, nullptr}};
+  spec_status st = run_graphed(ctx, key, [&]() -> spec_status {
   LAUNCH(SPEC_K_COMMIT, 1, commit_launch(B, ctx->last_K + 1, ctx->Rmax, ctx->Bmax, slots, ctx->m_ws, ctx->vtok, ctx->cand_ws, ctx->stage,
                    ctx->kv_pool, c.n_layers, c.n_pages_total, c.page_size, ctx->block_table, c.max_pages_per_seq,
                    ctx->seq_len, ctx->pending, ctx->b_ws, ctx->draft_b, ctx->draft_tok, ctx->draft_n, committed,
                    n_committed, ctx->d_err, ctx->stream));
+    return SPEC_OK;
+  });
+  if (st != SPEC_OK) return st;
   ctx->verified = false;
   return SPEC_OK;
 }
@@ -641,6 +757,8 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
   const int Rm = ctx->Rmax, T1 = B * Rm, ld = K + 1;
   const long long dstage_seq = static_cast<long long>(ctx->dstage_rows) * 2 * kD;
 
+  GraphKey key{3, B, K, 0, {slots, cand, nullptr, nullptr}};
+  spec_status st = run_graphed(ctx, key, [&]() -> spec_status {
   // depth 1: the rows committed by the last step enter the draft cache with their base states
   LAUNCH(SPEC_K_DRAFT_MISC, 1, draft_prep_launch(B, Rm, slots, ctx->seq_len, ctx->pending, ctx->draft_n, ctx->draft_b, ctx->draft_tok,
                        static_cast<const bf16*>(ctx->w.embed), c.vocab, static_cast<const bf16*>(ctx->w.enorm),
@@ -751,6 +869,9 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
                          static_cast<const bf16*>(ctx->w.hnorm), eps, ctx->dcat, ctx->pos, ctx->kv_rowoff, dstage_seq,
                          cand, ld, s));
   }
+    return SPEC_OK;
+  });
+  if (st != SPEC_OK) return st;
   ctx->last_draft_K = K;
   ctx->last_draft_B = B;
   return SPEC_OK;
@@ -773,9 +894,10 @@ extern "C" spec_status spec_sync(spec_ctx* ctx) {
   return SPEC_OK;
 }
 
-extern "C" spec_status spec_profile(spec_ctx* ctx, int32_t enable) {
+extern "C" spec_status spec_profile(spec_ctx* ctx, int32_t mode) {
   if (ctx == nullptr) return fail(nullptr, SPEC_EINVAL, "ctx is NULL");
-  if (enable) {
+  if (mode < 0 || mode > 2) return fail(ctx, SPEC_EINVAL, "mode must be 0, 1 or 2");
+  if (mode != 0) {
     CK(cudaStreamSynchronize(ctx->stream));
     for (auto& m : ctx->marks) {
       ctx->ev_free.push_back(m.second.first);
@@ -788,7 +910,7 @@ extern "C" spec_status spec_profile(spec_ctx* ctx, int32_t enable) {
     }
     CK(cudaMemsetAsync(ctx->d_expert_ctr, 0, 2 * sizeof(unsigned long long), ctx->stream));
   }
-  ctx->prof_on = enable != 0;
+  ctx->prof_on = mode == 1;
   return SPEC_OK;
 }
 
@@ -853,6 +975,7 @@ extern "C" spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, in
   if (!encode_map_2d(&g.a_map[0], W, Kdim, N, 128, &e)) return fail(nullptr, SPEC_EINVAL, e);
   if (!encode_act_maps(g.b_map[0], X, Kdim, M, &e)) return fail(nullptr, SPEC_EINVAL, e);
   int* err = nullptr;
+  CK(gemm_prepare());
   CK(cudaGetSymbolAddress(reinterpret_cast<void**>(&err), g_gemm_err));
   g.err = err;
   g.n_routed = 1 << 30;

@@ -111,19 +111,27 @@ __global__ void __launch_bounds__(128) router_kernel(const float* h, const bf16*
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int e = warp * 16; e < warp * 16 + 16; ++e) {
-    const bf16* w = wr + static_cast<size_t>(e) * kD;
-    float acc = 0.f;
+  for (int e0 = warp * 16; e0 < warp * 16 + 16; e0 += 4) {
+    // four experts at a time: 20 independent 16-byte weight loads in flight per lane
+    uint4 raw[4][5];
 #pragma unroll
-    for (int c = 0; c < 5; ++c) {
-      const int i0 = c * 256 + lane * 8;
-      const uint4 raw = *reinterpret_cast<const uint4*>(w + i0);
-      const bf16* wv = reinterpret_cast<const bf16*>(&raw);
+    for (int q = 0; q < 4; ++q)
 #pragma unroll
-      for (int u = 0; u < 8; ++u) acc += __bfloat162float(wv[u]) * xs[i0 + u];
+      for (int c = 0; c < 5; ++c)
+        raw[q][c] = *reinterpret_cast<const uint4*>(wr + static_cast<size_t>(e0 + q) * kD + c * 256 + lane * 8);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float acc = 0.f;
+#pragma unroll
+      for (int c = 0; c < 5; ++c) {
+        const int i0 = c * 256 + lane * 8;
+        const bf16* wv = reinterpret_cast<const bf16*>(&raw[q][c]);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc += __bfloat162float(wv[u]) * xs[i0 + u];
+      }
+      acc = warp_sum(acc);
+      if (lane == 0) lg[e0 + q] = acc + (bias ? bias[e0 + q] : 0.f);
     }
-    acc = warp_sum(acc);
-    if (lane == 0) lg[e] = acc + (bias ? bias[e] : 0.f);
   }
   __syncthreads();
   if (warp == 0) {
@@ -259,19 +267,17 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, i
   }
 }
 
+cudaError_t permute_prepare() {
+  return cudaFuncSetAttribute(permute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(sizeof(int) * (kMaxT * kTopK + 2 * kE * kMaxW + 4 * 67)));
+}
+
 cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
                            int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
                            unsigned long long* expert_ctr, cudaStream_t s) {
   if (T > kMaxT) return cudaErrorInvalidValue;
   const int W = (T + 31) / 32;
   const size_t smem = sizeof(int) * (static_cast<size_t>(T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(permute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(sizeof(int) * (kMaxT * kTopK + 2 * kE * kMaxW + 4 * 67)));
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
   const int pairs = T * kTopK;
   int grid = (pairs + 63) / 64;   // ~64 row copies per CTA
   if (grid > 64) grid = 64;

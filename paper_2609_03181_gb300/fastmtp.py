@@ -254,8 +254,9 @@ class Engine:
         self._check(self.lib.spec_read_workspace(self.ctx, which, out.data_ptr(), out.numel() * out.element_size()))
         return out
 
-    def profile(self, enable: bool):
-        self._check(self.lib.spec_profile(self.ctx, 1 if enable else 0))
+    def profile(self, mode: int):
+        """1: zero the counters and time every launch group; 2: zero the counters only; 0: stop."""
+        self._check(self.lib.spec_profile(self.ctx, int(mode)))
 
     def profile_read(self) -> dict:
         p = SpecProfile()
