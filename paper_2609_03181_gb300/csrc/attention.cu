@@ -6,10 +6,11 @@
 // range is cut into chunks of 128 positions fixed by absolute position; one CTA per
 // (chunk, head, sequence) stages the chunk's K and V in shared memory with 16-byte
 // cp.async copies, scores every (query, key) pair in fp32, and writes the chunk's
-// (max, sum, unnormalised output) per query.  A second kernel merges the chunks of each query
-// in chunk order.  Masked keys contribute exact zeros, so a query's result is the same
-// whether its key sits in a page or in staging and however many other queries share the
-// chunk: greedy decoding (K = 0) and speculative verification see identical rows.
+// (max, sum, unnormalised output) per query; the last chunk of a (sequence, head) to finish
+// merges the chunks of each query in chunk order.  Masked keys contribute exact zeros, so a
+// query's result is the same whether its key sits in a page or in staging and however many
+// other queries share the chunk: greedy decoding (K = 0) and speculative verification see
+// identical rows.
 #include <math.h>
 
 #include "common.cuh"
@@ -19,10 +20,28 @@ namespace fm {
 
 constexpr int kCH = kAttnChunk;
 constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 4 + kMaxR * kCH * 4;
+constexpr long long kStagedBit = 1ll << 62;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
                : "memory");
+}
+
+// Softmax-weighted combination of the chunks 0..lastc of one query, in chunk order.
+__device__ __forceinline__ void merge_query(const AttnArgs& a, int b, int h, int r, int lastc, int R) {
+  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * a.n_chunks * R * (kHD + 2);
+  float M = -INFINITY;
+  for (int c = 0; c <= lastc; ++c) M = fmaxf(M, __ldcg(&part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + kHD]));
+  float L = 0.f, O = 0.f;
+  for (int c = 0; c <= lastc; ++c) {
+    const float* pc = part + (static_cast<size_t>(c) * R + r) * (kHD + 2);
+    const float mc = __ldcg(&pc[kHD]);
+    const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
+    L += __ldcg(&pc[kHD + 1]) * w;
+    O += __ldcg(&pc[threadIdx.x]) * w;
+  }
+  a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + threadIdx.x] =
+      __float2bfloat16(O / L);
 }
 
 __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
@@ -31,6 +50,8 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   bf16* sV = sK + kCH * kHD;
   float* sq = reinterpret_cast<float*>(sV + kCH * kHD);    // [R][kHD]
   float* sp = sq + kMaxR * kHD;                           // [R][kCH] scores, then probabilities
+  __shared__ long long s_base[kCH];                       // element offset of each key row (-1: none)
+  __shared__ int s_last;
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int R = a.R;
@@ -43,36 +64,55 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   const int nk = min(kCH, last + 1 - start);
   const int tid = threadIdx.x;
 
-  // K and V rows of the chunk -> shared memory (zero-filled past the last key)
-  for (int v = tid; v < kCH * 16; v += 128) {
-    const int j = v >> 4, ch = v & 15;
+  // where each key row lives: a page of the pool (positions < ctx_len) or a staging row
+  {
+    const int j = tid;
     const int pos = start + j;
-    const bf16* srck = a.pool;
-    const bf16* srcv = a.pool;
-    int bytes = 0;
+    long long off = -1;
     if (j < nk) {
       if (pos < sl) {
         const int pi = pos / a.page_size;
         const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
-        if (page >= 0 && page < a.n_pages) {
-          const size_t base = ((static_cast<size_t>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
-          srck = a.pool + base;
-          srcv = a.pool + base + static_cast<size_t>(kH) * a.page_size * kHD;
-          bytes = 16;
-        } else if (ch == 0) {
+        if (page >= 0 && page < a.n_pages)
+          off = ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
+        else
           atomicOr(a.err, ERR_PAGE_RANGE);
-        }
       } else {
-        const size_t base = b * a.stage_seq_stride + static_cast<size_t>(pos - sl) * a.stage_row_stride +
-                            static_cast<size_t>(h) * kHD;
-        srck = a.stage + base;
-        srcv = a.stage + base + a.stage_kv_stride;
-        bytes = 16;
+        off = kStagedBit | (b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
+                            static_cast<long long>(h) * kHD);
       }
     }
-    const int sw = ((ch ^ (j & 7)) * 8);
-    cp_async16(sK + j * kHD + sw, srck + ch * 8 * (bytes ? 1 : 0), bytes);
-    cp_async16(sV + j * kHD + sw, srcv + ch * 8 * (bytes ? 1 : 0), bytes);
+    s_base[j] = off;
+  }
+  __syncthreads();
+
+  // K, then V, rows of the chunk -> shared memory (zero-filled where there is no key)
+  const long long v_pool = static_cast<long long>(kH) * a.page_size * kHD;
+#pragma unroll 4
+  for (int v = tid; v < kCH * 16; v += 128) {
+    const int j = v >> 4, ch = v & 15;
+    const long long off = s_base[j];
+    const bf16* src = a.pool;
+    int bytes = 0;
+    if (off >= 0) {
+      src = ((off & kStagedBit) ? a.stage + (off & (kStagedBit - 1)) : a.pool + off) + ch * 8;
+      bytes = 16;
+    }
+    cp_async16(sK + j * kHD + ((ch ^ (j & 7)) * 8), src, bytes);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+#pragma unroll 4
+  for (int v = tid; v < kCH * 16; v += 128) {
+    const int j = v >> 4, ch = v & 15;
+    const long long off = s_base[j];
+    const bf16* src = a.pool;
+    int bytes = 0;
+    if (off >= 0) {
+      src = ((off & kStagedBit) ? a.stage + (off & (kStagedBit - 1)) + a.stage_kv_stride : a.pool + off + v_pool) +
+            ch * 8;
+      bytes = 16;
+    }
+    cp_async16(sV + j * kHD + ((ch ^ (j & 7)) * 8), src, bytes);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
 
@@ -83,7 +123,7 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
     const int r = v / kHD, d = v % kHD;
     sq[v] = a.q[(static_cast<size_t>(qrow0 + r) * kH + h) * kHD + d] * qscale;
   }
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  asm volatile("cp.async.wait_group 1;" ::: "memory");   // K has landed; V may still be in flight
   __syncthreads();
 
   // scores: thread j owns key j of the chunk
@@ -136,6 +176,7 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
       part[r * (kHD + 2) + kHD + 1] = l;
     }
   }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncthreads();
 
   // P V: thread d owns output dim d
@@ -154,29 +195,22 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
     for (int r = 0; r < kMaxR; ++r)
       if (r < R) part[r * (kHD + 2) + d] = acc[r];
   }
-}
 
-// Merges the chunks 0..floor(p/128) of each query in chunk order: softmax-weighted combination.
-__global__ void __launch_bounds__(128) attn_merge_kernel(const AttnArgs a) {
-  const int R = a.R;
-  const int b = blockIdx.x / R, r = blockIdx.x % R, h = blockIdx.y;
-  const int slot = a.slots[b];
-  const int p = a.seq_len[slot] + a.qoff + r;
-  if (p < 0) return;
-  const int lastc = p / kCH;
-  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * a.n_chunks * R * (kHD + 2);
-  float M = -INFINITY;
-  for (int c = 0; c <= lastc; ++c) M = fmaxf(M, part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + kHD]);
-  float L = 0.f, O = 0.f;
-  for (int c = 0; c <= lastc; ++c) {
-    const float* pc = part + (static_cast<size_t>(c) * R + r) * (kHD + 2);
-    const float mc = pc[kHD];
-    const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
-    L += pc[kHD + 1] * w;
-    O += pc[threadIdx.x] * w;
+  // the last chunk of (sequence, head) to finish merges every query (atomic ticket, no wait)
+  __threadfence();
+  __syncthreads();
+  const int n_live = last / kCH + 1;
+  if (tid == 0) {
+    int* ticket = a.tickets + b * kH + h;
+    const int old = atomicAdd(ticket, 1);
+    s_last = (old == n_live - 1) ? 1 : 0;
+    if (s_last) *ticket = 0;
   }
-  a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + threadIdx.x] =
-      __float2bfloat16(O / L);
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    for (int r = 0; r < R; ++r) merge_query(a, b, h, r, (p0 + r) / kCH, R);
+  }
 }
 
 cudaError_t attention_prepare() {
@@ -185,9 +219,6 @@ cudaError_t attention_prepare() {
 
 cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s) {
   attn_chunk_kernel<<<dim3(a.n_chunks, kH, B), 128, kAttnSmem, s>>>(a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  attn_merge_kernel<<<dim3(B * a.R, kH), 128, 0, s>>>(a);
   return cudaGetLastError();
 }
 

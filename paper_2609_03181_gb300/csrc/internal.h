@@ -99,6 +99,7 @@ struct AttnArgs {
   const bf16* stage;           // keys at positions >= seq_len[slot]: staged row (pos - seq_len)
   long long stage_seq_stride, stage_row_stride, stage_kv_stride;
   float* part;                 // [B][H][n_chunks][R][kHD + 2]
+  int* tickets;                // [B][H] chunk counters, zero between launches
   int n_chunks;
   bf16* out;                   // [B*R][H*hd]
   int out_row_stride_seq;      // rows of out per sequence (R)

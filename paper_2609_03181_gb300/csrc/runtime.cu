@@ -73,6 +73,7 @@ struct spec_ctx {
   float* q = nullptr;
   bf16* stage = nullptr;
   float* attn_part = nullptr;
+  int* attn_tickets = nullptr;
   bf16* attn_out = nullptr;
   int* route_idx = nullptr;
   float* route_gate = nullptr;
@@ -395,6 +396,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->q, sizeof(float) * Tmax * d);
   add(&ctx->stage, sizeof(bf16) * L * Bmax * Rmax * 2 * d);
   add(&ctx->attn_part, sizeof(float) * static_cast<size_t>(Bmax) * kH * ctx->n_chunks * Rmax * (kHD + 2));
+  add(&ctx->attn_tickets, sizeof(int) * Bmax * kH);
   add(&ctx->attn_out, sizeof(bf16) * Tmax * d);
   add(&ctx->route_idx, sizeof(int) * L * Tmax * kTopK);
   add(&ctx->route_gate, sizeof(float) * L * Tmax * kTopK);
@@ -638,11 +640,12 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       a.stage_row_stride = 2 * kD;
       a.stage_kv_stride = kD;
       a.part = ctx->attn_part;
+      a.tickets = ctx->attn_tickets;
       a.n_chunks = ctx->n_chunks;
       a.out = ctx->attn_out;
       a.out_row_stride_seq = R;
       a.err = ctx->d_err;
-      LAUNCH(SPEC_K_ATTN, 2, attention_launch(a, B, s));
+      LAUNCH(SPEC_K_ATTN, 1, attention_launch(a, B, s));
     }
     // O-proj + residual
     {
@@ -817,11 +820,12 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       a.stage_row_stride = 2 * kD;
       a.stage_kv_stride = kD;
       a.part = ctx->attn_part;
+      a.tickets = ctx->attn_tickets;
       a.n_chunks = ctx->n_chunks;
       a.out = ctx->dattn;
       a.out_row_stride_seq = 1;
       a.err = ctx->d_err;
-      LAUNCH(SPEC_K_ATTN, 2, attention_launch(a, B, s));
+      LAUNCH(SPEC_K_ATTN, 1, attention_launch(a, B, s));
     }
     {
       GemmArgs g = base_args(ctx);

@@ -10,30 +10,39 @@
 
 namespace fm {
 
-// Sum over a 128-thread block in a fixed order (warp trees, then warps 0..3).
-__device__ __forceinline__ float block128_sum(float v, float* red) {
+// Sum over an NT-thread block in a fixed order (warp trees, then warps in index order).
+template <int NT>
+__device__ __forceinline__ float block_sum(float v, float* red) {
   v = warp_sum(v);
   const int w = threadIdx.x >> 5;
   if ((threadIdx.x & 31) == 0) red[w] = v;
   __syncthreads();
-  const float s = ((red[0] + red[1]) + red[2]) + red[3];
+  float s = red[0];
+#pragma unroll
+  for (int i = 1; i < NT / 32; ++i) s += red[i];
   __syncthreads();
   return s;
 }
+__device__ __forceinline__ float block128_sum(float v, float* red) { return block_sum<128>(v, red); }
 
-// x (10 values per thread, element i = tid + 128*k) -> bf16 x * rsqrt(mean(x^2) + eps) * gain
-__device__ __forceinline__ void norm_row_store(const float (&x)[10], const bf16* gain, float eps, bf16* out,
-                                               float* red) {
+// x (kD/NT values per thread, element i = tid + NT*k) -> bf16 x * rsqrt(mean(x^2) + eps) * gain
+template <int NT>
+__device__ __forceinline__ void norm_row_store_t(const float (&x)[kD / NT], const bf16* gain, float eps, bf16* out,
+                                                 float* red) {
   float ss = 0.f;
 #pragma unroll
-  for (int k = 0; k < 10; ++k) ss += x[k] * x[k];
-  ss = block128_sum(ss, red);
+  for (int k = 0; k < kD / NT; ++k) ss += x[k] * x[k];
+  ss = block_sum<NT>(ss, red);
   const float inv = rsqrtf(ss / kD + eps);
 #pragma unroll
-  for (int k = 0; k < 10; ++k) {
-    const int i = threadIdx.x + 128 * k;
+  for (int k = 0; k < kD / NT; ++k) {
+    const int i = threadIdx.x + NT * k;
     out[i] = __float2bfloat16(x[k] * inv * __bfloat162float(gain[i]));
   }
+}
+__device__ __forceinline__ void norm_row_store(const float (&x)[10], const bf16* gain, float eps, bf16* out,
+                                               float* red) {
+  norm_row_store_t<128>(x, gain, eps, out, red);
 }
 
 // ---------------------------------------------------------------- embedding + norm
@@ -93,25 +102,26 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
 // ---------------------------------------------------------------- router
 // RMSNorm of the residual row -> xn (bf16, also the experts' input); logits of the 64
 // experts from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).
-__global__ void __launch_bounds__(128) router_kernel(const float* h, const bf16* gain, float eps, const bf16* wr,
+__global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16* gain, float eps, const bf16* wr,
                                                      const float* bias, bf16* xn, int* idx, float* gate) {
-  __shared__ float red[4];
+  constexpr int NT = 256, EPT = kD / NT;
+  __shared__ float red[NT / 32];
   __shared__ __align__(16) float xs[kD];
   __shared__ float lg[kE];
   const size_t t = blockIdx.x;
-  float v[10];
+  float v[EPT];
 #pragma unroll
-  for (int k = 0; k < 10; ++k) v[k] = h[t * kD + threadIdx.x + 128 * k];
+  for (int k = 0; k < EPT; ++k) v[k] = h[t * kD + threadIdx.x + NT * k];
   bf16* xo = xn + t * kD;
-  norm_row_store(v, gain, eps, xo, red);
+  norm_row_store_t<NT>(v, gain, eps, xo, red);
 #pragma unroll
-  for (int k = 0; k < 10; ++k) {
-    const int i = threadIdx.x + 128 * k;
+  for (int k = 0; k < EPT; ++k) {
+    const int i = threadIdx.x + NT * k;
     xs[i] = __bfloat162float(xo[i]);   // the rounded row, as the experts see it
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int e0 = warp * 16; e0 < warp * 16 + 16; e0 += 4) {
+  for (int e0 = warp * 8; e0 < warp * 8 + 8; e0 += 4) {
     // four experts at a time: 20 independent 16-byte weight loads in flight per lane
     uint4 raw[4][5];
 #pragma unroll
@@ -159,7 +169,7 @@ __global__ void __launch_bounds__(128) router_kernel(const float* h, const bf16*
 
 cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
                           const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s) {
-  router_kernel<<<T, 128, 0, s>>>(h, gain, eps, w_router, bias, xn, idx, gate);
+  router_kernel<<<T, 256, 0, s>>>(h, gain, eps, w_router, bias, xn, idx, gate);
   return cudaGetLastError();
 }
 
@@ -279,8 +289,8 @@ cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted
   const int W = (T + 31) / 32;
   const size_t smem = sizeof(int) * (static_cast<size_t>(T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
   const int pairs = T * kTopK;
-  int grid = (pairs + 63) / 64;   // ~64 row copies per CTA
-  if (grid > 64) grid = 64;
+  int grid = (pairs + 7) / 8;     // one warp per (token, slot) row copy
+  if (grid > 512) grid = 512;
   if (grid < 1) grid = 1;
   permute_kernel<<<grid, kPermThreads, smem, s>>>(idx, T, xn, x_sorted, sorted_tok, sorted_slot, items_gu, items_dn,
                                                   n_items, counts, expert_ctr);
@@ -289,32 +299,37 @@ cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted
 
 // ---------------------------------------------------------------- combine
 // h += sum_{s<6} gate_s * y_s + y_shared0 + y_shared1 (fixed slot order), then RMSNorm -> out.
-__global__ void __launch_bounds__(128) combine_kernel(float* h, const float* y, const float* gate, const bf16* gain,
+__global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, const float* gate, const bf16* gain,
                                                       float eps, bf16* out) {
-  __shared__ float red[4];
+  constexpr int NT = 256, EPT = kD / NT;
+  __shared__ float red[NT / 32];
   const size_t t = blockIdx.x;
   float g[kTopK];
 #pragma unroll
   for (int s = 0; s < kTopK; ++s) g[s] = gate[t * kTopK + s];
-  float x[10];
+  float ys[EPT][kSlots];
 #pragma unroll
-  for (int k = 0; k < 10; ++k) {
-    const int i = threadIdx.x + 128 * k;
-    const float* yt = y + t * kSlots * kD + i;
+  for (int k = 0; k < EPT; ++k)
+#pragma unroll
+    for (int s = 0; s < kSlots; ++s) ys[k][s] = y[(t * kSlots + s) * kD + threadIdx.x + NT * k];
+  float x[EPT];
+#pragma unroll
+  for (int k = 0; k < EPT; ++k) {
+    const int i = threadIdx.x + NT * k;
     float acc = 0.f;
 #pragma unroll
-    for (int s = 0; s < kTopK; ++s) acc += g[s] * yt[s * kD];
-    acc += yt[kTopK * kD];
-    acc += yt[(kTopK + 1) * kD];
+    for (int s = 0; s < kTopK; ++s) acc += g[s] * ys[k][s];
+    acc += ys[k][kTopK];
+    acc += ys[k][kTopK + 1];
     x[k] = h[t * kD + i] + acc;
     h[t * kD + i] = x[k];
   }
-  norm_row_store(x, gain, eps, out + t * kD, red);
+  norm_row_store_t<NT>(x, gain, eps, out + t * kD, red);
 }
 
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
                            bf16* out, cudaStream_t s) {
-  combine_kernel<<<T, 128, 0, s>>>(h, y, gate, gain, eps, out);
+  combine_kernel<<<T, 256, 0, s>>>(h, y, gate, gain, eps, out);
   return cudaGetLastError();
 }
 

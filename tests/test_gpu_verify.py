@@ -38,23 +38,38 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
     eng.verify_step(slots, cand_d, vt, acc)
     eng.sync()
     T = B * (K + 1)
+    R = K + 1
     b_gpu = eng.read_workspace(F.WS_B, (T, shape.hidden), torch.bfloat16)
-    assert rel_err(b_gpu, ref.b.reshape(T, -1)) < REL_TOL
-
     ridx = eng.read_workspace(F.WS_ROUTE_IDX, (shape.n_layers, eng.max_batch * (eng.K_max + 1), shape.top_k),
                               torch.int32)
+    # Routing: bit-exact wherever the oracle's 6th/7th probability margin exceeds 1e-3.  A row
+    # whose expert set differs below the margin (a legitimate near-tie) leaves the comparison of
+    # hidden states from then on, together with the later candidates of its sequence (they
+    # attend to its K/V); such rows are counted.
+    diverged = np.zeros(T, dtype=bool)
     for l in range(shape.n_layers):
-        g = ridx[l, :T].numpy()
-        r = ref.route_idx[l].numpy()
-        n_ok, n_skip, n_bad = index_parity(np.sort(g, -1), np.sort(r, -1), ref.route_gap[l].numpy())
+        g = np.sort(ridx[l, :T].numpy(), -1)
+        r = np.sort(ref.route_idx[l].numpy(), -1)
+        live = ~diverged
+        n_ok, n_skip, n_bad = index_parity(g[live], r[live], ref.route_gap[l].numpy()[live])
         assert n_bad == 0, f"layer {l}: {n_bad} router mismatches over {n_ok} rows"
+        differ = (g != r).any(-1) & ~diverged
+        for row in np.nonzero(differ)[0]:
+            seq = row // R
+            diverged[row:(seq + 1) * R] = True
+    keep = ~diverged
+    errs = [rel_err(b_gpu[i], ref.b.reshape(T, -1)[i]) for i in range(T)]
+    assert keep.sum() >= T // 2, f"only {keep.sum()} of {T} rows comparable"
+    assert max(e for e, k in zip(errs, keep) if k) < REL_TOL, (
+        f"b rel err per row {['%.3g' % e for e in errs]}, diverged rows {np.nonzero(diverged)[0].tolist()}")
 
-    v_ok, v_skip, v_bad = index_parity(vt.cpu().numpy().reshape(-1), ref.v.numpy().reshape(-1),
-                                       ref.v_gap.numpy().reshape(-1))
+    v_ok, v_skip, v_bad = index_parity(vt.cpu().numpy().reshape(-1)[keep], ref.v.numpy().reshape(-1)[keep],
+                                       ref.v_gap.numpy().reshape(-1)[keep])
     assert v_bad == 0
-    for b in range(B):
-        if all(ref.v_gap[b, : K].numpy() > GAP):
-            assert int(acc[b]) == ref.m[b]
+    for bb in range(B):
+        rows = slice(bb * R, bb * R + K)
+        if keep[rows].all() and all(ref.v_gap[bb, :K].numpy() > GAP):
+            assert int(acc[bb]) == ref.m[bb]
 
     committed = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
     ncom = torch.empty(B, dtype=torch.int32, device=dev)
@@ -69,8 +84,12 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
         ln, pending = eng.seq_state(b)
         assert ln == ctx_lens[b] + m + 1 and pending == int(vt[b, m])
         bt = eng.block_table(b)
+        if m != ref.m[b]:
+            continue
         for l in range(shape.n_layers):
             for r in range(m + 1):
+                if diverged[b * R + r]:
+                    continue
                 p = ctx_lens[b] + r
                 page, off = bt[p // ps], p % ps
                 k_gpu = eng.kv_pool[l, page, 0, :, off, :].cpu()
