@@ -27,21 +27,51 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_b
                : "memory");
 }
 
-// Softmax-weighted combination of the chunks 0..lastc of one query, in chunk order.
-__device__ __forceinline__ void merge_query(const AttnArgs& a, int b, int h, int r, int lastc, int R) {
+// Merge of the chunks of every query of (sequence b, head h), run by the last chunk CTA:
+// query r combines chunks 0..floor(p_r/128) in chunk order, O = sum_c w_c acc_c / sum_c w_c l_c
+// with w_c = 2^(m_c - max_c m_c).  The (m, l) pairs are staged in shared memory by all threads
+// at once; the accumulator loads of the weighted sum are independent of each other.
+__device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R, int p0, int n_live, float* smem) {
   const float* part = a.part + (static_cast<size_t>(b) * kH + h) * a.n_chunks * R * (kHD + 2);
-  float M = -INFINITY;
-  for (int c = 0; c <= lastc; ++c) M = fmaxf(M, __ldcg(&part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + kHD]));
-  float L = 0.f, O = 0.f;
-  for (int c = 0; c <= lastc; ++c) {
-    const float* pc = part + (static_cast<size_t>(c) * R + r) * (kHD + 2);
-    const float mc = __ldcg(&pc[kHD]);
-    const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
-    L += __ldcg(&pc[kHD + 1]) * w;
-    O += __ldcg(&pc[threadIdx.x]) * w;
+  float* sm = smem;                      // [n_live * R] chunk max, then weight
+  float* sl = smem + n_live * R;         // [n_live * R] chunk sum
+  float* sL = sl + n_live * R;           // [R] total weight
+  for (int i = threadIdx.x; i < n_live * R; i += blockDim.x) {
+    const float* pc = part + static_cast<size_t>(i) * (kHD + 2);
+    sm[i] = __ldcg(&pc[kHD]);
+    sl[i] = __ldcg(&pc[kHD + 1]);
   }
-  a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + threadIdx.x] =
-      __float2bfloat16(O / L);
+  __syncthreads();
+  if (threadIdx.x < R) {
+    const int r = threadIdx.x, lastc = (p0 + r) / kCH;
+    float M = -INFINITY;
+    for (int c = 0; c <= lastc; ++c) M = fmaxf(M, sm[c * R + r]);
+    float L = 0.f;
+    for (int c = 0; c <= lastc; ++c) {
+      const float mc = sm[c * R + r];
+      const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
+      sm[c * R + r] = w;
+      L += sl[c * R + r] * w;
+    }
+    sL[r] = L;
+  }
+  __syncthreads();
+  const int d = threadIdx.x;
+  for (int r = 0; r < R; ++r) {
+    const int lastc = (p0 + r) / kCH;
+    float O = 0.f;
+    int c = 0;
+    for (; c + 4 <= lastc + 1; c += 4) {
+      float x[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) x[u] = __ldcg(&part[(static_cast<size_t>(c + u) * R + r) * (kHD + 2) + d]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) O += x[u] * sm[(c + u) * R + r];
+    }
+    for (; c <= lastc; ++c) O += __ldcg(&part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + d]) * sm[c * R + r];
+    a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d] =
+        __float2bfloat16(O / sL[r]);
+  }
 }
 
 __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
@@ -209,7 +239,7 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   __syncthreads();
   if (s_last) {
     __threadfence();
-    for (int r = 0; r < R; ++r) merge_query(a, b, h, r, (p0 + r) / kCH, R);
+    merge_all(a, b, h, R, p0, n_live, reinterpret_cast<float*>(asmem));   // K/V tiles are no longer needed
   }
 }
 

@@ -195,6 +195,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(fin + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   int* s_vote = const_cast<int*>(s_abort) + 1;   // [4]
+  int* s_last = s_vote + 4;
   float* xchg = reinterpret_cast<float*>(smem + C::STAGES * (C::A_BYTES + C::B_BYTES) + 256);
   float* am_s_val = xchg + C::XCHG_FLOATS;
   int* am_s_idx = reinterpret_cast<int*>(am_s_val + 64);
@@ -369,21 +370,62 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
       } else {
-        // split-K: raw fp32 partials; splitk_reduce_kernel sums them in split order and runs
-        // the epilogue
-        const int n = it.n_tile * 128 + row;
+        // split-K: each split writes its fp32 partial tile thread-major (a thread's 16 values
+        // of a chunk are 64 contiguous bytes); the last split of the tile to arrive (atomic
+        // ticket, no wait) sums the partials in split order and runs the epilogue.
+        const int box = 16 << it.box_log;
+        const int tile = it.n_tile * a.m_tiles + it.out_row / box;
+        const size_t tstride = static_cast<size_t>(box / 16) * 128 * 16;    // floats per split of a tile
+        float* mine = a.sk_ws + (static_cast<size_t>(tile) * a.split_k + it.split) * tstride;
         for (int c = 0; c < nchunks; ++c) {
           tc_ld16(tb + c * 16, v);
+          float4* dst = reinterpret_cast<float4*>(mine + (static_cast<size_t>(c) * 128 + row) * 16);
 #pragma unroll
-          for (int jj = 0; jj < 16; ++jj) {
-            const int r = c * 16 + jj;
-            if (r < it.rows && n < a.N)
-              a.sk_ws[(static_cast<size_t>(it.split) * a.sk_rows + it.out_row + r) * a.N + n] = v[jj];
-          }
+          for (int q4 = 0; q4 < 4; ++q4) dst[q4] = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (threadIdx.x == 64) {
+          const int old = atomicAdd(&a.sk_tickets[tile], 1);
+          *s_last = (old == a.split_k - 1) ? 1 : 0;
+          if (old == a.split_k - 1) a.sk_tickets[tile] = 0;
+        }
+        named_bar_sync(1, 128);
+        if (*s_last) {
+          __threadfence();
+          const float* base = a.sk_ws + static_cast<size_t>(tile) * a.split_k * tstride;
+          for (int c = 0; c < nchunks; ++c) {
+            float4 p[kMaxSplit][4];
+#pragma unroll
+            for (int sp = 0; sp < kMaxSplit; ++sp)
+              if (sp < a.split_k) {
+                const float4* src =
+                    reinterpret_cast<const float4*>(base + sp * tstride + (static_cast<size_t>(c) * 128 + row) * 16);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) p[sp][q4] = __ldcg(src + q4);
+              }
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+              float4 t = p[0][q4];
+#pragma unroll
+              for (int sp = 1; sp < kMaxSplit; ++sp)
+                if (sp < a.split_k) {
+                  t.x += p[sp][q4].x;
+                  t.y += p[sp][q4].y;
+                  t.z += p[sp][q4].z;
+                  t.w += p[sp][q4].w;
+                }
+              v[4 * q4] = t.x;
+              v[4 * q4 + 1] = t.y;
+              v[4 * q4 + 2] = t.z;
+              v[4 * q4 + 3] = t.w;
+            }
+            epi_chunk<EPI>(a, it, row, c * 16, v, xchg, am_s_val, am_s_idx);
+          }
+        }
       }
     }
   }
@@ -394,54 +436,6 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem_base, C::TMEM_COLS);
-  }
-}
-
-// ------------------------------------------------------------------ split-K reduction
-// One thread per output element (row r, feature n): the fp32 sum of the split partials in
-// split order, then the same epilogue arithmetic as the unsplit path.  RoPE and SwiGLU read
-// their partner rows (n ^ 64, n + 64) from the partials directly.
-__device__ __forceinline__ float sk_sum(const GemmArgs& a, int r, int n) {
-  float s = 0.f;
-  for (int sp = 0; sp < a.split_k; ++sp) s += a.sk_ws[(static_cast<size_t>(sp) * a.sk_rows + r) * a.N + n];
-  return s;
-}
-
-template <int EPI>
-__global__ void __launch_bounds__(256) splitk_reduce_kernel(const __grid_constant__ GemmArgs a) {
-  const int n = blockIdx.x * 256 + threadIdx.x;
-  const int r = blockIdx.y;
-  if (n >= a.N || r >= a.M) return;
-  if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
-    const float v = sk_sum(a, r, n);
-    float* p = a.out + static_cast<size_t>(r) * a.ldo + n;
-    if constexpr (EPI == EPI_RESID) *p += v;
-    else *p = v;
-  } else if constexpr (EPI == EPI_QKV) {
-    const int which = n / (kH * kHD), head = (n / kHD) % kH, i = n % kHD;
-    float val = sk_sum(a, r, n);
-    if (which < 2) {
-      const float partner = sk_sum(a, r, n ^ 64);
-      int p = a.pos[r];
-      if (p < 0 || p >= a.max_pos) {
-        atomicOr(a.err, ERR_POSITION);
-        p = 0;
-      }
-      const float2 cs = a.rope[static_cast<size_t>(p) * (kHD / 2) + (i & 63)];
-      val = (i < 64) ? (val * cs.x - partner * cs.y) : (val * cs.x + partner * cs.y);
-    }
-    if (which == 0) {
-      a.q_out[static_cast<size_t>(r) * (kH * kHD) + head * kHD + i] = val;
-    } else {
-      const long long off = a.kv_rowoff[r];
-      if (off >= 0) a.kv_base[off + (which == 2 ? a.v_off : 0) + head * a.head_stride + i] = __float2bfloat16(val);
-    }
-  } else if constexpr (EPI == EPI_SWIGLU) {
-    const int tile = n / 128, i = n % 128;
-    if (i < 64) {
-      const float g = sk_sum(a, r, n), u = sk_sum(a, r, n + 64);
-      a.act[static_cast<size_t>(r) * a.ld_act + tile * 64 + i] = __float2bfloat16(silu_f(g) * u);
-    }
   }
 }
 
@@ -549,34 +543,18 @@ int num_sms() {
 }
 
 int dense_split_k(int N, int K) {
+  // about 64 CTAs per dense matrix, at least 4 k-chunks (32 KB of weights) per split
   const int n_tiles = (N + 127) / 128;
   const int kc = K / 64;
-  int s = (148 + n_tiles - 1) / n_tiles;
-  if (s > kc) s = kc;
+  int s = (64 + n_tiles - 1) / n_tiles;
+  if (s > kc / 4) s = kc / 4;
+  if (s > kMaxSplit) s = kMaxSplit;
   if (s < 1) s = 1;
   return s;
 }
 
-template <int EPI>
-cudaError_t reduce_one(const GemmArgs& a, cudaStream_t s) {
-  splitk_reduce_kernel<EPI><<<dim3((a.N + 255) / 256, a.M), 256, 0, s>>>(a);
-  return cudaGetLastError();
-}
-
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s) {
   if (grid <= 0) return cudaSuccess;
-  if (a.split_k > 1) {
-    // the GEMM writes raw partials (epilogue-independent); the reduction applies the epilogue
-    cudaError_t e = nmax <= 64 ? launch_one<64, EPI_F32>(a, grid, s) : launch_one<256, EPI_F32>(a, grid, s);
-    if (e != cudaSuccess) return e;
-    switch (epi) {
-      case EPI_F32: return reduce_one<EPI_F32>(a, s);
-      case EPI_RESID: return reduce_one<EPI_RESID>(a, s);
-      case EPI_QKV: return reduce_one<EPI_QKV>(a, s);
-      case EPI_SWIGLU: return reduce_one<EPI_SWIGLU>(a, s);
-      default: return cudaErrorInvalidValue;
-    }
-  }
 #define FM_CASE(E)                                                                      \
   case E:                                                                               \
     return nmax <= 64 ? launch_one<64, E>(a, grid, s) : launch_one<256, E>(a, grid, s);

@@ -25,6 +25,7 @@ constexpr int kId = 3584;       // draft-block intermediate
 constexpr int kSlots = kTopK + kShared;   // per-token expert outputs combined
 constexpr int kAttnChunk = 128;           // split-KV chunk (keys), fixed by absolute position
 constexpr int kMaxR = 8;                  // K_max + 1 <= 8 candidate rows per sequence
+constexpr int kMaxSplit = 6;              // split-K ways of a dense GEMM
 
 // ------------------------------------------------------------------------- GEMM engine
 enum EpiKind : int {
@@ -63,7 +64,7 @@ struct GemmArgs {
   bf16* act; int ld_act;                                      // SWIGLU
   float* y; const int* sorted_tok; const int* sorted_slot;    // SCATTER
   float* am_val; int* am_idx; int am_ld;                      // ARGMAX partials [n_tile][am_ld]
-  float* sk_ws; int sk_rows;                                  // split-K partials [split][sk_rows][N]
+  float* sk_ws; int* sk_tickets;                              // split-K partials / per-tile tickets
   int* err;
 };
 
@@ -75,8 +76,7 @@ bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t ro
 // Fills b_map[src][*] for an activation buffer of `rows` x `inner` bf16.
 bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err);
 
-// Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).  With
-// split_k > 1 (dense only) it writes partials and a reduction kernel applies the epilogue.
+// Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s);
 int num_sms();
 // Kernel attributes (dynamic shared memory limits) set once, before any launch or capture.

@@ -110,6 +110,7 @@ struct spec_ctx {
   bf16* dstage = nullptr;
   int* last_row = nullptr;
   float* sk_ws = nullptr;
+  int* sk_tickets = nullptr;
   float2* rope = nullptr;
   int* d_err = nullptr;
 
@@ -158,7 +159,7 @@ GemmArgs base_args(spec_ctx* ctx) {
   g.rope = ctx->rope;
   g.max_pos = ctx->cfg.max_position;
   g.sk_ws = ctx->sk_ws;
-  g.sk_rows = ctx->Tmax;
+  g.sk_tickets = ctx->sk_tickets;
   g.am_ld = ctx->Tmax;
   g.err = ctx->d_err;
   return g;
@@ -373,16 +374,15 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ctx->dstage_rows = c.K_max > 1 ? c.K_max - 1 : 1;
   ctx->max_items = static_cast<size_t>(kE + kShared + (Tmax * kSlots) / 256 + 4) * (kI / 64);
   {
-    // split-K partials: max over the dense split launches of splits x N (x Tmax rows)
+    // split-K partials: per split, a tile's rows are padded to the row box (< 2 * rows + 16)
     const int shapes[][2] = {{3 * kD, kD}, {kD, kD}, {kD, 2 * kD}, {kD, kId}, {2 * kId, kD}};
     size_t mx = 0;
     for (auto& sh : shapes) {
-      const size_t v = static_cast<size_t>(dense_split_k(sh[0], sh[1])) * sh[0];
+      const size_t v = static_cast<size_t>(dense_split_k(sh[0], sh[1])) * ((sh[0] + 127) / 128) * 128;
       if (v > mx) mx = v;
     }
-    ctx->sk_floats = mx * Tmax + 16;
+    ctx->sk_floats = mx * (2 * static_cast<size_t>(Tmax) + 256) + 16;
   }
-
   // ---- workspace layout
   struct Sub {
     void** p;
@@ -433,6 +433,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->dstage, sizeof(bf16) * Bmax * ctx->dstage_rows * 2 * d);
   add(&ctx->last_row, sizeof(int) * Bmax);
   add(&ctx->sk_ws, sizeof(float) * ctx->sk_floats);
+  add(&ctx->sk_tickets, sizeof(int) * 8192);
   add(&ctx->rope, sizeof(float2) * static_cast<size_t>(c.max_position) * (kHD / 2));
   add(&ctx->d_err, sizeof(int) * 4);
   add(&ctx->d_expert_ctr, sizeof(unsigned long long) * 2);
