@@ -28,8 +28,9 @@ pre-norm attention + SwiGLU block with its own KV cache; argmax ties go to the l
 Precision: every quantity is fp64 computed from the bf16-stored weights and inputs.  With
 `rb=True` ("storage rounding") values are additionally rounded to bf16, in one step and ties
 to even, exactly where the GPU contract stores bf16 (norm outputs that feed a matrix product,
-K/V written to a cache, attention outputs, SwiGLU activations, the states b and u); everything
-between those points stays fp64.  `rb=False` is the plain definition.
+the rotated queries and K/V that feed the attention products, attention outputs, SwiGLU
+activations, the states b and u); everything between those points stays fp64.  `rb=False` is
+the plain definition.
 
 Parity of absolute hidden-state values on random weights is pinned only through the special
 cases and invariants in tests/test_oracle_pins.py (closed forms, brute force, the identity
@@ -282,7 +283,7 @@ def _attn_block(s, h, norm_w, wqkv, wo, seq_rows, keys, vals, pos, rb):
     new_k, new_v = [], []
     for i, rows in enumerate(seq_rows):
         p = torch.as_tensor(pos[i], dtype=F64)
-        qi = rope(q[rows], p, s.rope_theta)
+        qi = _rb(rope(q[rows], p, s.rope_theta), rb)
         ki = _rb(rope(k[rows], p, s.rope_theta), rb)
         vi = _rb(v[rows], rb)
         K_all = torch.cat([keys[i], ki], 0)

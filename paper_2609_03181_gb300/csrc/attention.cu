@@ -5,7 +5,9 @@
 // keys at positions >= ctx_len in a staging buffer (candidates not yet committed).  The key
 // range is cut into chunks of 128 positions fixed by absolute position; one CTA per
 // (chunk, head, sequence) stages the chunk's K and V in shared memory with 16-byte
-// cp.async copies, scores every (query, key) pair in fp32, and writes the chunk's
+// cp.async copies, forms the scores K q^T and the output V^T p^T with bf16 tensor-core
+// MMAs (fp32 accumulation; queries padded to 8; probabilities rounded to bf16 as the MMA
+// operand, their sum taken over the rounded values), and writes the chunk's
 // (max, sum, unnormalised output) per query; the last chunk of a (sequence, head) to finish
 // merges the chunks of each query in chunk order.  Masked keys contribute exact zeros, so a
 // query's result is the same whether its key sits in a page or in staging and however many
@@ -19,7 +21,7 @@
 namespace fm {
 
 constexpr int kCH = kAttnChunk;
-constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 4 + kMaxR * kCH * 4;
+constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 2 + kMaxR * kCH * 2 + kMaxR * kCH * 4;
 constexpr long long kStagedBit = 1ll << 62;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
@@ -74,13 +76,39 @@ __device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R
   }
 }
 
+// ---- warp-level tensor-core helpers (bf16 m16n8k16, fp32 accumulation)
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t (&r)[2]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+// Byte offset of 16-byte chunk `ch` of row `row` in a tile of 256-byte rows, chunks swizzled
+// by row (conflict-free for ldmatrix and row-wise cp.async).
+__device__ __forceinline__ uint32_t swz(int row, int ch) { return row * 256 + ((ch ^ (row & 7)) << 4); }
+
 __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   extern __shared__ __align__(16) uint8_t asmem[];
-  bf16* sK = reinterpret_cast<bf16*>(asmem);               // [kCH][kHD], 16-byte chunks swizzled by row
-  bf16* sV = sK + kCH * kHD;
-  float* sq = reinterpret_cast<float*>(sV + kCH * kHD);    // [R][kHD]
-  float* sp = sq + kMaxR * kHD;                           // [R][kCH] scores, then probabilities
-  __shared__ long long s_base[kCH];                       // element offset of each key row (-1: none)
+  uint8_t* sK = asmem;                                   // [128 keys][128 dims] bf16
+  uint8_t* sV = sK + kCH * kHD * 2;                      // [128 keys][128 dims] bf16
+  uint8_t* sQ = sV + kCH * kHD * 2;                      // [8 queries][128 dims] bf16
+  uint8_t* sP = sQ + kMaxR * kHD * 2;                    // [8 queries][128 keys] bf16 probabilities
+  float* sS = reinterpret_cast<float*>(sP + kMaxR * kCH * 2);   // [8][128] fp32 scores
+  __shared__ long long s_base[kCH];                      // element offset of each key row (-1: none)
   __shared__ int s_last;
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -92,7 +120,7 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   const int start = c * kCH;
   if (start > last || p0 < 0) return;
   const int nk = min(kCH, last + 1 - start);
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
   // where each key row lives: a page of the pool (positions < ctx_len) or a staging row
   {
@@ -128,7 +156,7 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
       src = ((off & kStagedBit) ? a.stage + (off & (kStagedBit - 1)) : a.pool + off) + ch * 8;
       bytes = 16;
     }
-    cp_async16(sK + j * kHD + ((ch ^ (j & 7)) * 8), src, bytes);
+    cp_async16(sK + swz(j, ch), src, bytes);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
 #pragma unroll 4
@@ -142,88 +170,101 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
             ch * 8;
       bytes = 16;
     }
-    cp_async16(sV + j * kHD + ((ch ^ (j & 7)) * 8), src, bytes);
+    cp_async16(sV + swz(j, ch), src, bytes);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
 
-  // queries, pre-scaled by log2(e) / sqrt(hd) so that softmax uses exp2
-  const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));
+  // queries (bf16, as the QKV epilogue stored them); rows R..7 are zero
   const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
-  for (int v = tid; v < R * kHD; v += 128) {
-    const int r = v / kHD, d = v % kHD;
-    sq[v] = a.q[(static_cast<size_t>(qrow0 + r) * kH + h) * kHD + d] * qscale;
+  {
+    const int q = tid >> 4, ch = tid & 15;   // 8 queries x 16 chunks
+    uint4 val = make_uint4(0, 0, 0, 0);
+    if (q < R) val = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
+    *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = val;
   }
   asm volatile("cp.async.wait_group 1;" ::: "memory");   // K has landed; V may still be in flight
   __syncthreads();
 
-  // scores: thread j owns key j of the chunk
+  const int g = lane >> 2, t4 = lane & 3;
+  const int mi = lane >> 3, ri = lane & 7;
+  // S^T[key][query] = K Q^T: warp w owns keys 32w..32w+31 (two 16-key tiles), 8 k-steps of 16 dims
   {
-    const int j = tid;
-    float s[kMaxR];
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    const uint32_t kbase = smem_u32(sK), qbase = smem_u32(sQ);
 #pragma unroll
-    for (int r = 0; r < kMaxR; ++r) s[r] = 0.f;
-#pragma unroll 4
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 raw = *reinterpret_cast<const uint4*>(sK + j * kHD + ((ch ^ (j & 7)) * 8));
-      const bf16* kv = reinterpret_cast<const bf16*>(&raw);
-      float kf[8];
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t bq[2];
+      ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), bq);
 #pragma unroll
-      for (int u = 0; u < 8; ++u) kf[u] = __bfloat162float(kv[u]);
-#pragma unroll
-      for (int r = 0; r < kMaxR; ++r) {
-        if (r < R) {
-          const float* qr = sq + r * kHD + ch * 8;
-#pragma unroll
-          for (int u = 0; u < 8; ++u) s[r] += qr[u] * kf[u];
-        }
+      for (int mt = 0; mt < 2; ++mt) {
+        uint32_t ak[4];
+        const int key = warp * 32 + mt * 16 + ri + ((mi & 1) ? 8 : 0);
+        ldsm_x4(kbase + swz(key, 2 * ks + (mi >> 1)), ak);
+        mma_bf16_16816(acc[mt], ak, bq);
       }
     }
-    const int pos = start + j;
+    const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));   // log2(e) / sqrt(hd)
 #pragma unroll
-    for (int r = 0; r < kMaxR; ++r)
-      if (r < R) sp[r * kCH + j] = (j < nk && pos <= p0 + r) ? s[r] : -INFINITY;
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = warp * 32 + mt * 16 + g + ((e >> 1) ? 8 : 0);
+        const int q = 2 * t4 + (e & 1);
+        const bool vis = q < R && key < nk && start + key <= p0 + q;
+        sS[q * kCH + key] = vis ? acc[mt][e] * scale : -INFINITY;
+      }
   }
   __syncthreads();
 
-  // per query: chunk max, probabilities (exact zeros where masked), sum
-  const int warp = tid >> 5, lane = tid & 31;
+  // per query: chunk max, probabilities rounded to bf16 (exact zeros where masked), their sum
   float* part = a.part + ((static_cast<size_t>(b) * kH + h) * a.n_chunks + c) * R * (kHD + 2);
-  for (int r = warp; r < R; r += 4) {
+  for (int q = warp; q < kMaxR; q += 4) {
     float x[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) x[i] = sp[r * kCH + lane + 32 * i];
+    for (int i = 0; i < 4; ++i) x[i] = sS[q * kCH + lane + 32 * i];
     const float m = warp_max(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])));
     float l = 0.f;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const float p = (m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m);
-      sp[r * kCH + lane + 32 * i] = p;
-      l += p;
+      const int key = lane + 32 * i;
+      const bf16 pb = __float2bfloat16((m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m));
+      *reinterpret_cast<bf16*>(sP + swz(q, key >> 3) + (key & 7) * 2) = pb;
+      l += __bfloat162float(pb);
     }
     l = warp_sum(l);
-    if (lane == 0) {
-      part[r * (kHD + 2) + kHD] = m;
-      part[r * (kHD + 2) + kHD + 1] = l;
+    if (lane == 0 && q < R) {
+      part[q * (kHD + 2) + kHD] = m;
+      part[q * (kHD + 2) + kHD + 1] = l;
     }
   }
   asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncthreads();
 
-  // P V: thread d owns output dim d
+  // O^T[dim][query] = V^T P^T: warp w owns dims 32w..32w+31, 8 k-steps of 16 keys
   {
-    const int d = tid;
-    float acc[kMaxR];
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    const uint32_t vbase = smem_u32(sV), pbase = smem_u32(sP);
 #pragma unroll
-    for (int r = 0; r < kMaxR; ++r) acc[r] = 0.f;
-    for (int j = 0; j < nk; ++j) {
-      const float vv = __bfloat162float(sV[j * kHD + (((d >> 3) ^ (j & 7)) * 8) + (d & 7)]);
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t bp[2];
+      ldsm_x2(pbase + swz(ri, 2 * ks + (mi & 1)), bp);
 #pragma unroll
-      for (int r = 0; r < kMaxR; ++r)
-        if (r < R) acc[r] += sp[r * kCH + j] * vv;
+      for (int mt = 0; mt < 2; ++mt) {
+        uint32_t av[4];
+        const int key = ks * 16 + ri + ((mi >> 1) ? 8 : 0);
+        const int dch = (warp * 32 + mt * 16) / 8 + (mi & 1);
+        ldsm_x4_t(vbase + swz(key, dch), av);
+        mma_bf16_16816(acc[mt], av, bp);
+      }
     }
 #pragma unroll
-    for (int r = 0; r < kMaxR; ++r)
-      if (r < R) part[r * (kHD + 2) + d] = acc[r];
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int d = warp * 32 + mt * 16 + g + ((e >> 1) ? 8 : 0);
+        const int q = 2 * t4 + (e & 1);
+        if (q < R) part[q * (kHD + 2) + d] = acc[mt][e];
+      }
   }
 
   // the last chunk of (sequence, head) to finish merges every query (atomic ticket, no wait)

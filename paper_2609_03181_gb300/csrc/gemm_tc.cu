@@ -136,7 +136,7 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
         val = (row < 64) ? (v[jj] * cs.x - partner[jj] * cs.y) : (v[jj] * cs.x + partner[jj] * cs.y);
       }
       if (which == 0) {
-        a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + row] = val;
+        a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + row] = __float2bfloat16(val);
       } else {
         const long long off = a.kv_rowoff[m];
         if (off >= 0)

@@ -59,7 +59,7 @@ struct GemmArgs {
   int n_tiles;                 // dense: weight tiles
   // epilogue operands
   float* out; int ldo;                                        // F32 / RESID
-  float* q_out; bf16* kv_base; const long long* kv_rowoff;   // QKV
+  bf16* q_out; bf16* kv_base; const long long* kv_rowoff;    // QKV (q stored bf16)
   long long head_stride, v_off; const int* pos; const float2* rope; int max_pos;
   bf16* act; int ld_act;                                      // SWIGLU
   float* y; const int* sorted_tok; const int* sorted_slot;    // SCATTER
@@ -90,7 +90,7 @@ int dense_split_k(int N, int K);
 
 // ------------------------------------------------------------------------- other kernels
 struct AttnArgs {
-  const float* q;              // [rows][H][hd] fp32
+  const bf16* q;               // [rows][H][hd] bf16
   const int* q_row0;           // per sequence first query row (NULL: b * R)
   int R;                       // queries per sequence
   int qoff;                    // query r of sequence b sits at seq_len[slot] + qoff + r

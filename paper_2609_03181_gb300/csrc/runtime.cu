@@ -70,7 +70,7 @@ struct spec_ctx {
   size_t ws_bytes = 0;
   float* h = nullptr;
   bf16* xn = nullptr;
-  float* q = nullptr;
+  bf16* q = nullptr;
   bf16* stage = nullptr;
   float* attn_part = nullptr;
   int* attn_tickets = nullptr;
@@ -393,7 +393,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   const size_t d = kD;
   add(&ctx->h, sizeof(float) * Tmax * d);
   add(&ctx->xn, sizeof(bf16) * Tmax * d);
-  add(&ctx->q, sizeof(float) * Tmax * d);
+  add(&ctx->q, sizeof(bf16) * Tmax * d);
   add(&ctx->stage, sizeof(bf16) * L * Bmax * Rmax * 2 * d);
   add(&ctx->attn_part, sizeof(float) * static_cast<size_t>(Bmax) * kH * ctx->n_chunks * Rmax * (kHD + 2));
   add(&ctx->attn_tickets, sizeof(int) * Bmax * kH);
