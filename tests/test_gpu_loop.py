@@ -99,18 +99,23 @@ def test_speculative_with_draft_head_equals_greedy(setup):
 
 
 def test_greedy_matches_oracle_greedy(setup):
+    """Token i of a stream is compared while every decision leading to it was unique: the
+    oracle's router margins (6th vs 7th expert) and argmax margins of steps 0..i all above 1e-3."""
     reset(setup)
     n = 6
     greedy, _ = run_loop(setup, n, 0)
     model = O.Verifier(setup["vw"])
-    for b in range(2):
+    compared = 0
+    for b in range(B):
         cache = O.SeqCache.from_prefix(setup["kvs"][b], setup["pend"][b])
         for i in range(n):
             vo = O.verify(model, [cache], [[cache.pending]], rb=True)
-            if float(vo.v_gap[0, 0]) <= GAP:
+            if float(vo.v_gap[0, 0]) <= GAP or min(float(g.min()) for g in vo.route_gap) <= GAP:
                 break
             assert greedy[b][i] == int(vo.v[0, 0]), (b, i)
+            compared += 1
             O.commit([cache], vo, [[cache.pending]])
+    assert compared >= 1
 
 
 def test_batch_invariance_alone_vs_in_batch(setup):
