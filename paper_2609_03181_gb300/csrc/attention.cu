@@ -6,8 +6,8 @@
 // range is cut into chunks of 128 positions fixed by absolute position; one CTA per
 // (chunk, head, sequence) stages the chunk's K and V in shared memory with 16-byte
 // cp.async copies, forms the scores K q^T and the output V^T p^T with bf16 tensor-core
-// MMAs (fp32 accumulation; queries padded to 8; probabilities rounded to bf16 as the MMA
-// operand, their sum taken over the rounded values), and writes the chunk's
+// MMAs (fp32 accumulation; queries padded to 8; the probabilities enter as a sum of two bf16
+// terms, so the product keeps about 16 bits of them), and writes the chunk's
 // (max, sum, unnormalised output) per query; the last chunk of a (sequence, head) to finish
 // merges the chunks of each query in chunk order.  Masked keys contribute exact zeros, so a
 // query's result is the same whether its key sits in a page or in staging and however many
@@ -21,7 +21,7 @@
 namespace fm {
 
 constexpr int kCH = kAttnChunk;
-constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 2 + kMaxR * kCH * 2 + kMaxR * kCH * 4;
+constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 2 + 2 * kMaxR * kCH * 2 + kMaxR * kCH * 4;
 constexpr long long kStagedBit = 1ll << 62;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
@@ -106,8 +106,9 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   uint8_t* sK = asmem;                                   // [128 keys][128 dims] bf16
   uint8_t* sV = sK + kCH * kHD * 2;                      // [128 keys][128 dims] bf16
   uint8_t* sQ = sV + kCH * kHD * 2;                      // [8 queries][128 dims] bf16
-  uint8_t* sP = sQ + kMaxR * kHD * 2;                    // [8 queries][128 keys] bf16 probabilities
-  float* sS = reinterpret_cast<float*>(sP + kMaxR * kCH * 2);   // [8][128] fp32 scores
+  uint8_t* sP = sQ + kMaxR * kHD * 2;                    // [8 queries][128 keys] bf16 p, high part
+  uint8_t* sPl = sP + kMaxR * kCH * 2;                   // [8 queries][128 keys] bf16 p - high part
+  float* sS = reinterpret_cast<float*>(sPl + kMaxR * kCH * 2);  // [8][128] fp32 scores
   __shared__ long long s_base[kCH];                      // element offset of each key row (-1: none)
   __shared__ int s_last;
 
@@ -216,7 +217,8 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   }
   __syncthreads();
 
-  // per query: chunk max, probabilities rounded to bf16 (exact zeros where masked), their sum
+  // per query: chunk max, probabilities (exact zeros where masked) split as p = hi + lo with
+  // hi, lo bf16 (about 16 significant bits for the P V product), and their fp32 sum
   float* part = a.part + ((static_cast<size_t>(b) * kH + h) * a.n_chunks + c) * R * (kHD + 2);
   for (int q = warp; q < kMaxR; q += 4) {
     float x[4];
@@ -227,9 +229,12 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int key = lane + 32 * i;
-      const bf16 pb = __float2bfloat16((m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m));
-      *reinterpret_cast<bf16*>(sP + swz(q, key >> 3) + (key & 7) * 2) = pb;
-      l += __bfloat162float(pb);
+      const float p = (m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m);
+      const bf16 hi = __float2bfloat16(p);
+      const bf16 lo = __float2bfloat16(p - __bfloat162float(hi));
+      *reinterpret_cast<bf16*>(sP + swz(q, key >> 3) + (key & 7) * 2) = hi;
+      *reinterpret_cast<bf16*>(sPl + swz(q, key >> 3) + (key & 7) * 2) = lo;
+      l += p;
     }
     l = warp_sum(l);
     if (lane == 0 && q < R) {
@@ -243,11 +248,12 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   // O^T[dim][query] = V^T P^T: warp w owns dims 32w..32w+31, 8 k-steps of 16 keys
   {
     float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    const uint32_t vbase = smem_u32(sV), pbase = smem_u32(sP);
+    const uint32_t vbase = smem_u32(sV), pbase = smem_u32(sP), plbase = smem_u32(sPl);
 #pragma unroll
     for (int ks = 0; ks < 8; ++ks) {
-      uint32_t bp[2];
+      uint32_t bp[2], bl[2];
       ldsm_x2(pbase + swz(ri, 2 * ks + (mi & 1)), bp);
+      ldsm_x2(plbase + swz(ri, 2 * ks + (mi & 1)), bl);
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt) {
         uint32_t av[4];
@@ -255,6 +261,7 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
         const int dch = (warp * 32 + mt * 16) / 8 + (mi & 1);
         ldsm_x4_t(vbase + swz(key, dch), av);
         mma_bf16_16816(acc[mt], av, bp);
+        mma_bf16_16816(acc[mt], av, bl);
       }
     }
 #pragma unroll
