@@ -64,6 +64,9 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it) {
 
 // ------------------------------------------------------------------ epilogues
 // v: 16 accumulator columns (activation rows j0..j0+15 of the item) of tile row `row`.
+// Every global load a chunk needs is issued before its first store: a store may alias a later
+// load as far as the compiler knows, so interleaving them would serialise one L2 round trip
+// per row.
 template <int EPI>
 __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int row, int j0, float (&v)[16],
                                           float* xchg, float* am_s_val, int* am_s_idx) {
@@ -71,27 +74,32 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
     const int n = it.n_tile * 128 + row;
     if (n < a.N) {
+      float* base = a.out + static_cast<size_t>(it.out_row + j0) * a.ldo + n;
+      if constexpr (EPI == EPI_RESID) {
+        float old[16];
 #pragma unroll
-      for (int jj = 0; jj < 16; ++jj) {
-        const int r = j0 + jj;
-        if (r < it.rows) {
-          float* p = a.out + static_cast<size_t>(it.out_row + r) * a.ldo + n;
-          if constexpr (EPI == EPI_RESID) *p += v[jj];
-          else *p = v[jj];
-        }
+        for (int jj = 0; jj < 16; ++jj) old[jj] = (j0 + jj < it.rows) ? base[static_cast<size_t>(jj) * a.ldo] : 0.f;
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj)
+          if (j0 + jj < it.rows) base[static_cast<size_t>(jj) * a.ldo] = old[jj] + v[jj];
+      } else {
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj)
+          if (j0 + jj < it.rows) base[static_cast<size_t>(jj) * a.ldo] = v[jj];
       }
     }
   } else if constexpr (EPI == EPI_SCATTER) {
     const int n = it.n_tile * 128 + row;
+    int tok[16], slt[16];
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
-      const int r = j0 + jj;
-      if (r < it.rows) {
-        const int m = it.out_row + r;
-        const int t = a.sorted_tok[m], s = a.sorted_slot[m];
-        a.y[(static_cast<size_t>(t) * kSlots + s) * kD + n] = v[jj];
-      }
+      const bool ok = j0 + jj < it.rows;
+      tok[jj] = ok ? a.sorted_tok[it.out_row + j0 + jj] : 0;
+      slt[jj] = ok ? a.sorted_slot[it.out_row + j0 + jj] : 0;
     }
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj)
+      if (j0 + jj < it.rows) a.y[(static_cast<size_t>(tok[jj]) * kSlots + slt[jj]) * kD + n] = v[jj];
   } else if constexpr (EPI == EPI_SWIGLU) {
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
@@ -111,36 +119,46 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
   } else if constexpr (EPI == EPI_QKV) {
     const int which = it.n_tile / kH;   // 0 q, 1 k, 2 v
     const int head = it.n_tile % kH;
-    float partner[16];
+    long long off[16];
+    float2 cs[16];
+    if (which > 0) {
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) off[jj] = (j0 + jj < it.rows) ? a.kv_rowoff[it.out_row + j0 + jj] : -1;
+    }
     if (which < 2) {
+      int p[16];
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) p[jj] = (j0 + jj < it.rows) ? a.pos[it.out_row + j0 + jj] : 0;
+      bool bad = false;
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) {
+        if (p[jj] < 0 || p[jj] >= a.max_pos) {
+          bad = true;
+          p[jj] = 0;
+        }
+        cs[jj] = a.rope[static_cast<size_t>(p[jj]) * (kHD / 2) + (row & 63)];
+      }
+      if (bad) atomicOr(a.err, ERR_POSITION);
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
       named_bar_sync(1, 128);
+      float partner[16];
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) partner[jj] = xchg[(row ^ 64) * 17 + jj];
       named_bar_sync(1, 128);
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj)
+        v[jj] = (row < 64) ? (v[jj] * cs[jj].x - partner[jj] * cs[jj].y) : (v[jj] * cs[jj].x + partner[jj] * cs[jj].y);
     }
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
       const int r = j0 + jj;
       if (r >= it.rows) continue;
       const int m = it.out_row + r;
-      float val = v[jj];
-      if (which < 2) {
-        int p = a.pos[m];
-        if (p < 0 || p >= a.max_pos) {
-          atomicOr(a.err, ERR_POSITION);
-          p = 0;
-        }
-        const float2 cs = a.rope[static_cast<size_t>(p) * (kHD / 2) + (row & 63)];
-        val = (row < 64) ? (v[jj] * cs.x - partner[jj] * cs.y) : (v[jj] * cs.x + partner[jj] * cs.y);
-      }
       if (which == 0) {
-        a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + row] = __float2bfloat16(val);
-      } else {
-        const long long off = a.kv_rowoff[m];
-        if (off >= 0)
-          a.kv_base[off + (which == 2 ? a.v_off : 0) + head * a.head_stride + row] = __float2bfloat16(val);
+        a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + row] = __float2bfloat16(v[jj]);
+      } else if (off[jj] >= 0) {
+        a.kv_base[off[jj] + (which == 2 ? a.v_off : 0) + head * a.head_stride + row] = __float2bfloat16(v[jj]);
       }
     }
   } else if constexpr (EPI == EPI_ARGMAX) {

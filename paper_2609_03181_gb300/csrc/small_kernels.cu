@@ -113,11 +113,19 @@ __global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16*
 #pragma unroll
   for (int k = 0; k < EPT; ++k) v[k] = h[t * kD + threadIdx.x + NT * k];
   bf16* xo = xn + t * kD;
-  norm_row_store_t<NT>(v, gain, eps, xo, red);
+  {
+    float ss = 0.f;
 #pragma unroll
-  for (int k = 0; k < EPT; ++k) {
-    const int i = threadIdx.x + NT * k;
-    xs[i] = __bfloat162float(xo[i]);   // the rounded row, as the experts see it
+    for (int k = 0; k < EPT; ++k) ss += v[k] * v[k];
+    ss = block_sum<NT>(ss, red);
+    const float inv = rsqrtf(ss / kD + eps);
+#pragma unroll
+    for (int k = 0; k < EPT; ++k) {
+      const int i = threadIdx.x + NT * k;
+      const bf16 r = __float2bfloat16(v[k] * inv * __bfloat162float(gain[i]));
+      xo[i] = r;
+      xs[i] = __bfloat162float(r);   // the rounded row, as the experts see it
+    }
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -314,15 +322,16 @@ __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, 
     for (int s = 0; s < kSlots; ++s) ys[k][s] = y[(t * kSlots + s) * kD + threadIdx.x + NT * k];
   float x[EPT];
 #pragma unroll
+  for (int k = 0; k < EPT; ++k) x[k] = h[t * kD + threadIdx.x + NT * k];   // all loads before any store
+#pragma unroll
   for (int k = 0; k < EPT; ++k) {
-    const int i = threadIdx.x + NT * k;
     float acc = 0.f;
 #pragma unroll
     for (int s = 0; s < kTopK; ++s) acc += g[s] * ys[k][s];
     acc += ys[k][kTopK];
     acc += ys[k][kTopK + 1];
-    x[k] = h[t * kD + i] + acc;
-    h[t * kD + i] = x[k];
+    x[k] += acc;
+    h[t * kD + threadIdx.x + NT * k] = x[k];
   }
   norm_row_store_t<NT>(x, gain, eps, out + t * kD, red);
 }
@@ -398,27 +407,38 @@ __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bma
   const int m = m_ws[b];
   const int c = seq_len[slot];
   constexpr int kVec = kHD / 8;   // 16-byte vectors per head row
+  constexpr int kBatch = 8;       // copies whose loads are issued before their stores
   const int total = (m + 1) * L * 2 * kH * kVec;
-  for (int v = threadIdx.x; v < total; v += blockDim.x) {
-    int t = v;
-    const int vec = t % kVec; t /= kVec;
-    const int h = t % kH; t /= kH;
-    const int kv = t % 2; t /= 2;
-    const int l = t % L;
-    const int r = t / L;
-    const int pos = c + r;
-    const int pi = pos / page_size;
-    const int page = (pi < max_pages) ? block_table[slot * max_pages + pi] : -1;
-    if (page < 0 || page >= n_pages) {
-      atomicOr(err, ERR_PAGE_RANGE);
-      continue;
+  for (int v0 = threadIdx.x; v0 < total; v0 += blockDim.x * kBatch) {
+    uint4 val[kBatch];
+    uint4* dst[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      dst[u] = nullptr;
+      const int v = v0 + u * blockDim.x;
+      if (v >= total) continue;
+      int t = v;
+      const int vec = t % kVec; t /= kVec;
+      const int h = t % kH; t /= kH;
+      const int kv = t % 2; t /= 2;
+      const int l = t % L;
+      const int r = t / L;
+      const int pos = c + r;
+      const int pi = pos / page_size;
+      const int page = (pi < max_pages) ? block_table[slot * max_pages + pi] : -1;
+      if (page < 0 || page >= n_pages) {
+        atomicOr(err, ERR_PAGE_RANGE);
+        continue;
+      }
+      val[u] = reinterpret_cast<const uint4*>(
+          stage + ((((static_cast<size_t>(l) * Bmax + b) * stage_R + r) * 2 + kv) * kH + h) * kHD)[vec];
+      dst[u] = reinterpret_cast<uint4*>(
+                   pool + ((((static_cast<size_t>(l) * n_pages + page) * 2 + kv) * kH + h) * page_size + pos % page_size) *
+                              kHD) + vec;
     }
-    const uint4* src = reinterpret_cast<const uint4*>(
-        stage + ((((static_cast<size_t>(l) * Bmax + b) * stage_R + r) * 2 + kv) * kH + h) * kHD) + vec;
-    uint4* dst = reinterpret_cast<uint4*>(
-        pool + ((((static_cast<size_t>(l) * n_pages + page) * 2 + kv) * kH + h) * page_size + pos % page_size) * kHD) +
-        vec;
-    *dst = *src;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u)
+      if (dst[u] != nullptr) *dst[u] = val[u];
   }
   // queue the new rows for the draft head: b_p and x_{p+1}
   for (int v = threadIdx.x; v < (m + 1) * (kD / 8); v += blockDim.x) {
