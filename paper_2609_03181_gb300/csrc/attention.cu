@@ -111,6 +111,8 @@ __global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
   float* sS = reinterpret_cast<float*>(sPl + kMaxR * kCH * 2);  // [8][128] fp32 scores
   __shared__ long long s_base[kCH];                      // element offset of each key row (-1: none)
   __shared__ int s_last;
+  pdl_trigger();
+  pdl_wait();
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int R = a.R;
@@ -296,8 +298,7 @@ cudaError_t attention_prepare() {
 }
 
 cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s) {
-  attn_chunk_kernel<<<dim3(a.n_chunks, kH, B), 128, kAttnSmem, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(attn_chunk_kernel, dim3(a.n_chunks, kH, B), dim3(128), kAttnSmem, s, a);
 }
 
 }  // namespace fm

@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  pdl_trigger();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -247,7 +248,12 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
 
-  const int n_items = (a.items != nullptr) ? *a.n_items_dev : a.n_items;
+  // Dense launches know their items from the arguments: the producer streams its first weight
+  // tiles (never written by earlier kernels) before it waits for the previous kernel; every
+  // other thread waits before its first global access.
+  const bool dense = (a.items == nullptr);
+  if (!(dense && warp == 0 && lane == 0)) pdl_wait();
+  const int n_items = dense ? a.n_items : *a.n_items_dev;
   const int kc_total = a.K / 64;
 
   if (warp == 0) {
@@ -257,6 +263,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       const uint64_t pol_x = l2_policy_evict_last();
       uint32_t g = 0;   // loads issued
       bool failed = false;
+      bool waited = !dense;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x) {
         Item it;
         get_item(a, i, it);
@@ -266,14 +273,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         const CUtensorMap* bmap = &a.b_map[src][it.box_log];
         const uint32_t bytes = C::A_BYTES + (16u << it.box_log) * 128u;
         const int kc0 = it.split * kc_total / a.split_k, kc1 = (it.split + 1) * kc_total / a.split_k;
-        for (int kc = kc0; kc < kc1; ++kc, ++g) {
-          const int st = g % C::STAGES;
-          const uint32_t ph = (g / C::STAGES) & 1u;
-          if (!mbar_wait(&empty[st], ph ^ 1u, s_abort)) {
-            failed = true;
-            break;
-          }
-          mbar_arrive_expect_tx(&full[st], bytes);
+        auto load_a = [&](int st, int kc) {
           uint8_t* sa = smA + st * C::A_BYTES;
           const int k = kc * 64;
           if (a.paired) {
@@ -290,9 +290,35 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
             if (a.a3d) tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
             else tma_load_2d(sa, amap, &full[st], k, r0, pol_w);
           }
-          tma_load_2d(smB + st * C::B_BYTES, bmap, &full[st], k, it.b_row, pol_x);
+        };
+        int kc = kc0;
+        if (!waited) {
+          // first item: the stages are all free (g == 0); weights first, activations after the wait
+          const int npre = min(C::STAGES, kc1 - kc0);
+          for (int q = 0; q < npre; ++q) {
+            mbar_arrive_expect_tx(&full[q], bytes);
+            load_a(q, kc0 + q);
+          }
+          pdl_wait();
+          waited = true;
+          for (int q = 0; q < npre; ++q)
+            tma_load_2d(smB + q * C::B_BYTES, bmap, &full[q], (kc0 + q) * 64, it.b_row, pol_x);
+          g = npre;
+          kc = kc0 + npre;
+        }
+        for (; kc < kc1; ++kc, ++g) {
+          const int st = g % C::STAGES;
+          const uint32_t ph = (g / C::STAGES) & 1u;
+          if (!mbar_wait(&empty[st], ph ^ 1u, s_abort)) {
+            failed = true;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[st], bytes);
+          load_a(st, kc);
+          tma_load_2d(smB + st * C::B_BYTES, bmap, &full[st], kc * 64, it.b_row, pol_x);
         }
       }
+      if (!waited) pdl_wait();
       if (failed) {
         *s_abort = 1;
         atomicOr(a.err, ERR_WAIT_TIMEOUT);
@@ -479,9 +505,8 @@ cudaError_t set_smem_attr() {
 }
 
 template <int NMAX, int EPI>
-cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s) {
-  gemm_tc_kernel<NMAX, EPI><<<grid, 192, Cfg<NMAX>::SMEM_BYTES, s>>>(a);
-  return cudaGetLastError();
+cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
+  return launch_k(pdl, gemm_tc_kernel<NMAX, EPI>, dim3(grid), dim3(192), Cfg<NMAX>::SMEM_BYTES, s, a);
 }
 }  // namespace
 
@@ -571,11 +596,11 @@ int dense_split_k(int N, int K) {
   return s;
 }
 
-cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s) {
+cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   if (grid <= 0) return cudaSuccess;
 #define FM_CASE(E)                                                                      \
   case E:                                                                               \
-    return nmax <= 64 ? launch_one<64, E>(a, grid, s) : launch_one<256, E>(a, grid, s);
+    return nmax <= 64 ? launch_one<64, E>(a, grid, s, pdl) : launch_one<256, E>(a, grid, s, pdl);
   switch (epi) {
     FM_CASE(EPI_F32)
     FM_CASE(EPI_RESID)

@@ -8,8 +8,33 @@
 #include <stdint.h>
 
 #include <string>
+#include <utility>
 
 namespace fm {
+
+// Launches `kernel` with programmatic stream serialization: it may start while the previous
+// kernel of the stream finishes; the kernel itself waits (griddepcontrol.wait) before it
+// touches memory that earlier kernels write.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  return launch_k(true, kernel, grid, block, smem, s, std::forward<Args>(args)...);
+}
 
 typedef __nv_bfloat16 bf16;
 
@@ -77,7 +102,9 @@ bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t ro
 bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err);
 
 // Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).
-cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s);
+// pdl = false launches without programmatic serialization (for streams whose earlier kernels
+// may still be writing the weights).
+cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl = true);
 int num_sms();
 // Kernel attributes (dynamic shared memory limits) set once, before any launch or capture.
 cudaError_t gemm_prepare();

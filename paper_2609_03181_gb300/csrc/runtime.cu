@@ -996,6 +996,6 @@ extern "C" spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, in
   g.out = Y;
   g.ldo = N;
   const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
-  CK(gemm_launch(EPI_F32, box <= 64 ? 64 : 256, g, grid, static_cast<cudaStream_t>(stream)));
+  CK(gemm_launch(EPI_F32, box <= 64 ? 64 : 256, g, grid, static_cast<cudaStream_t>(stream), false));
   return SPEC_OK;
 }

@@ -50,6 +50,8 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
                                                          const int* seq_len, const bf16* embed, int vocab,
                                                          const bf16* gain, float eps, float* h, bf16* xn, int* pos,
                                                          long long* kv_rowoff, int stage_R, int* err) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[4];
   const int row = blockIdx.x, b = row / R, r = row % R;
   const int slot = slots[b];
@@ -78,13 +80,14 @@ cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, c
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int* err,
                               cudaStream_t s) {
-  embed_norm_kernel<<<B * R, 128, 0, s>>>(cand, R, slots, pending, seq_len, embed, vocab, gain, eps, h, xn, pos,
+  return launch_pdl(embed_norm_kernel, dim3(B * R), dim3(128), 0, s, cand, R, slots, pending, seq_len, embed, vocab, gain, eps, h, xn, pos,
                                            kv_rowoff, stage_R, err);
-  return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- RMSNorm
 __global__ void __launch_bounds__(128) rmsnorm_kernel(const float* x, const bf16* gain, float eps, bf16* out) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[4];
   const size_t row = blockIdx.x;
   float v[10];
@@ -95,8 +98,7 @@ __global__ void __launch_bounds__(128) rmsnorm_kernel(const float* x, const bf16
 
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  rmsnorm_kernel<<<rows, 128, 0, s>>>(x, gain, eps, out);
-  return cudaGetLastError();
+  return launch_pdl(rmsnorm_kernel, dim3(rows), dim3(128), 0, s, x, gain, eps, out);
 }
 
 // ---------------------------------------------------------------- router
@@ -104,6 +106,8 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
 // experts from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).
 __global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16* gain, float eps, const bf16* wr,
                                                      const float* bias, bf16* xn, int* idx, float* gate) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int NT = 256, EPT = kD / NT;
   __shared__ float red[NT / 32];
   __shared__ __align__(16) float xs[kD];
@@ -177,8 +181,7 @@ __global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16*
 
 cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
                           const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s) {
-  router_kernel<<<T, 256, 0, s>>>(h, gain, eps, w_router, bias, xn, idx, gate);
-  return cudaGetLastError();
+  return launch_pdl(router_kernel, dim3(T), dim3(256), 0, s, h, gain, eps, w_router, bias, xn, idx, gate);
 }
 
 // ---------------------------------------------------------------- permute / scatter
@@ -195,6 +198,8 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, i
                                                                int* sorted_tok, int* sorted_slot, int4* items_gu,
                                                                int4* items_dn, int* n_items, int* counts,
                                                                unsigned long long* expert_ctr) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ int psm[];
   const int W = (T + 31) / 32;
   int* s_idx = psm;                       // [T*6]
@@ -300,15 +305,16 @@ cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted
   int grid = (pairs + 7) / 8;     // one warp per (token, slot) row copy
   if (grid > 512) grid = 512;
   if (grid < 1) grid = 1;
-  permute_kernel<<<grid, kPermThreads, smem, s>>>(idx, T, xn, x_sorted, sorted_tok, sorted_slot, items_gu, items_dn,
+  return launch_pdl(permute_kernel, dim3(grid), dim3(kPermThreads), smem, s, idx, T, xn, x_sorted, sorted_tok, sorted_slot, items_gu, items_dn,
                                                   n_items, counts, expert_ctr);
-  return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- combine
 // h += sum_{s<6} gate_s * y_s + y_shared0 + y_shared1 (fixed slot order), then RMSNorm -> out.
 __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, const float* gate, const bf16* gain,
                                                       float eps, bf16* out) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int NT = 256, EPT = kD / NT;
   __shared__ float red[NT / 32];
   const size_t t = blockIdx.x;
@@ -338,8 +344,7 @@ __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, 
 
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
                            bf16* out, cudaStream_t s) {
-  combine_kernel<<<T, 256, 0, s>>>(h, y, gate, gain, eps, out);
-  return cudaGetLastError();
+  return launch_pdl(combine_kernel, dim3(T), dim3(256), 0, s, h, y, gate, gain, eps, out);
 }
 
 // ---------------------------------------------------------------- argmax + greedy accept
@@ -361,6 +366,8 @@ __device__ __forceinline__ void reduce_partials(const float* am_val, const int* 
 
 __global__ void argmax_accept_kernel(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int R,
                                      const int* cand, int* vtok_out, int* accept_out, int* m_ws, int* vtok_ws) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ int sv[kMaxR];
   const int b = blockIdx.x, r = threadIdx.x >> 5;
   float bv;
@@ -387,9 +394,8 @@ cudaError_t argmax_final_launch(int mode, const float* am_val, const int* am_idx
                                 int R, const int* cand, int* vtok_out, int* accept_out, int* m_ws, int* vtok_ws,
                                 cudaStream_t s) {
   (void)mode;
-  argmax_accept_kernel<<<B, 32 * R, 0, s>>>(am_val, am_idx, n_tiles, am_ld, R, cand, vtok_out, accept_out, m_ws,
+  return launch_pdl(argmax_accept_kernel, dim3(B), dim3(32 * R), 0, s, am_val, am_idx, n_tiles, am_ld, R, cand, vtok_out, accept_out, m_ws,
                                              vtok_ws);
-  return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- KV commit
@@ -403,6 +409,8 @@ __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bma
                                                      int max_pages, int* seq_len, int* pending, const bf16* b_ws,
                                                      bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
                                                      int* n_committed, int* err) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x, slot = slots[b];
   const int m = m_ws[b];
   const int c = seq_len[slot];
@@ -466,10 +474,9 @@ cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots,
                           int page_size, const int* block_table, int max_pages, int* seq_len, int* pending,
                           const bf16* b_ws, bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
                           int* n_committed, int* err, cudaStream_t s) {
-  commit_kernel<<<B, 256, 0, s>>>(R, stage_R, Bmax, slots, m_ws, vtok_ws, cand_ws, stage, pool, L,
+  return launch_pdl(commit_kernel, dim3(B), dim3(256), 0, s, R, stage_R, Bmax, slots, m_ws, vtok_ws, cand_ws, stage, pool, L,
                                    n_pages, page_size, block_table, max_pages, seq_len, pending, b_ws, draft_b,
                                    draft_tok, draft_n, committed, n_committed, err);
-  return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- draft glue
@@ -483,6 +490,8 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
                                                          int* pos, long long* kv_rowoff, int* last_row, int page_size,
                                                          const int* block_table, int max_pages, int n_pages, int* cand,
                                                          int cand_ld, int* err) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[4];
   const int b = blockIdx.x / R, i = blockIdx.x % R, row = blockIdx.x;
   const int slot = slots[b];
@@ -536,13 +545,14 @@ cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len
                               int vocab, const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
                               long long* kv_rowoff, int* last_row, int page_size, const int* block_table,
                               int max_pages, int n_pages, int* cand, int cand_ld, int* err, cudaStream_t s) {
-  draft_prep_kernel<<<B * R, 128, 0, s>>>(R, slots, seq_len, pending, draft_n, draft_b, draft_tok, embed, vocab,
+  return launch_pdl(draft_prep_kernel, dim3(B * R), dim3(128), 0, s, R, slots, seq_len, pending, draft_n, draft_b, draft_tok, embed, vocab,
                                            enorm, hnorm, eps, dcat, pos, kv_rowoff, last_row, page_size, block_table,
                                            max_pages, n_pages, cand, cand_ld, err);
-  return cudaGetLastError();
 }
 
 __global__ void gather_rows_kernel(const float* src, const int* rows, float* dst) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const float4* s = reinterpret_cast<const float4*>(src + static_cast<size_t>(rows[b]) * kD);
   float4* d = reinterpret_cast<float4*>(dst + static_cast<size_t>(b) * kD);
@@ -550,8 +560,7 @@ __global__ void gather_rows_kernel(const float* src, const int* rows, float* dst
 }
 
 cudaError_t gather_rows_launch(const float* src, const int* rows, int B, float* dst, cudaStream_t s) {
-  gather_rows_kernel<<<B, 128, 0, s>>>(src, rows, dst);
-  return cudaGetLastError();
+  return launch_pdl(gather_rows_kernel, dim3(B), dim3(128), 0, s, src, rows, dst);
 }
 
 // After the LM head of depth k: x^_k = argmax; for k < K the inputs of depth k+1:
@@ -563,6 +572,8 @@ __global__ void __launch_bounds__(128) draft_next_kernel(const float* am_val, co
                                                          const bf16* hnorm, float eps, bf16* dcat, int* pos,
                                                          long long* kv_rowoff, long long dstage_seq_stride, int* cand,
                                                          int cand_ld) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[4];
   __shared__ int s_tok;
   const int b = blockIdx.x;
@@ -597,9 +608,8 @@ cudaError_t draft_next_launch(const float* am_val, const int* am_idx, int n_tile
                               const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
                               long long* kv_rowoff, long long dstage_seq_stride, int* cand, int cand_ld,
                               cudaStream_t s) {
-  draft_next_kernel<<<B, 128, 0, s>>>(am_val, am_idx, n_tiles, am_ld, k, K, slots, seq_len, u, embed, enorm, hnorm,
+  return launch_pdl(draft_next_kernel, dim3(B), dim3(128), 0, s, am_val, am_idx, n_tiles, am_ld, k, K, slots, seq_len, u, embed, enorm, hnorm,
                                        eps, dcat, pos, kv_rowoff, dstage_seq_stride, cand, cand_ld);
-  return cudaGetLastError();
 }
 
 }  // namespace fm
