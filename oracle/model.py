@@ -8,7 +8,7 @@ What it computes, in the paper's order and notation (arXiv 2609.03181, "Jina-OCR
 * the verifier: the DeepSeekMoE decoder of Table "Model specification" (12 layers, d=1280,
   64 routed + 2 shared experts, top-6, RoPE theta=1e6), run over the K+1 candidate tokens
   [bonus, x^_1..x^_K] of each sequence against its committed KV cache (Sec. 3, "Model
-  Architecture"; the router notation p_{i,t} of Sec. 6 "Auxiliary regularizers");
+  Architecture"; the router notation p_{i,t} of Sec. 5.4 "Auxiliary regularizers");
 * greedy verification: v_r = argmax q_r, the longest equality prefix m of the acceptance
   equation of Sec. 3.1, commit x^_{1:m} then v_{m+1} (bonus when m=K), discard the tail;
 * the FastMTP draft head, the draft-head equation of Sec. 3.1: a^(1)_p = b_p,

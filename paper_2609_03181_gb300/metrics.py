@@ -1,5 +1,5 @@
 """Speculative-decoding statistics with the definitions of the paper's efficiency table
-(Sec. 7.3, Table "Decoding efficiency ... with FastMTP"):
+(Sec. 6.4, Table "Decoding efficiency ... with FastMTP"):
 
 * tau: mean number of tokens committed per speculative step, bonus token included;
 * acceptance rate: the position-averaged (tau - 1) / k;
