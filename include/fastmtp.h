@@ -210,6 +210,23 @@ typedef struct spec_profile_t {
 spec_status spec_profile(spec_ctx* ctx, int32_t mode);
 spec_status spec_profile_read(spec_ctx* ctx, spec_profile_t* out);
 
+/* Y = X W^T like spec_gemm_bf16, computed split-K, for callers that cannot allocate device
+ * memory: code running while a stream is captured into a CUDA graph (an allocation there is
+ * rejected or breaks the capture), runtimes that give out device memory only from their own
+ * fixed pool, serving loops where a hidden cudaMalloc would stall the device.  (The paper has
+ * no counterpart; this is an interface for such callers.)  The split-K partial tiles and
+ * tickets live in a fixed file-scope device array of 4 MiB + 4 KiB that every GPU loading the
+ * library holds until the process exits; the call allocates and frees nothing.  The first call
+ * on a device looks the array up on that device (it must be current) and should come before
+ * any stream capture.  Every call shares the array and leaves its last contents there; the
+ * call clears the tickets it uses before its kernel runs.  Calls whose kernels overlap on the
+ * GPU race on the array: keep them on one stream.  Limits: n_tiles * m_tiles * splits * rows
+ * box * 128 floats <= 2^20 (e.g. M <= 64 with N <= 4096 at K = 1280); larger problems get
+ * SPEC_EINVAL with the reason in spec_last_error(NULL).  Same argument rules and errors as
+ * spec_gemm_bf16 otherwise; asynchronous on `stream`. */
+spec_status spec_gemm_bf16_noalloc(const void* X, const void* W, float* Y, int32_t M, int32_t N,
+                                   int32_t Kdim, void* stream);
+
 /* Frees the workspace.  Borrowed weights and pools are untouched.  NULL is ignored. */
 void spec_destroy(spec_ctx* ctx);
 

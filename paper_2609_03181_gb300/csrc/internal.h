@@ -106,6 +106,8 @@ bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, u
 // may still be writing the weights).
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl = true);
 int num_sms();
+// Sets the message spec_last_error(NULL) returns in this thread.
+void set_thread_error(const std::string& msg);
 // Kernel attributes (dynamic shared memory limits) set once, before any launch or capture.
 cudaError_t gemm_prepare();
 cudaError_t attention_prepare();

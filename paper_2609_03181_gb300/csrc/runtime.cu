@@ -522,6 +522,8 @@ extern "C" void spec_destroy(spec_ctx* ctx) {
   delete ctx;
 }
 
+void fm::set_thread_error(const std::string& msg) { g_tls_err = msg; }
+
 extern "C" const char* spec_last_error(const spec_ctx* ctx) {
   return ctx ? ctx->err.c_str() : g_tls_err.c_str();
 }

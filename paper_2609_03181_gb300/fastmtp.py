@@ -20,7 +20,8 @@ WS_B, WS_ROUTE_IDX, WS_ROUTE_GATE, WS_EXPERT_CNT, WS_DRAFT_U, WS_HIDDEN = range(
 # Public entry points, in the order include/fastmtp.h declares them.
 ENTRY_POINTS = ["spec_init", "spec_seq_reset", "spec_seq_set_draft_rows", "draft_step", "verify_step",
                 "accept_commit", "spec_sync", "spec_seq_state", "spec_read_workspace", "spec_gemm_bf16",
-                "spec_profile", "spec_profile_read", "spec_destroy", "spec_last_error"]
+                "spec_profile", "spec_profile_read", "spec_gemm_bf16_noalloc", "spec_destroy",
+                "spec_last_error"]
 KERNEL_CLASSES = ["embed", "qkv", "attention", "oproj", "router", "permute", "expert_gate_up", "expert_down",
                   "combine", "lm_head", "argmax", "commit", "draft_gemm", "draft_misc"]
 
@@ -81,6 +82,7 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
         "spec_gemm_bf16": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
         "spec_profile": (ctypes.c_int, [P, I32]),
         "spec_profile_read": (ctypes.c_int, [P, ctypes.POINTER(SpecProfile)]),
+        "spec_gemm_bf16_noalloc": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
         "spec_destroy": (None, [P]),
         "spec_last_error": (ctypes.c_char_p, [P]),
     }
@@ -110,6 +112,20 @@ def gemm_bf16(X: torch.Tensor, W: torch.Tensor, stream: Optional[torch.cuda.Stre
     N = W.shape[0]
     Y = torch.empty(M, N, dtype=torch.float32, device=X.device)
     st = lib.spec_gemm_bf16(X.data_ptr(), W.data_ptr(), Y.data_ptr(), M, N, K, _stream_handle(stream))
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+    return Y
+
+
+def gemm_bf16_noalloc(X: torch.Tensor, W: torch.Tensor, Y: torch.Tensor,
+                      stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Y = X W^T through spec_gemm_bf16_noalloc (split-K with the library's fixed scratch);
+    Y is a caller-provided fp32 CUDA tensor [M][N]."""
+    lib = load_library()
+    M, K = X.shape
+    N = W.shape[0]
+    assert Y.shape == (M, N) and Y.dtype == torch.float32 and Y.is_contiguous()
+    st = lib.spec_gemm_bf16_noalloc(X.data_ptr(), W.data_ptr(), Y.data_ptr(), M, N, K, _stream_handle(stream))
     if st != SPEC_OK:
         raise FastMTPError(st, lib.spec_last_error(None).decode())
     return Y
