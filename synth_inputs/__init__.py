@@ -202,3 +202,47 @@ def kv_prefix(seed: int, seq: int, n_layers: int, ctx: int, n_heads: int, head_d
 def draft_kv_prefix(seed: int, seq: int, ctx: int, n_heads: int, head_dim: int) -> torch.Tensor:
     """Committed draft-block KV for rows 0..ctx-1 of one sequence, bf16 [2][ctx][H][hd] ~N(0,1)."""
     return normal(seed, f"dkv.{seq}", (2, ctx, n_heads, head_dim), 1.0)
+
+
+def successor_weights(shape: ModelShape, seed: int, beta_over_alpha: float, alpha: float = 1.0,
+                      std: float = 0.02, gain_std: float = 0.0):
+    """Weights under which speculative decoding accepts a tunable share of the drafts.
+
+    Input construction only (seeded random matrices, a permutation and scalings):
+    * E ~ N(0, 1) (instead of 0.02) so the embedding dominates the residual stream of the
+      random std-0.02 layers, and W_lm[v] = E[pi^-1(v)] for a seeded permutation pi of the
+      vocabulary: the verifier's greedy successor of token x is pi(x), by a wide margin;
+    * P = [alpha * I | beta * M] with M ~ N(0, 1/d): the draft head sees the next token's
+      embedding through the identity half and a random rotation of its input state through the
+      other half; the ratio beta/alpha sets how often that perturbation moves the draft's argmax
+      away from pi(x), i.e. the acceptance rate.
+    Returns (VerifierWeights, DraftWeights, pi)."""
+    vw = verifier_weights(shape, seed, std=std, gain_std=gain_std)
+    dw = draft_weights(shape, seed, std=std, gain_std=gain_std)
+    d, V = shape.hidden, shape.vocab
+    E = normal(seed, "succ.embed", (V, d), 1.0)
+    pi = permutation(seed, "succ.pi", V)
+    inv = np.empty(V, dtype=np.int64)
+    inv[pi] = np.arange(V)
+    vw.embed = E
+    vw.lm_head = E[torch.from_numpy(inv)].contiguous()
+    M = normal(seed, "succ.M", (d, d), 1.0 / math.sqrt(d), dtype=torch.float32)
+    eye = torch.eye(d, dtype=torch.float32)
+    dw.eh_proj = torch.cat([alpha * eye, (alpha * beta_over_alpha) * M], dim=1).to(torch.bfloat16).contiguous()
+    return vw, dw, pi
+
+
+def kv_prefix_device(seed: int, seq: int, n_layers: int, ctx: int, n_heads: int, head_dim: int,
+                     device) -> torch.Tensor:
+    """Like kv_prefix, drawn on `device` by PyTorch's seeded generator (a different stream from
+    kv_prefix's): for large GPU-only workloads whose prefixes no CPU oracle has to reproduce."""
+    g = torch.Generator(device=device)
+    g.manual_seed((int(seed) * 1000003 + zlib.crc32(f"kvdev.{seq}".encode())) & 0x7FFFFFFFFFFFFFFF)
+    x = torch.randn(n_layers, 2, ctx, n_heads, head_dim, generator=g, device=device, dtype=torch.float32)
+    return x.to(torch.bfloat16)
+
+
+def draft_kv_prefix_device(seed: int, seq: int, ctx: int, n_heads: int, head_dim: int, device) -> torch.Tensor:
+    g = torch.Generator(device=device)
+    g.manual_seed((int(seed) * 1000003 + zlib.crc32(f"dkvdev.{seq}".encode())) & 0x7FFFFFFFFFFFFFFF)
+    return torch.randn(2, ctx, n_heads, head_dim, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)

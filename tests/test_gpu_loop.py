@@ -138,3 +138,26 @@ def test_batch_invariance_alone_vs_in_batch(setup):
         eng.sync()
         res.append((bst[: K + 1].clone(), vt[0].cpu().clone()))
     assert torch.equal(res[0][0], res[1][0]) and torch.equal(res[0][1], res[1][1])
+
+
+@pytest.fixture(scope="module")
+def succ():
+    """Acceptance-tuned (successor-map) weights: the draft head agrees with the verifier often."""
+    seed = 23
+    vw, dw, _ = S.successor_weights(SHAPE, seed, 7.0)
+    ctx = [int(c) for c in S.integers(seed, "ctx", B, 100, 300)]
+    kvs = [S.kv_prefix(seed, b, SHAPE.n_layers, ctx[b], SHAPE.n_heads, SHAPE.head_dim) for b in range(B)]
+    dkvs = [S.draft_kv_prefix(seed, b, ctx[b], SHAPE.n_heads, SHAPE.head_dim) for b in range(B)]
+    pend = [int(x) for x in S.integers(seed, "pending", B, 0, SHAPE.vocab - 1)]
+    eng = F.Engine(vw, dw, max_batch=8, K_max=K, max_ctx=max(ctx) + 2 * N_TOK + 16, page_size=64)
+    yield dict(vw=vw, dw=dw, ctx=ctx, kvs=kvs, dkvs=dkvs, pend=pend, eng=eng)
+    eng.close()
+
+
+def test_speculative_with_accepting_draft_head_equals_greedy(succ):
+    reset(succ)
+    greedy, _ = run_loop(succ, N_TOK, 0)
+    reset(succ)
+    got, ms = run_loop(succ, N_TOK, K, "head")
+    assert got == greedy
+    assert sum(ms) > 0, "the tuned draft head should get drafts accepted"

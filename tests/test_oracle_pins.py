@@ -431,6 +431,24 @@ def test_speculative_with_draft_head_equals_greedy():
     assert st.steps > 0
 
 
+def test_lossless_with_accepting_draft_head():
+    """Successor-map weights make the FastMTP head agree with the verifier often; the committed
+    stream must still equal plain greedy decoding, now with long accepted prefixes."""
+    sh = TINY.replace(hidden=64, n_heads=2, head_dim=8, vocab=60, n_layers=2)
+    vw, dw, pi = S.successor_weights(sh, 13, 1.0, gain_std=0.0)
+    model = O.Verifier(vw)
+    dr = O.Drafter(dw, model)
+    base = tiny_caches(sh, 13, 2, 3, 6)
+    greedy = O.greedy_decode(model, _clone(base), 16, rb=True)
+    assert greedy[0][:3] == [int(pi[base[0].pending]), int(pi[pi[base[0].pending]]),
+                             int(pi[pi[pi[base[0].pending]]])]      # the verifier follows pi
+    dcs = _dcaches(sh, base, 13)
+    st = O.DecodeStats()
+    got = O.speculative_decode(model, _clone(base), 16, 3, drafter=dr, dcaches=dcs, rb=True, stats=st)
+    assert got == greedy
+    assert sum(st.accept_hist[1:]) > 0
+
+
 # ----------------------------------------------------------------------------- paper numbers
 
 def test_shape_contract_parameter_counts_match_paper():
