@@ -3,8 +3,8 @@
 // Each sequence has R queries at consecutive positions p0..p0+R-1 (the K+1 verify
 // candidates, or one draft row).  Keys at positions < ctx_len live in the sequence's pages,
 // keys at positions >= ctx_len in a staging buffer (candidates not yet committed).  The key
-// range is cut into chunks of 128 positions fixed by absolute position; one CTA per
-// (chunk, head, sequence) stages the chunk's K and V in shared memory with 16-byte
+// range is cut into chunks of 128 positions fixed by absolute position; a persistent CTA per SM
+// walks the (chunk, head, sequence) items, stages each chunk's K and V in shared memory with 16-byte
 // cp.async copies, forms the scores K q^T and the output V^T p^T with bf16 tensor-core
 // MMAs (fp32 accumulation; queries padded to 8; the probabilities enter as a sum of two bf16
 // terms, so the product keeps about 16 bits of them), and writes the chunk's
@@ -21,7 +21,6 @@
 namespace fm {
 
 constexpr int kCH = kAttnChunk;
-constexpr int kAttnSmem = 2 * kCH * kHD * 2 + kMaxR * kHD * 2 + 2 * kMaxR * kCH * 2 + kMaxR * kCH * 4;
 constexpr long long kStagedBit = 1ll << 62;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
@@ -29,10 +28,10 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_b
                : "memory");
 }
 
-// Merge of the chunks of every query of (sequence b, head h), run by the last chunk CTA:
-// query r combines chunks 0..floor(p_r/128) in chunk order, O = sum_c w_c acc_c / sum_c w_c l_c
-// with w_c = 2^(m_c - max_c m_c).  The (m, l) pairs are staged in shared memory by all threads
-// at once; the accumulator loads of the weighted sum are independent of each other.
+// Merge of the chunks of every query of (sequence b, head h), run by the CTA that finishes the
+// last chunk: query r combines chunks 0..floor(p_r/128) in chunk order,
+// O = sum_c w_c acc_c / sum_c w_c l_c with w_c = 2^(m_c - max_c m_c).  The (m, l) pairs are
+// staged in shared memory by all threads at once; the accumulator loads are independent.
 __device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R, int p0, int n_live, float* smem) {
   const float* part = a.part + (static_cast<size_t>(b) * kH + h) * a.n_chunks * R * (kHD + 2);
   float* sm = smem;                      // [n_live * R] chunk max, then weight
@@ -59,20 +58,22 @@ __device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R
   }
   __syncthreads();
   const int d = threadIdx.x;
-  for (int r = 0; r < R; ++r) {
-    const int lastc = (p0 + r) / kCH;
-    float O = 0.f;
-    int c = 0;
-    for (; c + 4 <= lastc + 1; c += 4) {
-      float x[4];
+  if (d < kHD) {
+    for (int r = 0; r < R; ++r) {
+      const int lastc = (p0 + r) / kCH;
+      float O = 0.f;
+      int c = 0;
+      for (; c + 4 <= lastc + 1; c += 4) {
+        float x[4];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) x[u] = __ldcg(&part[(static_cast<size_t>(c + u) * R + r) * (kHD + 2) + d]);
+        for (int u = 0; u < 4; ++u) x[u] = __ldcg(&part[(static_cast<size_t>(c + u) * R + r) * (kHD + 2) + d]);
 #pragma unroll
-      for (int u = 0; u < 4; ++u) O += x[u] * sm[(c + u) * R + r];
+        for (int u = 0; u < 4; ++u) O += x[u] * sm[(c + u) * R + r];
+      }
+      for (; c <= lastc; ++c) O += __ldcg(&part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + d]) * sm[c * R + r];
+      a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d] =
+          __float2bfloat16(O / sL[r]);
     }
-    for (; c <= lastc; ++c) O += __ldcg(&part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + d]) * sm[c * R + r];
-    a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d] =
-        __float2bfloat16(O / sL[r]);
   }
 }
 
@@ -101,195 +102,228 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
 // by row (conflict-free for ldmatrix and row-wise cp.async).
 __device__ __forceinline__ uint32_t swz(int row, int ch) { return row * 256 + ((ch ^ (row & 7)) << 4); }
 
-__global__ void __launch_bounds__(128) attn_chunk_kernel(const AttnArgs a) {
-  extern __shared__ __align__(16) uint8_t asmem[];
-  uint8_t* sK = asmem;                                   // [128 keys][128 dims] bf16
-  uint8_t* sV = sK + kCH * kHD * 2;                      // [128 keys][128 dims] bf16
-  uint8_t* sQ = sV + kCH * kHD * 2;                      // [8 queries][128 dims] bf16
-  uint8_t* sP = sQ + kMaxR * kHD * 2;                    // [8 queries][128 keys] bf16 p, high part
-  uint8_t* sPl = sP + kMaxR * kCH * 2;                   // [8 queries][128 keys] bf16 p - high part
-  float* sS = reinterpret_cast<float*>(sPl + kMaxR * kCH * 2);  // [8][128] fp32 scores
-  __shared__ long long s_base[kCH];                      // element offset of each key row (-1: none)
-  __shared__ int s_last;
-  pdl_trigger();
-  pdl_wait();
+// One work item: 128 keys (a chunk fixed by absolute position) of one head of one sequence.
+struct ChunkItem {
+  int b, h, c, slot, sl, p0, last, start, nk;
+  bool live;
+};
+__device__ __forceinline__ void decode_item(const AttnArgs& a, int item, ChunkItem& it) {
+  it.c = item % a.n_chunks;
+  const int t = item / a.n_chunks;
+  it.h = t % kH;
+  it.b = t / kH;
+  it.slot = a.slots[it.b];
+  it.sl = a.seq_len[it.slot];
+  it.p0 = it.sl + a.qoff;
+  it.last = it.p0 + a.R - 1;
+  it.start = it.c * kCH;
+  it.live = !(it.start > it.last || it.p0 < 0);
+  it.nk = it.live ? min(kCH, it.last + 1 - it.start) : 0;
+}
 
-  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
-  const int R = a.R;
-  const int slot = a.slots[b];
-  const int sl = a.seq_len[slot];
-  const int p0 = sl + a.qoff;
-  const int last = p0 + R - 1;
-  const int start = c * kCH;
-  if (start > last || p0 < 0) return;
-  const int nk = min(kCH, last + 1 - start);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-  // where each key row lives: a page of the pool (positions < ctx_len) or a staging row
-  {
-    const int j = tid;
-    const int pos = start + j;
+// Locates the chunk's key rows (a page of the pool below ctx_len, else a staging row) and
+// issues their K and V copies into the stage buffer as one cp.async group.
+__device__ __forceinline__ void issue_chunk(const AttnArgs& a, const ChunkItem& it, long long* s_base, uint8_t* stage) {
+  const int tid = threadIdx.x;
+  if (tid < kCH) {
+    const int j = tid, pos = it.start + j;
     long long off = -1;
-    if (j < nk) {
-      if (pos < sl) {
+    if (j < it.nk) {
+      if (pos < it.sl) {
         const int pi = pos / a.page_size;
-        const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+        const int page = (pi < a.max_pages) ? a.block_table[it.slot * a.max_pages + pi] : -1;
         if (page >= 0 && page < a.n_pages)
-          off = ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
+          off = ((static_cast<long long>(page) * 2 * kH + it.h) * a.page_size + pos % a.page_size) * kHD;
         else
           atomicOr(a.err, ERR_PAGE_RANGE);
       } else {
-        off = kStagedBit | (b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
-                            static_cast<long long>(h) * kHD);
+        off = kStagedBit | (it.b * a.stage_seq_stride + static_cast<long long>(pos - it.sl) * a.stage_row_stride +
+                            static_cast<long long>(it.h) * kHD);
       }
     }
     s_base[j] = off;
   }
   __syncthreads();
-
-  // K, then V, rows of the chunk -> shared memory (zero-filled where there is no key)
   const long long v_pool = static_cast<long long>(kH) * a.page_size * kHD;
+  uint8_t* sK = stage;
+  uint8_t* sV = stage + kCH * kHD * 2;
 #pragma unroll 4
-  for (int v = tid; v < kCH * 16; v += 128) {
+  for (int v = tid; v < kCH * 16; v += blockDim.x) {
     const int j = v >> 4, ch = v & 15;
     const long long off = s_base[j];
-    const bf16* src = a.pool;
+    const bf16* srck = a.pool;
+    const bf16* srcv = a.pool;
     int bytes = 0;
     if (off >= 0) {
-      src = ((off & kStagedBit) ? a.stage + (off & (kStagedBit - 1)) : a.pool + off) + ch * 8;
+      if (off & kStagedBit) {
+        srck = a.stage + (off & (kStagedBit - 1)) + ch * 8;
+        srcv = srck + a.stage_kv_stride;
+      } else {
+        srck = a.pool + off + ch * 8;
+        srcv = srck + v_pool;
+      }
       bytes = 16;
     }
-    cp_async16(sK + swz(j, ch), src, bytes);
+    cp_async16(sK + swz(j, ch), srck, bytes);
+    cp_async16(sV + swz(j, ch), srcv, bytes);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
-#pragma unroll 4
-  for (int v = tid; v < kCH * 16; v += 128) {
-    const int j = v >> 4, ch = v & 15;
-    const long long off = s_base[j];
-    const bf16* src = a.pool;
-    int bytes = 0;
-    if (off >= 0) {
-      src = ((off & kStagedBit) ? a.stage + (off & (kStagedBit - 1)) + a.stage_kv_stride : a.pool + off + v_pool) +
-            ch * 8;
-      bytes = 16;
+}
+
+// Persistent kernel: each CTA walks the (sequence, head, chunk) items i = blockIdx.x + k*gridDim.x
+// and keeps two stage buffers, so the next live item's K/V are in flight while it computes the
+// current one.  Scores K q^T and output V^T p^T run on bf16 tensor cores (mma.sync m16n8k16,
+// fp32 accumulation, queries padded to 8, p entering as hi + lo bf16 terms).
+constexpr int kAttnThreads = 256;
+constexpr int kStageBytes = 2 * kCH * kHD * 2;   // K and V of one chunk
+constexpr int kAttnSmem = 2 * kStageBytes + kMaxR * kHD * 2 + 2 * kMaxR * kCH * 2 + kMaxR * kCH * 4;
+
+__global__ void __launch_bounds__(kAttnThreads, 1) attn_chunk_kernel(const AttnArgs a) {
+  extern __shared__ __align__(128) uint8_t asmem[];
+  uint8_t* stages = asmem;                                   // [2][K 32 KB | V 32 KB]
+  uint8_t* sQ = asmem + 2 * kStageBytes;                     // [8 queries][128 dims] bf16
+  uint8_t* sP = sQ + kMaxR * kHD * 2;                        // [8][128 keys] bf16 p, high part
+  uint8_t* sPl = sP + kMaxR * kCH * 2;                       // [8][128 keys] bf16 p - high part
+  float* sS = reinterpret_cast<float*>(sPl + kMaxR * kCH * 2);   // [8][128] fp32 scores
+  __shared__ long long s_base[2][kCH];
+  __shared__ int s_last;
+  pdl_trigger();
+  pdl_wait();
+
+  const int R = a.R;
+  const int total = a.n_seqs * kH * a.n_chunks;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
+
+  int item = blockIdx.x;
+  ChunkItem cur;
+  for (; item < total; item += gridDim.x) {
+    decode_item(a, item, cur);
+    if (cur.live) break;
+  }
+  if (item >= total) return;
+  issue_chunk(a, cur, s_base[0], stages);
+  int st = 0;
+  while (true) {
+    int nitem = item + gridDim.x;
+    ChunkItem nxt;
+    for (; nitem < total; nitem += gridDim.x) {
+      decode_item(a, nitem, nxt);
+      if (nxt.live) break;
     }
-    cp_async16(sV + swz(j, ch), src, bytes);
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
+    const bool has_next = nitem < total;
+    if (has_next) {
+      issue_chunk(a, nxt, s_base[st ^ 1], stages + (st ^ 1) * kStageBytes);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    // queries of the current item (bf16, as the QKV epilogue stored them); rows R..7 are zero
+    const int qrow0 = a.q_row0 ? a.q_row0[cur.b] : cur.b * R;
+    if (tid < kMaxR * 16) {
+      const int q = tid >> 4, ch = tid & 15;
+      uint4 val = make_uint4(0, 0, 0, 0);
+      if (q < R)
+        val = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + cur.h) * kHD + ch * 8);
+      *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = val;
+    }
+    __syncthreads();
+    const uint32_t kbase = smem_u32(stages + st * kStageBytes);
+    const uint32_t vbase = kbase + kCH * kHD * 2;
 
-  // queries (bf16, as the QKV epilogue stored them); rows R..7 are zero
-  const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
-  {
-    const int q = tid >> 4, ch = tid & 15;   // 8 queries x 16 chunks
-    uint4 val = make_uint4(0, 0, 0, 0);
-    if (q < R) val = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
-    *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = val;
-  }
-  asm volatile("cp.async.wait_group 1;" ::: "memory");   // K has landed; V may still be in flight
-  __syncthreads();
-
-  const int g = lane >> 2, t4 = lane & 3;
-  const int mi = lane >> 3, ri = lane & 7;
-  // S^T[key][query] = K Q^T: warp w owns keys 32w..32w+31 (two 16-key tiles), 8 k-steps of 16 dims
-  {
-    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    const uint32_t kbase = smem_u32(sK), qbase = smem_u32(sQ);
+    // S^T[key][query] = K Q^T: warp w owns keys 16w..16w+15, 8 k-steps of 16 dims
+    {
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint32_t qbase = smem_u32(sQ);
 #pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {
-      uint32_t bq[2];
-      ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), bq);
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        uint32_t ak[4];
-        const int key = warp * 32 + mt * 16 + ri + ((mi & 1) ? 8 : 0);
+      for (int ks = 0; ks < 8; ++ks) {
+        uint32_t bq[2], ak[4];
+        ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), bq);
+        const int key = warp * 16 + ri + ((mi & 1) ? 8 : 0);
         ldsm_x4(kbase + swz(key, 2 * ks + (mi >> 1)), ak);
-        mma_bf16_16816(acc[mt], ak, bq);
+        mma_bf16_16816(acc, ak, bq);
       }
-    }
-    const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));   // log2(e) / sqrt(hd)
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
+      const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));   // log2(e) / sqrt(hd)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const int key = warp * 32 + mt * 16 + g + ((e >> 1) ? 8 : 0);
+        const int key = warp * 16 + g + ((e >> 1) ? 8 : 0);
         const int q = 2 * t4 + (e & 1);
-        const bool vis = q < R && key < nk && start + key <= p0 + q;
-        sS[q * kCH + key] = vis ? acc[mt][e] * scale : -INFINITY;
+        const bool vis = q < R && key < cur.nk && cur.start + key <= cur.p0 + q;
+        sS[q * kCH + key] = vis ? acc[e] * scale : -INFINITY;
       }
-  }
-  __syncthreads();
-
-  // per query: chunk max, probabilities (exact zeros where masked) split as p = hi + lo with
-  // hi, lo bf16 (about 16 significant bits for the P V product), and their fp32 sum
-  float* part = a.part + ((static_cast<size_t>(b) * kH + h) * a.n_chunks + c) * R * (kHD + 2);
-  for (int q = warp; q < kMaxR; q += 4) {
-    float x[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) x[i] = sS[q * kCH + lane + 32 * i];
-    const float m = warp_max(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])));
-    float l = 0.f;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int key = lane + 32 * i;
-      const float p = (m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m);
-      const bf16 hi = __float2bfloat16(p);
-      const bf16 lo = __float2bfloat16(p - __bfloat162float(hi));
-      *reinterpret_cast<bf16*>(sP + swz(q, key >> 3) + (key & 7) * 2) = hi;
-      *reinterpret_cast<bf16*>(sPl + swz(q, key >> 3) + (key & 7) * 2) = lo;
-      l += p;
     }
-    l = warp_sum(l);
-    if (lane == 0 && q < R) {
-      part[q * (kHD + 2) + kHD] = m;
-      part[q * (kHD + 2) + kHD + 1] = l;
-    }
-  }
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
-  __syncthreads();
+    __syncthreads();
 
-  // O^T[dim][query] = V^T P^T: warp w owns dims 32w..32w+31, 8 k-steps of 16 keys
-  {
-    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    const uint32_t vbase = smem_u32(sV), pbase = smem_u32(sP), plbase = smem_u32(sPl);
+    // per query (warp w owns query w): chunk max, p = hi + lo (exact zeros where masked), sum
+    float* part = a.part + ((static_cast<size_t>(cur.b) * kH + cur.h) * a.n_chunks + cur.c) * R * (kHD + 2);
+    {
+      const int q = warp;
+      float x[4];
 #pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {
-      uint32_t bp[2], bl[2];
-      ldsm_x2(pbase + swz(ri, 2 * ks + (mi & 1)), bp);
-      ldsm_x2(plbase + swz(ri, 2 * ks + (mi & 1)), bl);
+      for (int i = 0; i < 4; ++i) x[i] = sS[q * kCH + lane + 32 * i];
+      const float m = warp_max(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])));
+      float l = 0.f;
 #pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        uint32_t av[4];
+      for (int i = 0; i < 4; ++i) {
+        const int key = lane + 32 * i;
+        const float p = (m == -INFINITY || x[i] == -INFINITY) ? 0.f : exp2f(x[i] - m);
+        const bf16 hi = __float2bfloat16(p);
+        const bf16 lo = __float2bfloat16(p - __bfloat162float(hi));
+        *reinterpret_cast<bf16*>(sP + swz(q, key >> 3) + (key & 7) * 2) = hi;
+        *reinterpret_cast<bf16*>(sPl + swz(q, key >> 3) + (key & 7) * 2) = lo;
+        l += p;
+      }
+      l = warp_sum(l);
+      if (lane == 0 && q < R) {
+        part[q * (kHD + 2) + kHD] = m;
+        part[q * (kHD + 2) + kHD + 1] = l;
+      }
+    }
+    __syncthreads();
+
+    // O^T[dim][query] = V^T P^T: warp w owns dims 16w..16w+15, 8 k-steps of 16 keys
+    {
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint32_t pbase = smem_u32(sP), plbase = smem_u32(sPl);
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        uint32_t bp[2], bl[2], av[4];
+        ldsm_x2(pbase + swz(ri, 2 * ks + (mi & 1)), bp);
+        ldsm_x2(plbase + swz(ri, 2 * ks + (mi & 1)), bl);
         const int key = ks * 16 + ri + ((mi >> 1) ? 8 : 0);
-        const int dch = (warp * 32 + mt * 16) / 8 + (mi & 1);
-        ldsm_x4_t(vbase + swz(key, dch), av);
-        mma_bf16_16816(acc[mt], av, bp);
-        mma_bf16_16816(acc[mt], av, bl);
+        ldsm_x4_t(vbase + swz(key, 2 * warp + (mi & 1)), av);
+        mma_bf16_16816(acc, av, bp);
+        mma_bf16_16816(acc, av, bl);
       }
-    }
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const int d = warp * 32 + mt * 16 + g + ((e >> 1) ? 8 : 0);
+        const int d = warp * 16 + g + ((e >> 1) ? 8 : 0);
         const int q = 2 * t4 + (e & 1);
-        if (q < R) part[q * (kHD + 2) + d] = acc[mt][e];
+        if (q < R) part[q * (kHD + 2) + d] = acc[e];
       }
-  }
+    }
 
-  // the last chunk of (sequence, head) to finish merges every query (atomic ticket, no wait)
-  __threadfence();
-  __syncthreads();
-  const int n_live = last / kCH + 1;
-  if (tid == 0) {
-    int* ticket = a.tickets + b * kH + h;
-    const int old = atomicAdd(ticket, 1);
-    s_last = (old == n_live - 1) ? 1 : 0;
-    if (s_last) *ticket = 0;
-  }
-  __syncthreads();
-  if (s_last) {
+    // the CTA that finishes the last chunk of (sequence, head) merges every query
     __threadfence();
-    merge_all(a, b, h, R, p0, n_live, reinterpret_cast<float*>(asmem));   // K/V tiles are no longer needed
+    __syncthreads();
+    const int n_live = cur.last / kCH + 1;
+    if (tid == 0) {
+      int* ticket = a.tickets + cur.b * kH + cur.h;
+      const int old = atomicAdd(ticket, 1);
+      s_last = (old == n_live - 1) ? 1 : 0;
+      if (s_last) *ticket = 0;
+    }
+    __syncthreads();
+    if (s_last) {
+      __threadfence();
+      // the current stage's K tile is no longer needed: scratch for the merge
+      merge_all(a, cur.b, cur.h, R, cur.p0, n_live, reinterpret_cast<float*>(stages + st * kStageBytes));
+    }
+    __syncthreads();   // stage st, sQ, sS and sP are reused by the next item
+    if (!has_next) break;
+    item = nitem;
+    cur = nxt;
+    st ^= 1;
   }
 }
 
@@ -297,8 +331,12 @@ cudaError_t attention_prepare() {
   return cudaFuncSetAttribute(attn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
 }
 
-cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s) {
-  return launch_pdl(attn_chunk_kernel, dim3(a.n_chunks, kH, B), dim3(128), kAttnSmem, s, a);
+cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
+  AttnArgs a = a_in;
+  a.n_seqs = B;
+  const int total = B * kH * a.n_chunks;
+  const int grid = total < num_sms() ? total : num_sms();
+  return launch_pdl(attn_chunk_kernel, dim3(grid), dim3(kAttnThreads), kAttnSmem, s, a);
 }
 
 }  // namespace fm
