@@ -48,7 +48,7 @@ constexpr int kShared = 2;
 constexpr int kI = 896;         // expert intermediate
 constexpr int kId = 3584;       // draft-block intermediate
 constexpr int kSlots = kTopK + kShared;   // per-token expert outputs combined
-constexpr int kAttnChunk = 128;           // split-KV chunk (keys), fixed by absolute position
+constexpr int kAttnChunk = 64;            // split-KV chunk (keys), fixed by absolute position
 constexpr int kMaxR = 8;                  // K_max + 1 <= 8 candidate rows per sequence
 constexpr int kMaxSplit = 6;              // split-K ways of a dense GEMM
 
@@ -130,7 +130,6 @@ struct AttnArgs {
   float* part;                 // [B][H][n_chunks][R][kHD + 2]
   int* tickets;                // [B][H] chunk counters, zero between launches
   int n_chunks;
-  int n_seqs;                  // B
   bf16* out;                   // [B*R][H*hd]
   int out_row_stride_seq;      // rows of out per sequence (R)
   int* err;
