@@ -9,7 +9,7 @@
 // bf16 tensor cores (mma.sync m16n8k16, fp32 accumulation, queries padded to 8; p enters as a
 // sum of two bf16 terms so the product keeps about 16 bits of it).
 //
-// Scheduling: one CTA per (unit of 8 consecutive chunks, head, sequence); it resolves the
+// Scheduling: one CTA per (unit of consecutive chunks, head, sequence); it resolves the
 // page offsets of all its keys at once, then streams its chunks through two shared-memory
 // stages (16-byte cp.async), computing one chunk while the next is in flight.  The CTA that
 // finishes the last unit of a (sequence, head) merges (atomic ticket, no wait).  Masked keys
@@ -25,7 +25,7 @@
 namespace fm {
 
 constexpr int kCH = kAttnChunk;                  // keys per chunk (64)
-constexpr int kUnit = 8;                         // chunks per CTA
+constexpr int kUnitMax = 16;                     // most chunks one CTA streams
 constexpr int kAttnThreads = 128;
 constexpr int kStageBytes = 2 * kCH * kHD * 2;   // K and V of one chunk: 32 KB
 constexpr int kAttnSmem = 2 * kStageBytes + kMaxR * kHD * 2 + 2 * kMaxR * kCH * 2 + kMaxR * kCH * 4;
@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const AttnArgs
   uint8_t* sP = sQ + kMaxR * kHD * 2;                        // [8][64 keys] bf16 p, high part
   uint8_t* sPl = sP + kMaxR * kCH * 2;                       // [8][64 keys] bf16 p - high part
   float* sS = reinterpret_cast<float*>(sPl + kMaxR * kCH * 2);   // [8][64] fp32 scores
-  __shared__ long long s_base[kUnit * kCH];                  // element offset of every key row of the unit
+  __shared__ long long s_base[kUnitMax * kCH];               // element offset of every key row of the unit
   __shared__ int s_last;
   pdl_trigger();
   pdl_wait();
@@ -161,9 +161,9 @@ __global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const AttnArgs
   const int last = p0 + R - 1;
   if (p0 < 0) return;
   const int n_live = last / kCH + 1;                         // chunks holding keys 0..last
-  const int c0 = u * kUnit;
+  const int c0 = u * a.unit;
   if (c0 >= n_live) return;
-  const int c1 = min(c0 + kUnit, n_live);
+  const int c1 = min(c0 + a.unit, n_live);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
 
@@ -293,7 +293,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const AttnArgs
   // the CTA that finishes the last unit of (sequence, head) merges every query
   __threadfence();
   __syncthreads();
-  const int n_units = (n_live + kUnit - 1) / kUnit;
+  const int n_units = (n_live + a.unit - 1) / a.unit;
   if (tid == 0) {
     int* ticket = a.tickets + b * kH + h;
     const int old = atomicAdd(ticket, 1);
@@ -311,8 +311,18 @@ cudaError_t attention_prepare() {
   return cudaFuncSetAttribute(attn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
 }
 
-cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s) {
-  const int n_units = (a.n_chunks + kUnit - 1) / kUnit;
+cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
+  // Chunks per CTA: enough CTAs for about three resident per SM over the largest context the
+  // pools allow.  Pure scheduling: the arithmetic of every chunk and of the merge is the same
+  // for any grouping.
+  AttnArgs a = a_in;
+  const long long target = 3ll * num_sms();
+  const long long per_unit = static_cast<long long>(B) * kH;
+  int unit = static_cast<int>((per_unit * a.n_chunks + target - 1) / target);
+  if (unit < 1) unit = 1;
+  if (unit > kUnitMax) unit = kUnitMax;
+  a.unit = unit;
+  const int n_units = (a.n_chunks + unit - 1) / unit;
   return launch_pdl(attn_chunk_kernel, dim3(n_units, kH, B), dim3(kAttnThreads), kAttnSmem, s, a);
 }
 

@@ -130,6 +130,7 @@ struct AttnArgs {
   float* part;                 // [B][H][n_chunks][R][kHD + 2]
   int* tickets;                // [B][H] chunk counters, zero between launches
   int n_chunks;
+  int unit;                    // chunks per CTA (set by attention_launch)
   bf16* out;                   // [B*R][H*hd]
   int out_row_stride_seq;      // rows of out per sequence (R)
   int* err;

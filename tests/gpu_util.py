@@ -50,3 +50,13 @@ def index_parity(gpu_idx, ref_idx, gaps, gap=GAP):
     ok = gaps > gap
     mism = int(((gpu_idx != ref_idx).reshape(len(gaps), -1).any(-1) & ok).sum())
     return int(ok.sum()), int((~ok).sum()), mism
+
+
+def argmax_margin(lm_head, b_gpu, b_ref, k_sigma=8.0, floor=GAP):
+    """Per-row margin for comparing argmax tokens: the oracle's top-2 logit gap must exceed
+    k_sigma standard deviations of the logit-difference noise that the measured state
+    difference implies, sqrt(2) * rms(W_lm) * ||b_gpu - b_ref||_2 (and at least `floor`).
+    Twelve bf16 layers leave ~1% state noise, so a fixed 1e-3 logit margin would flip by chance."""
+    w_rms = float(lm_head.float().pow(2).mean().sqrt())
+    d = (b_gpu.double().cpu() - b_ref.double().cpu()).reshape(b_ref.shape[0], -1)
+    return np.maximum(floor, k_sigma * np.sqrt(2.0) * w_rms * d.norm(dim=-1).numpy())

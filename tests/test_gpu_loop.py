@@ -100,7 +100,9 @@ def test_speculative_with_draft_head_equals_greedy(setup):
 
 def test_greedy_matches_oracle_greedy(setup):
     """Token i of a stream is compared while every decision leading to it was unique: the
-    oracle's router margins (6th vs 7th expert) and argmax margins of steps 0..i all above 1e-3."""
+    oracle's router margins (6th vs 7th expert) above 1e-3 and argmax margins above 5e-2 logits
+    (two bf16 layers leave <0.5% state noise, a logit-difference noise of ~4e-3 here) at steps
+    0..i."""
     reset(setup)
     n = 6
     greedy, _ = run_loop(setup, n, 0)
@@ -110,7 +112,7 @@ def test_greedy_matches_oracle_greedy(setup):
         cache = O.SeqCache.from_prefix(setup["kvs"][b], setup["pend"][b])
         for i in range(n):
             vo = O.verify(model, [cache], [[cache.pending]], rb=True)
-            if float(vo.v_gap[0, 0]) <= GAP or min(float(g.min()) for g in vo.route_gap) <= GAP:
+            if float(vo.v_gap[0, 0]) <= 5e-2 or min(float(g.min()) for g in vo.route_gap) <= GAP:
                 break
             assert greedy[b][i] == int(vo.v[0, 0]), (b, i)
             compared += 1

@@ -11,7 +11,7 @@ import torch
 import oracle as O
 import synth_inputs as S
 from paper_2609_03181_gb300 import fastmtp as F
-from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, index_parity
+from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, index_parity, argmax_margin
 
 pytestmark = pytest.mark.gpu
 
@@ -65,12 +65,17 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
     assert max(e for e, k in zip(errs, keep) if k) < REL_TOL, (
         f"b rel err per row {['%.3g' % e for e in errs]}, diverged rows {np.nonzero(diverged)[0].tolist()}")
 
-    v_ok, v_skip, v_bad = index_parity(vt.cpu().numpy().reshape(-1)[keep], ref.v.numpy().reshape(-1)[keep],
-                                       ref.v_gap.numpy().reshape(-1)[keep])
-    assert v_bad == 0
+    # verifier tokens: exact where the oracle's logit margin exceeds the noise the measured state
+    # difference implies (at least 1e-3); accept lengths where all of a sequence's tokens are
+    margin = argmax_margin(vw.lm_head, b_gpu, ref.b.reshape(T, -1))
+    gaps = ref.v_gap.numpy().reshape(-1)
+    sure = keep & (gaps > margin)
+    g_tok, r_tok = vt.cpu().numpy().reshape(-1), ref.v.numpy().reshape(-1)
+    assert (g_tok[sure] == r_tok[sure]).all(), (
+        f"token mismatch at rows {np.nonzero(sure & (g_tok != r_tok))[0].tolist()}")
     for bb in range(B):
         rows = slice(bb * R, bb * R + K)
-        if keep[rows].all() and all(ref.v_gap[bb, :K].numpy() > GAP):
+        if sure[rows].all():
             assert int(acc[bb]) == ref.m[bb]
 
     committed = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
