@@ -99,10 +99,10 @@ def test_speculative_with_draft_head_equals_greedy(setup):
 
 
 def test_greedy_matches_oracle_greedy(setup):
-    """Token i of a stream is compared while every decision leading to it was unique: the
-    oracle's router margins (6th vs 7th expert) above 1e-3 and argmax margins above 5e-2 logits
-    (two bf16 layers leave <0.5% state noise, a logit-difference noise of ~4e-3 here) at steps
-    0..i."""
+    """Token i of a stream is compared while every decision leading to it was unique at steps
+    0..i: oracle router margins (6th vs 7th expert probability) above 3e-4 and argmax margins
+    above 2e-2 logits.  Two bf16 layers leave ~0.15% rms state noise here: router-probability
+    noise ~2e-5 and logit-difference noise ~1.5e-3, so both margins are over 10 sigma."""
     reset(setup)
     n = 6
     greedy, _ = run_loop(setup, n, 0)
@@ -112,7 +112,7 @@ def test_greedy_matches_oracle_greedy(setup):
         cache = O.SeqCache.from_prefix(setup["kvs"][b], setup["pend"][b])
         for i in range(n):
             vo = O.verify(model, [cache], [[cache.pending]], rb=True)
-            if float(vo.v_gap[0, 0]) <= 5e-2 or min(float(g.min()) for g in vo.route_gap) <= GAP:
+            if float(vo.v_gap[0, 0]) <= 2e-2 or min(float(g.min()) for g in vo.route_gap) <= 3e-4:
                 break
             assert greedy[b][i] == int(vo.v[0, 0]), (b, i)
             compared += 1
