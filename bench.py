@@ -12,9 +12,13 @@ Metric: accepted (committed) tokens per second, sum over sequences of (m + 1) pe
 whole job over all GPUs.  Prints one JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl fastmtp|reference]
+  python bench.py --sweep [--sweep-batch 1,4,16,64,256] [--sweep-ctx 1024,4096,8192]
+                  [--sweep-k 1,2,3] [--sweep-router uniform,zipf]
 
 `--impl reference` times the fp64 CPU oracle on a bounded sample of the same workload (the
-method's only other implementation here); under torchrun only rank 0 runs it.
+method's only other implementation here); under torchrun only rank 0 runs it.  `--sweep`
+measures the step at every (batch, context, K, router) point of the verify-throughput grid,
+one JSON line per point (one GPU).
 """
 from __future__ import annotations
 
@@ -56,6 +60,11 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--weights", default="successor", choices=["successor", "random"],
                    help="successor: acceptance-tuned seeded weights (tau ~2.7); random: N(0,0.02) everywhere")
+    p.add_argument("--sweep", action="store_true", help="run the (batch, context, K, router) grid")
+    p.add_argument("--sweep-batch", default="1,4,16,64,256")
+    p.add_argument("--sweep-ctx", default="1024,4096,8192")
+    p.add_argument("--sweep-k", default="1,2,3")
+    p.add_argument("--sweep-router", default="uniform,zipf")
     return p.parse_args()
 
 
@@ -441,9 +450,115 @@ def run_fastmtp(args):
         dist.destroy_process_group()
 
 
+# ----------------------------------------------------------------------------- sweep
+def run_sweep(args):
+    """Every (router, context, batch, K) point of the grid on one engine per router mode:
+    committed contexts of exactly `ctx` tokens (N(0,1) KV drawn on the device), one K=0 step
+    to seed the draft head, `warmup` steps, then `steps` timed steps with an event pair around
+    each phase.  Weights: the acceptance-tuned seeded set (seed 4); the Zipf mode adds the
+    per-expert router bias -1.2 ln(rank).  Pending tokens use seeds 4..8 by batch size."""
+    import torch
+
+    import synth_inputs as S
+    from paper_2609_03181_gb300 import fastmtp as F
+
+    batches = [int(x) for x in args.sweep_batch.split(",")]
+    ctxs = [int(x) for x in args.sweep_ctx.split(",")]
+    Ks = [int(x) for x in args.sweep_k.split(",")]
+    routers = args.sweep_router.split(",")
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peak, peak_kind = measured_peaks()
+    shape = S.ModelShape(n_layers=args.layers)
+    Bmax, Kmax = max(batches), max(Ks)
+    grow = (args.warmup + args.steps + 2) * (Kmax + 1)
+    clocks = ClockSampler(0)
+    clocks.start()
+    for router in routers:
+        vw, dw, _ = S.successor_weights(shape, 4, ACCEPT_RATIO)
+        if router == "zipf":
+            for l, lw in enumerate(vw.layers):
+                lw.router_bias = S.zipf_router_bias(4, l, shape.n_experts, 1.2)
+        stream = torch.cuda.Stream(dev)
+        eng = F.Engine(vw, dw, max_batch=Bmax, K_max=Kmax, max_ctx=max(ctxs) + grow, page_size=64,
+                       device=str(dev), stream=stream)
+        g = torch.Generator(device=dev)
+        g.manual_seed(4)
+        for l in range(shape.n_layers):
+            eng.kv_pool[l].normal_(generator=g)
+        eng.dkv_pool.normal_(generator=g)
+        # tensors made on PyTorch's current stream are complete before the engine's stream reads them
+        torch.cuda.synchronize(dev)
+        for ctx in ctxs:
+            for bi, B in enumerate(batches):
+                pend = [int(t) for t in S.integers(4 + bi, "pending", B, 0, shape.vocab - 1)]
+                slots = torch.arange(B, dtype=torch.int32, device=dev)
+                c0 = torch.tensor([[p] for p in pend], dtype=torch.int32, device=dev)
+                v0 = torch.empty(B, 1, dtype=torch.int32, device=dev)
+                for K in Ks:
+                    for b in range(B):
+                        eng.reset_seq(b, ctx, eng.block_table(b), pend[b])
+                    acc = torch.empty(B, dtype=torch.int32, device=dev)
+                    cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+                    vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+                    com = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+                    n_all = args.warmup + args.steps
+                    hist = torch.zeros(n_all, B, dtype=torch.int32, device=dev)
+                    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_all)]
+                    torch.cuda.synchronize(dev)
+                    with torch.cuda.stream(stream):
+                        eng.verify_step(slots, c0, v0, acc)
+                        eng.accept_commit(slots, v0, acc)
+                    eng.sync()
+                    with torch.cuda.stream(stream):
+                        for i in range(n_all):
+                            if i == args.warmup:
+                                eng.profile(2)
+                            ev[i][0].record(stream)
+                            eng.draft_step(slots, K, cand)
+                            ev[i][1].record(stream)
+                            eng.verify_step(slots, cand, vt, acc)
+                            ev[i][2].record(stream)
+                            eng.accept_commit(slots, com, hist[i])
+                            ev[i][3].record(stream)
+                    eng.sync()
+                    counted = eng.profile_read()
+                    eng.profile(0)
+                    cnt = eng.read_workspace(F.WS_EXPERT_CNT, (shape.n_layers, shape.n_experts), torch.int32).double()
+                    timed = range(args.warmup, n_all)
+                    ms = lambda a, b: statistics.mean(ev[i][a].elapsed_time(ev[i][b]) for i in timed)
+                    ms_step, ms_draft, ms_verify = ms(0, 3), ms(0, 1), ms(1, 2)
+                    h = hist.double().cpu()
+                    lens = ctx + 1 + torch.cumsum(h, 0) - h          # committed length seen by each verify
+                    ctx_mean = float(lens[args.warmup:].mean())
+                    tok = float(h[args.warmup:].sum())
+                    touched = counted["experts_touched"] / max(1, counted["launches"]["permute"])
+                    vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
+                    load = cnt / cnt.mean(-1, keepdim=True)
+                    out = {"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K,
+                           "tokens_per_s": tok / (ms_step * args.steps / 1000.0), "ms_step": ms_step,
+                           "ms_draft": ms_draft, "ms_verify": ms_verify, "ms_commit": ms(2, 3),
+                           "tau": tok / (args.steps * B),
+                           "verify_roofline": {"bytes": vbytes, "achieved_gbs": vbytes / ms_verify / 1e6,
+                                               "peak": peak, "peak_source": peak_kind,
+                                               "frac": vbytes / ms_verify / 1e6 / peak},
+                           "experts_touched_per_layer": touched,
+                           "expert_load_max_over_mean": float(load.max(-1).values.mean()),
+                           "expert_share_top1": float((cnt.max(-1).values / cnt.sum(-1)).mean()),
+                           "steps": args.steps, "warmup": args.warmup}
+                    print(json.dumps(out), flush=True)
+        eng.close()
+        del eng
+        torch.cuda.empty_cache()
+    clk = clocks.stop()
+    print(json.dumps({"sweep_clocks": clk}), flush=True)
+
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.sweep:
+        run_sweep(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_fastmtp(args)

@@ -26,9 +26,11 @@
  *  - Every step is asynchronous on the stream given to spec_init.  Arguments are validated
  *    on the host before any launch; a rejected call launches nothing and leaves the state
  *    unchanged.  Data-dependent faults found on the device (a token id out of range, a page
- *    index outside the pool, a candidate 0 that is not the pending token, a wait that ran
- *    out) set a device guard flag instead of trapping; spec_sync() reports it as
- *    SPEC_EDEVICE.  Kernels never trap and never spin without a time limit.
+ *    index outside the pool, a slot id in a device array outside [0, max_batch), a
+ *    candidate 0 that is not the pending token, a non-finite router row, a wait that ran
+ *    out) set a device guard flag instead of trapping, and the affected work is skipped or
+ *    clamped to a valid index; spec_sync() reports it as SPEC_EDEVICE.  Kernels never trap
+ *    and never spin without a time limit.
  *  - bf16 tensors are row-major with the last dimension contiguous; matrices are stored
  *    [out_features][in_features].
  *  - Layout of the verifier KV pool (bf16): [n_layers][n_pages_total][2 (K,V)][n_heads]

@@ -156,6 +156,10 @@ __global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const AttnArgs
   const int u = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int R = a.R;
   const int slot = a.slots[b];
+  if (slot < 0 || slot >= a.n_slots) {   // every CTA of the sequence leaves; no ticket, no merge
+    if (u == 0 && h == 0 && threadIdx.x == 0) atomicOr(a.err, ERR_SLOT_RANGE);
+    return;
+  }
   const int sl = a.seq_len[slot];
   const int p0 = sl + a.qoff;
   const int last = p0 + R - 1;

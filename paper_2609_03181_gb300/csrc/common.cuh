@@ -19,7 +19,9 @@ enum : int {
   ERR_PAGE_RANGE = 4,       // a position outside the block table or a page id outside the pool
   ERR_PENDING = 8,          // candidate 0 is not the slot's pending token
   ERR_NO_DRAFT_ROWS = 16,   // draft_step on a slot with no queued rows
-  ERR_POSITION = 32         // a position beyond the RoPE table
+  ERR_POSITION = 32,        // a position beyond the RoPE table
+  ERR_SLOT_RANGE = 64,      // a slot id outside [0, max_batch)
+  ERR_NONFINITE = 128       // a router row with a non-finite probability
 };
 
 // Time limit of every spin on an mbarrier (ns).  A correct pipeline never comes near it.
@@ -204,6 +206,17 @@ __device__ __forceinline__ void warp_argmax(float& v, int& i) {
     int oi = __shfl_xor_sync(0xffffffffu, i, o);
     if (better(ov, oi, v, i)) { v = ov; i = oi; }
   }
+}
+
+// (value, index) as one 64-bit key whose unsigned order is better(): the float's bits mapped
+// to an order-preserving unsigned integer (-0 taken as +0) above the complemented index.
+__device__ __forceinline__ unsigned long long argmax_key(float v, int i) {
+  const uint32_t u = __float_as_uint(v + 0.0f);
+  const uint32_t o = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return (static_cast<unsigned long long>(o) << 32) | static_cast<uint32_t>(~static_cast<uint32_t>(i));
+}
+__device__ __forceinline__ int argmax_key_index(unsigned long long k) {
+  return static_cast<int>(~static_cast<uint32_t>(k & 0xffffffffull));
 }
 
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }

@@ -186,9 +186,7 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
             bv = am_s_val[w * 16 + row];
             bi = am_s_idx[w * 16 + row];
           }
-        const size_t o = static_cast<size_t>(it.n_tile) * a.am_ld + it.out_row + r;
-        a.am_val[o] = bv;
-        a.am_idx[o] = bi;
+        atomicMax(a.am_key + it.out_row + r, argmax_key(bv, bi));
       }
     }
     named_bar_sync(1, 128);
@@ -468,6 +466,41 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
               v[4 * q4 + 3] = t.w;
             }
             epi_chunk<EPI>(a, it, row, c * 16, v, xchg, am_s_val, am_s_idx);
+          }
+        }
+      }
+    }
+    if constexpr (EPI == EPI_ARGMAX) {
+      if (a.fin_B > 0) {
+        // every CTA's keys are final once the last CTA takes the ticket: it decodes the tokens,
+        // then m = longest prefix r with cand[b][r+1] == v[b][r] (acceptance rule of Sec. 3.1)
+        __threadfence();
+        named_bar_sync(1, 128);
+        const int et = threadIdx.x - 64;
+        if (et == 0) {
+          const int old = atomicAdd(a.am_done, 1);
+          *s_last = (old == static_cast<int>(gridDim.x) - 1) ? 1 : 0;
+          if (*s_last) *a.am_done = 0;
+        }
+        named_bar_sync(1, 128);
+        if (*s_last) {
+          __threadfence();
+          const int T = a.fin_B * a.fin_R;
+          for (int t = et; t < T; t += 128) {
+            const int tok = argmax_key_index(__ldcg(a.am_key + t));
+            a.am_key[t] = 0ull;
+            a.fin_vtok_out[t] = tok;
+            a.fin_vtok_ws[t] = tok;
+          }
+          named_bar_sync(1, 128);
+          for (int b = et; b < a.fin_B; b += 128) {
+            int m = 0;
+            for (int r = 1; r < a.fin_R; ++r) {
+              if (a.fin_cand[b * a.fin_R + r] == a.fin_vtok_ws[b * a.fin_R + r - 1]) m = r;
+              else break;
+            }
+            a.fin_accept_out[b] = m;
+            a.fin_m_ws[b] = m;
           }
         }
       }

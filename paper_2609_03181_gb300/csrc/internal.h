@@ -59,7 +59,7 @@ enum EpiKind : int {
   EPI_QKV = 2,      // RoPE on q/k, q -> fp32 buffer, k/v -> bf16 cache rows
   EPI_SWIGLU = 3,   // tile = 64 gate rows + 64 up rows -> bf16 silu(g)*u
   EPI_SCATTER = 4,  // expert down: out row (token, slot) from the sorted index
-  EPI_ARGMAX = 5    // per-tile (max, argmax) of each column (LM head)
+  EPI_ARGMAX = 5    // running (max, argmax) of each column in a packed key (LM head)
 };
 
 // One work item: weight tile x activation rows.  x = expert | n_tile << 16, y = TMA row of
@@ -88,7 +88,11 @@ struct GemmArgs {
   long long head_stride, v_off; const int* pos; const float2* rope; int max_pos;
   bf16* act; int ld_act;                                      // SWIGLU
   float* y; const int* sorted_tok; const int* sorted_slot;    // SCATTER
-  float* am_val; int* am_idx; int am_ld;                      // ARGMAX partials [n_tile][am_ld]
+  // ARGMAX: am_key[row] = max over tiles of (ordered logit << 32 | ~token) (atomicMax; zero =
+  // empty).  fin_B > 0: the last CTA (ticket am_done) decodes the tokens of fin_B x fin_R rows,
+  // computes the greedy accept lengths and clears the keys.
+  unsigned long long* am_key; int* am_done;
+  int fin_B, fin_R; const int* fin_cand; int* fin_vtok_out; int* fin_vtok_ws; int* fin_accept_out; int* fin_m_ws;
   float* sk_ws; int* sk_tickets;                              // split-K partials / per-tile tickets
   int* err;
 };
@@ -124,6 +128,7 @@ struct AttnArgs {
   int R;                       // queries per sequence
   int qoff;                    // query r of sequence b sits at seq_len[slot] + qoff + r
   const int* slots; const int* seq_len;   // keys at positions < seq_len[slot] are in pages
+  int n_slots;                 // valid slot ids are 0..n_slots-1
   const bf16* pool; int page_size; int n_pages; const int* block_table; int max_pages;
   const bf16* stage;           // keys at positions >= seq_len[slot]: staged row (pos - seq_len)
   long long stage_seq_stride, stage_row_stride, stage_kv_stride;
@@ -139,33 +144,30 @@ cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s);
 
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
-                              float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int* err,
-                              cudaStream_t s);
+                              float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
+                              int* err, cudaStream_t s);
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
 cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
-                          const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s);
+                          const float* bias, bf16* xn, int* idx, float* gate, int* err, cudaStream_t s);
 cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
                            int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
                            unsigned long long* expert_ctr, cudaStream_t s);
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
                            bf16* out, cudaStream_t s);
-cudaError_t argmax_final_launch(int mode, const float* am_val, const int* am_idx, int n_tiles, int am_ld,
-                                int B, int R, const int* cand, int* vtok_out, int* accept_out,
-                                int* m_ws, int* vtok_ws, cudaStream_t s);
 cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots, const int* m_ws, const int* vtok_ws,
                           const int* cand_ws, const bf16* stage, bf16* pool, int L, int n_pages,
                           int page_size, const int* block_table, int max_pages, int* seq_len, int* pending,
                           const bf16* b_ws, bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
-                          int* n_committed, int* err, cudaStream_t s);
+                          int* n_committed, int* tickets, int* err, cudaStream_t s);
 cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len, const int* pending,
                               const int* draft_n, const bf16* draft_b, const int* draft_tok,
                               const bf16* embed, int vocab, const bf16* enorm, const bf16* hnorm, float eps,
                               bf16* dcat, int* pos, long long* kv_rowoff, int* last_row, int page_size,
                               const int* block_table, int max_pages, int n_pages, int* cand, int cand_ld,
-                              int* err, cudaStream_t s);
+                              int n_slots, int* err, cudaStream_t s);
 cudaError_t gather_rows_launch(const float* src, const int* rows, int B, float* dst, cudaStream_t s);
-cudaError_t draft_next_launch(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int B, int k,
-                              int K, const int* slots, const int* seq_len, const bf16* u, const bf16* embed,
+cudaError_t draft_next_launch(unsigned long long* am_key, int vocab, int* err, int B, int k, int K, const int* slots,
+                              int n_slots, const int* seq_len, const bf16* u, const bf16* embed,
                               const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
                               long long* kv_rowoff, long long dstage_seq_stride, int* cand, int cand_ld,
                               cudaStream_t s);

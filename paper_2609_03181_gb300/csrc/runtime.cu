@@ -74,6 +74,7 @@ struct spec_ctx {
   bf16* stage = nullptr;
   float* attn_part = nullptr;
   int* attn_tickets = nullptr;
+  int* commit_tickets = nullptr;
   bf16* attn_out = nullptr;
   int* route_idx = nullptr;
   float* route_gate = nullptr;
@@ -87,8 +88,8 @@ struct spec_ctx {
   bf16* act = nullptr;
   float* y = nullptr;
   bf16* b_ws = nullptr;
-  float* am_val = nullptr;
-  int* am_idx = nullptr;
+  unsigned long long* am_key = nullptr;   // packed (logit, token) per row of the LM head
+  int* am_done = nullptr;                 // CTA ticket of the verify LM head
   int* vtok = nullptr;
   int* m_ws = nullptr;
   int* cand_ws = nullptr;
@@ -120,6 +121,10 @@ struct spec_ctx {
   std::vector<Mark> marks;
   // CUDA graphs: one per distinct call key, replayed on later calls with the same key
   bool use_graphs = true;
+  // FASTMTP_CHECK_LAUNCHES: no graphs, and the stream is synchronised after every launch group
+  // so that a fault or a guard flag is reported with the kernel class that raised it
+  bool check_launches = false;
+  int64_t launch_seq = 0;
   std::vector<CallGraph*> graphs;
   CallGraph* capturing = nullptr;
   int64_t launches[SPEC_K_COUNT] = {};
@@ -160,7 +165,6 @@ GemmArgs base_args(spec_ctx* ctx) {
   g.max_pos = ctx->cfg.max_position;
   g.sk_ws = ctx->sk_ws;
   g.sk_tickets = ctx->sk_tickets;
-  g.am_ld = ctx->Tmax;
   g.err = ctx->d_err;
   return g;
 }
@@ -304,11 +308,29 @@ spec_status run_graphed(spec_ctx* ctx, GraphKey key, F body) {
 
 }  // namespace
 
-#define LAUNCH(cls, nk, call)          \
-  do {                                 \
-    ProfScope ps_(ctx, cls);           \
-    CK(call);                          \
-    ps_.done(nk);                      \
+// Synchronises after one launch group in checking mode and names the group in the error.
+spec_status check_launch(spec_ctx* ctx, int cls, const char* what) {
+  ++ctx->launch_seq;
+  if (!ctx->check_launches || ctx->capturing != nullptr) return SPEC_OK;
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);
+  int flag = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&flag, ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess || flag != 0) {
+    char buf[256];
+    snprintf(buf, sizeof(buf), "launch %lld (class %d: %s): %s, guard flag 0x%x",
+             static_cast<long long>(ctx->launch_seq), cls, what, cudaGetErrorString(e), flag);
+    return fail(ctx, e != cudaSuccess ? SPEC_ECUDA : SPEC_EDEVICE, buf);
+  }
+  return SPEC_OK;
+}
+
+#define LAUNCH(cls, nk, call)                             \
+  do {                                                    \
+    ProfScope ps_(ctx, cls);                              \
+    CK(call);                                             \
+    ps_.done(nk);                                         \
+    spec_status cs_ = check_launch(ctx, cls, #call);      \
+    if (cs_ != SPEC_OK) return cs_;                       \
   } while (0)
 
 // ============================================================================ init / destroy
@@ -362,7 +384,8 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ctx->w.layers = ctx->layers.data();
   ctx->kv_pool = static_cast<bf16*>(kv_pool);
   ctx->dkv_pool = static_cast<bf16*>(draft_kv_pool);
-  ctx->use_graphs = getenv("FASTMTP_NO_GRAPHS") == nullptr;
+  ctx->check_launches = getenv("FASTMTP_CHECK_LAUNCHES") != nullptr;
+  ctx->use_graphs = getenv("FASTMTP_NO_GRAPHS") == nullptr && !ctx->check_launches;
 
   const int L = c.n_layers;
   ctx->Bmax = c.max_batch;
@@ -397,6 +420,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->stage, sizeof(bf16) * L * Bmax * Rmax * 2 * d);
   add(&ctx->attn_part, sizeof(float) * static_cast<size_t>(Bmax) * kH * ctx->n_chunks * Rmax * (kHD + 2));
   add(&ctx->attn_tickets, sizeof(int) * Bmax * kH);
+  add(&ctx->commit_tickets, sizeof(int) * Bmax);
   add(&ctx->attn_out, sizeof(bf16) * Tmax * d);
   add(&ctx->route_idx, sizeof(int) * L * Tmax * kTopK);
   add(&ctx->route_gate, sizeof(float) * L * Tmax * kTopK);
@@ -410,8 +434,8 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->act, sizeof(bf16) * Tmax * kSlots * kI);
   add(&ctx->y, sizeof(float) * Tmax * kSlots * d);
   add(&ctx->b_ws, sizeof(bf16) * Tmax * d);
-  add(&ctx->am_val, sizeof(float) * ctx->lm_tiles * Tmax);
-  add(&ctx->am_idx, sizeof(int) * ctx->lm_tiles * Tmax);
+  add(&ctx->am_key, sizeof(unsigned long long) * Tmax);
+  add(&ctx->am_done, sizeof(int));
   add(&ctx->vtok, sizeof(int) * Tmax);
   add(&ctx->m_ws, sizeof(int) * Bmax);
   add(&ctx->cand_ws, sizeof(int) * Tmax);
@@ -608,7 +632,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   CK(cudaMemcpyAsync(ctx->cand_ws, cand, sizeof(int) * T, cudaMemcpyDeviceToDevice, s));
   LAUNCH(SPEC_K_EMBED, 1, embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
                        c.vocab, static_cast<const bf16*>(ctx->layers[0].attn_norm), eps, ctx->h, ctx->xn, ctx->pos,
-                       ctx->kv_rowoff, ctx->Rmax, ctx->d_err, s));
+                       ctx->kv_rowoff, ctx->Rmax, ctx->Bmax, ctx->d_err, s));
   const int nmax_grouped = T <= 64 ? 64 : 256;
   for (int l = 0; l < L; ++l) {
     const spec_layer_weights& W = ctx->layers[l];
@@ -633,6 +657,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       a.qoff = 0;
       a.slots = slots;
       a.seq_len = ctx->seq_len;
+      a.n_slots = ctx->Bmax;
       a.pool = ctx->kv_pool + l * pool_layer;
       a.page_size = c.page_size;
       a.n_pages = c.n_pages_total;
@@ -660,7 +685,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
     int* ridx = ctx->route_idx + static_cast<size_t>(l) * ctx->Tmax * kTopK;
     float* rgate = ctx->route_gate + static_cast<size_t>(l) * ctx->Tmax * kTopK;
     LAUNCH(SPEC_K_ROUTER, 1, router_launch(ctx->h, T, static_cast<const bf16*>(W.moe_norm), eps, static_cast<const bf16*>(W.router),
-                     W.router_bias, ctx->xn, ridx, rgate, s));
+                     W.router_bias, ctx->xn, ridx, rgate, ctx->d_err, s));
     LAUNCH(SPEC_K_PERMUTE, 1, permute_launch(ridx, T, ctx->xn, ctx->x_sorted, ctx->sorted_tok, ctx->sorted_slot,
                                               ctx->items_gu, ctx->items_dn, ctx->n_items, ctx->counts + l * kE,
                                               ctx->d_expert_ctr, s));
@@ -712,11 +737,16 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   // LM head + argmax (logits never leave the SM) + greedy accept
   {
     GemmArgs g = base_args(ctx);
-    g.am_val = ctx->am_val;
-    g.am_idx = ctx->am_idx;
+    g.am_key = ctx->am_key;
+    g.am_done = ctx->am_done;
+    g.fin_B = B;
+    g.fin_R = R;
+    g.fin_cand = ctx->cand_ws;
+    g.fin_vtok_out = verifier_tokens;
+    g.fin_vtok_ws = ctx->vtok;
+    g.fin_accept_out = accept_len;
+    g.fin_m_ws = ctx->m_ws;
     LAUNCH(SPEC_K_LMHEAD, 1, run_dense(ctx, g, EPI_ARGMAX, ctx->lm, ctx->a_b, c.vocab, kD, T, false));
-    LAUNCH(SPEC_K_ARGMAX, 1, argmax_final_launch(0, ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, R, ctx->cand_ws,
-                           verifier_tokens, accept_len, ctx->m_ws, ctx->vtok, s));
   }
     return SPEC_OK;
   });
@@ -742,7 +772,7 @@ extern "C" spec_status accept_commit(spec_ctx* ctx, int32_t B, const int32_t* sl
   LAUNCH(SPEC_K_COMMIT, 1, commit_launch(B, ctx->last_K + 1, ctx->Rmax, ctx->Bmax, slots, ctx->m_ws, ctx->vtok, ctx->cand_ws, ctx->stage,
                    ctx->kv_pool, c.n_layers, c.n_pages_total, c.page_size, ctx->block_table, c.max_pages_per_seq,
                    ctx->seq_len, ctx->pending, ctx->b_ws, ctx->draft_b, ctx->draft_tok, ctx->draft_n, committed,
-                   n_committed, ctx->d_err, ctx->stream));
+                   n_committed, ctx->commit_tickets, ctx->d_err, ctx->stream));
     return SPEC_OK;
   });
   if (st != SPEC_OK) return st;
@@ -769,7 +799,8 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
   LAUNCH(SPEC_K_DRAFT_MISC, 1, draft_prep_launch(B, Rm, slots, ctx->seq_len, ctx->pending, ctx->draft_n, ctx->draft_b, ctx->draft_tok,
                        static_cast<const bf16*>(ctx->w.embed), c.vocab, static_cast<const bf16*>(ctx->w.enorm),
                        static_cast<const bf16*>(ctx->w.hnorm), eps, ctx->dcat, ctx->pos, ctx->kv_rowoff, ctx->last_row,
-                       c.page_size, ctx->block_table, c.max_pages_per_seq, c.n_pages_total, cand, ld, ctx->d_err, s));
+                       c.page_size, ctx->block_table, c.max_pages_per_seq, c.n_pages_total, cand, ld, ctx->Bmax,
+                       ctx->d_err, s));
   {
     GemmArgs g = base_args(ctx);
     g.out = ctx->z;
@@ -813,6 +844,7 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       a.qoff = (k == 1) ? -1 : k - 2;
       a.slots = slots;
       a.seq_len = ctx->seq_len;
+      a.n_slots = ctx->Bmax;
       a.pool = ctx->dkv_pool;
       a.page_size = c.page_size;
       a.n_pages = c.n_pages_total;
@@ -853,8 +885,7 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
     LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.final_norm), eps, uk, s));
     {
       GemmArgs g = base_args(ctx);
-      g.am_val = ctx->am_val;
-      g.am_idx = ctx->am_idx;
+      g.am_key = ctx->am_key;
       // rows of depth k start at (k-1) * Bmax in the u buffer
       g.a_map[0] = ctx->lm;
       for (int b = 0; b < 5; ++b) g.b_map[0][b] = ctx->a_u.m[b];
@@ -871,7 +902,7 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
       LAUNCH(SPEC_K_LMHEAD, 1, gemm_launch(EPI_ARGMAX, box <= 64 ? 64 : 256, g, grid, s));
     }
-    LAUNCH(SPEC_K_ARGMAX, 1, draft_next_launch(ctx->am_val, ctx->am_idx, ctx->lm_tiles, ctx->Tmax, B, k, K, slots, ctx->seq_len, uk,
+    LAUNCH(SPEC_K_ARGMAX, 1, draft_next_launch(ctx->am_key, c.vocab, ctx->d_err, B, k, K, slots, ctx->Bmax, ctx->seq_len, uk,
                          static_cast<const bf16*>(ctx->w.embed), static_cast<const bf16*>(ctx->w.enorm),
                          static_cast<const bf16*>(ctx->w.hnorm), eps, ctx->dcat, ctx->pos, ctx->kv_rowoff, dstage_seq,
                          cand, ld, s));
@@ -893,9 +924,9 @@ extern "C" spec_status spec_sync(spec_ctx* ctx) {
   if (flag != 0) {
     const int zero = 0;
     CK(cudaMemcpy(ctx->d_err, &zero, sizeof(int), cudaMemcpyHostToDevice));
-    char buf[160];
+    char buf[256];
     snprintf(buf, sizeof(buf), "device guard flag 0x%x (1 wait timeout, 2 token range, 4 page range, 8 pending "
-             "mismatch, 16 no draft rows, 32 position)", flag);
+             "mismatch, 16 no draft rows, 32 position, 64 slot range, 128 non-finite router row)", flag);
     return fail(ctx, SPEC_EDEVICE, buf);
   }
   return SPEC_OK;

@@ -1,8 +1,7 @@
 // Latency-bound kernels of the FastMTP step: embedding + RMSNorm, RMSNorm, router
 // (norm, logits, softmax, top-6), token permute/scatter by expert, MoE combine (+ the next
-// RMSNorm), the argmax reduction with the greedy-accept epilogue, the KV commit, and the
-// glue of the draft chain.  Every reduction runs in a fixed order, so a row's result never
-// depends on the other rows of the batch.
+// RMSNorm), the KV commit, and the glue of the draft chain.  Every reduction runs in a fixed
+// order, so a row's result never depends on the other rows of the batch.
 #include <math.h>
 
 #include "common.cuh"
@@ -49,18 +48,20 @@ __device__ __forceinline__ void norm_row_store(const float (&x)[10], const bf16*
 __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R, const int* slots, const int* pending,
                                                          const int* seq_len, const bf16* embed, int vocab,
                                                          const bf16* gain, float eps, float* h, bf16* xn, int* pos,
-                                                         long long* kv_rowoff, int stage_R, int* err) {
+                                                         long long* kv_rowoff, int stage_R, int n_slots, int* err) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[4];
   const int row = blockIdx.x, b = row / R, r = row % R;
   const int slot = slots[b];
+  const bool slot_ok = slot >= 0 && slot < n_slots;
+  if (!slot_ok && r == 0 && threadIdx.x == 0) atomicOr(err, ERR_SLOT_RANGE);
   int tok = cand[row];
   if (tok < 0 || tok >= vocab) {
     if (threadIdx.x == 0) atomicOr(err, ERR_TOKEN_RANGE);
     tok = 0;
   }
-  if (r == 0 && tok != pending[slot] && threadIdx.x == 0) atomicOr(err, ERR_PENDING);
+  if (slot_ok && r == 0 && tok != pending[slot] && threadIdx.x == 0) atomicOr(err, ERR_PENDING);
   const bf16* e = embed + static_cast<size_t>(tok) * kD;
   float x[10];
 #pragma unroll
@@ -71,17 +72,17 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
   }
   norm_row_store(x, gain, eps, xn + static_cast<size_t>(row) * kD, red);
   if (threadIdx.x == 0) {
-    pos[row] = seq_len[slot] + r;
+    pos[row] = (slot_ok ? seq_len[slot] : 0) + r;
     kv_rowoff[row] = static_cast<long long>(b * stage_R + r) * 2 * kH * kHD;
   }
 }
 
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
-                              float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int* err,
-                              cudaStream_t s) {
-  return launch_pdl(embed_norm_kernel, dim3(B * R), dim3(128), 0, s, cand, R, slots, pending, seq_len, embed, vocab, gain, eps, h, xn, pos,
-                                           kv_rowoff, stage_R, err);
+                              float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
+                              int* err, cudaStream_t s) {
+  return launch_pdl(embed_norm_kernel, dim3(B * R), dim3(128), 0, s, cand, R, slots, pending, seq_len, embed, vocab, gain,
+                    eps, h, xn, pos, kv_rowoff, stage_R, n_slots, err);
 }
 
 // ---------------------------------------------------------------- RMSNorm
@@ -105,7 +106,7 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
 // RMSNorm of the residual row -> xn (bf16, also the experts' input); logits of the 64
 // experts from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).
 __global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16* gain, float eps, const bf16* wr,
-                                                     const float* bias, bf16* xn, int* idx, float* gate) {
+                                                     const float* bias, bf16* xn, int* idx, float* gate, int* err) {
   pdl_trigger();
   pdl_wait();
   constexpr int NT = 256, EPT = kD / NT;
@@ -162,6 +163,13 @@ __global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16*
     const float e0 = expf(l0 - m), e1 = expf(l1 - m);
     const float sum = warp_sum(e0 + e1);
     float p0 = e0 / sum, p1 = e1 / sum;
+    // a non-finite row still selects six distinct valid experts (NaN ranks below every number)
+    const bool bad = __any_sync(0xffffffffu, !(p0 == p0) || !(p1 == p1));
+    if (bad) {
+      if (lane == 0) atomicOr(err, ERR_NONFINITE);
+      if (!(p0 == p0)) p0 = -1.f;
+      if (!(p1 == p1)) p1 = -1.f;
+    }
     bool taken0 = false, taken1 = false;
     for (int k = 0; k < kTopK; ++k) {
       float bv = -1.f;
@@ -180,8 +188,8 @@ __global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16*
 }
 
 cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
-                          const float* bias, bf16* xn, int* idx, float* gate, cudaStream_t s) {
-  return launch_pdl(router_kernel, dim3(T), dim3(256), 0, s, h, gain, eps, w_router, bias, xn, idx, gate);
+                          const float* bias, bf16* xn, int* idx, float* gate, int* err, cudaStream_t s) {
+  return launch_pdl(router_kernel, dim3(T), dim3(256), 0, s, h, gain, eps, w_router, bias, xn, idx, gate, err);
 }
 
 // ---------------------------------------------------------------- permute / scatter
@@ -347,76 +355,36 @@ cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, c
   return launch_pdl(combine_kernel, dim3(T), dim3(256), 0, s, h, y, gate, gain, eps, out);
 }
 
-// ---------------------------------------------------------------- argmax + greedy accept
-// Row (b, r) of the verify batch: v = argmax over the LM-head tile partials (value, lower
-// id on ties).  Then m = longest prefix r with cand[b][r+1] == v[b][r] (acceptance equation
-// of Sec. 3.1).
-__device__ __forceinline__ void reduce_partials(const float* am_val, const int* am_idx, int n_tiles, int am_ld,
-                                                int row, float& bv, int& bi) {
-  const int lane = threadIdx.x & 31;
-  bv = -INFINITY;
-  bi = 0x7fffffff;
-  for (int t = lane; t < n_tiles; t += 32) {
-    const float v = am_val[static_cast<size_t>(t) * am_ld + row];
-    const int i = am_idx[static_cast<size_t>(t) * am_ld + row];
-    if (better(v, i, bv, bi)) { bv = v; bi = i; }
-  }
-  warp_argmax(bv, bi);
-}
-
-__global__ void argmax_accept_kernel(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int R,
-                                     const int* cand, int* vtok_out, int* accept_out, int* m_ws, int* vtok_ws) {
-  pdl_trigger();
-  pdl_wait();
-  __shared__ int sv[kMaxR];
-  const int b = blockIdx.x, r = threadIdx.x >> 5;
-  float bv;
-  int bi;
-  reduce_partials(am_val, am_idx, n_tiles, am_ld, b * R + r, bv, bi);
-  if ((threadIdx.x & 31) == 0) {
-    sv[r] = bi;
-    vtok_out[b * R + r] = bi;
-    vtok_ws[b * R + r] = bi;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int m = 0;
-    for (int s = 1; s < R; ++s) {
-      if (cand[b * R + s] == sv[s - 1]) m = s;
-      else break;
-    }
-    accept_out[b] = m;
-    m_ws[b] = m;
-  }
-}
-
-cudaError_t argmax_final_launch(int mode, const float* am_val, const int* am_idx, int n_tiles, int am_ld, int B,
-                                int R, const int* cand, int* vtok_out, int* accept_out, int* m_ws, int* vtok_ws,
-                                cudaStream_t s) {
-  (void)mode;
-  return launch_pdl(argmax_accept_kernel, dim3(B), dim3(32 * R), 0, s, am_val, am_idx, n_tiles, am_ld, R, cand, vtok_out, accept_out, m_ws,
-                                             vtok_ws);
-}
-
 // ---------------------------------------------------------------- KV commit
 // Appends the staged K/V of candidates 0..m of each sequence to its pages (16-byte
 // vectors), advances the slot, writes the committed tokens and queues the m+1 new rows
 // (base states b and next tokens) for the draft head.  The rejected tail stays in the
-// staging buffer and is overwritten by the next verify.
+// staging buffer and is overwritten by the next verify.  One CTA per (sequence, layer); the
+// last CTA of a sequence to finish its copies (atomic ticket) updates the sequence's state,
+// after every CTA of that sequence has read the old length.
 __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bmax, const int* slots, const int* m_ws,
                                                      const int* vtok, const int* cand, const bf16* stage, bf16* pool,
                                                      int L, int n_pages, int page_size, const int* block_table,
                                                      int max_pages, int* seq_len, int* pending, const bf16* b_ws,
                                                      bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
-                                                     int* n_committed, int* err) {
+                                                     int* n_committed, int* tickets, int* err) {
   pdl_trigger();
   pdl_wait();
-  const int b = blockIdx.x, slot = slots[b];
-  const int m = m_ws[b];
+  __shared__ int s_last;
+  const int b = blockIdx.x, l = blockIdx.y, slot = slots[b];
+  if (slot < 0 || slot >= Bmax) {   // every CTA of the sequence skips it, none takes the ticket
+    if (threadIdx.x == 0 && l == 0) atomicOr(err, ERR_SLOT_RANGE);
+    return;
+  }
+  int m = m_ws[b];
+  if (m < 0 || m >= R) {   // an accept length the verify cannot produce: flag it, commit the bonus only
+    if (threadIdx.x == 0 && l == 0) atomicOr(err, ERR_TOKEN_RANGE);
+    m = 0;
+  }
   const int c = seq_len[slot];
   constexpr int kVec = kHD / 8;   // 16-byte vectors per head row
   constexpr int kBatch = 8;       // copies whose loads are issued before their stores
-  const int total = (m + 1) * L * 2 * kH * kVec;
+  const int total = (m + 1) * 2 * kH * kVec;
   for (int v0 = threadIdx.x; v0 < total; v0 += blockDim.x * kBatch) {
     uint4 val[kBatch];
     uint4* dst[kBatch];
@@ -428,9 +396,8 @@ __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bma
       int t = v;
       const int vec = t % kVec; t /= kVec;
       const int h = t % kH; t /= kH;
-      const int kv = t % 2; t /= 2;
-      const int l = t % L;
-      const int r = t / L;
+      const int kv = t % 2;
+      const int r = t / 2;
       const int pos = c + r;
       const int pi = pos / page_size;
       const int page = (pi < max_pages) ? block_table[slot * max_pages + pi] : -1;
@@ -448,13 +415,19 @@ __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bma
     for (int u = 0; u < kBatch; ++u)
       if (dst[u] != nullptr) *dst[u] = val[u];
   }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(&tickets[b], 1) == L - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
   // queue the new rows for the draft head: b_p and x_{p+1}
   for (int v = threadIdx.x; v < (m + 1) * (kD / 8); v += blockDim.x) {
     const int r = v / (kD / 8), c8 = v % (kD / 8);
     reinterpret_cast<uint4*>(draft_b + (static_cast<size_t>(slot) * kMaxR + r) * kD)[c8] =
         reinterpret_cast<const uint4*>(b_ws + static_cast<size_t>(b * R + r) * kD)[c8];
   }
-  __syncthreads();
   if (threadIdx.x < R) {
     const int r = threadIdx.x;
     const int tok = (r < m) ? cand[b * R + r + 1] : (r == m ? vtok[b * R + m] : -1);
@@ -462,6 +435,7 @@ __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bma
     if (r <= m) draft_tok[slot * kMaxR + r] = tok;
   }
   if (threadIdx.x == 0) {
+    tickets[b] = 0;
     n_committed[b] = m + 1;
     pending[slot] = vtok[b * R + m];
     seq_len[slot] = c + m + 1;
@@ -473,10 +447,10 @@ cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots,
                           const int* vtok_ws, const int* cand_ws, const bf16* stage, bf16* pool, int L, int n_pages,
                           int page_size, const int* block_table, int max_pages, int* seq_len, int* pending,
                           const bf16* b_ws, bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
-                          int* n_committed, int* err, cudaStream_t s) {
-  return launch_pdl(commit_kernel, dim3(B), dim3(256), 0, s, R, stage_R, Bmax, slots, m_ws, vtok_ws, cand_ws, stage, pool, L,
-                                   n_pages, page_size, block_table, max_pages, seq_len, pending, b_ws, draft_b,
-                                   draft_tok, draft_n, committed, n_committed, err);
+                          int* n_committed, int* tickets, int* err, cudaStream_t s) {
+  return launch_pdl(commit_kernel, dim3(B, L), dim3(256), 0, s, R, stage_R, Bmax, slots, m_ws, vtok_ws, cand_ws, stage,
+                    pool, L, n_pages, page_size, block_table, max_pages, seq_len, pending, b_ws, draft_b, draft_tok,
+                    draft_n, committed, n_committed, tickets, err);
 }
 
 // ---------------------------------------------------------------- draft glue
@@ -489,19 +463,23 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
                                                          const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat,
                                                          int* pos, long long* kv_rowoff, int* last_row, int page_size,
                                                          const int* block_table, int max_pages, int n_pages, int* cand,
-                                                         int cand_ld, int* err) {
+                                                         int cand_ld, int n_slots, int* err) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[4];
   const int b = blockIdx.x / R, i = blockIdx.x % R, row = blockIdx.x;
-  const int slot = slots[b];
-  int n = draft_n[slot];
-  if (n < 1 || n > kMaxR) {
+  int slot = slots[b];
+  if (slot < 0 || slot >= n_slots) {   // treated as a slot with no queued rows
+    if (threadIdx.x == 0 && i == 0) atomicOr(err, ERR_SLOT_RANGE);
+    slot = -1;
+  }
+  int n = slot >= 0 ? draft_n[slot] : 0;
+  if (slot >= 0 && (n < 1 || n > kMaxR)) {
     if (threadIdx.x == 0 && i == 0) atomicOr(err, ERR_NO_DRAFT_ROWS);
     n = 0;
   }
   if (i == 0 && threadIdx.x == 0) {
-    cand[b * cand_ld] = pending[slot];
+    cand[b * cand_ld] = slot >= 0 ? pending[slot] : 0;
     last_row[b] = b * R + (n > 0 ? n - 1 : 0);
   }
   bf16* out = dcat + static_cast<size_t>(row) * 2 * kD;
@@ -544,10 +522,11 @@ cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len
                               const int* draft_n, const bf16* draft_b, const int* draft_tok, const bf16* embed,
                               int vocab, const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
                               long long* kv_rowoff, int* last_row, int page_size, const int* block_table,
-                              int max_pages, int n_pages, int* cand, int cand_ld, int* err, cudaStream_t s) {
-  return launch_pdl(draft_prep_kernel, dim3(B * R), dim3(128), 0, s, R, slots, seq_len, pending, draft_n, draft_b, draft_tok, embed, vocab,
-                                           enorm, hnorm, eps, dcat, pos, kv_rowoff, last_row, page_size, block_table,
-                                           max_pages, n_pages, cand, cand_ld, err);
+                              int max_pages, int n_pages, int* cand, int cand_ld, int n_slots, int* err,
+                              cudaStream_t s) {
+  return launch_pdl(draft_prep_kernel, dim3(B * R), dim3(128), 0, s, R, slots, seq_len, pending, draft_n, draft_b,
+                    draft_tok, embed, vocab, enorm, hnorm, eps, dcat, pos, kv_rowoff, last_row, page_size, block_table,
+                    max_pages, n_pages, cand, cand_ld, n_slots, err);
 }
 
 __global__ void gather_rows_kernel(const float* src, const int* rows, float* dst) {
@@ -563,28 +542,30 @@ cudaError_t gather_rows_launch(const float* src, const int* rows, int B, float* 
   return launch_pdl(gather_rows_kernel, dim3(B), dim3(128), 0, s, src, rows, dst);
 }
 
-// After the LM head of depth k: x^_k = argmax; for k < K the inputs of depth k+1:
-// dcat = [N_e(E x^_k); N_h(u^(k))], position p = j + k (j = ctx_len - 1) and the staging
-// row k-1 of its tentative draft K/V.
-__global__ void __launch_bounds__(128) draft_next_kernel(const float* am_val, const int* am_idx, int n_tiles, int am_ld,
-                                                         int k, int K, const int* slots, const int* seq_len,
-                                                         const bf16* u, const bf16* embed, const bf16* enorm,
-                                                         const bf16* hnorm, float eps, bf16* dcat, int* pos,
-                                                         long long* kv_rowoff, long long dstage_seq_stride, int* cand,
-                                                         int cand_ld) {
+// After the LM head of depth k: x^_k = argmax (decoded from the LM head's packed key, which
+// is cleared for the next use); for k < K the inputs of depth k+1: dcat = [N_e(E x^_k);
+// N_h(u^(k))], position p = j + k (j = ctx_len - 1) and the staging row k-1 of its tentative
+// draft K/V.
+__global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_key, int vocab, int* err, int k, int K,
+                                                         const int* slots, int n_slots,
+                                                         const int* seq_len, const bf16* u, const bf16* embed,
+                                                         const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat,
+                                                         int* pos, long long* kv_rowoff, long long dstage_seq_stride,
+                                                         int* cand, int cand_ld) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[4];
   __shared__ int s_tok;
   const int b = blockIdx.x;
-  if (threadIdx.x < 32) {
-    float bv;
-    int bi;
-    reduce_partials(am_val, am_idx, n_tiles, am_ld, b, bv, bi);
-    if (threadIdx.x == 0) {
-      s_tok = bi;
-      cand[b * cand_ld + k] = bi;
+  if (threadIdx.x == 0) {
+    int tok = argmax_key_index(am_key[b]);
+    am_key[b] = 0ull;
+    if (tok < 0 || tok >= vocab) {   // no logit reached this row
+      atomicOr(err, ERR_TOKEN_RANGE);
+      tok = 0;
     }
+    s_tok = tok;
+    cand[b * cand_ld + k] = tok;
   }
   __syncthreads();
   if (k >= K) return;
@@ -598,18 +579,21 @@ __global__ void __launch_bounds__(128) draft_next_kernel(const float* am_val, co
   for (int q = 0; q < 10; ++q) x[q] = __bfloat162float(u[static_cast<size_t>(b) * kD + threadIdx.x + 128 * q]);
   norm_row_store(x, hnorm, eps, out + kD, red);
   if (threadIdx.x == 0) {
-    pos[b] = seq_len[slots[b]] + k - 1;
+    const int slot = slots[b];
+    const bool slot_ok = slot >= 0 && slot < n_slots;
+    if (!slot_ok) atomicOr(err, ERR_SLOT_RANGE);
+    pos[b] = (slot_ok ? seq_len[slot] : 0) + k - 1;
     kv_rowoff[b] = b * dstage_seq_stride + static_cast<long long>(k - 1) * 2 * kH * kHD;
   }
 }
 
-cudaError_t draft_next_launch(const float* am_val, const int* am_idx, int n_tiles, int am_ld, int B, int k, int K,
-                              const int* slots, const int* seq_len, const bf16* u, const bf16* embed,
-                              const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat, int* pos,
-                              long long* kv_rowoff, long long dstage_seq_stride, int* cand, int cand_ld,
-                              cudaStream_t s) {
-  return launch_pdl(draft_next_kernel, dim3(B), dim3(128), 0, s, am_val, am_idx, n_tiles, am_ld, k, K, slots, seq_len, u, embed, enorm, hnorm,
-                                       eps, dcat, pos, kv_rowoff, dstage_seq_stride, cand, cand_ld);
+cudaError_t draft_next_launch(unsigned long long* am_key, int vocab, int* err, int B, int k, int K, const int* slots,
+                              int n_slots, const int* seq_len,
+                              const bf16* u, const bf16* embed, const bf16* enorm, const bf16* hnorm, float eps,
+                              bf16* dcat, int* pos, long long* kv_rowoff, long long dstage_seq_stride, int* cand,
+                              int cand_ld, cudaStream_t s) {
+  return launch_pdl(draft_next_kernel, dim3(B), dim3(128), 0, s, am_key, vocab, err, k, K, slots, n_slots, seq_len, u, embed, enorm, hnorm,
+                    eps, dcat, pos, kv_rowoff, dstage_seq_stride, cand, cand_ld);
 }
 
 }  // namespace fm

@@ -80,3 +80,27 @@ def test_device_guard_flags_and_recovery(eng):
     eng.accept_commit(slots, torch.empty(2, 2, dtype=torch.int32, device="cuda"), acc)
     eng.sync()
     assert eng.seq_state(0)[0] == 50 + int(acc[0])
+
+
+def test_slot_id_out_of_range_sets_guard_flag(eng):
+    """A slot id in the device slots array outside [0, max_batch) is caught by every kernel that
+    indexes by slot: its sequence is skipped (no page, state or staging access) and the flag
+    reads 64; the valid sequence of the same call is still committed."""
+    dev = torch.device("cuda")
+    for b in range(2):
+        eng.load_prefix(b, S.kv_prefix(9, b, 1, 50, 10, 128), S.draft_kv_prefix(9, b, 50, 10, 128), 7)
+    bad = torch.tensor([0, 1 << 20], dtype=torch.int32, device=dev)
+    vt = torch.empty(2, 2, dtype=torch.int32, device=dev)
+    acc = torch.empty(2, dtype=torch.int32, device=dev)
+    eng.verify_step(bad, torch.tensor([[7, 1], [7, 2]], dtype=torch.int32, device=dev), vt, acc)
+    eng.accept_commit(bad, torch.empty(2, 2, dtype=torch.int32, device=dev), acc)
+    with pytest.raises(F.FastMTPError) as e:
+        eng.sync()
+    assert e.value.status == F.SPEC_EDEVICE and "0x40" in str(e.value)
+    assert eng.seq_state(0)[0] == 50 + int(acc[0])
+    assert eng.seq_state(1)[0] == 50
+    # the draft head's kernels check the same ids
+    eng.draft_step(bad, 1, torch.empty(2, 2, dtype=torch.int32, device=dev))
+    with pytest.raises(F.FastMTPError) as e:
+        eng.sync()
+    assert "0x40" in str(e.value) or "0x50" in str(e.value)

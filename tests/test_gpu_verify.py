@@ -16,16 +16,24 @@ from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, ind
 pytestmark = pytest.mark.gpu
 
 
-def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
+def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None):
+    """One verify_step + accept_commit of len(ctx_lens) sequences on the GPU; the sequences in
+    `check` (default: all) are compared with the oracle, the others get uniform random drafts and
+    only fill the batch.  Returns (tokens compared, tokens skipped below the margin)."""
     B = len(ctx_lens)
+    check = list(range(B)) if check is None else list(check)
     vw = S.verifier_weights(shape, seed, gain_std=gain_std)
     dw = S.draft_weights(shape, seed, gain_std=gain_std)
     model = O.Verifier(vw)
     kvs, dkvs = seq_prefixes(shape, seed, ctx_lens)
     pend = S.integers(seed, "pending", B, 0, shape.vocab - 1)
-    caches = [O.SeqCache.from_prefix(kvs[b], int(pend[b])) for b in range(B)]
-    cand = make_drafts(model, caches, K, seed)
-    ref = O.verify(model, caches, cand, rb=True)
+    caches = [O.SeqCache.from_prefix(kvs[b], int(pend[b])) for b in check]
+    cand_chk = make_drafts(model, caches, K, seed)
+    other = S.integers(seed, "draft.other", B * K, 0, shape.vocab - 1).reshape(B, K)
+    cand = [[int(pend[b])] + [int(t) for t in other[b]] for b in range(B)]
+    for j, b in enumerate(check):
+        cand[b] = cand_chk[j]
+    ref = O.verify(model, caches, cand_chk, rb=True)
 
     eng = F.Engine(vw, dw, max_batch=B, K_max=max(K, 3), max_ctx=max(ctx_lens) + 8, page_size=64)
     for b in range(B):
@@ -37,9 +45,11 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
     acc = torch.empty(B, dtype=torch.int32, device=dev)
     eng.verify_step(slots, cand_d, vt, acc)
     eng.sync()
-    T = B * (K + 1)
     R = K + 1
-    b_gpu = eng.read_workspace(F.WS_B, (T, shape.hidden), torch.bfloat16)
+    rows = [b * R + r for b in check for r in range(R)]   # GPU rows of the checked sequences
+    T = len(rows)
+    b_all = eng.read_workspace(F.WS_B, (B * R, shape.hidden), torch.bfloat16)
+    b_gpu = b_all[rows]
     ridx = eng.read_workspace(F.WS_ROUTE_IDX, (shape.n_layers, eng.max_batch * (eng.K_max + 1), shape.top_k),
                               torch.int32)
     # Routing: bit-exact wherever the oracle's 6th/7th probability margin exceeds 1e-3.  A row
@@ -48,7 +58,7 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
     # attend to its K/V); such rows are counted.
     diverged = np.zeros(T, dtype=bool)
     for l in range(shape.n_layers):
-        g = np.sort(ridx[l, :T].numpy(), -1)
+        g = np.sort(ridx[l, rows].numpy(), -1)
         r = np.sort(ref.route_idx[l].numpy(), -1)
         live = ~diverged
         n_ok, n_skip, n_bad = index_parity(g[live], r[live], ref.route_gap[l].numpy()[live])
@@ -70,13 +80,13 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
     margin = argmax_margin(vw.lm_head, b_gpu, ref.b.reshape(T, -1))
     gaps = ref.v_gap.numpy().reshape(-1)
     sure = keep & (gaps > margin)
-    g_tok, r_tok = vt.cpu().numpy().reshape(-1), ref.v.numpy().reshape(-1)
+    g_tok, r_tok = vt.cpu().numpy()[check].reshape(-1), ref.v.numpy().reshape(-1)
     assert (g_tok[sure] == r_tok[sure]).all(), (
         f"token mismatch at rows {np.nonzero(sure & (g_tok != r_tok))[0].tolist()}")
-    for bb in range(B):
-        rows = slice(bb * R, bb * R + K)
-        if sure[rows].all():
-            assert int(acc[bb]) == ref.m[bb]
+    for j, bb in enumerate(check):
+        rr = slice(j * R, j * R + K)
+        if sure[rr].all():
+            assert int(acc[bb]) == ref.m[j]
 
     committed = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
     ncom = torch.empty(B, dtype=torch.int32, device=dev)
@@ -90,19 +100,21 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1):
         assert toks[:m + 1] == cand[b][1:m + 1] + [int(vt[b, m])] and all(t == -1 for t in toks[m + 1:])
         ln, pending = eng.seq_state(b)
         assert ln == ctx_lens[b] + m + 1 and pending == int(vt[b, m])
+    for j, b in enumerate(check):
+        m = int(acc[b])
         bt = eng.block_table(b)
-        if m != ref.m[b]:
+        if m != ref.m[j]:
             continue
         for l in range(shape.n_layers):
             for r in range(m + 1):
-                if diverged[b * R + r]:
+                if diverged[j * R + r]:
                     continue
                 p = ctx_lens[b] + r
                 page, off = bt[p // ps], p % ps
                 k_gpu = eng.kv_pool[l, page, 0, :, off, :].cpu()
                 v_gpu = eng.kv_pool[l, page, 1, :, off, :].cpu()
-                assert rel_err(k_gpu, ref.new_k[b][l][r]) < REL_TOL
-                assert rel_err(v_gpu, ref.new_v[b][l][r]) < REL_TOL
+                assert rel_err(k_gpu, ref.new_k[j][l][r]) < REL_TOL
+                assert rel_err(v_gpu, ref.new_v[j][l][r]) < REL_TOL
     eng.close()
     return int(sure.sum()), int((~sure).sum())
 
@@ -122,3 +134,12 @@ def test_verify_twelve_layers_cfg1():
     shape = S.ModelShape()
     ctx = [int(c) for c in S.integers(1, "ctx", 8, 768, 1024)]
     run_verify_case(shape, 1, ctx, K=3, gain_std=0.0)
+
+
+def test_verify_max_batch_256():
+    """The largest batch of the throughput sweep, B=256 (T=1024 candidate rows, four 256-row
+    GEMM tiles per weight tile): 16 sequences spread over the batch are checked against the
+    oracle."""
+    shape = S.ModelShape(n_layers=1, vocab=4096)
+    ctx = [int(c) for c in S.integers(9, "ctx", 256, 1, 160)]
+    run_verify_case(shape, 9, ctx, K=3, check=range(3, 256, 16))
