@@ -60,6 +60,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--weights", default="successor", choices=["successor", "random"],
                    help="successor: acceptance-tuned seeded weights (tau ~2.7); random: N(0,0.02) everywhere")
+    p.add_argument("--device-kv", action="store_true",
+                   help="draw the KV prefixes on the GPU (PyTorch's generator) instead of the host Philox stream")
     p.add_argument("--sweep", action="store_true", help="run the (batch, context, K, router) grid")
     p.add_argument("--sweep-batch", default="1,4,16,64,256")
     p.add_argument("--sweep-ctx", default="1024,4096,8192")
@@ -97,9 +99,16 @@ def workload(args, rank=0):
     B = args.batch
     ctx = [int(c) for c in S.integers(seed + 1000 * rank, "ctx", B, args.ctx_lo, args.ctx_hi)]
     pend = [int(t) for t in S.integers(seed + 1000 * rank, "pending", B, 0, shape.vocab - 1)]
-    kvs = [S.kv_prefix(seed + 1000 * rank, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim)
-           for b in range(B)]
-    dkvs = [S.draft_kv_prefix(seed + 1000 * rank, b, ctx[b], shape.n_heads, shape.head_dim) for b in range(B)]
+    if args.device_kv:
+        dev = f"cuda:{int(os.environ.get('LOCAL_RANK', '0'))}"
+        kvs = [S.kv_prefix_device(seed + 1000 * rank, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim, dev)
+               for b in range(B)]
+        dkvs = [S.draft_kv_prefix_device(seed + 1000 * rank, b, ctx[b], shape.n_heads, shape.head_dim, dev)
+                for b in range(B)]
+    else:
+        kvs = [S.kv_prefix(seed + 1000 * rank, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim)
+               for b in range(B)]
+        dkvs = [S.draft_kv_prefix(seed + 1000 * rank, b, ctx[b], shape.n_heads, shape.head_dim) for b in range(B)]
     return shape, vw, dw, ctx, pend, kvs, dkvs
 
 
@@ -183,8 +192,8 @@ class OracleRunner:
         self.K = args.K
         self.model = O.Verifier(vw)
         self.dr = O.Drafter(dw, self.model)
-        self.cache = O.SeqCache.from_prefix(kvs[0], pend[0])
-        self.dcache = O.DraftCache.from_prefix(dkvs[0])
+        self.cache = O.SeqCache.from_prefix(kvs[0].cpu(), pend[0])
+        self.dcache = O.DraftCache.from_prefix(dkvs[0].cpu())
         vo = O.verify(self.model, [self.cache], [[self.cache.pending]], rb=True)
         O.commit([self.cache], vo, [[self.cache.pending]], [self.dcache])
 

@@ -3,20 +3,29 @@
 // Each sequence has R queries at consecutive positions p0..p0+R-1 (the K+1 verify
 // candidates, or one draft row).  Keys at positions < ctx_len live in the sequence's pages,
 // keys at positions >= ctx_len in a staging buffer (candidates not yet committed).  The key
-// range is cut into chunks of 64 positions fixed by absolute position.  For each chunk and
-// query the kernel forms (max, sum, unnormalised output) of the chunk's softmax terms; a query's
-// result is the chunk-ordered merge of its chunks.  Scores K q^T and outputs V^T p^T run on
-// bf16 tensor cores (mma.sync m16n8k16, fp32 accumulation, queries padded to 8; p enters as a
-// sum of two bf16 terms so the product keeps about 16 bits of it).
+// range is cut into chunks of 64 positions and super-chunks of 4 chunks (256 positions), both
+// fixed by absolute position.
 //
-// Scheduling: one CTA per (unit of consecutive chunks, head, sequence); it resolves the
-// page offsets of all its keys at once, then streams its chunks through two shared-memory
-// stages (16-byte cp.async), computing one chunk while the next is in flight.  The CTA that
-// finishes the last unit of a (sequence, head) merges (atomic ticket, no wait).  Masked keys
-// contribute exact zeros and the chunk grouping does not enter the arithmetic, so a query's
-// result is the same whether its keys sit in pages or in staging and however many queries or
-// sequences share the launch: greedy decoding (K = 0) and speculative verification see
-// identical rows.
+// Arithmetic (fixed by position, never by the launch shape): a super-chunk's chunks are
+// folded in chunk order by the online softmax (running max M, sum L and unnormalised output O
+// per query, rescaled by 2^(M_old - M_new) when the max grows); a query's result is the merge
+// of its super-chunks in order, O = sum_s w_s O_s / sum_s w_s L_s with w_s = 2^(M_s - max M).
+// Scores K q^T and outputs V^T p^T run on bf16 tensor cores (mma.sync m16n8k16, fp32
+// accumulation, queries padded to 8); p enters the product as two bf16 terms (hi + lo, about
+// 16 bits); the transposes between the score and the product layouts stay in registers
+// (movmatrix).  Masked keys contribute exact zeros, so a query's result is the same whether
+// its keys sit in pages or in staging and however many queries or sequences share the launch:
+// greedy decoding (K = 0) and speculative verification see identical rows.
+//
+// Scheduling: one warp per CTA, two CTAs per SM.  A CTA owns a unit of consecutive
+// super-chunks of one (sequence, head) and streams its chunks through three private shared-
+// memory stages.  A chunk whose 64 keys are all committed is one page segment per head: its K
+// and V rows are two contiguous 16 KB blocks, fetched as four TMA boxes (64 rows x 128 bytes,
+// 128-byte swizzle) onto the stage's mbarrier, issued up to three chunks ahead.  The chunk
+// holding the newest keys (staged candidates, masked positions) is gathered row by row with
+// 16-byte cp.async into the same swizzled layout, zero-filled where there is no key.  Each
+// super-chunk's (M, L, O) goes to global memory; the CTA that finishes the last unit of a
+// (sequence, head) merges them (atomic ticket, no wait).
 #include <math.h>
 
 #include "common.cuh"
@@ -25,11 +34,15 @@
 namespace fm {
 
 constexpr int kCH = kAttnChunk;                  // keys per chunk (64)
-constexpr int kUnitMax = 16;                     // most chunks one CTA streams
-constexpr int kAttnThreads = 128;
-constexpr int kStageBytes = 2 * kCH * kHD * 2;   // K and V of one chunk: 32 KB
-constexpr int kAttnSmem = 2 * kStageBytes + kMaxR * kHD * 2 + 2 * kMaxR * kCH * 2 + kMaxR * kCH * 4;
-constexpr long long kStagedBit = 1ll << 62;
+constexpr int kSuper = kAttnSuper;               // chunks per super-chunk
+constexpr int kUnitMaxSuper = 4;                 // most super-chunks one CTA streams
+constexpr int kUnitMaxChunks = kSuper * kUnitMaxSuper;
+constexpr int kStages = 3;
+constexpr int kHalfBytes = kCH * 128;            // 64 rows x 64 dims of K or V: 8 KB
+constexpr int kTileBytes = 2 * kHalfBytes;       // K (or V) of a chunk: 16 KB
+constexpr int kStageBytes = 2 * kTileBytes;      // K and V of a chunk: 32 KB
+constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
+constexpr int kAttnSmem = 1024 + kStages * kStageBytes + kMaxR * kHD * 2 + kStages * 8;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
@@ -57,107 +70,152 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
-// Byte offset of 16-byte chunk `ch` of row `row` in a tile of 256-byte rows (a K or V row of
-// 128 bf16), chunks swizzled by row: conflict-free for ldmatrix and for row-wise cp.async.
-__device__ __forceinline__ uint32_t swz(int row, int ch) { return row * 256 + ((ch ^ (row & 7)) << 4); }
-// Same for the 128-byte rows of the probability tiles (64 keys per query).
-__device__ __forceinline__ uint32_t swz_p(int row, int ch) { return row * 128 + ((ch ^ (row & 7)) << 4); }
+// Transpose of an 8x8 b16 matrix held in the warp's fragment layout (lane 4i+j: row i,
+// columns 2j, 2j+1).
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
 
-// Merge of the chunks of every query of (sequence b, head h), run by the CTA that finishes the
-// last unit: query r combines chunks 0..floor(p_r/64) in chunk order,
-// O = sum_c w_c acc_c / sum_c w_c l_c with w_c = 2^(m_c - max_c m_c).  The (m, l) pairs are
-// staged in shared memory by all threads at once; the accumulator loads are independent.
-__device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R, int p0, int n_live, float* smem) {
-  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * a.n_chunks * R * (kHD + 2);
-  float* sm = smem;                      // [n_live * R] chunk max, then weight
-  float* sl = smem + n_live * R;         // [n_live * R] chunk sum
-  float* sL = sl + n_live * R;           // [R] total weight
-  for (int i = threadIdx.x; i < n_live * R; i += blockDim.x) {
-    const float* pc = part + static_cast<size_t>(i) * (kHD + 2);
+// Byte offset of 16-byte chunk `ch` of row `row` in a tile of 256-byte rows (the 8 query rows
+// of 128 bf16), chunks swizzled by row: conflict-free for ldmatrix.
+__device__ __forceinline__ uint32_t swz(int row, int ch) { return row * 256 + ((ch ^ (row & 7)) << 4); }
+// Byte offset of 16-byte chunk `ch` (dims 8ch..8ch+7) of key row `row` in a K or V tile: two
+// halves of 64 dims, each 64 rows of 128 bytes in the 128-byte swizzle a TMA box writes (chunk
+// index XOR row mod 8, from a 1024-byte aligned base).  Conflict-free for ldmatrix.
+__device__ __forceinline__ uint32_t swt(int row, int ch) {
+  return (ch >> 3) * kHalfBytes + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
+}
+
+// Merge of the super-chunks of every query of (sequence b, head h), run by the CTA that
+// finishes the last unit: query r combines super-chunks 0..floor(p_r/256) in order.
+__device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R, int p0, int n_sup, float* smem) {
+  const int lane = threadIdx.x & 31;
+  const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
+  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * n_super * R * kPartStride;
+  float* sm = smem;                      // [n_sup * R] super-chunk max, then weight
+  float* sl = smem + n_sup * R;          // [n_sup * R] super-chunk sum
+  float* sL = sl + n_sup * R;            // [R] total weight
+  for (int i = lane; i < n_sup * R; i += 32) {
+    const float* pc = part + static_cast<size_t>(i) * kPartStride;
     sm[i] = __ldcg(&pc[kHD]);
     sl[i] = __ldcg(&pc[kHD + 1]);
   }
-  __syncthreads();
-  if (threadIdx.x < R) {
-    const int r = threadIdx.x, lastc = (p0 + r) / kCH;
+  __syncwarp();
+  if (lane < R) {
+    const int r = lane, lasts = (p0 + r) / (kCH * kSuper);
     float M = -INFINITY;
-    for (int c = 0; c <= lastc; ++c) M = fmaxf(M, sm[c * R + r]);
+    for (int s = 0; s <= lasts; ++s) M = fmaxf(M, sm[s * R + r]);
     float L = 0.f;
-    for (int c = 0; c <= lastc; ++c) {
-      const float mc = sm[c * R + r];
-      const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
-      sm[c * R + r] = w;
-      L += sl[c * R + r] * w;
+    for (int s = 0; s <= lasts; ++s) {
+      const float ms = sm[s * R + r];
+      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+      sm[s * R + r] = w;
+      L += sl[s * R + r] * w;
     }
     sL[r] = L;
   }
-  __syncthreads();
-  const int d = threadIdx.x;
-  if (d < kHD) {
-    for (int r = 0; r < R; ++r) {
-      const int lastc = (p0 + r) / kCH;
-      float O = 0.f;
-      int c = 0;
-      for (; c + 4 <= lastc + 1; c += 4) {
-        float x[4];
+  __syncwarp();
+  const int d = lane * 4;   // four dims per lane
+  for (int r = 0; r < R; ++r) {
+    const int lasts = (p0 + r) / (kCH * kSuper);
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    int s = 0;
+    for (; s + 4 <= lasts + 1; s += 4) {
+      float4 x[4];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) x[u] = __ldcg(&part[(static_cast<size_t>(c + u) * R + r) * (kHD + 2) + d]);
+      for (int u = 0; u < 4; ++u)
+        x[u] = __ldcg(reinterpret_cast<const float4*>(part + (static_cast<size_t>(s + u) * R + r) * kPartStride + d));
 #pragma unroll
-        for (int u = 0; u < 4; ++u) O += x[u] * sm[(c + u) * R + r];
+      for (int u = 0; u < 4; ++u) {
+        const float w = sm[(s + u) * R + r];
+        O.x += x[u].x * w;
+        O.y += x[u].y * w;
+        O.z += x[u].z * w;
+        O.w += x[u].w * w;
       }
-      for (; c <= lastc; ++c) O += __ldcg(&part[(static_cast<size_t>(c) * R + r) * (kHD + 2) + d]) * sm[c * R + r];
-      a.out[(static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d] =
-          __float2bfloat16(O / sL[r]);
     }
+    for (; s <= lasts; ++s) {
+      const float4 x =
+          __ldcg(reinterpret_cast<const float4*>(part + (static_cast<size_t>(s) * R + r) * kPartStride + d));
+      const float w = sm[s * R + r];
+      O.x += x.x * w;
+      O.y += x.y * w;
+      O.z += x.z * w;
+      O.w += x.w * w;
+    }
+    const float inv = 1.f / sL[r];
+    bf16* o = a.out + (static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d;
+    *reinterpret_cast<__nv_bfloat162*>(o) = __floats2bfloat162_rn(O.x * inv, O.y * inv);
+    *reinterpret_cast<__nv_bfloat162*>(o + 2) = __floats2bfloat162_rn(O.z * inv, O.w * inv);
   }
 }
 
-// Copies the K and V rows j0..j0+63 of the unit into a stage as one cp.async group; rows
-// without a key are zero-filled.
-__device__ __forceinline__ void issue_chunk(const AttnArgs& a, const long long* s_base, int j0, uint8_t* stage) {
-  const long long v_pool = static_cast<long long>(kH) * a.page_size * kHD;
-  uint8_t* sK = stage;
-  uint8_t* sV = stage + kCH * kHD * 2;
-#pragma unroll 4
-  for (int v = threadIdx.x; v < kCH * 16; v += kAttnThreads) {
-    const int j = v >> 4, ch = v & 15;
-    const long long off = s_base[j0 + j];
+// Gathers the K and V rows of chunk c into a stage with 16-byte cp.async (each lane two keys,
+// sixteen 16-byte pieces of K and of V each); rows without a visible key are zero-filled.
+// Used for the chunk that holds staged candidates or masked positions, and for every chunk
+// when the pool has no TMA map.
+__device__ __forceinline__ void gather_chunk(const AttnArgs& a, int b, int h, int slot, int sl, int last, int c,
+                                             uint8_t* stage) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int key = lane * 2 + j;
+    const int pos = c * kCH + key;
     const bf16* srck = a.pool;
     const bf16* srcv = a.pool;
     int bytes = 0;
-    if (off >= 0) {
-      if (off & kStagedBit) {
-        srck = a.stage + (off & (kStagedBit - 1)) + ch * 8;
-        srcv = srck + a.stage_kv_stride;
+    if (pos <= last) {
+      if (pos < sl) {
+        const int pi = pos / a.page_size;
+        const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+        if (page >= 0 && page < a.n_pages) {
+          srck = a.pool + ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
+          srcv = srck + static_cast<long long>(kH) * a.page_size * kHD;
+          bytes = 16;
+        } else {
+          atomicOr(a.err, ERR_PAGE_RANGE);
+        }
       } else {
-        srck = a.pool + off + ch * 8;
-        srcv = srck + v_pool;
+        srck = a.stage + b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
+               static_cast<long long>(h) * kHD;
+        srcv = srck + a.stage_kv_stride;
+        bytes = 16;
       }
-      bytes = 16;
     }
-    cp_async16(sK + swz(j, ch), srck, bytes);
-    cp_async16(sV + swz(j, ch), srcv, bytes);
+#pragma unroll
+    for (int ch = 0; ch < 16; ++ch) {
+      const int o = bytes ? ch * 8 : 0;
+      cp_async16(stage + swt(key, ch), srck + o, bytes);
+      cp_async16(stage + kTileBytes + swt(key, ch), srcv + o, bytes);
+    }
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
 
-__global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const AttnArgs a) {
-  extern __shared__ __align__(128) uint8_t asmem[];
-  uint8_t* stages = asmem;                                   // [2][K 16 KB | V 16 KB]
-  uint8_t* sQ = asmem + 2 * kStageBytes;                     // [8 queries][128 dims] bf16
-  uint8_t* sP = sQ + kMaxR * kHD * 2;                        // [8][64 keys] bf16 p, high part
-  uint8_t* sPl = sP + kMaxR * kCH * 2;                       // [8][64 keys] bf16 p - high part
-  float* sS = reinterpret_cast<float*>(sPl + kMaxR * kCH * 2);   // [8][64] fp32 scores
-  __shared__ long long s_base[kUnitMax * kCH];               // element offset of every key row of the unit
-  __shared__ int s_last;
+__global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ AttnArgs a) {
+  extern __shared__ uint8_t asmem_raw[];
+  const uint32_t raw_u32 = smem_u32(asmem_raw);
+  uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [3][K 16 KB | V 16 KB]
+  uint8_t* sQ = stages + kStages * kStageBytes;              // [8 queries][128 dims] bf16
+  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + kMaxR * kHD * 2);   // [3] TMA stage barriers
+  __shared__ int s_page[kUnitMaxChunks];                     // page of each TMA chunk of the unit
+  __shared__ int s_abort;
   pdl_trigger();
   pdl_wait();
 
   const int u = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int lane = threadIdx.x;
+  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
   const int R = a.R;
   const int slot = a.slots[b];
   if (slot < 0 || slot >= a.n_slots) {   // every CTA of the sequence leaves; no ticket, no merge
-    if (u == 0 && h == 0 && threadIdx.x == 0) atomicOr(a.err, ERR_SLOT_RANGE);
+    if (u == 0 && h == 0 && lane == 0) atomicOr(a.err, ERR_SLOT_RANGE);
     return;
   }
   const int sl = a.seq_len[slot];
@@ -165,149 +223,240 @@ __global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const AttnArgs
   const int last = p0 + R - 1;
   if (p0 < 0) return;
   const int n_live = last / kCH + 1;                         // chunks holding keys 0..last
-  const int c0 = u * a.unit;
+  const int c0 = u * a.unit * kSuper;
   if (c0 >= n_live) return;
-  const int c1 = min(c0 + a.unit, n_live);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
+  const int c1 = min(c0 + a.unit * kSuper, n_live);
+  const int n = c1 - c0;
+  // chunks c0..c0+n_tma-1 hold committed keys only and come by TMA; the rest are gathered
+  const int n_tma = a.use_tma ? max(0, min(c1, sl / kCH) - c0) : 0;
 
-  // page offsets of every key of the unit, all lookups in flight at once
-  for (int j = tid; j < (c1 - c0) * kCH; j += kAttnThreads) {
-    const int pos = c0 * kCH + j;
-    long long off = -1;
-    if (pos <= last) {
-      if (pos < sl) {
-        const int pi = pos / a.page_size;
-        const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
-        if (page >= 0 && page < a.n_pages)
-          off = ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
-        else
-          atomicOr(a.err, ERR_PAGE_RANGE);
-      } else {
-        off = kStagedBit | (b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
-                            static_cast<long long>(h) * kHD);
-      }
+  for (int i = lane; i < n_tma; i += 32) {
+    const int pi = (c0 + i) * kCH / a.page_size;
+    int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+    if (page < 0 || page >= a.n_pages) {
+      atomicOr(a.err, ERR_PAGE_RANGE);
+      page = -1;
     }
-    s_base[j] = off;
+    s_page[i] = page;
+  }
+  if (lane == 0) {
+    for (int st = 0; st < kStages; ++st) mbar_init(&full[st], 1);
+    s_abort = 0;
+    fence_mbar_init();
   }
   // queries (bf16, as the QKV epilogue stored them); rows R..7 are zero
   const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
-  {
-    const int q = tid >> 4, ch = tid & 15;   // 8 queries x 16 chunks of 16 bytes
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int v = lane + 32 * i, q = v >> 4, ch = v & 15;   // 8 queries x 16 pieces of 16 bytes
     uint4 val = make_uint4(0, 0, 0, 0);
     if (q < R) val = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
     *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = val;
   }
-  __syncthreads();
-  issue_chunk(a, s_base, 0, stages);
+  __syncwarp();
+
+  // TMA of chunk i of the unit into stage i % 3; a chunk whose page is invalid completes its
+  // barrier without data (the guard flag is already set)
+  const uint64_t pol = l2_policy_evict_first();
+  auto issue = [&](int i) {
+    const int st = i % kStages;
+    uint8_t* dst = stages + st * kStageBytes;
+    const int page = s_page[i];
+    if (page < 0) {
+      mbar_arrive(&full[st]);
+      return;
+    }
+    const int c = c0 + i;
+    const int row_k = (page * 2 * kH + h) * a.page_size + (c * kCH) % a.page_size;
+    const int row_v = row_k + kH * a.page_size;
+    mbar_arrive_expect_tx(&full[st], kStageBytes);
+    tma_load_2d(dst, &a.kv_map, &full[st], 0, row_k, pol);
+    tma_load_2d(dst + kHalfBytes, &a.kv_map, &full[st], 64, row_k, pol);
+    tma_load_2d(dst + kTileBytes, &a.kv_map, &full[st], 0, row_v, pol);
+    tma_load_2d(dst + kTileBytes + kHalfBytes, &a.kv_map, &full[st], 64, row_v, pol);
+  };
+  if (lane == 0) {
+    if (n_tma > 0) tma_prefetch_desc(&a.kv_map);
+    for (int i = 0; i < min(n_tma, kStages); ++i) issue(i);
+  }
+
+  // Q^T fragments (B operand of S^T = K Q^T), the same for every chunk
+  const uint32_t qbase = smem_u32(sQ);
+  uint32_t qf[8][2];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), qf[ks]);
 
   const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));   // log2(e) / sqrt(hd)
-  const uint32_t qbase = smem_u32(sQ), pbase = smem_u32(sP), plbase = smem_u32(sPl);
-  int st = 0;
-  for (int c = c0; c < c1; ++c) {
-    const bool has_next = c + 1 < c1;
-    if (has_next) {
-      issue_chunk(a, s_base, (c + 1 - c0) * kCH, stages + (st ^ 1) * kStageBytes);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
-    __syncthreads();
-    const uint32_t kbase = smem_u32(stages + st * kStageBytes);
-    const uint32_t vbase = kbase + kCH * kHD * 2;
-    const int start = c * kCH;
-    const int nk = min(kCH, last + 1 - start);
-
-    // S^T[key][query] = K Q^T: warp w owns keys 16w..16w+15, 8 k-steps of 16 dims
-    {
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  const int qa = 2 * t4, qb = 2 * t4 + 1;                    // the two queries of this lane
+  float* part = a.part + (static_cast<size_t>(b) * kH + h) * ((a.n_chunks + kSuper - 1) / kSuper) * R * kPartStride;
+  float M_a = -INFINITY, M_b = -INFINITY, L_a = 0.f, L_b = 0.f;
+  float O[8][4];
+  int consumed = 0;   // TMA chunks waited for
+  bool aborted = false;
+  for (int i = 0; i < n; ++i) {
+    const int c = c0 + i;
+    const int st = i % kStages;
+    uint8_t* stage = stages + st * kStageBytes;
+    if (c % kSuper == 0 || i == 0) {
+      M_a = M_b = -INFINITY;
+      L_a = L_b = 0.f;
 #pragma unroll
-      for (int ks = 0; ks < 8; ++ks) {
-        uint32_t bq[2], ak[4];
-        ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), bq);
-        const int key = warp * 16 + ri + ((mi & 1) ? 8 : 0);
-        ldsm_x4(kbase + swz(key, 2 * ks + (mi >> 1)), ak);
-        mma_bf16_16816(acc, ak, bq);
+      for (int dt = 0; dt < 8; ++dt) O[dt][0] = O[dt][1] = O[dt][2] = O[dt][3] = 0.f;
+    }
+    if (i < n_tma) {
+      const bool ok = mbar_wait(&full[st], static_cast<uint32_t>(i / kStages) & 1u, &s_abort);
+      if (!__all_sync(0xffffffffu, ok)) {
+        aborted = true;
+        break;
       }
+      consumed = i + 1;
+    } else {
+      gather_chunk(a, b, h, slot, sl, last, c, stage);
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+      __syncwarp();
+    }
+    const uint32_t kbase = smem_u32(stage);
+    const uint32_t vbase = kbase + kTileBytes;
+
+    // S^T[key][query] = K Q^T over four 16-key tiles, 8 k-steps of 16 dims
+    float s[4][4];
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt) s[kt][0] = s[kt][1] = s[kt][2] = s[kt][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+#pragma unroll
+      for (int kt = 0; kt < 4; ++kt) {
+        uint32_t ak[4];
+        ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + (mi >> 1)), ak);
+        mma_bf16_16816(s[kt], ak, qf[ks]);
+      }
+    }
+    // visibility, chunk max per query (lanes sharing t4 hold the same two queries)
+    const int kb = c * kCH;
+    float m_a = -INFINITY, m_b = -INFINITY;
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const int key = warp * 16 + g + ((e >> 1) ? 8 : 0);
-        const int q = 2 * t4 + (e & 1);
-        const bool vis = q < R && key < nk && start + key <= p0 + q;
-        sS[q * kCH + key] = vis ? acc[e] * scale : -INFINITY;
+        const int key = kb + 16 * kt + g + ((e >> 1) ? 8 : 0);
+        const int q = (e & 1) ? qb : qa;
+        const float x = (q < R && key <= p0 + q) ? s[kt][e] * scale : -INFINITY;
+        s[kt][e] = x;
+        if (e & 1) m_b = fmaxf(m_b, x);
+        else m_a = fmaxf(m_a, x);
+      }
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      m_a = fmaxf(m_a, __shfl_xor_sync(0xffffffffu, m_a, o));
+      m_b = fmaxf(m_b, __shfl_xor_sync(0xffffffffu, m_b, o));
+    }
+    const float Mn_a = fmaxf(M_a, m_a), Mn_b = fmaxf(M_b, m_b);
+    const float al_a = (M_a == -INFINITY) ? 0.f : exp2f(M_a - Mn_a);
+    const float al_b = (M_b == -INFINITY) ? 0.f : exp2f(M_b - Mn_b);
+    M_a = Mn_a;
+    M_b = Mn_b;
+    // p = 2^(x - M) (exact zeros where masked), row sums, and P^T as bf16 hi + lo fragments
+    float l_a = 0.f, l_b = 0.f;
+    uint32_t ph[4][2], pl[4][2];
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt) {
+      float p[4], lo[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float Mq = (e & 1) ? M_b : M_a;
+        p[e] = (s[kt][e] == -INFINITY) ? 0.f : exp2f(s[kt][e] - Mq);
+        if (e & 1) l_b += p[e];
+        else l_a += p[e];
+        lo[e] = p[e] - __bfloat162float(__float2bfloat16(p[e]));
+      }
+      ph[kt][0] = movmatrix_t(pack_bf16(p[0], p[1]));     // keys 16kt+0..7
+      ph[kt][1] = movmatrix_t(pack_bf16(p[2], p[3]));     // keys 16kt+8..15
+      pl[kt][0] = movmatrix_t(pack_bf16(lo[0], lo[1]));
+      pl[kt][1] = movmatrix_t(pack_bf16(lo[2], lo[3]));
+    }
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      l_a += __shfl_xor_sync(0xffffffffu, l_a, o);
+      l_b += __shfl_xor_sync(0xffffffffu, l_b, o);
+    }
+    L_a = L_a * al_a + l_a;
+    L_b = L_b * al_b + l_b;
+    // O^T[dim][query] = al * O^T + V^T P^T: eight 16-dim tiles, 4 k-steps of 16 keys
+#pragma unroll
+    for (int dt = 0; dt < 8; ++dt) {
+      O[dt][0] *= al_a;
+      O[dt][1] *= al_b;
+      O[dt][2] *= al_a;
+      O[dt][3] *= al_b;
+    }
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt) {
+#pragma unroll
+      for (int dt = 0; dt < 8; ++dt) {
+        uint32_t av[4];
+        ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * dt + (mi & 1)), av);
+        mma_bf16_16816(O[dt], av, ph[kt]);
+        mma_bf16_16816(O[dt], av, pl[kt]);
       }
     }
-    __syncthreads();
+    __syncwarp();   // every lane is done with this stage
+    if (lane == 0 && i + kStages < n_tma) issue(i + kStages);
 
-    // per query: chunk max, p = hi + lo (exact zeros where masked), sum
-    float* part = a.part + ((static_cast<size_t>(b) * kH + h) * a.n_chunks + c) * R * (kHD + 2);
-    for (int q = warp; q < kMaxR; q += 4) {
-      const float x0 = sS[q * kCH + lane], x1 = sS[q * kCH + lane + 32];
-      const float m = warp_max(fmaxf(x0, x1));
-      float l = 0.f;
+    // end of a super-chunk: its (M, L, O) per query
+    if ((c + 1) % kSuper == 0 || i + 1 == n) {
+      float* ps = part + static_cast<size_t>(c / kSuper) * R * kPartStride;
 #pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const int key = lane + 32 * i;
-        const float x = i ? x1 : x0;
-        const float p = (m == -INFINITY || x == -INFINITY) ? 0.f : exp2f(x - m);
-        const bf16 hi = __float2bfloat16(p);
-        const bf16 lo = __float2bfloat16(p - __bfloat162float(hi));
-        *reinterpret_cast<bf16*>(sP + swz_p(q, key >> 3) + (key & 7) * 2) = hi;
-        *reinterpret_cast<bf16*>(sPl + swz_p(q, key >> 3) + (key & 7) * 2) = lo;
-        l += p;
-      }
-      l = warp_sum(l);
-      if (lane == 0 && q < R) {
-        part[q * (kHD + 2) + kHD] = m;
-        part[q * (kHD + 2) + kHD + 1] = l;
-      }
-    }
-    __syncthreads();
-
-    // O^T[dim][query] = V^T P^T: warp w owns dims 32w..32w+31 (two tiles), 4 k-steps of 16 keys
-    {
-      float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-#pragma unroll
-      for (int ks = 0; ks < kCH / 16; ++ks) {
-        uint32_t bp[2], bl[2];
-        ldsm_x2(pbase + swz_p(ri, 2 * ks + (mi & 1)), bp);
-        ldsm_x2(plbase + swz_p(ri, 2 * ks + (mi & 1)), bl);
-#pragma unroll
-        for (int mt = 0; mt < 2; ++mt) {
-          uint32_t av[4];
-          const int key = ks * 16 + ri + ((mi >> 1) ? 8 : 0);
-          ldsm_x4_t(vbase + swz(key, (warp * 32 + mt * 16) / 8 + (mi & 1)), av);
-          mma_bf16_16816(acc[mt], av, bp);
-          mma_bf16_16816(acc[mt], av, bl);
+      for (int dt = 0; dt < 8; ++dt) {
+        const int d = 16 * dt + g;
+        if (qa < R) {
+          ps[qa * kPartStride + d] = O[dt][0];
+          ps[qa * kPartStride + d + 8] = O[dt][2];
+        }
+        if (qb < R) {
+          ps[qb * kPartStride + d] = O[dt][1];
+          ps[qb * kPartStride + d + 8] = O[dt][3];
         }
       }
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int d = warp * 32 + mt * 16 + g + ((e >> 1) ? 8 : 0);
-          const int q = 2 * t4 + (e & 1);
-          if (q < R) part[q * (kHD + 2) + d] = acc[mt][e];
+      if (g == 0) {
+        if (qa < R) {
+          ps[qa * kPartStride + kHD] = M_a;
+          ps[qa * kPartStride + kHD + 1] = L_a;
         }
+        if (qb < R) {
+          ps[qb * kPartStride + kHD] = M_b;
+          ps[qb * kPartStride + kHD + 1] = L_b;
+        }
+      }
     }
-    __syncthreads();   // this stage and the score/probability tiles are reused next
-    st ^= 1;
+  }
+  if (aborted) {
+    // a stage wait ran out: flag it and let the copies still in flight land, then take the
+    // ticket as usual so that the counters stay consistent (the merged result is invalid)
+    if (lane == 0) {
+      atomicOr(a.err, ERR_WAIT_TIMEOUT);
+      const int issued = min(n_tma, consumed + kStages);
+      int never = 0;
+      for (int i = consumed; i < issued; ++i)
+        mbar_wait(&full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, &never, 100000000ull);
+    }
+    __syncwarp();
   }
 
   // the CTA that finishes the last unit of (sequence, head) merges every query
   __threadfence();
-  __syncthreads();
-  const int n_units = (n_live + a.unit - 1) / a.unit;
-  if (tid == 0) {
+  __syncwarp();
+  const int n_units = (n_live + a.unit * kSuper - 1) / (a.unit * kSuper);
+  int is_last = 0;
+  if (lane == 0) {
     int* ticket = a.tickets + b * kH + h;
     const int old = atomicAdd(ticket, 1);
-    s_last = (old == n_units - 1) ? 1 : 0;
-    if (s_last) *ticket = 0;
+    is_last = (old == n_units - 1) ? 1 : 0;
+    if (is_last) *ticket = 0;
   }
-  __syncthreads();
-  if (s_last) {
+  is_last = __shfl_sync(0xffffffffu, is_last, 0);
+  if (is_last) {
     __threadfence();
-    merge_all(a, b, h, R, p0, n_live, reinterpret_cast<float*>(stages));   // the K/V stages are free
+    merge_all(a, b, h, R, p0, (n_live + kSuper - 1) / kSuper, reinterpret_cast<float*>(stages));
   }
 }
 
@@ -316,18 +465,19 @@ cudaError_t attention_prepare() {
 }
 
 cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
-  // Chunks per CTA: enough CTAs for about three resident per SM over the largest context the
-  // pools allow.  Pure scheduling: the arithmetic of every chunk and of the merge is the same
-  // for any grouping.
+  // Super-chunks per CTA: enough CTAs for about two waves of two per SM over the largest
+  // context the pools allow.  Pure scheduling: the arithmetic of every super-chunk and of the
+  // merge is the same for any grouping.
   AttnArgs a = a_in;
-  const long long target = 3ll * num_sms();
+  const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
+  const long long target = 4ll * num_sms();
   const long long per_unit = static_cast<long long>(B) * kH;
-  int unit = static_cast<int>((per_unit * a.n_chunks + target - 1) / target);
+  int unit = static_cast<int>((per_unit * n_super + target - 1) / target);
   if (unit < 1) unit = 1;
-  if (unit > kUnitMax) unit = kUnitMax;
+  if (unit > kUnitMaxSuper) unit = kUnitMaxSuper;
   a.unit = unit;
-  const int n_units = (a.n_chunks + unit - 1) / unit;
-  return launch_pdl(attn_chunk_kernel, dim3(n_units, kH, B), dim3(kAttnThreads), kAttnSmem, s, a);
+  const int n_units = (n_super + unit - 1) / unit;
+  return launch_pdl(attn_chunk_kernel, dim3(n_units, kH, B), dim3(32), kAttnSmem, s, a);
 }
 
 }  // namespace fm

@@ -49,6 +49,8 @@ constexpr int kI = 896;         // expert intermediate
 constexpr int kId = 3584;       // draft-block intermediate
 constexpr int kSlots = kTopK + kShared;   // per-token expert outputs combined
 constexpr int kAttnChunk = 64;            // split-KV chunk (keys), fixed by absolute position
+constexpr int kAttnSuper = 4;             // chunks per attention super-chunk (one partial each)
+constexpr int kAttnPartStride = 132;      // floats per (super-chunk, query) partial: O[128], M, L, pad
 constexpr int kMaxR = 8;                  // K_max + 1 <= 8 candidate rows per sequence
 constexpr int kMaxSplit = 6;              // split-K ways of a dense GEMM
 
@@ -123,6 +125,11 @@ int dense_split_k(int N, int K);
 
 // ------------------------------------------------------------------------- other kernels
 struct AttnArgs {
+  // The pool of this launch as a 2-D bf16 tensor [n_pages * 2 * H * page_size][hd], box 64 x
+  // 64 with the 128-byte swizzle; used for chunks whose 64 keys are all committed when
+  // use_tma is set (page_size a multiple of 64).
+  CUtensorMap kv_map;
+  int use_tma;
   const bf16* q;               // [rows][H][hd] bf16
   const int* q_row0;           // per sequence first query row (NULL: b * R)
   int R;                       // queries per sequence
@@ -132,7 +139,7 @@ struct AttnArgs {
   const bf16* pool; int page_size; int n_pages; const int* block_table; int max_pages;
   const bf16* stage;           // keys at positions >= seq_len[slot]: staged row (pos - seq_len)
   long long stage_seq_stride, stage_row_stride, stage_kv_stride;
-  float* part;                 // [B][H][n_chunks][R][kHD + 2]
+  float* part;                 // [B][H][ceil(n_chunks / 4)][R][132] super-chunk partials
   int* tickets;                // [B][H] chunk counters, zero between launches
   int n_chunks;
   int unit;                    // chunks per CTA (set by attention_launch)

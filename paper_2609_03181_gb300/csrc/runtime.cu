@@ -57,6 +57,11 @@ struct spec_ctx {
   std::vector<spec_layer_weights> layers;
   bf16* kv_pool = nullptr;
   bf16* dkv_pool = nullptr;
+  // attention: the pools as TMA tensors (per verifier layer, and the draft pool), when the
+  // page size allows whole-chunk boxes
+  bool attn_tma = false;
+  std::vector<CUtensorMap> kv_maps;
+  CUtensorMap dkv_map;
 
   std::vector<LayerMaps> lmaps;
   CUtensorMap lm{}, eh{}, mqkv{}, mwo{}, mgu{}, mdn{};
@@ -418,7 +423,8 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->xn, sizeof(bf16) * Tmax * d);
   add(&ctx->q, sizeof(bf16) * Tmax * d);
   add(&ctx->stage, sizeof(bf16) * L * Bmax * Rmax * 2 * d);
-  add(&ctx->attn_part, sizeof(float) * static_cast<size_t>(Bmax) * kH * ctx->n_chunks * Rmax * (kHD + 2));
+  add(&ctx->attn_part, sizeof(float) * static_cast<size_t>(Bmax) * kH * ((ctx->n_chunks + kAttnSuper - 1) / kAttnSuper) *
+                           Rmax * kAttnPartStride);
   add(&ctx->attn_tickets, sizeof(int) * Bmax * kH);
   add(&ctx->commit_tickets, sizeof(int) * Bmax);
   add(&ctx->attn_out, sizeof(bf16) * Tmax * d);
@@ -526,6 +532,17 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ok = ok && encode_act_maps(ctx->a_dattn.m, ctx->dattn, kD, Bmax, &e);
   ok = ok && encode_act_maps(ctx->a_dact.m, ctx->dact, kId, Bmax, &e);
   ok = ok && encode_act_maps(ctx->a_u.m, ctx->u, kD, static_cast<uint64_t>(c.K_max > 0 ? c.K_max : 1) * Bmax, &e);
+  {
+    const long long pool_rows = static_cast<long long>(c.n_pages_total) * 2 * kH * c.page_size;
+    ctx->attn_tma = (c.page_size % kAttnChunk == 0) && pool_rows < (1ll << 31);
+    if (ctx->attn_tma) {
+      const size_t pool_layer = static_cast<size_t>(pool_rows) * kHD;
+      ctx->kv_maps.resize(L);
+      for (int l = 0; l < L && ok; ++l)
+        ok = encode_map_2d(&ctx->kv_maps[l], ctx->kv_pool + l * pool_layer, kHD, pool_rows, kAttnChunk, &e);
+      ok = ok && encode_map_2d(&ctx->dkv_map, ctx->dkv_pool, kHD, pool_rows, kAttnChunk, &e);
+    }
+  }
   if (!ok) return bail(SPEC_EINVAL, "tensor map: " + e);
   if (cudaStreamSynchronize(ctx->stream) != cudaSuccess) return bail(SPEC_ECUDA, "stream synchronize failed");
   *out = ctx;
@@ -659,6 +676,10 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       a.seq_len = ctx->seq_len;
       a.n_slots = ctx->Bmax;
       a.pool = ctx->kv_pool + l * pool_layer;
+      if (ctx->attn_tma) {
+        a.kv_map = ctx->kv_maps[l];
+        a.use_tma = 1;
+      }
       a.page_size = c.page_size;
       a.n_pages = c.n_pages_total;
       a.block_table = ctx->block_table;
@@ -846,6 +867,10 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       a.seq_len = ctx->seq_len;
       a.n_slots = ctx->Bmax;
       a.pool = ctx->dkv_pool;
+      if (ctx->attn_tma) {
+        a.kv_map = ctx->dkv_map;
+        a.use_tma = 1;
+      }
       a.page_size = c.page_size;
       a.n_pages = c.n_pages_total;
       a.block_table = ctx->block_table;
