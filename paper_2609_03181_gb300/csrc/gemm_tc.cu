@@ -29,7 +29,11 @@ struct Cfg {
   static constexpr int STAGES = (NMAX <= 64) ? 8 : 4;
   static constexpr int TMEM_COLS = 2 * NMAX;           // two accumulator buffers
   static constexpr int XCHG_FLOATS = 128 * 17;
-  static constexpr int SMEM_BYTES = 1024 + STAGES * (A_BYTES + B_BYTES) + 256 + XCHG_FLOATS * 4 + 4 * 16 * 8;
+  static constexpr int AM_BYTES = 128 * 8;             // argmax partials of 8 row groups x 16 columns
+  static constexpr int META_BYTES = 256 * 16;          // per-row metadata of an item (QKV, SCATTER)
+  static constexpr int ROPE_BYTES = 2 * 16 * 64 * 8;   // QKV: RoPE factors of two 16-row chunks
+  static constexpr int SMEM_BYTES =
+      1024 + STAGES * (A_BYTES + B_BYTES) + 256 + XCHG_FLOATS * 4 + AM_BYTES + META_BYTES + ROPE_BYTES;
 };
 
 struct Item {
@@ -51,8 +55,9 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it) {
   } else {
     const int mt = i % a.m_tiles;
     const int t = i / a.m_tiles;
-    it.split = t % a.split_k;
-    it.n_tile = t / a.split_k;
+    const int ns = a.seq_split ? 1 : a.split_k;   // in-CTA splits: one item covers every split
+    it.split = t % ns;
+    it.n_tile = t / ns;
     it.e = 0;
     const int box = 16 << a.box_log;
     it.out_row = mt * box;
@@ -64,43 +69,107 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it) {
 
 // ------------------------------------------------------------------ epilogues
 // v: 16 accumulator columns (activation rows j0..j0+15 of the item) of tile row `row`.
-// Every global load a chunk needs is issued before its first store: a store may alias a later
-// load as far as the compiler knows, so interleaving them would serialise one L2 round trip
-// per row.
+// epi_pre issues the global loads a chunk needs (the old residuals, the scatter targets, the
+// RoPE factors) into registers; the chunk loops call it one chunk ahead, so a chunk's loads
+// are in flight while the previous chunk computes and stores.  epi_post computes and
+// stores.  Shared scratch: xchg [128][17] floats, am_val/am_idx [128], s_pos/s_off [256].
+struct EpiPre {
+  float old[16];
+};
+
+struct EpiSmem {
+  float* xchg;
+  float* am_val;
+  int* am_idx;
+  int* s_pos;         // QKV: position of each row of the item; SCATTER: token
+  int* s_aux;         // SCATTER: slot
+  long long* s_off;   // QKV: staging offset
+  float2* rope;       // QKV: [2][16 rows][64] cos/sin of a chunk's positions (double-buffered)
+};
+
 template <int EPI>
-__device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int row, int j0, float (&v)[16],
-                                          float* xchg, float* am_s_val, int* am_s_idx) {
-  const int lane = threadIdx.x & 31;
+__device__ __forceinline__ void epi_pre(const GemmArgs& a, const Item& it, int row, int j0, const EpiSmem& sm,
+                                        EpiPre& p) {
+  if constexpr (EPI == EPI_RESID) {
+    const int n = it.n_tile * 128 + row;
+    if (n < a.N) {
+      const float* base = a.out + static_cast<size_t>(it.out_row + j0) * a.ldo + n;
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) p.old[jj] = (j0 + jj < it.rows) ? base[static_cast<size_t>(jj) * a.ldo] : 0.f;
+    }
+  }
+}
+
+// QKV with RoPE (q and k tiles): the cos/sin rows of a chunk's 16 positions, fetched by all
+// 128 epilogue threads as 16-byte pieces (rope_load, issued a chunk ahead) and put into one of
+// two shared buffers (rope_store) before the barrier that precedes their use.
+struct RopeRegs {
+  float4 r[4];
+};
+__device__ __forceinline__ void rope_load(const GemmArgs& a, const Item& it, int j0, const EpiSmem& sm, RopeRegs& rr) {
+  const int t = threadIdx.x - 64;
+  bool bad = false;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int idx = t + 128 * k, r = idx >> 5, piece = idx & 31;   // 16 rows x 32 pieces of 16 bytes
+    int q = (j0 + r < it.rows) ? sm.s_pos[j0 + r] : 0;
+    if (q < 0 || q >= a.max_pos) {
+      bad = true;
+      q = 0;
+    }
+    rr.r[k] = *reinterpret_cast<const float4*>(a.rope + static_cast<size_t>(q) * (kHD / 2) + piece * 2);
+  }
+  if (bad) atomicOr(a.err, ERR_POSITION);
+}
+__device__ __forceinline__ void rope_store(const EpiSmem& sm, int buf, const RopeRegs& rr) {
+  const int t = threadIdx.x - 64;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int idx = t + 128 * k, r = idx >> 5, piece = idx & 31;
+    *reinterpret_cast<float4*>(sm.rope + (buf * 16 + r) * 64 + piece * 2) = rr.r[k];
+  }
+}
+
+// The per-row metadata of an item into shared memory, loaded once by all 128 epilogue
+// threads (QKV: positions and staging offsets; SCATTER: token and slot of each sorted row).
+// The barriers keep the previous item's readers and this item's readers apart.
+template <int EPI>
+__device__ __forceinline__ void stage_meta(const GemmArgs& a, const Item& it, const EpiSmem& sm) {
+  if constexpr (EPI == EPI_QKV || EPI == EPI_SCATTER) {
+    const int t = threadIdx.x - 64;
+    named_bar_sync(1, 128);
+    for (int r = t; r < it.rows; r += 128) {
+      if constexpr (EPI == EPI_QKV) {
+        sm.s_pos[r] = a.pos[it.out_row + r];
+        sm.s_off[r] = a.kv_rowoff[it.out_row + r];
+      } else {
+        sm.s_pos[r] = a.sorted_tok[it.out_row + r];
+        sm.s_aux[r] = a.sorted_slot[it.out_row + r];
+      }
+    }
+    named_bar_sync(1, 128);
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int row, int j0, float (&v)[16],
+                                         const EpiPre& p, const EpiSmem& sm, int rope_buf) {
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
     const int n = it.n_tile * 128 + row;
     if (n < a.N) {
       float* base = a.out + static_cast<size_t>(it.out_row + j0) * a.ldo + n;
-      if constexpr (EPI == EPI_RESID) {
-        float old[16];
 #pragma unroll
-        for (int jj = 0; jj < 16; ++jj) old[jj] = (j0 + jj < it.rows) ? base[static_cast<size_t>(jj) * a.ldo] : 0.f;
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj)
-          if (j0 + jj < it.rows) base[static_cast<size_t>(jj) * a.ldo] = old[jj] + v[jj];
-      } else {
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj)
-          if (j0 + jj < it.rows) base[static_cast<size_t>(jj) * a.ldo] = v[jj];
-      }
+      for (int jj = 0; jj < 16; ++jj)
+        if (j0 + jj < it.rows) base[static_cast<size_t>(jj) * a.ldo] = (EPI == EPI_RESID) ? p.old[jj] + v[jj] : v[jj];
     }
   } else if constexpr (EPI == EPI_SCATTER) {
     const int n = it.n_tile * 128 + row;
-    int tok[16], slt[16];
-#pragma unroll
-    for (int jj = 0; jj < 16; ++jj) {
-      const bool ok = j0 + jj < it.rows;
-      tok[jj] = ok ? a.sorted_tok[it.out_row + j0 + jj] : 0;
-      slt[jj] = ok ? a.sorted_slot[it.out_row + j0 + jj] : 0;
-    }
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj)
-      if (j0 + jj < it.rows) a.y[(static_cast<size_t>(tok[jj]) * kSlots + slt[jj]) * kD + n] = v[jj];
+      if (j0 + jj < it.rows)
+        a.y[(static_cast<size_t>(sm.s_pos[j0 + jj]) * kSlots + sm.s_aux[j0 + jj]) * kD + n] = v[jj];
   } else if constexpr (EPI == EPI_SWIGLU) {
+    float* xchg = sm.xchg;
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
     named_bar_sync(1, 128);
@@ -119,26 +188,8 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
   } else if constexpr (EPI == EPI_QKV) {
     const int which = it.n_tile / kH;   // 0 q, 1 k, 2 v
     const int head = it.n_tile % kH;
-    long long off[16];
-    float2 cs[16];
-    if (which > 0) {
-#pragma unroll
-      for (int jj = 0; jj < 16; ++jj) off[jj] = (j0 + jj < it.rows) ? a.kv_rowoff[it.out_row + j0 + jj] : -1;
-    }
     if (which < 2) {
-      int p[16];
-#pragma unroll
-      for (int jj = 0; jj < 16; ++jj) p[jj] = (j0 + jj < it.rows) ? a.pos[it.out_row + j0 + jj] : 0;
-      bool bad = false;
-#pragma unroll
-      for (int jj = 0; jj < 16; ++jj) {
-        if (p[jj] < 0 || p[jj] >= a.max_pos) {
-          bad = true;
-          p[jj] = 0;
-        }
-        cs[jj] = a.rope[static_cast<size_t>(p[jj]) * (kHD / 2) + (row & 63)];
-      }
-      if (bad) atomicOr(a.err, ERR_POSITION);
+      float* xchg = sm.xchg;
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
       named_bar_sync(1, 128);
@@ -146,9 +197,12 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) partner[jj] = xchg[(row ^ 64) * 17 + jj];
       named_bar_sync(1, 128);
+      const float2* cs = sm.rope + rope_buf * 16 * 64 + (row & 63);
 #pragma unroll
-      for (int jj = 0; jj < 16; ++jj)
-        v[jj] = (row < 64) ? (v[jj] * cs[jj].x - partner[jj] * cs[jj].y) : (v[jj] * cs[jj].x + partner[jj] * cs[jj].y);
+      for (int jj = 0; jj < 16; ++jj) {
+        const float2 f = cs[jj * 64];
+        v[jj] = (row < 64) ? (v[jj] * f.x - partner[jj] * f.y) : (v[jj] * f.x + partner[jj] * f.y);
+      }
     }
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
@@ -157,37 +211,47 @@ __device__ __forceinline__ void epi_chunk(const GemmArgs& a, const Item& it, int
       const int m = it.out_row + r;
       if (which == 0) {
         a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + row] = __float2bfloat16(v[jj]);
-      } else if (off[jj] >= 0) {
-        a.kv_base[off[jj] + (which == 2 ? a.v_off : 0) + head * a.head_stride + row] = __float2bfloat16(v[jj]);
+      } else {
+        const long long off = sm.s_off[r];
+        if (off >= 0) a.kv_base[off + (which == 2 ? a.v_off : 0) + head * a.head_stride + row] = __float2bfloat16(v[jj]);
       }
     }
   } else if constexpr (EPI == EPI_ARGMAX) {
-    const int q = (threadIdx.x >> 5) & 3;
+    // per activation row: max over the tile's 128 logits (lower id on ties), through a
+    // transpose in shared memory: 8 groups of 16 tile rows per column, then the 8 groups
     const int n = it.n_tile * 128 + row;
+    float* xchg = sm.xchg;
 #pragma unroll
-    for (int jj = 0; jj < 16; ++jj) {
-      float bv = (n < a.N) ? v[jj] : -INFINITY;
-      int bi = n;
-      warp_argmax(bv, bi);
-      if (lane == 0) {
-        am_s_val[q * 16 + jj] = bv;
-        am_s_idx[q * 16 + jj] = bi;
+    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = (n < a.N) ? v[jj] : -INFINITY;
+    named_bar_sync(1, 128);
+    const int t = threadIdx.x - 64, j = t & 15, grp = t >> 4;
+    {
+      float bv = xchg[(grp * 16) * 17 + j];
+      int bi = grp * 16;
+#pragma unroll
+      for (int rr = 1; rr < 16; ++rr) {
+        const float x = xchg[(grp * 16 + rr) * 17 + j];
+        if (x > bv) {
+          bv = x;
+          bi = grp * 16 + rr;
+        }
       }
+      sm.am_val[grp * 16 + j] = bv;
+      sm.am_idx[grp * 16 + j] = bi;
     }
     named_bar_sync(1, 128);
-    if (row < 16) {
-      const int r = j0 + row;
-      if (r < it.rows) {
-        float bv = am_s_val[row];
-        int bi = am_s_idx[row];
+    if (t < 16 && j0 + t < it.rows) {
+      float bv = sm.am_val[t];
+      int bi = sm.am_idx[t];
 #pragma unroll
-        for (int w = 1; w < 4; ++w)
-          if (better(am_s_val[w * 16 + row], am_s_idx[w * 16 + row], bv, bi)) {
-            bv = am_s_val[w * 16 + row];
-            bi = am_s_idx[w * 16 + row];
-          }
-        atomicMax(a.am_key + it.out_row + r, argmax_key(bv, bi));
+      for (int g2 = 1; g2 < 8; ++g2) {
+        const float x = sm.am_val[g2 * 16 + t];
+        if (x > bv) {
+          bv = x;
+          bi = sm.am_idx[g2 * 16 + t];
+        }
       }
+      atomicMax(a.am_key + it.out_row + j0 + t, argmax_key(bv, it.n_tile * 128 + bi));
     }
     named_bar_sync(1, 128);
   }
@@ -212,9 +276,14 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   int* s_vote = const_cast<int*>(s_abort) + 1;   // [4]
   int* s_last = s_vote + 4;
-  float* xchg = reinterpret_cast<float*>(smem + C::STAGES * (C::A_BYTES + C::B_BYTES) + 256);
-  float* am_s_val = xchg + C::XCHG_FLOATS;
-  int* am_s_idx = reinterpret_cast<int*>(am_s_val + 64);
+  EpiSmem esm;
+  esm.xchg = reinterpret_cast<float*>(smem + C::STAGES * (C::A_BYTES + C::B_BYTES) + 256);
+  esm.am_val = esm.xchg + C::XCHG_FLOATS;
+  esm.am_idx = reinterpret_cast<int*>(esm.am_val + 128);
+  esm.s_off = reinterpret_cast<long long*>(esm.am_idx + 128);
+  esm.s_pos = reinterpret_cast<int*>(esm.s_off + 256);
+  esm.s_aux = esm.s_pos + 256;
+  esm.rope = reinterpret_cast<float2*>(esm.s_aux + 256);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -237,8 +306,13 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     tma_prefetch_desc(&a.a_map[0]);
     tma_prefetch_desc(&a.a_map[1]);
   }
+  // accumulator buffers: two of NMAX columns, or with in-CTA splits one (split_k > 4) or two
+  // groups of split_k x 64 columns
+  const uint32_t tmem_cols = a.seq_split ? 512u : static_cast<uint32_t>(C::TMEM_COLS);
+  const int nbuf = (a.seq_split && a.split_k > 4) ? 1 : 2;
+  const uint32_t acc_stride = a.seq_split ? static_cast<uint32_t>(a.split_k) * 64u : static_cast<uint32_t>(NMAX);
   if (warp == 1) {
-    tmem_alloc(s_tmem, C::TMEM_COLS);
+    tmem_alloc(s_tmem, tmem_cols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -270,7 +344,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         const CUtensorMap* amap = &a.a_map[src];
         const CUtensorMap* bmap = &a.b_map[src][it.box_log];
         const uint32_t bytes = C::A_BYTES + (16u << it.box_log) * 128u;
-        const int kc0 = it.split * kc_total / a.split_k, kc1 = (it.split + 1) * kc_total / a.split_k;
+        const int kc0 = a.seq_split ? 0 : it.split * kc_total / a.split_k;
+        const int kc1 = a.seq_split ? kc_total : (it.split + 1) * kc_total / a.split_k;
         auto load_a = [&](int st, int kc) {
           uint8_t* sa = smA + st * C::A_BYTES;
           const int k = kc * 64;
@@ -338,17 +413,26 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x, ++local) {
         Item it;
         get_item(a, i, it);
-        const int acc = local & 1;
-        const uint32_t acc_ph = (local >> 1) & 1;
+        const int acc = local % nbuf;
+        const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
         if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, s_abort)) {
           failed = true;
           break;
         }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * NMAX;
         const uint32_t idesc = idesc_bf16(128, 16 << it.box_log);
-        const int kc0 = it.split * kc_total / a.split_k, kc1 = (it.split + 1) * kc_total / a.split_k;
+        const int kc0 = a.seq_split ? 0 : it.split * kc_total / a.split_k;
+        const int kc1 = a.seq_split ? kc_total : (it.split + 1) * kc_total / a.split_k;
+        // with in-CTA splits, split sp accumulates k-chunks [sp*kc/S, (sp+1)*kc/S) into its own
+        // 64 columns, starting from zero, exactly as a separate CTA would
+        int sp = 0, sp_begin = kc0, sp_end = a.seq_split ? kc_total / a.split_k : kc1;
         for (int kc = kc0; kc < kc1; ++kc, ++g) {
+          if (kc == sp_end) {
+            ++sp;
+            sp_begin = kc;
+            sp_end = (sp + 1) * kc_total / a.split_k;
+          }
+          const uint32_t d_tmem = tmem_base + acc * acc_stride + sp * 64;
           const int st = g % C::STAGES;
           const uint32_t ph = (g / C::STAGES) & 1u;
           if (!mbar_wait(&full[st], ph, s_abort)) {
@@ -360,7 +444,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           const uint64_t bd = sw128_kmajor_desc(smem_u32(smB + st * C::B_BYTES));
 #pragma unroll
           for (int s = 0; s < 4; ++s)   // 4 x K=16 per 64-column chunk: +32 B in the swizzled row
-            tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > kc0 || s > 0) ? 1u : 0u);
+            tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
           tc_commit(&empty[st]);
         }
         if (failed) break;
@@ -386,8 +470,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     for (int i = blockIdx.x; i < n_items; i += gridDim.x, ++local) {
       Item it;
       get_item(a, i, it);
-      const int acc = local & 1;
-      const uint32_t acc_ph = (local >> 1) & 1;
+      const int acc = local % nbuf;
+      const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
       bool ok = mbar_wait(&tfull[acc], acc_ph, s_abort);
       ok = __all_sync(0xffffffffu, ok);
       if (lane == 0) s_vote[ew] = ok ? 1 : 0;
@@ -400,13 +484,39 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         break;
       }
       tc_fence_after();
-      const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * NMAX;
+      const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * acc_stride;
       const int nchunks = (it.rows + 15) >> 4;
       float v[16];
-      if (a.split_k == 1) {
+      if (a.split_k == 1 || a.seq_split) {
+        stage_meta<EPI>(a, it, esm);
+        const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
+        RopeRegs rr;
+        if (rope) {
+          rope_load(a, it, 0, esm, rr);
+          rope_store(esm, 0, rr);
+          named_bar_sync(1, 128);
+        }
+        EpiPre cur, nxt;
+        epi_pre<EPI>(a, it, row, 0, esm, cur);
         for (int c = 0; c < nchunks; ++c) {
+          if (c + 1 < nchunks) {
+            epi_pre<EPI>(a, it, row, (c + 1) * 16, esm, nxt);
+            if (rope) rope_load(a, it, (c + 1) * 16, esm, rr);
+          }
           tc_ld16(tb + c * 16, v);
-          epi_chunk<EPI>(a, it, row, c * 16, v, xchg, am_s_val, am_s_idx);
+          for (int sp = 1; sp < (a.seq_split ? a.split_k : 1); ++sp) {
+            // in-CTA splits: partial sums added in split order, as the cross-CTA reduction does
+            float w[16];
+            tc_ld16(tb + sp * 64 + c * 16, w);
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
+          }
+          epi_post<EPI>(a, it, row, c * 16, v, cur, esm, c & 1);
+          cur = nxt;
+          if (rope && c + 1 < nchunks) {
+            rope_store(esm, (c + 1) & 1, rr);
+            named_bar_sync(1, 128);
+          }
         }
         tc_fence_before();
         __syncwarp();
@@ -439,33 +549,57 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         if (*s_last) {
           __threadfence();
           const float* base = a.sk_ws + static_cast<size_t>(tile) * a.split_k * tstride;
+          stage_meta<EPI>(a, it, esm);
+          const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
+          RopeRegs rr;
+          if (rope) {
+            rope_load(a, it, 0, esm, rr);
+            rope_store(esm, 0, rr);
+            named_bar_sync(1, 128);
+          }
+          EpiPre cur, nxt;
+          epi_pre<EPI>(a, it, row, 0, esm, cur);
           for (int c = 0; c < nchunks; ++c) {
-            float4 p[kMaxSplit][4];
-#pragma unroll
-            for (int sp = 0; sp < kMaxSplit; ++sp)
-              if (sp < a.split_k) {
-                const float4* src =
-                    reinterpret_cast<const float4*>(base + sp * tstride + (static_cast<size_t>(c) * 128 + row) * 16);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) p[sp][q4] = __ldcg(src + q4);
-              }
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-              float4 t = p[0][q4];
-#pragma unroll
-              for (int sp = 1; sp < kMaxSplit; ++sp)
-                if (sp < a.split_k) {
-                  t.x += p[sp][q4].x;
-                  t.y += p[sp][q4].y;
-                  t.z += p[sp][q4].z;
-                  t.w += p[sp][q4].w;
-                }
-              v[4 * q4] = t.x;
-              v[4 * q4 + 1] = t.y;
-              v[4 * q4 + 2] = t.z;
-              v[4 * q4 + 3] = t.w;
+            if (c + 1 < nchunks) {
+              epi_pre<EPI>(a, it, row, (c + 1) * 16, esm, nxt);
+              if (rope) rope_load(a, it, (c + 1) * 16, esm, rr);
             }
-            epi_chunk<EPI>(a, it, row, c * 16, v, xchg, am_s_val, am_s_idx);
+            // two halves of the 16 values, each with all splits' loads in flight
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf) {
+              float4 p[kMaxSplit][2];
+#pragma unroll
+              for (int sp = 0; sp < kMaxSplit; ++sp)
+                if (sp < a.split_k) {
+                  const float4* src = reinterpret_cast<const float4*>(
+                      base + sp * tstride + (static_cast<size_t>(c) * 128 + row) * 16) + 2 * hf;
+                  p[sp][0] = __ldcg(src);
+                  p[sp][1] = __ldcg(src + 1);
+                }
+#pragma unroll
+              for (int q2 = 0; q2 < 2; ++q2) {
+                float4 t = p[0][q2];
+#pragma unroll
+                for (int sp = 1; sp < kMaxSplit; ++sp)
+                  if (sp < a.split_k) {
+                    t.x += p[sp][q2].x;
+                    t.y += p[sp][q2].y;
+                    t.z += p[sp][q2].z;
+                    t.w += p[sp][q2].w;
+                  }
+                const int q4 = 2 * hf + q2;
+                v[4 * q4] = t.x;
+                v[4 * q4 + 1] = t.y;
+                v[4 * q4 + 2] = t.z;
+                v[4 * q4 + 3] = t.w;
+              }
+            }
+            epi_post<EPI>(a, it, row, c * 16, v, cur, esm, c & 1);
+            cur = nxt;
+            if (rope && c + 1 < nchunks) {
+              rope_store(esm, (c + 1) & 1, rr);
+              named_bar_sync(1, 128);
+            }
           }
         }
       }
@@ -512,7 +646,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, C::TMEM_COLS);
+    tmem_dealloc(tmem_base, tmem_cols);
   }
 }
 

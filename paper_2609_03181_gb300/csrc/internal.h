@@ -77,6 +77,8 @@ struct GemmArgs {
   int half_rows;
   int n_routed;                // experts with id >= n_routed read a_map[1] and source 1
   int split_k;                 // >= 1, fixed per matrix shape
+  int seq_split;               // dense, split_k > 1: one CTA computes every split of a tile into
+                               // its own TMEM accumulator (64-row boxes), no partials in memory
   const int4* items;           // grouped: device item list
   const int* n_items_dev;      //          and its length
   int n_items;                 // dense: number of items
@@ -117,11 +119,13 @@ void set_thread_error(const std::string& msg);
 // Kernel attributes (dynamic shared memory limits) set once, before any launch or capture.
 cudaError_t gemm_prepare();
 cudaError_t attention_prepare();
-cudaError_t permute_prepare();
+cudaError_t router_prepare();
 
 // Split-K count of a dense matrix: depends on (N, K) only, never on M, so every row's sum
-// order is the same at any batch size.
+// order is the same at any batch size.  From kSeqSplitRows activation rows on, the splits of
+// a tile are computed by one CTA (GemmArgs::seq_split) instead of one CTA each.
 int dense_split_k(int N, int K);
+constexpr int kSeqSplitRows = 128;
 
 // ------------------------------------------------------------------------- other kernels
 struct AttnArgs {
@@ -154,11 +158,15 @@ cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, c
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
                               int* err, cudaStream_t s);
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
-cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
-                          const float* bias, bf16* xn, int* idx, float* gate, int* err, cudaStream_t s);
-cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
-                           int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
-                           unsigned long long* expert_ctr, cudaStream_t s);
+// Router (+ expert grouping by the last CTA) and the permute row gather.
+struct RouteArgs {
+  const float* h; const bf16* gain; float eps; const bf16* wr; const float* bias;
+  bf16* xn; int* idx; float* gate; int* err; int T;
+  int* dst_row; int* sorted_tok; int* sorted_slot; int4* items_gu; int4* items_dn; int* n_items; int* counts;
+  unsigned long long* expert_ctr; int* ticket;
+};
+cudaError_t router_launch(const RouteArgs& a, cudaStream_t s);
+cudaError_t permute_launch(const int* dst_row, int T, const bf16* xn, bf16* x_sorted, cudaStream_t s);
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
                            bf16* out, cudaStream_t s);
 cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots, const int* m_ws, const int* vtok_ws,

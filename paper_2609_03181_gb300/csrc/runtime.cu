@@ -80,6 +80,8 @@ struct spec_ctx {
   float* attn_part = nullptr;
   int* attn_tickets = nullptr;
   int* commit_tickets = nullptr;
+  int* route_ticket = nullptr;
+  int* dst_row = nullptr;       // [Tmax * top_k] expert-sorted row of each (token, slot) pair
   bf16* attn_out = nullptr;
   int* route_idx = nullptr;
   float* route_gate = nullptr;
@@ -191,11 +193,17 @@ cudaError_t run_dense(spec_ctx* ctx, GemmArgs g, int epi, const CUtensorMap& wma
   g.paired = paired ? 1 : 0;
   g.half_rows = half_rows;
   g.box_log = box_log_for(M < 256 ? M : 256);
-  const int box = 16 << g.box_log;
-  g.m_tiles = (M + box - 1) / box;
   g.n_tiles = paired ? (N / 128) : (N + 127) / 128;
   g.split_k = split ? dense_split_k(N, K) : 1;
-  g.n_items = g.n_tiles * g.split_k * g.m_tiles;
+  if (g.split_k > 1 && M >= kSeqSplitRows) {
+    // many rows: one CTA per (weight tile, 64 rows) computes every split into its own TMEM
+    // accumulator and adds them in split order -- the same sums as the cross-CTA split
+    g.seq_split = 1;
+    g.box_log = 2;
+  }
+  const int box = 16 << g.box_log;
+  g.m_tiles = (M + box - 1) / box;
+  g.n_items = g.n_tiles * (g.seq_split ? 1 : g.split_k) * g.m_tiles;
   const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
   return gemm_launch(epi, box <= 64 ? 64 : 256, g, grid, ctx->stream);
 }
@@ -377,7 +385,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   {
     cudaError_t e = gemm_prepare();
     if (e == cudaSuccess) e = attention_prepare();
-    if (e == cudaSuccess) e = permute_prepare();
+    if (e == cudaSuccess) e = router_prepare();
     if (e != cudaSuccess) return fail(nullptr, SPEC_ECUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
   }
   ctx = new spec_ctx();
@@ -427,6 +435,8 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
                            Rmax * kAttnPartStride);
   add(&ctx->attn_tickets, sizeof(int) * Bmax * kH);
   add(&ctx->commit_tickets, sizeof(int) * Bmax);
+  add(&ctx->route_ticket, sizeof(int));
+  add(&ctx->dst_row, sizeof(int) * Tmax * kTopK);
   add(&ctx->attn_out, sizeof(bf16) * Tmax * d);
   add(&ctx->route_idx, sizeof(int) * L * Tmax * kTopK);
   add(&ctx->route_gate, sizeof(float) * L * Tmax * kTopK);
@@ -705,11 +715,30 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
     }
     int* ridx = ctx->route_idx + static_cast<size_t>(l) * ctx->Tmax * kTopK;
     float* rgate = ctx->route_gate + static_cast<size_t>(l) * ctx->Tmax * kTopK;
-    LAUNCH(SPEC_K_ROUTER, 1, router_launch(ctx->h, T, static_cast<const bf16*>(W.moe_norm), eps, static_cast<const bf16*>(W.router),
-                     W.router_bias, ctx->xn, ridx, rgate, ctx->d_err, s));
-    LAUNCH(SPEC_K_PERMUTE, 1, permute_launch(ridx, T, ctx->xn, ctx->x_sorted, ctx->sorted_tok, ctx->sorted_slot,
-                                              ctx->items_gu, ctx->items_dn, ctx->n_items, ctx->counts + l * kE,
-                                              ctx->d_expert_ctr, s));
+    {
+      RouteArgs ra;
+      ra.h = ctx->h;
+      ra.gain = static_cast<const bf16*>(W.moe_norm);
+      ra.eps = eps;
+      ra.wr = static_cast<const bf16*>(W.router);
+      ra.bias = W.router_bias;
+      ra.xn = ctx->xn;
+      ra.idx = ridx;
+      ra.gate = rgate;
+      ra.err = ctx->d_err;
+      ra.T = T;
+      ra.dst_row = ctx->dst_row;
+      ra.sorted_tok = ctx->sorted_tok;
+      ra.sorted_slot = ctx->sorted_slot;
+      ra.items_gu = ctx->items_gu;
+      ra.items_dn = ctx->items_dn;
+      ra.n_items = ctx->n_items;
+      ra.counts = ctx->counts + l * kE;
+      ra.expert_ctr = ctx->d_expert_ctr;
+      ra.ticket = ctx->route_ticket;
+      LAUNCH(SPEC_K_ROUTER, 1, router_launch(ra, s));
+    }
+    LAUNCH(SPEC_K_PERMUTE, 1, permute_launch(ctx->dst_row, T, ctx->xn, ctx->x_sorted, s));
     // routed + shared experts: gate/up + SwiGLU
     {
       GemmArgs g = base_args(ctx);

@@ -102,128 +102,35 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
   return launch_pdl(rmsnorm_kernel, dim3(rows), dim3(128), 0, s, x, gain, eps, out);
 }
 
-// ---------------------------------------------------------------- router
-// RMSNorm of the residual row -> xn (bf16, also the experts' input); logits of the 64
-// experts from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).
-__global__ void __launch_bounds__(256) router_kernel(const float* h, const bf16* gain, float eps, const bf16* wr,
-                                                     const float* bias, bf16* xn, int* idx, float* gate, int* err) {
-  pdl_trigger();
-  pdl_wait();
-  constexpr int NT = 256, EPT = kD / NT;
-  __shared__ float red[NT / 32];
-  __shared__ __align__(16) float xs[kD];
-  __shared__ float lg[kE];
-  const size_t t = blockIdx.x;
-  float v[EPT];
-#pragma unroll
-  for (int k = 0; k < EPT; ++k) v[k] = h[t * kD + threadIdx.x + NT * k];
-  bf16* xo = xn + t * kD;
-  {
-    float ss = 0.f;
-#pragma unroll
-    for (int k = 0; k < EPT; ++k) ss += v[k] * v[k];
-    ss = block_sum<NT>(ss, red);
-    const float inv = rsqrtf(ss / kD + eps);
-#pragma unroll
-    for (int k = 0; k < EPT; ++k) {
-      const int i = threadIdx.x + NT * k;
-      const bf16 r = __float2bfloat16(v[k] * inv * __bfloat162float(gain[i]));
-      xo[i] = r;
-      xs[i] = __bfloat162float(r);   // the rounded row, as the experts see it
-    }
-  }
-  __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int e0 = warp * 8; e0 < warp * 8 + 8; e0 += 4) {
-    // four experts at a time: 20 independent 16-byte weight loads in flight per lane
-    uint4 raw[4][5];
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-#pragma unroll
-      for (int c = 0; c < 5; ++c)
-        raw[q][c] = *reinterpret_cast<const uint4*>(wr + static_cast<size_t>(e0 + q) * kD + c * 256 + lane * 8);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      float acc = 0.f;
-#pragma unroll
-      for (int c = 0; c < 5; ++c) {
-        const int i0 = c * 256 + lane * 8;
-        const bf16* wv = reinterpret_cast<const bf16*>(&raw[q][c]);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) acc += __bfloat162float(wv[u]) * xs[i0 + u];
-      }
-      acc = warp_sum(acc);
-      if (lane == 0) lg[e0 + q] = acc + (bias ? bias[e0 + q] : 0.f);
-    }
-  }
-  __syncthreads();
-  if (warp == 0) {
-    const float l0 = lg[lane], l1 = lg[lane + 32];
-    const float m = warp_max(fmaxf(l0, l1));
-    const float e0 = expf(l0 - m), e1 = expf(l1 - m);
-    const float sum = warp_sum(e0 + e1);
-    float p0 = e0 / sum, p1 = e1 / sum;
-    // a non-finite row still selects six distinct valid experts (NaN ranks below every number)
-    const bool bad = __any_sync(0xffffffffu, !(p0 == p0) || !(p1 == p1));
-    if (bad) {
-      if (lane == 0) atomicOr(err, ERR_NONFINITE);
-      if (!(p0 == p0)) p0 = -1.f;
-      if (!(p1 == p1)) p1 = -1.f;
-    }
-    bool taken0 = false, taken1 = false;
-    for (int k = 0; k < kTopK; ++k) {
-      float bv = -1.f;
-      int bi = 1 << 30;
-      if (!taken0) { bv = p0; bi = lane; }
-      if (!taken1 && better(p1, lane + 32, bv, bi)) { bv = p1; bi = lane + 32; }
-      warp_argmax(bv, bi);
-      if (bi == lane) taken0 = true;
-      if (bi == lane + 32) taken1 = true;
-      if (lane == 0) {
-        idx[t * kTopK + k] = bi;
-        gate[t * kTopK + k] = bv;
-      }
-    }
-  }
-}
-
-cudaError_t router_launch(const float* h, int T, const bf16* gain, float eps, const bf16* w_router,
-                          const float* bias, bf16* xn, int* idx, float* gate, int* err, cudaStream_t s) {
-  return launch_pdl(router_kernel, dim3(T), dim3(256), 0, s, h, gain, eps, w_router, bias, xn, idx, gate, err);
-}
-
-// ---------------------------------------------------------------- permute / scatter
-// Groups the (token, slot) pairs of this layer by expert.  Routed rows of expert e take
-// act rows offs[e] .. offs[e+1]-1 in token order; the two shared experts follow with all T
-// tokens each.  Every CTA builds the ranking in shared memory (a per-expert token bitmap and
-// its prefix popcounts); the copies of the selected activation rows are spread over the
-// grid; CTA 0 writes the sorted index and the GEMM work lists.
-constexpr int kPermThreads = 256;
+// ---------------------------------------------------------------- router + expert grouping
+// RR rows per CTA: 1 for small batches (latency), 4 above 128 rows (the 64 x 1280 router
+// matrix is then read once per four rows).  Per row:
+// RMSNorm of the residual row -> xn (bf16, also the experts' input); logits of the 64 experts
+// from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).  Every row's
+// arithmetic is the same whatever rows share its CTA.
+//
+// Then the CTA that finishes last (atomic ticket, no wait) groups the (token, slot) pairs of
+// the layer by expert: routed rows of expert e take act rows offs[e] .. offs[e+1]-1 in token
+// order (rank from a per-expert token bitmap and its prefix popcounts); the two shared experts
+// follow with all T tokens each.  It writes the destination row of every pair, the sorted
+// token/slot lists, the GEMM work lists and the expert counters.
+constexpr int kRouterRows = 4;
 constexpr int kMaxT = 2048;
 constexpr int kMaxW = kMaxT / 32;
 
-__global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, int T, const bf16* xn, bf16* xs,
-                                                               int* sorted_tok, int* sorted_slot, int4* items_gu,
-                                                               int4* items_dn, int* n_items, int* counts,
-                                                               unsigned long long* expert_ctr) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ int psm[];
-  const int W = (T + 31) / 32;
-  int* s_idx = psm;                       // [T*6]
-  unsigned* bits = reinterpret_cast<unsigned*>(s_idx + T * kTopK);   // [64][W]
-  int* pre = reinterpret_cast<int*>(bits + kE * W);                // [64][W]
+__device__ __forceinline__ void group_by_expert(const RouteArgs& a, int* gsm) {
+  const int T = a.T, W = (T + 31) / 32, T6 = T * kTopK, tid = threadIdx.x;
+  int* s_idx = gsm;                       // [T*6]
+  unsigned* bits = reinterpret_cast<unsigned*>(s_idx + T6);   // [64][W]
+  int* pre = reinterpret_cast<int*>(bits + kE * W);          // [64][W]
   int* cnt = pre + kE * W;                // [66]
   int* offs = cnt + kE + kShared;         // [67]
   int* ibase = offs + kE + kShared + 1;   // [67] gate_up item offsets
   int* dbase = ibase + kE + kShared + 1;  // [67]
-  const int tid = threadIdx.x;
-  const int T6 = T * kTopK;
-  for (int p = tid; p < T6; p += kPermThreads) s_idx[p] = idx[p];
-  for (int p = tid; p < kE * W; p += kPermThreads) bits[p] = 0u;
-  for (int p = tid; p < kE + kShared; p += kPermThreads) cnt[p] = 0;
+  for (int p = tid; p < T6; p += blockDim.x) s_idx[p] = __ldcg(a.idx + p);
+  for (int p = tid; p < kE * W; p += blockDim.x) bits[p] = 0u;
   __syncthreads();
-  for (int p = tid; p < T6; p += kPermThreads) {
+  for (int p = tid; p < T6; p += blockDim.x) {
     const int t = p / kTopK, e = s_idx[p];
     atomicOr(&bits[e * W + (t >> 5)], 1u << (t & 31));
   }
@@ -239,51 +146,63 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, i
     cnt[tid] = T;
   }
   __syncthreads();
-  if (tid == 0) {
-    offs[0] = 0;
-    ibase[0] = 0;
-    dbase[0] = 0;
-    for (int e = 0; e < kE + kShared; ++e) {
-      offs[e + 1] = offs[e] + cnt[e];
-      const int mt = (cnt[e] + 255) / 256;
-      ibase[e + 1] = ibase[e] + mt * (kI / 64);
-      dbase[e + 1] = dbase[e] + mt * (kD / 128);
+  if (tid < 32) {
+    // exclusive prefix sums over the 66 experts (three per lane, lanes in order)
+    int c3[3], m3[3];
+    int sc = 0, sm = 0;
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      const int e = tid * 3 + k;
+      c3[k] = (e < kE + kShared) ? cnt[e] : 0;
+      m3[k] = (c3[k] + 255) / 256;
+      sc += c3[k];
+      sm += m3[k];
     }
-    if (blockIdx.x == 0) {
-      n_items[0] = ibase[kE + kShared];
-      n_items[1] = dbase[kE + kShared];
+    int ic = sc, im = sm;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int xc = __shfl_up_sync(0xffffffffu, ic, o), xm = __shfl_up_sync(0xffffffffu, im, o);
+      if (tid >= o) {
+        ic += xc;
+        im += xm;
+      }
+    }
+    int rc = ic - sc, rm = im - sm;   // exclusive
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      const int e = tid * 3 + k;
+      if (e <= kE + kShared) {
+        offs[e] = rc;
+        ibase[e] = rm * (kI / 64);
+        dbase[e] = rm * (kD / 128);
+      }
+      rc += c3[k];
+      rm += m3[k];
+    }
+    if (tid == 31) {
+      a.n_items[0] = im * (kI / 64);
+      a.n_items[1] = im * (kD / 128);
     }
   }
   __syncthreads();
-  // copies of the routed activation rows, one warp per pair, spread over the grid
-  const int warp = tid >> 5, lane = tid & 31;
-  const int gw = blockIdx.x * (kPermThreads / 32) + warp, nw = gridDim.x * (kPermThreads / 32);
-  for (int p = gw; p < T6; p += nw) {
-    const int t = p / kTopK, e = s_idx[p];
-    const int rank = pre[e * W + (t >> 5)] + __popc(bits[e * W + (t >> 5)] & ((1u << (t & 31)) - 1u));
-    const int dst = offs[e] + rank;
-    const uint4* src = reinterpret_cast<const uint4*>(xn + static_cast<size_t>(t) * kD);
-    uint4* d = reinterpret_cast<uint4*>(xs + static_cast<size_t>(dst) * kD);
-    for (int c = lane; c < kD / 8; c += 32) d[c] = src[c];
+  for (int p = tid; p < T6; p += blockDim.x) {
+    const int t = p / kTopK, sl = p % kTopK, e = s_idx[p];
+    const int dst = offs[e] + pre[e * W + (t >> 5)] + __popc(bits[e * W + (t >> 5)] & ((1u << (t & 31)) - 1u));
+    a.dst_row[p] = dst;
+    a.sorted_tok[dst] = t;
+    a.sorted_slot[dst] = sl;
   }
-  if (blockIdx.x != 0) return;
-  for (int p = tid; p < T6; p += kPermThreads) {
-    const int t = p / kTopK, s = p % kTopK, e = s_idx[p];
-    const int rank = pre[e * W + (t >> 5)] + __popc(bits[e * W + (t >> 5)] & ((1u << (t & 31)) - 1u));
-    sorted_tok[offs[e] + rank] = t;
-    sorted_slot[offs[e] + rank] = s;
-  }
-  for (int p = tid; p < kShared * T; p += kPermThreads) {
+  for (int p = tid; p < kShared * T; p += blockDim.x) {
     const int j = p / T, t = p % T;
-    sorted_tok[offs[kE + j] + t] = t;
-    sorted_slot[offs[kE + j] + t] = kTopK + j;
+    a.sorted_tok[offs[kE + j] + t] = t;
+    a.sorted_slot[offs[kE + j] + t] = kTopK + j;
   }
   if (tid < kE + kShared) {
     const int e = tid, n = cnt[e];
-    if (e < kE) counts[e] = n;
+    if (e < kE) a.counts[e] = n;
     if (n > 0) {
-      atomicAdd(&expert_ctr[0], 1ull);
-      atomicAdd(&expert_ctr[1], static_cast<unsigned long long>(n));
+      atomicAdd(&a.expert_ctr[0], 1ull);
+      atomicAdd(&a.expert_ctr[1], static_cast<unsigned long long>(n));
     }
     const int mt = (n + 255) / 256;
     for (int m = 0; m < mt; ++m) {
@@ -291,30 +210,173 @@ __global__ void __launch_bounds__(kPermThreads) permute_kernel(const int* idx, i
       const int out_row = offs[e] + 256 * m;
       const int b_row_gu = (e < kE) ? out_row : 256 * m;   // shared experts read xn rows directly
       for (int nt = 0; nt < kI / 64; ++nt)
-        items_gu[ibase[e] + m * (kI / 64) + nt] = make_int4(e | (nt << 16), b_row_gu, out_row, rows);
+        a.items_gu[ibase[e] + m * (kI / 64) + nt] = make_int4(e | (nt << 16), b_row_gu, out_row, rows);
       for (int nt = 0; nt < kD / 128; ++nt)
-        items_dn[dbase[e] + m * (kD / 128) + nt] = make_int4(e | (nt << 16), out_row, out_row, rows);
+        a.items_dn[dbase[e] + m * (kD / 128) + nt] = make_int4(e | (nt << 16), out_row, out_row, rows);
     }
   }
 }
 
-cudaError_t permute_prepare() {
-  return cudaFuncSetAttribute(permute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(sizeof(int) * (kMaxT * kTopK + 2 * kE * kMaxW + 4 * 67)));
+template <int RR>
+__global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ RouteArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  constexpr int NT = 256, EPT = kD / NT;
+  __shared__ float red[NT / 32][RR];
+  __shared__ __align__(16) float xs[RR][kD];
+  __shared__ float lg[RR][kE];
+  __shared__ int s_last;
+  extern __shared__ int gsm[];
+  const int t0 = blockIdx.x * RR;
+  const int nr = min(RR, a.T - t0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  {
+    float v[RR][EPT];
+    float ss[RR];
+#pragma unroll
+    for (int r = 0; r < RR; ++r) {
+#pragma unroll
+      for (int k = 0; k < EPT; ++k) v[r][k] = (r < nr) ? a.h[static_cast<size_t>(t0 + r) * kD + threadIdx.x + NT * k] : 0.f;
+      ss[r] = 0.f;
+#pragma unroll
+      for (int k = 0; k < EPT; ++k) ss[r] += v[r][k] * v[r][k];
+      ss[r] = warp_sum(ss[r]);
+    }
+    if (lane == 0)
+#pragma unroll
+      for (int r = 0; r < RR; ++r) red[warp][r] = ss[r];
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < RR; ++r) {
+      if (r >= nr) break;
+      float tot = red[0][r];
+#pragma unroll
+      for (int w = 1; w < NT / 32; ++w) tot += red[w][r];
+      const float inv = rsqrtf(tot / kD + a.eps);
+      bf16* xo = a.xn + static_cast<size_t>(t0 + r) * kD;
+#pragma unroll
+      for (int k = 0; k < EPT; ++k) {
+        const int i = threadIdx.x + NT * k;
+        const bf16 rb = __float2bfloat16(v[r][k] * inv * __bfloat162float(a.gain[i]));
+        xo[i] = rb;
+        xs[r][i] = __bfloat162float(rb);   // the rounded row, as the experts see it
+      }
+    }
+  }
+  __syncthreads();
+  for (int e0 = warp * 8; e0 < warp * 8 + 8; e0 += 4) {
+    // four experts at a time: 20 independent 16-byte weight loads in flight per lane, each
+    // weight used for every row of the CTA
+    uint4 raw[4][5];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int c = 0; c < 5; ++c)
+        raw[q][c] = *reinterpret_cast<const uint4*>(a.wr + static_cast<size_t>(e0 + q) * kD + c * 256 + lane * 8);
+#pragma unroll
+    for (int r = 0; r < RR; ++r) {
+      if (r >= nr) break;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float acc = 0.f;
+#pragma unroll
+        for (int c = 0; c < 5; ++c) {
+          const int i0 = c * 256 + lane * 8;
+          const bf16* wv = reinterpret_cast<const bf16*>(&raw[q][c]);
+#pragma unroll
+          for (int u = 0; u < 8; ++u) acc += __bfloat162float(wv[u]) * xs[r][i0 + u];
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) lg[r][e0 + q] = acc + (a.bias ? a.bias[e0 + q] : 0.f);
+      }
+    }
+  }
+  __syncthreads();
+  if (warp < nr) {
+    const int r = warp;
+    const size_t t = t0 + r;
+    const float l0 = lg[r][lane], l1 = lg[r][lane + 32];
+    const float m = warp_max(fmaxf(l0, l1));
+    const float e0 = expf(l0 - m), e1 = expf(l1 - m);
+    const float sum = warp_sum(e0 + e1);
+    float p0 = e0 / sum, p1 = e1 / sum;
+    // a non-finite row still selects six distinct valid experts (NaN ranks below every number)
+    const bool bad = __any_sync(0xffffffffu, !(p0 == p0) || !(p1 == p1));
+    if (bad) {
+      if (lane == 0) atomicOr(a.err, ERR_NONFINITE);
+      if (!(p0 == p0)) p0 = -1.f;
+      if (!(p1 == p1)) p1 = -1.f;
+    }
+    bool taken0 = false, taken1 = false;
+    for (int k = 0; k < kTopK; ++k) {
+      float bv = -1.f;
+      int bi = 1 << 30;
+      if (!taken0) { bv = p0; bi = lane; }
+      if (!taken1 && better(p1, lane + 32, bv, bi)) { bv = p1; bi = lane + 32; }
+      warp_argmax(bv, bi);
+      if (bi == lane) taken0 = true;
+      if (bi == lane + 32) taken1 = true;
+      if (lane == 0) {
+        a.idx[t * kTopK + k] = bi;
+        a.gate[t * kTopK + k] = bv;
+      }
+    }
+  }
+  // the last CTA to finish groups the layer's pairs by expert
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int old = atomicAdd(a.ticket, 1);
+    s_last = (old == static_cast<int>(gridDim.x) - 1) ? 1 : 0;
+    if (s_last) *a.ticket = 0;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  group_by_expert(a, gsm);
 }
 
-cudaError_t permute_launch(const int* idx, int T, const bf16* xn, bf16* x_sorted, int* sorted_tok,
-                           int* sorted_slot, int4* items_gu, int4* items_dn, int* n_items, int* counts,
-                           unsigned long long* expert_ctr, cudaStream_t s) {
-  if (T > kMaxT) return cudaErrorInvalidValue;
-  const int W = (T + 31) / 32;
-  const size_t smem = sizeof(int) * (static_cast<size_t>(T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
+cudaError_t router_prepare() {
+  const int smem = static_cast<int>(sizeof(int) * (kMaxT * kTopK + 2 * kE * kMaxW + 4 * 67));
+  cudaError_t e = cudaFuncSetAttribute(router_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(router_kernel<kRouterRows>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  return e;
+}
+
+cudaError_t router_launch(const RouteArgs& a, cudaStream_t s) {
+  if (a.T > kMaxT || a.T < 1) return cudaErrorInvalidValue;
+  const int W = (a.T + 31) / 32;
+  const size_t smem = sizeof(int) * (static_cast<size_t>(a.T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
+  if (a.T <= 128) return launch_pdl(router_kernel<1>, dim3(a.T), dim3(256), smem, s, a);
+  return launch_pdl(router_kernel<kRouterRows>, dim3((a.T + kRouterRows - 1) / kRouterRows), dim3(256), smem, s, a);
+}
+
+// ---------------------------------------------------------------- permute (row gather)
+// Copies the normalised row of every routed (token, slot) pair to its expert-sorted row of
+// the experts' input, one warp per pair, all of a row's loads issued before its stores.
+__global__ void __launch_bounds__(256) permute_kernel(const int* dst_row, int T6, const bf16* xn, bf16* xs) {
+  pdl_trigger();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * 8 + warp, nw = gridDim.x * 8;
+  for (int p = gw; p < T6; p += nw) {
+    const int t = p / kTopK, dst = dst_row[p];
+    const uint4* src = reinterpret_cast<const uint4*>(xn + static_cast<size_t>(t) * kD);
+    uint4* d = reinterpret_cast<uint4*>(xs + static_cast<size_t>(dst) * kD);
+    uint4 v[kD / 8 / 32];
+#pragma unroll
+    for (int c = 0; c < kD / 8 / 32; ++c) v[c] = src[lane + 32 * c];
+#pragma unroll
+    for (int c = 0; c < kD / 8 / 32; ++c) d[lane + 32 * c] = v[c];
+  }
+}
+
+cudaError_t permute_launch(const int* dst_row, int T, const bf16* xn, bf16* x_sorted, cudaStream_t s) {
   const int pairs = T * kTopK;
   int grid = (pairs + 7) / 8;     // one warp per (token, slot) row copy
-  if (grid > 512) grid = 512;
+  if (grid > 1024) grid = 1024;
   if (grid < 1) grid = 1;
-  return launch_pdl(permute_kernel, dim3(grid), dim3(kPermThreads), smem, s, idx, T, xn, x_sorted, sorted_tok, sorted_slot, items_gu, items_dn,
-                                                  n_items, counts, expert_ctr);
+  return launch_pdl(permute_kernel, dim3(grid), dim3(256), 0, s, dst_row, pairs, xn, x_sorted);
 }
 
 // ---------------------------------------------------------------- combine

@@ -163,3 +163,41 @@ def test_speculative_with_accepting_draft_head_equals_greedy(succ):
     got, ms = run_loop(succ, N_TOK, K, "head")
     assert got == greedy
     assert sum(ms) > 0, "the tuned draft head should get drafts accepted"
+
+
+def test_rows_identical_across_gemm_schedules():
+    """Batch invariance across the two dense-GEMM schedules: with few rows every split of K runs
+    in its own CTA (partials reduced through memory), from 128 rows on one CTA runs all splits of
+    a tile into separate TMEM accumulators.  Sequence 0 verified alone (4 rows) and as row 0 of
+    a batch of 40 (160 rows), then drafted alone (4 depth-1 rows) and in the batch (160 rows):
+    the b rows, verifier tokens, draft states u and draft tokens are bit-identical."""
+    seed, Bb = 31, 40
+    vw = S.verifier_weights(SHAPE, seed, gain_std=0.1)
+    dw = S.draft_weights(SHAPE, seed, gain_std=0.1)
+    ctx = [int(c) for c in S.integers(seed, "ctx", Bb, 30, 120)]
+    kvs = [S.kv_prefix(seed, b, SHAPE.n_layers, ctx[b], SHAPE.n_heads, SHAPE.head_dim) for b in range(Bb)]
+    dkvs = [S.draft_kv_prefix(seed, b, ctx[b], SHAPE.n_heads, SHAPE.head_dim) for b in range(Bb)]
+    pend = [int(x) for x in S.integers(seed, "pending", Bb, 0, SHAPE.vocab - 1)]
+    eng = F.Engine(vw, dw, max_batch=Bb, K_max=K, max_ctx=max(ctx) + 16, page_size=64)
+    dev = torch.device("cuda")
+    res = []
+    for bsz in (1, Bb):
+        for b in range(bsz):
+            eng.load_prefix(b, kvs[b], dkvs[b], pend[b])
+        slots = torch.arange(bsz, dtype=torch.int32, device=dev)
+        cand = torch.tensor([[pend[b], 11, 12, 13] for b in range(bsz)], dtype=torch.int32, device=dev)
+        vt = torch.empty(bsz, K + 1, dtype=torch.int32, device=dev)
+        acc = torch.empty(bsz, dtype=torch.int32, device=dev)
+        eng.verify_step(slots, cand, vt, acc)
+        bst = eng.read_workspace(F.WS_B, (bsz * (K + 1), SHAPE.hidden), torch.bfloat16)
+        com = torch.empty(bsz, K + 1, dtype=torch.int32, device=dev)
+        nc = torch.empty(bsz, dtype=torch.int32, device=dev)
+        eng.accept_commit(slots, com, nc)
+        dcand = torch.empty(bsz, K + 1, dtype=torch.int32, device=dev)
+        eng.draft_step(slots, K, dcand)
+        u = eng.read_workspace(F.WS_DRAFT_U, (K, eng.max_batch, SHAPE.hidden), torch.bfloat16)
+        eng.sync()
+        res.append((bst[: K + 1].clone(), vt[0].cpu().clone(), u[:, 0].clone(), dcand[0].cpu().clone()))
+    eng.close()
+    for x, y in zip(res[0], res[1]):
+        assert torch.equal(x, y)
