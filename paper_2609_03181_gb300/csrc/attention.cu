@@ -11,15 +11,16 @@
 // per query, rescaled by 2^(M_old - M_new) when the max grows); a query's result is the merge
 // of its super-chunks in order, O = sum_s w_s O_s / sum_s w_s L_s with w_s = 2^(M_s - max M).
 // Scores K q^T and outputs V^T p^T run on bf16 tensor cores (mma.sync m16n8k16, fp32
-// accumulation, queries padded to 8); p enters the product as two bf16 terms (hi + lo, about
-// 16 bits); the transposes between the score and the product layouts stay in registers
-// (movmatrix).  Masked keys contribute exact zeros, so a query's result is the same whether
+// accumulation, queries padded to 8); a score sums its even and its odd 16-dim steps
+// separately, then adds the two; p enters the product as two bf16 terms (hi + lo, about 16
+// bits) whose products accumulate separately over a super-chunk and are added at its end; the
+// transposes between the score and the product layouts stay in registers (movmatrix).  Masked keys contribute exact zeros, so a query's result is the same whether
 // its keys sit in pages or in staging and however many queries or sequences share the launch:
 // greedy decoding (K = 0) and speculative verification see identical rows.
 //
-// Scheduling: one warp per CTA, two CTAs per SM.  A CTA owns a unit of consecutive
-// super-chunks of one (sequence, head) and streams its chunks through three private shared-
-// memory stages.  A chunk whose 64 keys are all committed is one page segment per head: its K
+// Scheduling: one warp per CTA, two CTAs per SM.  The CTAs of one (sequence, head) take its
+// super-chunks in turn (CTA u: super-chunks u, u + n, u + 2n, ...), each streaming its chunks
+// through three private shared-memory stages.  A chunk whose 64 keys are all committed is one page segment per head: its K
 // and V rows are two contiguous 16 KB blocks, fetched as four TMA boxes (64 rows x 128 bytes,
 // 128-byte swizzle) onto the stage's mbarrier, issued up to three chunks ahead.  The chunk
 // holding the newest keys (staged candidates, masked positions) is gathered row by row with
@@ -37,12 +38,12 @@ constexpr int kCH = kAttnChunk;                  // keys per chunk (64)
 constexpr int kSuper = kAttnSuper;               // chunks per super-chunk
 constexpr int kUnitMaxSuper = 4;                 // most super-chunks one CTA streams
 constexpr int kUnitMaxChunks = kSuper * kUnitMaxSuper;
-constexpr int kStages = 3;
 constexpr int kHalfBytes = kCH * 128;            // 64 rows x 64 dims of K or V: 8 KB
 constexpr int kTileBytes = 2 * kHalfBytes;       // K (or V) of a chunk: 16 KB
 constexpr int kStageBytes = 2 * kTileBytes;      // K and V of a chunk: 32 KB
 constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
-constexpr int kAttnSmem = 1024 + kStages * kStageBytes + kMaxR * kHD * 2 + kStages * 8;
+// shared memory of a CTA with `stages` stages: 1 KB alignment slack, the stages, Q, barriers
+constexpr int attn_smem(int stages) { return 1024 + stages * kStageBytes + kMaxR * kHD * 2 + stages * 8; }
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
@@ -198,12 +199,15 @@ __device__ __forceinline__ void gather_chunk(const AttnArgs& a, int b, int h, in
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
 
+// kStages stages per CTA: 3 (two CTAs per SM) when the launch spans many waves, 2 (three CTAs
+// per SM) when it fits in about two.
+template <int kStages>
 __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ uint8_t asmem_raw[];
   const uint32_t raw_u32 = smem_u32(asmem_raw);
-  uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [3][K 16 KB | V 16 KB]
+  uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [S][K 16 KB | V 16 KB]
   uint8_t* sQ = stages + kStages * kStageBytes;              // [8 queries][128 dims] bf16
-  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + kMaxR * kHD * 2);   // [3] TMA stage barriers
+  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + kMaxR * kHD * 2);   // [S] TMA stage barriers
   __shared__ int s_page[kUnitMaxChunks];                     // page of each TMA chunk of the unit
   __shared__ int s_abort;
   pdl_trigger();
@@ -213,45 +217,66 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   const int lane = threadIdx.x;
   const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
   const int R = a.R;
+  // the queries first (bf16, as the QKV epilogue stored them; rows R..7 zero): their loads need
+  // no slot and overlap the slot -> length -> page lookups
+  uint4 qv[4];
+  {
+    const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int v = lane + 32 * i, q = v >> 4, ch = v & 15;   // 8 queries x 16 pieces of 16 bytes
+      qv[i] = make_uint4(0, 0, 0, 0);
+      if (q < R) qv[i] = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
+    }
+  }
   const int slot = a.slots[b];
   if (slot < 0 || slot >= a.n_slots) {   // every CTA of the sequence leaves; no ticket, no merge
     if (u == 0 && h == 0 && lane == 0) atomicOr(a.err, ERR_SLOT_RANGE);
     return;
+  }
+  // this CTA's super-chunks: u, u + n_units, u + 2 n_units, ... (strided, so that short contexts
+  // spread over the CTAs of the (sequence, head) as evenly as long ones); its chunk list, in
+  // increasing order, is chunk_of(i)
+  const int n_units = gridDim.x;
+  auto chunk_of = [&](int i) { return (u + (i / kSuper) * n_units) * kSuper + i % kSuper; };
+  // the pages of every chunk the CTA may own are looked up now, alongside the length
+  int spec_page = -1;
+  if (lane < a.unit * kSuper) {
+    const int pi = chunk_of(lane) * kCH / a.page_size;
+    if (pi < a.max_pages) spec_page = a.block_table[slot * a.max_pages + pi];
   }
   const int sl = a.seq_len[slot];
   const int p0 = sl + a.qoff;
   const int last = p0 + R - 1;
   if (p0 < 0) return;
   const int n_live = last / kCH + 1;                         // chunks holding keys 0..last
-  const int c0 = u * a.unit * kSuper;
-  if (c0 >= n_live) return;
-  const int c1 = min(c0 + a.unit * kSuper, n_live);
-  const int n = c1 - c0;
-  // chunks c0..c0+n_tma-1 hold committed keys only and come by TMA; the rest are gathered
-  const int n_tma = a.use_tma ? max(0, min(c1, sl / kCH) - c0) : 0;
+  const int n_sup_live = (n_live + kSuper - 1) / kSuper;
+  if (u >= n_sup_live) return;
+  const int n_mine = (n_sup_live - 1 - u) / n_units + 1;            // super-chunks of this CTA
+  const int last_sup = u + (n_mine - 1) * n_units;
+  const int n = (n_mine - 1) * kSuper + (min(n_live, (last_sup + 1) * kSuper) - last_sup * kSuper);
+  // a prefix of the list holds committed keys only and comes by TMA; the rest are gathered
+  int n_tma = 0;
+  if (a.use_tma)
+    while (n_tma < n && (chunk_of(n_tma) + 1) * kCH <= sl) ++n_tma;
 
-  for (int i = lane; i < n_tma; i += 32) {
-    const int pi = (c0 + i) * kCH / a.page_size;
-    int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+  if (lane < n_tma) {
+    int page = spec_page;
     if (page < 0 || page >= a.n_pages) {
       atomicOr(a.err, ERR_PAGE_RANGE);
       page = -1;
     }
-    s_page[i] = page;
+    s_page[lane] = page;
   }
   if (lane == 0) {
     for (int st = 0; st < kStages; ++st) mbar_init(&full[st], 1);
     s_abort = 0;
     fence_mbar_init();
   }
-  // queries (bf16, as the QKV epilogue stored them); rows R..7 are zero
-  const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const int v = lane + 32 * i, q = v >> 4, ch = v & 15;   // 8 queries x 16 pieces of 16 bytes
-    uint4 val = make_uint4(0, 0, 0, 0);
-    if (q < R) val = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
-    *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = val;
+    const int v = lane + 32 * i, q = v >> 4, ch = v & 15;
+    *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = qv[i];
   }
   __syncwarp();
 
@@ -266,7 +291,7 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
       mbar_arrive(&full[st]);
       return;
     }
-    const int c = c0 + i;
+    const int c = chunk_of(i);
     const int row_k = (page * 2 * kH + h) * a.page_size + (c * kCH) % a.page_size;
     const int row_v = row_k + kH * a.page_size;
     mbar_arrive_expect_tx(&full[st], kStageBytes);
@@ -290,18 +315,20 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   const int qa = 2 * t4, qb = 2 * t4 + 1;                    // the two queries of this lane
   float* part = a.part + (static_cast<size_t>(b) * kH + h) * ((a.n_chunks + kSuper - 1) / kSuper) * R * kPartStride;
   float M_a = -INFINITY, M_b = -INFINITY, L_a = 0.f, L_b = 0.f;
-  float O[8][4];
+  float O[8][4], Ol[8][4];   // hi and lo parts of the unnormalised output
   int consumed = 0;   // TMA chunks waited for
   bool aborted = false;
   for (int i = 0; i < n; ++i) {
-    const int c = c0 + i;
+    const int c = chunk_of(i);
     const int st = i % kStages;
     uint8_t* stage = stages + st * kStageBytes;
     if (c % kSuper == 0 || i == 0) {
       M_a = M_b = -INFINITY;
       L_a = L_b = 0.f;
 #pragma unroll
-      for (int dt = 0; dt < 8; ++dt) O[dt][0] = O[dt][1] = O[dt][2] = O[dt][3] = 0.f;
+      for (int dt = 0; dt < 8; ++dt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) O[dt][e] = Ol[dt][e] = 0.f;
     }
     if (i < n_tma) {
       const bool ok = mbar_wait(&full[st], static_cast<uint32_t>(i / kStages) & 1u, &s_abort);
@@ -318,19 +345,28 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
     const uint32_t kbase = smem_u32(stage);
     const uint32_t vbase = kbase + kTileBytes;
 
-    // S^T[key][query] = K Q^T over four 16-key tiles, 8 k-steps of 16 dims
-    float s[4][4];
+    // S^T[key][query] = K Q^T over four 16-key tiles, 8 k-steps of 16 dims: even and odd
+    // k-steps in separate accumulators (eight independent MMA chains), added at the end
+    float s[4][4], s1[4][4];
 #pragma unroll
-    for (int kt = 0; kt < 4; ++kt) s[kt][0] = s[kt][1] = s[kt][2] = s[kt][3] = 0.f;
+    for (int kt = 0; kt < 4; ++kt)
 #pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {
+      for (int e = 0; e < 4; ++e) s[kt][e] = s1[kt][e] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < 8; ks += 2) {
 #pragma unroll
       for (int kt = 0; kt < 4; ++kt) {
-        uint32_t ak[4];
+        uint32_t ak[4], ak1[4];
         ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + (mi >> 1)), ak);
+        ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + 2 + (mi >> 1)), ak1);
         mma_bf16_16816(s[kt], ak, qf[ks]);
+        mma_bf16_16816(s1[kt], ak1, qf[ks + 1]);
       }
     }
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) s[kt][e] += s1[kt][e];
     // visibility, chunk max per query (lanes sharing t4 hold the same two queries)
     const int kb = c * kCH;
     float m_a = -INFINITY, m_b = -INFINITY;
@@ -381,13 +417,18 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
     }
     L_a = L_a * al_a + l_a;
     L_b = L_b * al_b + l_b;
-    // O^T[dim][query] = al * O^T + V^T P^T: eight 16-dim tiles, 4 k-steps of 16 keys
+    // O^T[dim][query] = al * O^T + V^T P^T: eight 16-dim tiles, 4 k-steps of 16 keys; the hi
+    // and lo products accumulate separately (sixteen independent chains), summed per super-chunk
 #pragma unroll
     for (int dt = 0; dt < 8; ++dt) {
       O[dt][0] *= al_a;
       O[dt][1] *= al_b;
       O[dt][2] *= al_a;
       O[dt][3] *= al_b;
+      Ol[dt][0] *= al_a;
+      Ol[dt][1] *= al_b;
+      Ol[dt][2] *= al_a;
+      Ol[dt][3] *= al_b;
     }
 #pragma unroll
     for (int kt = 0; kt < 4; ++kt) {
@@ -396,25 +437,25 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
         uint32_t av[4];
         ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * dt + (mi & 1)), av);
         mma_bf16_16816(O[dt], av, ph[kt]);
-        mma_bf16_16816(O[dt], av, pl[kt]);
+        mma_bf16_16816(Ol[dt], av, pl[kt]);
       }
     }
     __syncwarp();   // every lane is done with this stage
     if (lane == 0 && i + kStages < n_tma) issue(i + kStages);
 
     // end of a super-chunk: its (M, L, O) per query
-    if ((c + 1) % kSuper == 0 || i + 1 == n) {
+    if ((c + 1) % kSuper == 0 || c + 1 == n_live) {
       float* ps = part + static_cast<size_t>(c / kSuper) * R * kPartStride;
 #pragma unroll
       for (int dt = 0; dt < 8; ++dt) {
         const int d = 16 * dt + g;
         if (qa < R) {
-          ps[qa * kPartStride + d] = O[dt][0];
-          ps[qa * kPartStride + d + 8] = O[dt][2];
+          ps[qa * kPartStride + d] = O[dt][0] + Ol[dt][0];
+          ps[qa * kPartStride + d + 8] = O[dt][2] + Ol[dt][2];
         }
         if (qb < R) {
-          ps[qb * kPartStride + d] = O[dt][1];
-          ps[qb * kPartStride + d + 8] = O[dt][3];
+          ps[qb * kPartStride + d] = O[dt][1] + Ol[dt][1];
+          ps[qb * kPartStride + d + 8] = O[dt][3] + Ol[dt][3];
         }
       }
       if (g == 0) {
@@ -445,12 +486,12 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   // the CTA that finishes the last unit of (sequence, head) merges every query
   __threadfence();
   __syncwarp();
-  const int n_units = (n_live + a.unit * kSuper - 1) / (a.unit * kSuper);
+  const int n_busy = min(n_units, n_sup_live);   // CTAs of this (sequence, head) with work
   int is_last = 0;
   if (lane == 0) {
     int* ticket = a.tickets + b * kH + h;
     const int old = atomicAdd(ticket, 1);
-    is_last = (old == n_units - 1) ? 1 : 0;
+    is_last = (old == n_busy - 1) ? 1 : 0;
     if (is_last) *ticket = 0;
   }
   is_last = __shfl_sync(0xffffffffu, is_last, 0);
@@ -461,13 +502,16 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
 }
 
 cudaError_t attention_prepare() {
-  return cudaFuncSetAttribute(attn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+  cudaError_t e = cudaFuncSetAttribute(attn_chunk_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, attn_smem(2));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_chunk_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, attn_smem(3));
+  return e;
 }
 
 cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
-  // Super-chunks per CTA: enough CTAs for about two waves of two per SM over the largest
-  // context the pools allow.  Pure scheduling: the arithmetic of every super-chunk and of the
-  // merge is the same for any grouping.
+  // At most `unit` super-chunks per CTA: enough CTAs for about two waves of two per SM over the
+  // largest context the pools allow.  Pure scheduling: the arithmetic of every super-chunk and
+  // of the merge is the same for any assignment.
   AttnArgs a = a_in;
   const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
   const long long target = 4ll * num_sms();
@@ -477,7 +521,10 @@ cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
   if (unit > kUnitMaxSuper) unit = kUnitMaxSuper;
   a.unit = unit;
   const int n_units = (n_super + unit - 1) / unit;
-  return launch_pdl(attn_chunk_kernel, dim3(n_units, kH, B), dim3(32), kAttnSmem, s, a);
+  const long long ctas = static_cast<long long>(n_units) * kH * B;
+  if (ctas <= 6ll * num_sms())
+    return launch_pdl(attn_chunk_kernel<2>, dim3(n_units, kH, B), dim3(32), attn_smem(2), s, a);
+  return launch_pdl(attn_chunk_kernel<3>, dim3(n_units, kH, B), dim3(32), attn_smem(3), s, a);
 }
 
 }  // namespace fm

@@ -472,6 +472,17 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       get_item(a, i, it);
       const int acc = local % nbuf;
       const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
+      // the item's metadata, RoPE factors and first old residuals are fetched while its MMAs run
+      stage_meta<EPI>(a, it, esm);
+      const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
+      RopeRegs rr;
+      if (rope) {
+        rope_load(a, it, 0, esm, rr);
+        rope_store(esm, 0, rr);
+        named_bar_sync(1, 128);
+      }
+      EpiPre cur, nxt;
+      epi_pre<EPI>(a, it, row, 0, esm, cur);
       bool ok = mbar_wait(&tfull[acc], acc_ph, s_abort);
       ok = __all_sync(0xffffffffu, ok);
       if (lane == 0) s_vote[ew] = ok ? 1 : 0;
@@ -488,16 +499,6 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       const int nchunks = (it.rows + 15) >> 4;
       float v[16];
       if (a.split_k == 1 || a.seq_split) {
-        stage_meta<EPI>(a, it, esm);
-        const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
-        RopeRegs rr;
-        if (rope) {
-          rope_load(a, it, 0, esm, rr);
-          rope_store(esm, 0, rr);
-          named_bar_sync(1, 128);
-        }
-        EpiPre cur, nxt;
-        epi_pre<EPI>(a, it, row, 0, esm, cur);
         for (int c = 0; c < nchunks; ++c) {
           if (c + 1 < nchunks) {
             epi_pre<EPI>(a, it, row, (c + 1) * 16, esm, nxt);
@@ -549,16 +550,6 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         if (*s_last) {
           __threadfence();
           const float* base = a.sk_ws + static_cast<size_t>(tile) * a.split_k * tstride;
-          stage_meta<EPI>(a, it, esm);
-          const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
-          RopeRegs rr;
-          if (rope) {
-            rope_load(a, it, 0, esm, rr);
-            rope_store(esm, 0, rr);
-            named_bar_sync(1, 128);
-          }
-          EpiPre cur, nxt;
-          epi_pre<EPI>(a, it, row, 0, esm, cur);
           for (int c = 0; c < nchunks; ++c) {
             if (c + 1 < nchunks) {
               epi_pre<EPI>(a, it, row, (c + 1) * 16, esm, nxt);

@@ -126,6 +126,8 @@ cudaError_t router_prepare();
 // a tile are computed by one CTA (GemmArgs::seq_split) instead of one CTA each.
 int dense_split_k(int N, int K);
 constexpr int kSeqSplitRows = 128;
+// Row tile of the grouped expert launches (work-list items cover at most this many rows).
+constexpr int kExpertTileRows = 64;
 
 // ------------------------------------------------------------------------- other kernels
 struct AttnArgs {

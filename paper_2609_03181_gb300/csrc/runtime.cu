@@ -408,7 +408,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ctx->n_chunks = (c.max_pages_per_seq * c.page_size + Rmax + kAttnChunk - 1) / kAttnChunk;
   ctx->lm_tiles = (c.vocab + 127) / 128;
   ctx->dstage_rows = c.K_max > 1 ? c.K_max - 1 : 1;
-  ctx->max_items = static_cast<size_t>(kE + kShared + (Tmax * kSlots) / 256 + 4) * (kI / 64);
+  ctx->max_items = static_cast<size_t>(kE + kShared + (Tmax * kSlots) / kExpertTileRows + 4) * (kI / 64);
   {
     // split-K partials: per split, a tile's rows are padded to the row box (< 2 * rows + 16)
     const int shapes[][2] = {{3 * kD, kD}, {kD, kD}, {kD, 2 * kD}, {kD, kId}, {2 * kId, kD}};
@@ -660,7 +660,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   LAUNCH(SPEC_K_EMBED, 1, embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
                        c.vocab, static_cast<const bf16*>(ctx->layers[0].attn_norm), eps, ctx->h, ctx->xn, ctx->pos,
                        ctx->kv_rowoff, ctx->Rmax, ctx->Bmax, ctx->d_err, s));
-  const int nmax_grouped = T <= 64 ? 64 : 256;
+  const int nmax_grouped = kExpertTileRows;
   for (int l = 0; l < L; ++l) {
     const spec_layer_weights& W = ctx->layers[l];
     const LayerMaps& M = ctx->lmaps[l];

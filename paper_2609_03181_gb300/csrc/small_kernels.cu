@@ -113,7 +113,8 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
 // the layer by expert: routed rows of expert e take act rows offs[e] .. offs[e+1]-1 in token
 // order (rank from a per-expert token bitmap and its prefix popcounts); the two shared experts
 // follow with all T tokens each.  It writes the destination row of every pair, the sorted
-// token/slot lists, the GEMM work lists and the expert counters.
+// token/slot lists, the GEMM work lists (row tiles of at most 64 rows, so every grouped launch
+// runs the deep 8-stage weight pipeline) and the expert counters.
 constexpr int kRouterRows = 4;
 constexpr int kMaxT = 2048;
 constexpr int kMaxW = kMaxT / 32;
@@ -154,7 +155,7 @@ __device__ __forceinline__ void group_by_expert(const RouteArgs& a, int* gsm) {
     for (int k = 0; k < 3; ++k) {
       const int e = tid * 3 + k;
       c3[k] = (e < kE + kShared) ? cnt[e] : 0;
-      m3[k] = (c3[k] + 255) / 256;
+      m3[k] = (c3[k] + kExpertTileRows - 1) / kExpertTileRows;
       sc += c3[k];
       sm += m3[k];
     }
@@ -204,11 +205,11 @@ __device__ __forceinline__ void group_by_expert(const RouteArgs& a, int* gsm) {
       atomicAdd(&a.expert_ctr[0], 1ull);
       atomicAdd(&a.expert_ctr[1], static_cast<unsigned long long>(n));
     }
-    const int mt = (n + 255) / 256;
+    const int mt = (n + kExpertTileRows - 1) / kExpertTileRows;
     for (int m = 0; m < mt; ++m) {
-      const int rows = min(256, n - 256 * m);
-      const int out_row = offs[e] + 256 * m;
-      const int b_row_gu = (e < kE) ? out_row : 256 * m;   // shared experts read xn rows directly
+      const int rows = min(kExpertTileRows, n - kExpertTileRows * m);
+      const int out_row = offs[e] + kExpertTileRows * m;
+      const int b_row_gu = (e < kE) ? out_row : kExpertTileRows * m;   // shared experts read xn rows directly
       for (int nt = 0; nt < kI / 64; ++nt)
         a.items_gu[ibase[e] + m * (kI / 64) + nt] = make_int4(e | (nt << 16), b_row_gu, out_row, rows);
       for (int nt = 0; nt < kD / 128; ++nt)
