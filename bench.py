@@ -87,6 +87,21 @@ def data_desc(args):
     return "synthetic: seeded random-init weights N(0,0.02), N(0,1) KV prefixes"
 
 
+def rank_seed(seed, rank):
+    """Replica r draws its own sequences (contexts, pending tokens, KV prefixes) from seed + 1000 r;
+    the weights are the same on every replica."""
+    return seed + 1000 * rank
+
+
+def sequence_inputs(args, shape, rank=0):
+    """Contexts and pending tokens of the replica's B sequences (host, cheap)."""
+    import synth_inputs as S
+    sd = rank_seed(args.seed, rank)
+    ctx = [int(c) for c in S.integers(sd, "ctx", args.batch, args.ctx_lo, args.ctx_hi)]
+    pend = [int(t) for t in S.integers(sd, "pending", args.batch, 0, shape.vocab - 1)]
+    return ctx, pend
+
+
 def workload(args, rank=0):
     import synth_inputs as S
     shape = S.ModelShape(n_layers=args.layers)
@@ -97,19 +112,30 @@ def workload(args, rank=0):
         vw = S.verifier_weights(shape, seed)
         dw = S.draft_weights(shape, seed)
     B = args.batch
-    ctx = [int(c) for c in S.integers(seed + 1000 * rank, "ctx", B, args.ctx_lo, args.ctx_hi)]
-    pend = [int(t) for t in S.integers(seed + 1000 * rank, "pending", B, 0, shape.vocab - 1)]
+    ctx, pend = sequence_inputs(args, shape, rank)
+    sd = rank_seed(seed, rank)
     if args.device_kv:
         dev = f"cuda:{int(os.environ.get('LOCAL_RANK', '0'))}"
-        kvs = [S.kv_prefix_device(seed + 1000 * rank, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim, dev)
-               for b in range(B)]
-        dkvs = [S.draft_kv_prefix_device(seed + 1000 * rank, b, ctx[b], shape.n_heads, shape.head_dim, dev)
-                for b in range(B)]
+        kvs = [S.kv_prefix_device(sd, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim, dev) for b in range(B)]
+        dkvs = [S.draft_kv_prefix_device(sd, b, ctx[b], shape.n_heads, shape.head_dim, dev) for b in range(B)]
     else:
-        kvs = [S.kv_prefix(seed + 1000 * rank, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim)
-               for b in range(B)]
-        dkvs = [S.draft_kv_prefix(seed + 1000 * rank, b, ctx[b], shape.n_heads, shape.head_dim) for b in range(B)]
+        kvs = [S.kv_prefix(sd, b, shape.n_layers, ctx[b], shape.n_heads, shape.head_dim) for b in range(B)]
+        dkvs = [S.draft_kv_prefix(sd, b, ctx[b], shape.n_heads, shape.head_dim) for b in range(B)]
     return shape, vw, dw, ctx, pend, kvs, dkvs
+
+
+def job_totals(ms, tokens, world, device):
+    """Whole-job (time, tokens) of the replicas: the slowest rank's time and the sum of the
+    committed tokens (a collective over the default process group when world > 1)."""
+    if world <= 1:
+        return float(ms), int(tokens)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    n = torch.tensor([int(tokens)], dtype=torch.int64, device=device)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(n.item())
 
 
 def algorithmic_bytes(shape, B, K, ctx_mean, experts_touched_routed_per_layer):
@@ -353,14 +379,7 @@ def run_fastmtp(args):
     m_hist = [0] * (K + 1)
     for n in hist.flatten().tolist():
         m_hist[n - 1] += 1
-    if world > 1:
-        t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        n = torch.tensor([accepted], dtype=torch.int64, device=dev)
-        dist.all_reduce(n, op=dist.ReduceOp.SUM)
-        ms_total, accepted_all = float(t.item()), int(n.item())
-    else:
-        accepted_all = accepted
+    ms_total, accepted_all = job_totals(ms_total, accepted, world, dev)
     value = accepted_all / (ms_total / 1000.0)
 
     # -------- e2e through the public API: pinned H2D of the step's input, D2H of its result
@@ -388,13 +407,7 @@ def run_fastmtp(args):
                 h_n.copy_(d_n, non_blocking=True)
                 stream.synchronize()
                 tok += int(h_n.sum())
-        dt = time.perf_counter() - t0
-        if world > 1:
-            t = torch.tensor([dt], dtype=torch.float64, device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            n = torch.tensor([tok], dtype=torch.int64, device=dev)
-            dist.all_reduce(n, op=dist.ReduceOp.SUM)
-            dt, tok = float(t.item()), int(n.item())
+        dt, tok = job_totals(time.perf_counter() - t0, tok, world, dev)
         e2e = {"value": tok / dt, "unit": "tokens/s", "h2d_bytes_per_step": B * 4,
                "d2h_bytes_per_step": B * (K + 1) * 4 + B * 4}
     eng.close()
@@ -464,8 +477,9 @@ def run_sweep(args):
     """Every (router, context, batch, K) point of the grid on one engine per router mode:
     committed contexts of exactly `ctx` tokens (N(0,1) KV drawn on the device), one K=0 step
     to seed the draft head, `warmup` steps, then `steps` timed steps with an event pair around
-    each phase.  Weights: the acceptance-tuned seeded set (seed 4); the Zipf mode adds the
-    per-expert router bias -1.2 ln(rank).  Pending tokens use seeds 4..8 by batch size."""
+    each phase (medians over the timed steps).  Weights: the acceptance-tuned seeded set
+    (seed 4); the Zipf mode adds the per-expert router bias -1.2 ln(rank).  Pending tokens use
+    seeds 4..8 by batch size."""
     import torch
 
     import synth_inputs as S
@@ -535,7 +549,9 @@ def run_sweep(args):
                     eng.profile(0)
                     cnt = eng.read_workspace(F.WS_EXPERT_CNT, (shape.n_layers, shape.n_experts), torch.int32).double()
                     timed = range(args.warmup, n_all)
-                    ms = lambda a, b: statistics.mean(ev[i][a].elapsed_time(ev[i][b]) for i in timed)
+                    # medians over the timed steps: a host stall between two launches shows up
+                    # in one step's event pair and would skew a mean
+                    ms = lambda a, b: statistics.median(ev[i][a].elapsed_time(ev[i][b]) for i in timed)
                     ms_step, ms_draft, ms_verify = ms(0, 3), ms(0, 1), ms(1, 2)
                     h = hist.double().cpu()
                     lens = ctx + 1 + torch.cumsum(h, 0) - h          # committed length seen by each verify
@@ -546,6 +562,7 @@ def run_sweep(args):
                     load = cnt / cnt.mean(-1, keepdim=True)
                     out = {"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K,
                            "tokens_per_s": tok / (ms_step * args.steps / 1000.0), "ms_step": ms_step,
+                           "ms_step_mean": statistics.mean(ev[i][0].elapsed_time(ev[i][3]) for i in timed),
                            "ms_draft": ms_draft, "ms_verify": ms_verify, "ms_commit": ms(2, 3),
                            "tau": tok / (args.steps * B),
                            "verify_roofline": {"bytes": vbytes, "achieved_gbs": vbytes / ms_verify / 1e6,

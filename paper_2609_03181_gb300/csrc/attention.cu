@@ -14,19 +14,21 @@
 // accumulation, queries padded to 8); a score sums its even and its odd 16-dim steps
 // separately, then adds the two; p enters the product as two bf16 terms (hi + lo, about 16
 // bits) whose products accumulate separately over a super-chunk and are added at its end; the
-// transposes between the score and the product layouts stay in registers (movmatrix).  Masked keys contribute exact zeros, so a query's result is the same whether
-// its keys sit in pages or in staging and however many queries or sequences share the launch:
-// greedy decoding (K = 0) and speculative verification see identical rows.
+// transposes between the score and the product layouts stay in registers (movmatrix).  Masked
+// keys contribute exact zeros, so a query's result is the same whether its keys sit in pages
+// or in staging and however many queries or sequences share the launch: greedy decoding
+// (K = 0) and speculative verification see identical rows.
 //
-// Scheduling: one warp per CTA, two CTAs per SM.  The CTAs of one (sequence, head) take its
-// super-chunks in turn (CTA u: super-chunks u, u + n, u + 2n, ...), each streaming its chunks
-// through three private shared-memory stages.  A chunk whose 64 keys are all committed is one page segment per head: its K
-// and V rows are two contiguous 16 KB blocks, fetched as four TMA boxes (64 rows x 128 bytes,
-// 128-byte swizzle) onto the stage's mbarrier, issued up to three chunks ahead.  The chunk
-// holding the newest keys (staged candidates, masked positions) is gathered row by row with
-// 16-byte cp.async into the same swizzled layout, zero-filled where there is no key.  Each
-// super-chunk's (M, L, O) goes to global memory; the CTA that finishes the last unit of a
-// (sequence, head) merges them (atomic ticket, no wait).
+// Scheduling: one warp per CTA; two stages per CTA (three CTAs per SM) for launches of about
+// two waves or fewer, three stages (two CTAs per SM) above.  The CTAs of one (sequence, head)
+// take its super-chunks in turn (CTA u: super-chunks u, u + n, u + 2n, ...).  A chunk whose 64
+// keys are all committed is one page segment per head: its K and V rows are two contiguous
+// 16 KB blocks, fetched as four TMA boxes (64 rows x 128 bytes, 128-byte swizzle) onto the
+// stage's mbarrier, issued ahead of the compute.  The chunk holding the newest keys (staged
+// candidates, masked positions) is gathered row by row with 16-byte cp.async into the same
+// swizzled layout, zero-filled where there is no key.  Each super-chunk's (M, L, O) goes to
+// global memory; the CTA that finishes last for a (sequence, head) merges them (atomic
+// ticket, no wait).
 #include <math.h>
 
 #include "common.cuh"
