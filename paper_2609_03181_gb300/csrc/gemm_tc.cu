@@ -257,6 +257,60 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
   }
 }
 
+// Cluster split-K reduction, run by the 128 epilogue threads of every CTA of the cluster after
+// the first cluster barrier: CTA `rank` takes chunks rank, rank + S, ..., adds the S partial
+// tiles of each (read from the cluster's shared memory) in split order -- the same sums as the
+// other schedules -- and runs the epilogue on them.
+template <int EPI>
+__device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem& esm, uint32_t part_saddr, int row) {
+  Item it;
+  get_item(a, blockIdx.x, it);
+  const int S = a.cluster;
+  const int rank = static_cast<int>(cluster_ctarank());
+  const int nchunks = (it.rows + 15) >> 4;
+  const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
+  int k = 0;
+  for (int c = rank; c < nchunks; c += S, ++k) {
+    if (rope) {
+      RopeRegs rr;
+      rope_load(a, it, c * 16, esm, rr);
+      rope_store(esm, k & 1, rr);
+      named_bar_sync(1, 128);
+    }
+    EpiPre cur;
+    epi_pre<EPI>(a, it, row, c * 16, esm, cur);
+    float v[16];
+#pragma unroll
+    for (int hf = 0; hf < 2; ++hf) {
+      float4 p[kMaxSplit][2];
+#pragma unroll
+      for (int sp = 0; sp < kMaxSplit; ++sp)
+        if (sp < S)
+#pragma unroll
+          for (int q2 = 0; q2 < 2; ++q2)
+            p[sp][q2] = ld_dsmem_f4(part_saddr + ((c * 4 + 2 * hf + q2) * 128 + row) * 16, sp);
+#pragma unroll
+      for (int q2 = 0; q2 < 2; ++q2) {
+        float4 t = p[0][q2];
+#pragma unroll
+        for (int sp = 1; sp < kMaxSplit; ++sp)
+          if (sp < S) {
+            t.x += p[sp][q2].x;
+            t.y += p[sp][q2].y;
+            t.z += p[sp][q2].z;
+            t.w += p[sp][q2].w;
+          }
+        const int q4 = 2 * hf + q2;
+        v[4 * q4] = t.x;
+        v[4 * q4 + 1] = t.y;
+        v[4 * q4 + 2] = t.z;
+        v[4 * q4 + 3] = t.w;
+      }
+    }
+    epi_post<EPI>(a, it, row, c * 16, v, cur, esm, k & 1);
+  }
+}
+
 // ------------------------------------------------------------------ kernel
 template <int NMAX, int EPI>
 __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
@@ -522,6 +576,20 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
+      } else if (a.cluster > 1) {
+        // cluster split-K: the partial tile goes to this CTA's shared memory (the pipeline
+        // stages are free once the tile's MMAs have completed), laid out [chunk][quad][row];
+        // the reduction follows the cluster barrier at the end of the kernel
+        float4* part = reinterpret_cast<float4*>(smA);
+        for (int c = 0; c < nchunks; ++c) {
+          tc_ld16(tb + c * 16, v);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4)
+            part[(c * 4 + q4) * 128 + row] = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
       } else {
         // split-K: each split writes its fp32 partial tile thread-major (a thread's 16 values
         // of a chunk are 64 contiguous bytes); the last split of the tile to arrive (atomic
@@ -632,6 +700,11 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     }
   }
 
+  if (a.cluster > 1) {
+    cluster_sync_all();   // every split's partial tile is in its CTA's shared memory
+    if (warp >= 2) cluster_reduce<EPI>(a, esm, smem_u32(smA), (warp & 3) * 32 + lane);
+    cluster_sync_all();   // no CTA leaves while the others still read its shared memory
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -664,7 +737,28 @@ cudaError_t set_smem_attr() {
 
 template <int NMAX, int EPI>
 cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
-  return launch_k(pdl, gemm_tc_kernel<NMAX, EPI>, dim3(grid), dim3(192), Cfg<NMAX>::SMEM_BYTES, s, a);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = Cfg<NMAX>::SMEM_BYTES;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  if (pdl) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (a.cluster > 1) {   // the split_k CTAs of a tile form one thread-block cluster
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = a.cluster;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI>, a);
 }
 }  // namespace
 

@@ -79,6 +79,8 @@ struct GemmArgs {
   int split_k;                 // >= 1, fixed per matrix shape
   int seq_split;               // dense, split_k > 1: one CTA computes every split of a tile into
                                // its own TMEM accumulator (64-row boxes), no partials in memory
+  int cluster;                 // dense, split_k > 1, one item per CTA: the split_k CTAs of a tile
+                               // are a cluster and add their partials through shared memory
   const int4* items;           // grouped: device item list
   const int* n_items_dev;      //          and its length
   int n_items;                 // dense: number of items

@@ -200,11 +200,15 @@ cudaError_t run_dense(spec_ctx* ctx, GemmArgs g, int epi, const CUtensorMap& wma
     // accumulator and adds them in split order -- the same sums as the cross-CTA split
     g.seq_split = 1;
     g.box_log = 2;
+  } else if (g.split_k > 1) {
+    // few rows: one CTA per split, the splits of a tile form a cluster and add their partial
+    // tiles through distributed shared memory, in split order
+    g.cluster = g.split_k;
   }
   const int box = 16 << g.box_log;
   g.m_tiles = (M + box - 1) / box;
   g.n_items = g.n_tiles * (g.seq_split ? 1 : g.split_k) * g.m_tiles;
-  const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
+  const int grid = g.cluster ? g.n_items : (g.n_items < num_sms() ? g.n_items : num_sms());
   return gemm_launch(epi, box <= 64 ? 64 : 256, g, grid, ctx->stream);
 }
 
