@@ -19,16 +19,16 @@
 // or in staging and however many queries or sequences share the launch: greedy decoding
 // (K = 0) and speculative verification see identical rows.
 //
-// Scheduling: one warp per CTA; two stages per CTA (three CTAs per SM) for launches of about
-// two waves or fewer, three stages (two CTAs per SM) above.  The CTAs of one (sequence, head)
-// take its super-chunks in turn (CTA u: super-chunks u, u + n, u + 2n, ...).  A chunk whose 64
-// keys are all committed is one page segment per head: its K and V rows are two contiguous
-// 16 KB blocks, fetched as four TMA boxes (64 rows x 128 bytes, 128-byte swizzle) onto the
-// stage's mbarrier, issued ahead of the compute.  The chunk holding the newest keys (staged
-// candidates, masked positions) is gathered row by row with 16-byte cp.async into the same
-// swizzled layout, zero-filled where there is no key.  Each super-chunk's (M, L, O) goes to
-// global memory; the CTA that finishes last for a (sequence, head) merges them (atomic
-// ticket, no wait).
+// Scheduling: four warps per CTA, each recomputing a chunk's 64 x 8 scores and owning 32 of
+// the 128 output dims; two stages per CTA (three CTAs per SM) for launches of about two waves
+// or fewer, three stages (two per SM) above.  The CTAs of one (sequence, head) take its
+// super-chunks in turn (CTA u: super-chunks u, u + n, u + 2n, ...).  A chunk whose 64 keys are
+// all committed is one page segment per head: its K and V rows are two contiguous 16 KB
+// blocks, fetched as four TMA boxes (64 rows x 128 bytes, 128-byte swizzle) onto the stage's
+// mbarrier, issued ahead of the compute.  The chunk holding the newest keys (staged candidates,
+// masked positions) is gathered row by row with 16-byte cp.async into the same swizzled layout,
+// zero-filled where there is no key.  Each super-chunk's (M, L, O) goes to global memory; the
+// CTA that finishes last for a (sequence, head) merges them (atomic ticket, no wait).
 #include <math.h>
 
 #include "common.cuh"
@@ -43,6 +43,7 @@ constexpr int kUnitMaxChunks = kSuper * kUnitMaxSuper;
 constexpr int kHalfBytes = kCH * 128;            // 64 rows x 64 dims of K or V: 8 KB
 constexpr int kTileBytes = 2 * kHalfBytes;       // K (or V) of a chunk: 16 KB
 constexpr int kStageBytes = 2 * kTileBytes;      // K and V of a chunk: 32 KB
+constexpr int kAttnThreads = 128;                // four warps, each owning 32 of the 128 dims
 constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
 // shared memory of a CTA with `stages` stages: 1 KB alignment slack, the stages, Q, barriers
 constexpr int attn_smem(int stages) { return 1024 + stages * kStageBytes + kMaxR * kHD * 2 + stages * 8; }
@@ -96,22 +97,23 @@ __device__ __forceinline__ uint32_t swt(int row, int ch) {
 }
 
 // Merge of the super-chunks of every query of (sequence b, head h), run by the CTA that
-// finishes the last unit: query r combines super-chunks 0..floor(p_r/256) in order.
+// finishes last for it: query r combines super-chunks 0..floor(p_r/256) in order.  Warp w
+// writes queries w, w + 4; each lane four dims.
 __device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R, int p0, int n_sup, float* smem) {
-  const int lane = threadIdx.x & 31;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
   const float* part = a.part + (static_cast<size_t>(b) * kH + h) * n_super * R * kPartStride;
   float* sm = smem;                      // [n_sup * R] super-chunk max, then weight
   float* sl = smem + n_sup * R;          // [n_sup * R] super-chunk sum
   float* sL = sl + n_sup * R;            // [R] total weight
-  for (int i = lane; i < n_sup * R; i += 32) {
+  for (int i = tid; i < n_sup * R; i += kAttnThreads) {
     const float* pc = part + static_cast<size_t>(i) * kPartStride;
     sm[i] = __ldcg(&pc[kHD]);
     sl[i] = __ldcg(&pc[kHD + 1]);
   }
-  __syncwarp();
-  if (lane < R) {
-    const int r = lane, lasts = (p0 + r) / (kCH * kSuper);
+  __syncthreads();
+  if (tid < R) {
+    const int r = tid, lasts = (p0 + r) / (kCH * kSuper);
     float M = -INFINITY;
     for (int s = 0; s <= lasts; ++s) M = fmaxf(M, sm[s * R + r]);
     float L = 0.f;
@@ -123,9 +125,9 @@ __device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R
     }
     sL[r] = L;
   }
-  __syncwarp();
+  __syncthreads();
   const int d = lane * 4;   // four dims per lane
-  for (int r = 0; r < R; ++r) {
+  for (int r = warp; r < R; r += kAttnThreads / 32) {
     const int lasts = (p0 + r) / (kCH * kSuper);
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     int s = 0;
@@ -159,52 +161,50 @@ __device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R
   }
 }
 
-// Gathers the K and V rows of chunk c into a stage with 16-byte cp.async (each lane two keys,
-// sixteen 16-byte pieces of K and of V each); rows without a visible key are zero-filled.
-// Used for the chunk that holds staged candidates or masked positions, and for every chunk
-// when the pool has no TMA map.
+// Gathers the K and V rows of chunk c into a stage with 16-byte cp.async (two threads per key,
+// eight 16-byte pieces of K and of V each); rows without a visible key are zero-filled.  Used
+// for the chunk that holds staged candidates or masked positions, and for every chunk when the
+// pool has no TMA map.
 __device__ __forceinline__ void gather_chunk(const AttnArgs& a, int b, int h, int slot, int sl, int last, int c,
                                              uint8_t* stage) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int j = 0; j < 2; ++j) {
-    const int key = lane * 2 + j;
-    const int pos = c * kCH + key;
-    const bf16* srck = a.pool;
-    const bf16* srcv = a.pool;
-    int bytes = 0;
-    if (pos <= last) {
-      if (pos < sl) {
-        const int pi = pos / a.page_size;
-        const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
-        if (page >= 0 && page < a.n_pages) {
-          srck = a.pool + ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
-          srcv = srck + static_cast<long long>(kH) * a.page_size * kHD;
-          bytes = 16;
-        } else {
-          atomicOr(a.err, ERR_PAGE_RANGE);
-        }
-      } else {
-        srck = a.stage + b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
-               static_cast<long long>(h) * kHD;
-        srcv = srck + a.stage_kv_stride;
+  const int key = threadIdx.x >> 1, half = threadIdx.x & 1;
+  const int pos = c * kCH + key;
+  const bf16* srck = a.pool;
+  const bf16* srcv = a.pool;
+  int bytes = 0;
+  if (pos <= last) {
+    if (pos < sl) {
+      const int pi = pos / a.page_size;
+      const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+      if (page >= 0 && page < a.n_pages) {
+        srck = a.pool + ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
+        srcv = srck + static_cast<long long>(kH) * a.page_size * kHD;
         bytes = 16;
+      } else {
+        atomicOr(a.err, ERR_PAGE_RANGE);
       }
+    } else {
+      srck = a.stage + b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
+             static_cast<long long>(h) * kHD;
+      srcv = srck + a.stage_kv_stride;
+      bytes = 16;
     }
+  }
 #pragma unroll
-    for (int ch = 0; ch < 16; ++ch) {
-      const int o = bytes ? ch * 8 : 0;
-      cp_async16(stage + swt(key, ch), srck + o, bytes);
-      cp_async16(stage + kTileBytes + swt(key, ch), srcv + o, bytes);
-    }
+  for (int i = 0; i < 8; ++i) {
+    const int ch = half * 8 + i;
+    const int o = bytes ? ch * 8 : 0;
+    cp_async16(stage + swt(key, ch), srck + o, bytes);
+    cp_async16(stage + kTileBytes + swt(key, ch), srcv + o, bytes);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
 
 // kStages stages per CTA: 3 (two CTAs per SM) when the launch spans many waves, 2 (three CTAs
-// per SM) when it fits in about two.
+// per SM) when it fits in about two.  Four warps: each recomputes the chunk's 64 x 8 scores
+// (cheap) and owns 32 of the 128 output dims, so its dependent MMA chain is short.
 template <int kStages>
-__global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ uint8_t asmem_raw[];
   const uint32_t raw_u32 = smem_u32(asmem_raw);
   uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [S][K 16 KB | V 16 KB]
@@ -212,28 +212,25 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   uint64_t* full = reinterpret_cast<uint64_t*>(sQ + kMaxR * kHD * 2);   // [S] TMA stage barriers
   __shared__ int s_page[kUnitMaxChunks];                     // page of each TMA chunk of the unit
   __shared__ int s_abort;
+  __shared__ int s_last;
   pdl_trigger();
   pdl_wait();
 
   const int u = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
-  const int lane = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
   const int R = a.R;
   // the queries first (bf16, as the QKV epilogue stored them; rows R..7 zero): their loads need
   // no slot and overlap the slot -> length -> page lookups
-  uint4 qv[4];
+  uint4 qv = make_uint4(0, 0, 0, 0);
   {
     const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int v = lane + 32 * i, q = v >> 4, ch = v & 15;   // 8 queries x 16 pieces of 16 bytes
-      qv[i] = make_uint4(0, 0, 0, 0);
-      if (q < R) qv[i] = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
-    }
+    const int q = tid >> 4, ch = tid & 15;   // 8 queries x 16 pieces of 16 bytes
+    if (q < R) qv = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
   }
   const int slot = a.slots[b];
   if (slot < 0 || slot >= a.n_slots) {   // every CTA of the sequence leaves; no ticket, no merge
-    if (u == 0 && h == 0 && lane == 0) atomicOr(a.err, ERR_SLOT_RANGE);
+    if (u == 0 && h == 0 && tid == 0) atomicOr(a.err, ERR_SLOT_RANGE);
     return;
   }
   // this CTA's super-chunks: u, u + n_units, u + 2 n_units, ... (strided, so that short contexts
@@ -243,8 +240,8 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   auto chunk_of = [&](int i) { return (u + (i / kSuper) * n_units) * kSuper + i % kSuper; };
   // the pages of every chunk the CTA may own are looked up now, alongside the length
   int spec_page = -1;
-  if (lane < a.unit * kSuper) {
-    const int pi = chunk_of(lane) * kCH / a.page_size;
+  if (tid < a.unit * kSuper) {
+    const int pi = chunk_of(tid) * kCH / a.page_size;
     if (pi < a.max_pages) spec_page = a.block_table[slot * a.max_pages + pi];
   }
   const int sl = a.seq_len[slot];
@@ -262,27 +259,23 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   if (a.use_tma)
     while (n_tma < n && (chunk_of(n_tma) + 1) * kCH <= sl) ++n_tma;
 
-  if (lane < n_tma) {
+  if (tid < n_tma) {
     int page = spec_page;
     if (page < 0 || page >= a.n_pages) {
       atomicOr(a.err, ERR_PAGE_RANGE);
       page = -1;
     }
-    s_page[lane] = page;
+    s_page[tid] = page;
   }
-  if (lane == 0) {
+  if (tid == 0) {
     for (int st = 0; st < kStages; ++st) mbar_init(&full[st], 1);
     s_abort = 0;
     fence_mbar_init();
   }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int v = lane + 32 * i, q = v >> 4, ch = v & 15;
-    *reinterpret_cast<uint4*>(sQ + swz(q, ch)) = qv[i];
-  }
-  __syncwarp();
+  *reinterpret_cast<uint4*>(sQ + swz(tid >> 4, tid & 15)) = qv;
+  __syncthreads();
 
-  // TMA of chunk i of the unit into stage i % 3; a chunk whose page is invalid completes its
+  // TMA of chunk i of the unit into stage i % S; a chunk whose page is invalid completes its
   // barrier without data (the guard flag is already set)
   const uint64_t pol = l2_policy_evict_first();
   auto issue = [&](int i) {
@@ -302,7 +295,7 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
     tma_load_2d(dst + kTileBytes, &a.kv_map, &full[st], 0, row_v, pol);
     tma_load_2d(dst + kTileBytes + kHalfBytes, &a.kv_map, &full[st], 64, row_v, pol);
   };
-  if (lane == 0) {
+  if (tid == 0) {
     if (n_tma > 0) tma_prefetch_desc(&a.kv_map);
     for (int i = 0; i < min(n_tma, kStages); ++i) issue(i);
   }
@@ -317,8 +310,8 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   const int qa = 2 * t4, qb = 2 * t4 + 1;                    // the two queries of this lane
   float* part = a.part + (static_cast<size_t>(b) * kH + h) * ((a.n_chunks + kSuper - 1) / kSuper) * R * kPartStride;
   float M_a = -INFINITY, M_b = -INFINITY, L_a = 0.f, L_b = 0.f;
-  float O[8][4], Ol[8][4];   // hi and lo parts of the unnormalised output
-  int consumed = 0;   // TMA chunks waited for
+  float O[2][4], Ol[2][4];   // hi and lo parts of the unnormalised output, dims 32 warp + 16 j
+  int consumed = 0;          // TMA chunks waited for
   bool aborted = false;
   for (int i = 0; i < n; ++i) {
     const int c = chunk_of(i);
@@ -328,13 +321,13 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
       M_a = M_b = -INFINITY;
       L_a = L_b = 0.f;
 #pragma unroll
-      for (int dt = 0; dt < 8; ++dt)
+      for (int j = 0; j < 2; ++j)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) O[dt][e] = Ol[dt][e] = 0.f;
+        for (int e = 0; e < 4; ++e) O[j][e] = Ol[j][e] = 0.f;
     }
     if (i < n_tma) {
       const bool ok = mbar_wait(&full[st], static_cast<uint32_t>(i / kStages) & 1u, &s_abort);
-      if (!__all_sync(0xffffffffu, ok)) {
+      if (__syncthreads_or(!ok)) {
         aborted = true;
         break;
       }
@@ -342,7 +335,7 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
     } else {
       gather_chunk(a, b, h, slot, sl, last, c, stage);
       asm volatile("cp.async.wait_group 0;" ::: "memory");
-      __syncwarp();
+      __syncthreads();
     }
     const uint32_t kbase = smem_u32(stage);
     const uint32_t vbase = kbase + kTileBytes;
@@ -419,48 +412,48 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
     }
     L_a = L_a * al_a + l_a;
     L_b = L_b * al_b + l_b;
-    // O^T[dim][query] = al * O^T + V^T P^T: eight 16-dim tiles, 4 k-steps of 16 keys; the hi
-    // and lo products accumulate separately (sixteen independent chains), summed per super-chunk
+    // O^T[dim][query] = al * O^T + V^T P^T for this warp's two 16-dim tiles (dims 32w..32w+31),
+    // 4 k-steps of 16 keys; hi and lo products in separate accumulators, summed per super-chunk
 #pragma unroll
-    for (int dt = 0; dt < 8; ++dt) {
-      O[dt][0] *= al_a;
-      O[dt][1] *= al_b;
-      O[dt][2] *= al_a;
-      O[dt][3] *= al_b;
-      Ol[dt][0] *= al_a;
-      Ol[dt][1] *= al_b;
-      Ol[dt][2] *= al_a;
-      Ol[dt][3] *= al_b;
+    for (int j = 0; j < 2; ++j) {
+      O[j][0] *= al_a;
+      O[j][1] *= al_b;
+      O[j][2] *= al_a;
+      O[j][3] *= al_b;
+      Ol[j][0] *= al_a;
+      Ol[j][1] *= al_b;
+      Ol[j][2] *= al_a;
+      Ol[j][3] *= al_b;
     }
 #pragma unroll
     for (int kt = 0; kt < 4; ++kt) {
 #pragma unroll
-      for (int dt = 0; dt < 8; ++dt) {
+      for (int j = 0; j < 2; ++j) {
         uint32_t av[4];
-        ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * dt + (mi & 1)), av);
-        mma_bf16_16816(O[dt], av, ph[kt]);
-        mma_bf16_16816(Ol[dt], av, pl[kt]);
+        ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * (2 * warp + j) + (mi & 1)), av);
+        mma_bf16_16816(O[j], av, ph[kt]);
+        mma_bf16_16816(Ol[j], av, pl[kt]);
       }
     }
-    __syncwarp();   // every lane is done with this stage
-    if (lane == 0 && i + kStages < n_tma) issue(i + kStages);
+    __syncthreads();   // every warp is done with this stage
+    if (tid == 0 && i + kStages < n_tma) issue(i + kStages);
 
-    // end of a super-chunk: its (M, L, O) per query
+    // end of a super-chunk: its (M, L, O) per query (each warp its 32 dims)
     if ((c + 1) % kSuper == 0 || c + 1 == n_live) {
       float* ps = part + static_cast<size_t>(c / kSuper) * R * kPartStride;
 #pragma unroll
-      for (int dt = 0; dt < 8; ++dt) {
-        const int d = 16 * dt + g;
+      for (int j = 0; j < 2; ++j) {
+        const int d = 16 * (2 * warp + j) + g;
         if (qa < R) {
-          ps[qa * kPartStride + d] = O[dt][0] + Ol[dt][0];
-          ps[qa * kPartStride + d + 8] = O[dt][2] + Ol[dt][2];
+          ps[qa * kPartStride + d] = O[j][0] + Ol[j][0];
+          ps[qa * kPartStride + d + 8] = O[j][2] + Ol[j][2];
         }
         if (qb < R) {
-          ps[qb * kPartStride + d] = O[dt][1] + Ol[dt][1];
-          ps[qb * kPartStride + d + 8] = O[dt][3] + Ol[dt][3];
+          ps[qb * kPartStride + d] = O[j][1] + Ol[j][1];
+          ps[qb * kPartStride + d + 8] = O[j][3] + Ol[j][3];
         }
       }
-      if (g == 0) {
+      if (warp == 0 && g == 0) {
         if (qa < R) {
           ps[qa * kPartStride + kHD] = M_a;
           ps[qa * kPartStride + kHD + 1] = L_a;
@@ -475,29 +468,28 @@ __global__ void __launch_bounds__(32) attn_chunk_kernel(const __grid_constant__ 
   if (aborted) {
     // a stage wait ran out: flag it and let the copies still in flight land, then take the
     // ticket as usual so that the counters stay consistent (the merged result is invalid)
-    if (lane == 0) {
+    if (tid == 0) {
       atomicOr(a.err, ERR_WAIT_TIMEOUT);
       const int issued = min(n_tma, consumed + kStages);
       int never = 0;
       for (int i = consumed; i < issued; ++i)
         mbar_wait(&full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, &never, 100000000ull);
     }
-    __syncwarp();
+    __syncthreads();
   }
 
-  // the CTA that finishes the last unit of (sequence, head) merges every query
+  // the CTA that finishes last for (sequence, head) merges every query
   __threadfence();
-  __syncwarp();
+  __syncthreads();
   const int n_busy = min(n_units, n_sup_live);   // CTAs of this (sequence, head) with work
-  int is_last = 0;
-  if (lane == 0) {
+  if (tid == 0) {
     int* ticket = a.tickets + b * kH + h;
     const int old = atomicAdd(ticket, 1);
-    is_last = (old == n_busy - 1) ? 1 : 0;
-    if (is_last) *ticket = 0;
+    s_last = (old == n_busy - 1) ? 1 : 0;
+    if (s_last) *ticket = 0;
   }
-  is_last = __shfl_sync(0xffffffffu, is_last, 0);
-  if (is_last) {
+  __syncthreads();
+  if (s_last) {
     __threadfence();
     merge_all(a, b, h, R, p0, (n_live + kSuper - 1) / kSuper, reinterpret_cast<float*>(stages));
   }
@@ -525,8 +517,8 @@ cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
   const int n_units = (n_super + unit - 1) / unit;
   const long long ctas = static_cast<long long>(n_units) * kH * B;
   if (ctas <= 6ll * num_sms())
-    return launch_pdl(attn_chunk_kernel<2>, dim3(n_units, kH, B), dim3(32), attn_smem(2), s, a);
-  return launch_pdl(attn_chunk_kernel<3>, dim3(n_units, kH, B), dim3(32), attn_smem(3), s, a);
+    return launch_pdl(attn_chunk_kernel<2>, dim3(n_units, kH, B), dim3(kAttnThreads), attn_smem(2), s, a);
+  return launch_pdl(attn_chunk_kernel<3>, dim3(n_units, kH, B), dim3(kAttnThreads), attn_smem(3), s, a);
 }
 
 }  // namespace fm
