@@ -221,16 +221,28 @@ __device__ __forceinline__ void group_by_expert(const RouteArgs& a, int* gsm) {
 template <int RR>
 __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ RouteArgs a) {
   pdl_trigger();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // the first four experts of this warp's eight: router weights are never written by earlier
+  // kernels, so their loads go out before the wait for the previous kernel
+  uint4 raw[4][5];
+  auto load_group = [&](int e0) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int c = 0; c < 5; ++c)
+        raw[q][c] = *reinterpret_cast<const uint4*>(a.wr + static_cast<size_t>(e0 + q) * kD + c * 256 + lane * 8);
+  };
+  load_group(warp * 8);
   pdl_wait();
   constexpr int NT = 256, EPT = kD / NT;
   __shared__ float red[NT / 32][RR];
   __shared__ __align__(16) float xs[RR][kD];
   __shared__ float lg[RR][kE];
+  __shared__ float sp[RR][kE];
   __shared__ int s_last;
   extern __shared__ int gsm[];
   const int t0 = blockIdx.x * RR;
   const int nr = min(RR, a.T - t0);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   {
     float v[RR][EPT];
     float ss[RR];
@@ -268,12 +280,7 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
   for (int e0 = warp * 8; e0 < warp * 8 + 8; e0 += 4) {
     // four experts at a time: 20 independent 16-byte weight loads in flight per lane, each
     // weight used for every row of the CTA
-    uint4 raw[4][5];
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-#pragma unroll
-      for (int c = 0; c < 5; ++c)
-        raw[q][c] = *reinterpret_cast<const uint4*>(a.wr + static_cast<size_t>(e0 + q) * kD + c * 256 + lane * 8);
+    if (e0 != warp * 8) load_group(e0);
 #pragma unroll
     for (int r = 0; r < RR; ++r) {
       if (r >= nr) break;
@@ -308,19 +315,25 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
       if (!(p0 == p0)) p0 = -1.f;
       if (!(p1 == p1)) p1 = -1.f;
     }
-    bool taken0 = false, taken1 = false;
-    for (int k = 0; k < kTopK; ++k) {
-      float bv = -1.f;
-      int bi = 1 << 30;
-      if (!taken0) { bv = p0; bi = lane; }
-      if (!taken1 && better(p1, lane + 32, bv, bi)) { bv = p1; bi = lane + 32; }
-      warp_argmax(bv, bi);
-      if (bi == lane) taken0 = true;
-      if (bi == lane + 32) taken1 = true;
-      if (lane == 0) {
-        a.idx[t * kTopK + k] = bi;
-        a.gate[t * kTopK + k] = bv;
-      }
+    // top-6: the rank of each expert among the 64 (a higher probability, or an equal one with a
+    // lower id, ranks ahead) -- the experts of rank 0..5 are the selection, in that order
+    sp[r][lane] = p0;
+    sp[r][lane + 32] = p1;
+    __syncwarp();
+    int rk0 = 0, rk1 = 0;
+#pragma unroll 16
+    for (int j = 0; j < kE; ++j) {
+      const float pj = sp[r][j];
+      rk0 += better(pj, j, p0, lane) ? 1 : 0;
+      rk1 += better(pj, j, p1, lane + 32) ? 1 : 0;
+    }
+    if (rk0 < kTopK) {
+      a.idx[t * kTopK + rk0] = lane;
+      a.gate[t * kTopK + rk0] = p0;
+    }
+    if (rk1 < kTopK) {
+      a.idx[t * kTopK + rk1] = lane + 32;
+      a.gate[t * kTopK + rk1] = p1;
     }
   }
   // the last CTA to finish groups the layer's pairs by expert
