@@ -19,16 +19,21 @@
 // or in staging and however many queries or sequences share the launch: greedy decoding
 // (K = 0) and speculative verification see identical rows.
 //
-// Scheduling: four warps per CTA, each recomputing a chunk's 64 x 8 scores and owning 32 of
-// the 128 output dims; two stages per CTA (three CTAs per SM) for launches of about two waves
-// or fewer, three stages (two per SM) above.  The CTAs of one (sequence, head) take its
-// super-chunks in turn (CTA u: super-chunks u, u + n, u + 2n, ...).  A chunk whose 64 keys are
-// all committed is one page segment per head: its K and V rows are two contiguous 16 KB
-// blocks, fetched as four TMA boxes (64 rows x 128 bytes, 128-byte swizzle) onto the stage's
-// mbarrier, issued ahead of the compute.  The chunk holding the newest keys (staged candidates,
-// masked positions) is gathered row by row with 16-byte cp.async into the same swizzled layout,
-// zero-filled where there is no key.  Each super-chunk's (M, L, O) goes to global memory; the
-// CTA that finishes last for a (sequence, head) merges them (atomic ticket, no wait).
+// Scheduling: the launch's work is the list of (sequence, head, super-chunk) items, sequences
+// in order, then heads, then super-chunks.  Every CTA builds the list's per-sequence prefix
+// from the lengths and takes one contiguous share of ceil(W / grid) items, so that it streams
+// many chunks back to back whatever the mix of lengths, and all shares but the last are equal.
+// One producer warp fetches up to two chunks ahead: a chunk whose 64 keys are all committed
+// is one page segment per head, its K and V rows two contiguous 16 KB blocks fetched as four
+// TMA boxes (64 rows x 128 bytes, 128-byte swizzle); a chunk holding the newest keys (staged
+// candidates, masked positions) is gathered row by row with 16-byte cp.async into the same
+// swizzled layout, zero-filled where there is no key; the queries of each (sequence, head)
+// go to one of two query slots.  Four consumer warps each recompute a chunk's 64 x 8 scores
+// (cheap) and own 32 of the 128 output dims.  Each super-chunk's (M, L, O) goes to global
+// memory; the CTA whose atomic count completes the super-chunks of a (sequence, head) merges
+// them (no wait on other CTAs).  In the verify step, where nothing in the step writes the
+// pages, the producer fetches the first committed chunks before it waits for the previous
+// kernel.
 #include <math.h>
 
 #include "common.cuh"
@@ -38,15 +43,25 @@ namespace fm {
 
 constexpr int kCH = kAttnChunk;                  // keys per chunk (64)
 constexpr int kSuper = kAttnSuper;               // chunks per super-chunk
-constexpr int kUnitMaxSuper = 4;                 // most super-chunks one CTA streams
-constexpr int kUnitMaxChunks = kSuper * kUnitMaxSuper;
 constexpr int kHalfBytes = kCH * 128;            // 64 rows x 64 dims of K or V: 8 KB
 constexpr int kTileBytes = 2 * kHalfBytes;       // K (or V) of a chunk: 16 KB
 constexpr int kStageBytes = 2 * kTileBytes;      // K and V of a chunk: 32 KB
-constexpr int kAttnThreads = 128;                // four warps, each owning 32 of the 128 dims
+constexpr int kQBytes = kMaxR * kHD * 2;         // the queries of one (sequence, head): 2 KB
+// Chunks in flight per CTA: two stages keep a CTA at 64 KB of shared memory and 128 registers
+// a thread, three CTAs per SM (192 KB in flight per SM, as three stages at two CTAs would) --
+// more CTAs, so that a small launch spreads over more of them.
+constexpr int kAttnStages = 2;
+constexpr int kConsumers = 128;                  // four warps, each owning 32 of the 128 dims
+constexpr int kAttnThreads = kConsumers + 32;    // plus the producer warp
 constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
-// shared memory of a CTA with `stages` stages: 1 KB alignment slack, the stages, Q, barriers
-constexpr int attn_smem(int stages) { return 1024 + stages * kStageBytes + kMaxR * kHD * 2 + stages * 8; }
+
+// Shared memory of a CTA of a launch over B sequences: 1 KB alignment slack, the stages, two
+// query slots, the barriers, the merge scratch and flags, and the per-sequence tables (first
+// query position, slot, item prefix).
+constexpr size_t attn_smem(int stages, int B) {
+  return 1024 + stages * kStageBytes + 2 * kQBytes + (2 * stages + 4) * 8 + (2 * kMaxR + 8) * 4 +
+         (3 * static_cast<size_t>(B) + 1) * 4;
+}
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
@@ -96,361 +111,522 @@ __device__ __forceinline__ uint32_t swt(int row, int ch) {
   return (ch >> 3) * kHalfBytes + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
 }
 
-// Merge of the super-chunks of every query of (sequence b, head h), run by the CTA that
-// finishes last for it: query r combines super-chunks 0..floor(p_r/256) in order.  Warp w
-// writes queries w, w + 4; each lane four dims.
-__device__ __forceinline__ void merge_all(const AttnArgs& a, int b, int h, int R, int p0, int n_sup, float* smem) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
-  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * n_super * R * kPartStride;
-  float* sm = smem;                      // [n_sup * R] super-chunk max, then weight
-  float* sl = smem + n_sup * R;          // [n_sup * R] super-chunk sum
-  float* sL = sl + n_sup * R;            // [R] total weight
-  for (int i = tid; i < n_sup * R; i += kAttnThreads) {
-    const float* pc = part + static_cast<size_t>(i) * kPartStride;
-    sm[i] = __ldcg(&pc[kHD]);
-    sl[i] = __ldcg(&pc[kHD + 1]);
+// Arrives on the mbarrier when every cp.async this thread issued before has landed; the
+// arrival counts against the barrier's expected count.
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+// Orders this thread's earlier generic-proxy shared-memory accesses before its later TMA writes.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// A position in a CTA's share of the item list: item i is super-chunk s of head h of
+// sequence b, which has nsup super-chunks.  pref[b] is the index of sequence b's first item
+// (pref[B] = the launch's item count).
+struct Walk {
+  int i, b, h, s, nsup;
+  __device__ __forceinline__ void seek(const int* pref, int B, int item) {
+    int lo = 0, hi = B - 1;   // the last sequence whose first item is <= item has items
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (pref[mid] <= item) lo = mid;
+      else hi = mid - 1;
+    }
+    i = item;
+    b = lo;
+    nsup = (pref[b + 1] - pref[b]) / kH;
+    const int r = item - pref[b];
+    h = r / nsup;
+    s = r - h * nsup;
   }
-  __syncthreads();
+  // the next item (the caller has checked that there is one)
+  __device__ __forceinline__ void next(const int* pref) {
+    ++i;
+    if (++s < nsup) return;
+    s = 0;
+    if (++h < kH) return;
+    h = 0;
+    do ++b;
+    while (pref[b + 1] == pref[b]);
+    nsup = (pref[b + 1] - pref[b]) / kH;
+  }
+};
+
+__device__ __forceinline__ int chunks_live(int p0, int R) { return (p0 + R - 1) / kCH + 1; }
+
+// Merge of the super-chunks of every query of (sequence b, head h), run by the 128 consumer
+// threads of the CTA that completed its count: query r combines super-chunks 0..floor(p_r/256)
+// in order.  Threads 0..R-1 find each query's max and weighted sum; warp w then writes queries
+// w, w + 4, each lane four dims.
+__device__ __forceinline__ void merge_seq_head(const AttnArgs& a, int b, int h, int R, int p0, int n_super,
+                                               float* s_mrg, int tid) {
+  const int lane = tid & 31, warp = tid >> 5;
+  const float* part = a.part + (static_cast<size_t>(b) * kH + h) * n_super * R * kPartStride;
   if (tid < R) {
     const int r = tid, lasts = (p0 + r) / (kCH * kSuper);
     float M = -INFINITY;
-    for (int s = 0; s <= lasts; ++s) M = fmaxf(M, sm[s * R + r]);
+#pragma unroll 4
+    for (int s = 0; s <= lasts; ++s) M = fmaxf(M, __ldcg(part + (static_cast<size_t>(s) * R + r) * kPartStride + kHD));
     float L = 0.f;
+#pragma unroll 4
     for (int s = 0; s <= lasts; ++s) {
-      const float ms = sm[s * R + r];
+      const float* pc = part + (static_cast<size_t>(s) * R + r) * kPartStride;
+      const float ms = __ldcg(pc + kHD);
       const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      sm[s * R + r] = w;
-      L += sl[s * R + r] * w;
+      L += __ldcg(pc + kHD + 1) * w;
     }
-    sL[r] = L;
+    s_mrg[r] = M;
+    s_mrg[kMaxR + r] = L;
   }
-  __syncthreads();
-  const int d = lane * 4;   // four dims per lane
-  for (int r = warp; r < R; r += kAttnThreads / 32) {
+  named_bar_sync(1, kConsumers);
+  const int d = lane * 4;
+  for (int r = warp; r < R; r += kConsumers / 32) {
     const int lasts = (p0 + r) / (kCH * kSuper);
+    const float M = s_mrg[r];
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-    int s = 0;
-    for (; s + 4 <= lasts + 1; s += 4) {
-      float4 x[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        x[u] = __ldcg(reinterpret_cast<const float4*>(part + (static_cast<size_t>(s + u) * R + r) * kPartStride + d));
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float w = sm[(s + u) * R + r];
-        O.x += x[u].x * w;
-        O.y += x[u].y * w;
-        O.z += x[u].z * w;
-        O.w += x[u].w * w;
-      }
-    }
-    for (; s <= lasts; ++s) {
-      const float4 x =
-          __ldcg(reinterpret_cast<const float4*>(part + (static_cast<size_t>(s) * R + r) * kPartStride + d));
-      const float w = sm[s * R + r];
+#pragma unroll 4
+    for (int s = 0; s <= lasts; ++s) {
+      const float* pc = part + (static_cast<size_t>(s) * R + r) * kPartStride;
+      const float ms = __ldcg(pc + kHD);
+      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+      const float4 x = __ldcg(reinterpret_cast<const float4*>(pc + d));
       O.x += x.x * w;
       O.y += x.y * w;
       O.z += x.z * w;
       O.w += x.w * w;
     }
-    const float inv = 1.f / sL[r];
+    const float inv = 1.f / s_mrg[kMaxR + r];
     bf16* o = a.out + (static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d;
     *reinterpret_cast<__nv_bfloat162*>(o) = __floats2bfloat162_rn(O.x * inv, O.y * inv);
     *reinterpret_cast<__nv_bfloat162*>(o + 2) = __floats2bfloat162_rn(O.z * inv, O.w * inv);
   }
 }
 
-// Gathers the K and V rows of chunk c into a stage with 16-byte cp.async (two threads per key,
-// eight 16-byte pieces of K and of V each); rows without a visible key are zero-filled.  Used
-// for the chunk that holds staged candidates or masked positions, and for every chunk when the
-// pool has no TMA map.
-__device__ __forceinline__ void gather_chunk(const AttnArgs& a, int b, int h, int slot, int sl, int last, int c,
-                                             uint8_t* stage) {
-  const int key = threadIdx.x >> 1, half = threadIdx.x & 1;
-  const int pos = c * kCH + key;
-  const bf16* srck = a.pool;
-  const bf16* srcv = a.pool;
-  int bytes = 0;
-  if (pos <= last) {
-    if (pos < sl) {
-      const int pi = pos / a.page_size;
-      const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
-      if (page >= 0 && page < a.n_pages) {
-        srck = a.pool + ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
-        srcv = srck + static_cast<long long>(kH) * a.page_size * kHD;
-        bytes = 16;
-      } else {
-        atomicOr(a.err, ERR_PAGE_RANGE);
-      }
-    } else {
-      srck = a.stage + b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
-             static_cast<long long>(h) * kHD;
-      srcv = srck + a.stage_kv_stride;
-      bytes = 16;
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int ch = half * 8 + i;
-    const int o = bytes ? ch * 8 : 0;
-    cp_async16(stage + swt(key, ch), srck + o, bytes);
-    cp_async16(stage + kTileBytes + swt(key, ch), srcv + o, bytes);
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-
-// kStages stages per CTA: 3 (two CTAs per SM) when the launch spans many waves, 2 (three CTAs
-// per SM) when it fits in about two.  Four warps: each recomputes the chunk's 64 x 8 scores
-// (cheap) and owns 32 of the 128 output dims, so its dependent MMA chain is short.
 template <int kStages>
-__global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 2) attn_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ uint8_t asmem_raw[];
   const uint32_t raw_u32 = smem_u32(asmem_raw);
   uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [S][K 16 KB | V 16 KB]
-  uint8_t* sQ = stages + kStages * kStageBytes;              // [8 queries][128 dims] bf16
-  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + kMaxR * kHD * 2);   // [S] TMA stage barriers
-  __shared__ int s_page[kUnitMaxChunks];                     // page of each TMA chunk of the unit
-  __shared__ int s_abort;
-  __shared__ int s_last;
+  uint8_t* sQ = stages + kStages * kStageBytes;                             // [2][8 queries][128] bf16
+  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + 2 * kQBytes);           // [S] chunk landed
+  uint64_t* empty = full + kStages;                                         // [S] chunk consumed
+  uint64_t* qfull = empty + kStages;                                        // [2] queries landed
+  uint64_t* qempty = qfull + 2;                                             // [2] queries loaded
+  float* s_mrg = reinterpret_cast<float*>(qempty + 2);                      // [2 * kMaxR] merge M, L
+  int* s_flag = reinterpret_cast<int*>(s_mrg + 2 * kMaxR);                  // abort, last, err, warp sums[5]
+  volatile int* s_abort = s_flag;
+  int* s_p0 = s_flag + 8;                                                   // [B] first query position
+  int* s_slot = s_p0 + a.B;                                                 // [B] slot
+  int* s_pref = s_slot + a.B;                                               // [B + 1] first item
   pdl_trigger();
-  pdl_wait();
+  if (!a.prewait) pdl_wait();
 
-  const int u = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
-  const int R = a.R;
-  // the queries first (bf16, as the QKV epilogue stored them; rows R..7 zero): their loads need
-  // no slot and overlap the slot -> length -> page lookups
-  uint4 qv = make_uint4(0, 0, 0, 0);
-  {
-    const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
-    const int q = tid >> 4, ch = tid & 15;   // 8 queries x 16 pieces of 16 bytes
-    if (q < R) qv = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(qrow0 + q) * kH + h) * kHD + ch * 8);
-  }
-  const int slot = a.slots[b];
-  if (slot < 0 || slot >= a.n_slots) {   // every CTA of the sequence leaves; no ticket, no merge
-    if (u == 0 && h == 0 && tid == 0) atomicOr(a.err, ERR_SLOT_RANGE);
-    return;
-  }
-  // this CTA's super-chunks: u, u + n_units, u + 2 n_units, ... (strided, so that short contexts
-  // spread over the CTAs of the (sequence, head) as evenly as long ones); its chunk list, in
-  // increasing order, is chunk_of(i)
-  const int n_units = gridDim.x;
-  auto chunk_of = [&](int i) { return (u + (i / kSuper) * n_units) * kSuper + i % kSuper; };
-  // the pages of every chunk the CTA may own are looked up now, alongside the length
-  int spec_page = -1;
-  if (tid < a.unit * kSuper) {
-    const int pi = chunk_of(tid) * kCH / a.page_size;
-    if (pi < a.max_pages) spec_page = a.block_table[slot * a.max_pages + pi];
-  }
-  const int sl = a.seq_len[slot];
-  const int p0 = sl + a.qoff;
-  const int last = p0 + R - 1;
-  if (p0 < 0) return;
-  const int n_live = last / kCH + 1;                         // chunks holding keys 0..last
-  const int n_sup_live = (n_live + kSuper - 1) / kSuper;
-  if (u >= n_sup_live) return;
-  const int n_mine = (n_sup_live - 1 - u) / n_units + 1;            // super-chunks of this CTA
-  const int last_sup = u + (n_mine - 1) * n_units;
-  const int n = (n_mine - 1) * kSuper + (min(n_live, (last_sup + 1) * kSuper) - last_sup * kSuper);
-  // a prefix of the list holds committed keys only and comes by TMA; the rest are gathered
-  int n_tma = 0;
-  if (a.use_tma)
-    while (n_tma < n && (chunk_of(n_tma) + 1) * kCH <= sl) ++n_tma;
-
-  if (tid < n_tma) {
-    int page = spec_page;
-    if (page < 0 || page >= a.n_pages) {
-      atomicOr(a.err, ERR_PAGE_RANGE);
-      page = -1;
-    }
-    s_page[tid] = page;
-  }
+  const int B = a.B, R = a.R;
   if (tid == 0) {
-    for (int st = 0; st < kStages; ++st) mbar_init(&full[st], 1);
-    s_abort = 0;
+    for (int st = 0; st < kStages; ++st) {
+      mbar_init(&full[st], 32);
+      mbar_init(&empty[st], kConsumers / 32);
+    }
+    for (int q = 0; q < 2; ++q) {
+      mbar_init(&qfull[q], 32);
+      mbar_init(&qempty[q], kConsumers / 32);
+    }
+    s_flag[0] = 0;
+    s_flag[2] = 0;
     fence_mbar_init();
   }
-  *reinterpret_cast<uint4*>(sQ + swz(tid >> 4, tid & 15)) = qv;
-  __syncthreads();
+  if (tid == kConsumers && a.use_tma) tma_prefetch_desc(&a.kv_map);
 
-  // TMA of chunk i of the unit into stage i % S; a chunk whose page is invalid completes its
-  // barrier without data (the guard flag is already set)
-  const uint64_t pol = l2_policy_evict_first();
-  auto issue = [&](int i) {
-    const int st = i % kStages;
-    uint8_t* dst = stages + st * kStageBytes;
-    const int page = s_page[i];
-    if (page < 0) {
-      mbar_arrive(&full[st]);
-      return;
+  // ---- per-sequence tables: slot, first query position and super-chunk count, then the
+  // exclusive prefix of the item counts (thread t scans a contiguous block of sequences)
+  for (int bb = tid; bb < B; bb += kAttnThreads) s_slot[bb] = a.slots[bb];
+  __syncthreads();
+  int errbits = 0;
+  for (int bb = tid; bb < B; bb += kAttnThreads) {
+    const int slot = s_slot[bb];
+    int p0 = -1, nsup = 0;
+    if (slot < 0 || slot >= a.n_slots) {
+      errbits |= ERR_SLOT_RANGE;
+    } else {
+      p0 = a.seq_len[slot] + a.qoff;
+      if (p0 >= 0) {
+        const int n_live = chunks_live(p0, R);
+        if (n_live > a.n_chunks) errbits |= ERR_PAGE_RANGE;
+        else nsup = (n_live + kSuper - 1) / kSuper;
+      }
     }
-    const int c = chunk_of(i);
-    const int row_k = (page * 2 * kH + h) * a.page_size + (c * kCH) % a.page_size;
-    const int row_v = row_k + kH * a.page_size;
-    mbar_arrive_expect_tx(&full[st], kStageBytes);
-    tma_load_2d(dst, &a.kv_map, &full[st], 0, row_k, pol);
-    tma_load_2d(dst + kHalfBytes, &a.kv_map, &full[st], 64, row_k, pol);
-    tma_load_2d(dst + kTileBytes, &a.kv_map, &full[st], 0, row_v, pol);
-    tma_load_2d(dst + kTileBytes + kHalfBytes, &a.kv_map, &full[st], 64, row_v, pol);
-  };
-  if (tid == 0) {
-    if (n_tma > 0) tma_prefetch_desc(&a.kv_map);
-    for (int i = 0; i < min(n_tma, kStages); ++i) issue(i);
+    s_p0[bb] = p0;
+    s_pref[bb] = nsup * kH;
+  }
+  if (errbits) atomicOr(&s_flag[2], errbits);
+  __syncthreads();
+  {
+    const int per = (B + kAttnThreads - 1) / kAttnThreads;
+    const int b0 = min(B, tid * per), b1 = min(B, b0 + per);
+    int own = 0;
+    for (int bb = b0; bb < b1; ++bb) own += s_pref[bb];
+    int incl = own;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) s_flag[3 + warp] = incl;
+    __syncthreads();
+    int acc = incl - own;
+    for (int w = 0; w < warp; ++w) acc += s_flag[3 + w];
+    for (int bb = b0; bb < b1; ++bb) {
+      const int n = s_pref[bb];
+      s_pref[bb] = acc;
+      acc += n;
+    }
+    if (tid == kAttnThreads - 1) s_pref[B] = acc;
+  }
+  __syncthreads();
+  if (blockIdx.x == 0 && tid == 0 && s_flag[2]) {
+    pdl_wait();
+    atomicOr(a.err, s_flag[2]);
+  }
+  const int W = s_pref[B];
+  const int per_cta = (W + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
+  const int i_begin = static_cast<int>(blockIdx.x) * per_cta;
+  const int i_end = min(W, i_begin + per_cta);
+  if (i_begin >= i_end) return;
+  const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
+
+  if (warp == kConsumers / 32) {
+    // ------------------------------------------------------------------ producer warp
+    const uint64_t pol = l2_policy_evict_first();
+    int perr = 0;
+    // lanes 0..3: the page of chunk 4 s + lane of item w if it can come by TMA (its 64 keys
+    // all committed), -1 if it is gathered, -2 if its page is outside the table or the pool
+    auto lookup = [&](const Walk& w) -> int {
+      int pg = -1;
+      if (lane < kSuper && a.use_tma) {
+        const int p0 = s_p0[w.b], c = kSuper * w.s + lane;
+        if (c < chunks_live(p0, R) && (c + 1) * kCH <= p0 - a.qoff) {
+          const int pi = c * kCH / a.page_size;
+          pg = (pi < a.max_pages) ? a.block_table[s_slot[w.b] * a.max_pages + pi] : -2;
+          if (pg < 0 || pg >= a.n_pages) pg = -2;
+        }
+      }
+      return pg;
+    };
+    auto issue_tma = [&](int st, int page, int h, int c) {
+      if (lane == 0) {
+        if (page < 0) {   // completes the stage without data; the guard flag reports it
+          perr |= ERR_PAGE_RANGE;
+          mbar_arrive(&full[st]);
+        } else {
+          uint8_t* dst = stages + st * kStageBytes;
+          const int row_k = (page * 2 * kH + h) * a.page_size + (c * kCH) % a.page_size;
+          const int row_v = row_k + kH * a.page_size;
+          fence_proxy_async_smem();
+          mbar_arrive_expect_tx(&full[st], kStageBytes);
+          tma_load_2d(dst, &a.kv_map, &full[st], 0, row_k, pol);
+          tma_load_2d(dst + kHalfBytes, &a.kv_map, &full[st], 64, row_k, pol);
+          tma_load_2d(dst + kTileBytes, &a.kv_map, &full[st], 0, row_v, pol);
+          tma_load_2d(dst + kTileBytes + kHalfBytes, &a.kv_map, &full[st], 64, row_v, pol);
+        }
+      } else {
+        mbar_arrive(&full[st]);
+      }
+    };
+    // keys lane and lane + 32 of chunk c, K and V, eight... sixteen 16-byte pieces each
+    auto issue_gather = [&](int st, int b, int h, int c) {
+      uint8_t* stage = stages + st * kStageBytes;
+      const int slot = s_slot[b], p0 = s_p0[b];
+      const int sl = p0 - a.qoff, last = p0 + R - 1;
+#pragma unroll
+      for (int k2 = 0; k2 < 2; ++k2) {
+        const int key = lane + 32 * k2, pos = c * kCH + key;
+        const bf16* srck = a.pool;
+        const bf16* srcv = a.pool;
+        int bytes = 0;
+        if (pos <= last) {
+          if (pos < sl) {
+            const int pi = pos / a.page_size;
+            const int page = (pi < a.max_pages) ? a.block_table[slot * a.max_pages + pi] : -1;
+            if (page >= 0 && page < a.n_pages) {
+              srck = a.pool + ((static_cast<long long>(page) * 2 * kH + h) * a.page_size + pos % a.page_size) * kHD;
+              srcv = srck + static_cast<long long>(kH) * a.page_size * kHD;
+              bytes = 16;
+            } else {
+              perr |= ERR_PAGE_RANGE;
+            }
+          } else {
+            srck = a.stage + b * a.stage_seq_stride + static_cast<long long>(pos - sl) * a.stage_row_stride +
+                   static_cast<long long>(h) * kHD;
+            srcv = srck + a.stage_kv_stride;
+            bytes = 16;
+          }
+        }
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          const int o = bytes ? ch * 8 : 0;
+          cp_async16(stage + swt(key, ch), srck + o, bytes);
+          cp_async16(stage + kTileBytes + swt(key, ch), srcv + o, bytes);
+        }
+      }
+      cp_async_mbar_arrive(&full[st]);
+    };
+    // the queries of run r (rows R..7 zero) into slot r & 1, four 16-byte pieces per lane
+    auto issue_q = [&](int r, int b, int h) -> bool {
+      const int qs = r & 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&qempty[qs], ((r >> 1) & 1) ^ 1u, s_abort));
+      if (!ok) return false;
+      const int qrow0 = a.q_row0 ? a.q_row0[b] : b * R;
+      const int row = lane >> 2;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int ch = (lane & 3) * 4 + k;
+        const bool has = row < R;
+        const bf16* src = has ? a.q + (static_cast<size_t>(qrow0 + row) * kH + h) * kHD + ch * 8 : a.q;
+        cp_async16(sQ + qs * kQBytes + swz(row, ch), src, has ? 16 : 0);
+      }
+      cp_async_mbar_arrive(&qfull[qs]);
+      return true;
+    };
+
+    Walk w;
+    w.seek(s_pref, B, i_begin);
+    // pass 1 (verify step): the K/V of the leading committed chunks, before the wait
+    int j_pre = 0;
+    if (a.prewait) {
+      Walk v = w;
+      bool go = true;
+      while (go) {
+        const int pg = lookup(v);
+        const int c0 = kSuper * v.s, c1 = min(c0 + kSuper, chunks_live(s_p0[v.b], R));
+        for (int c = c0; c < c1 && go; ++c) {
+          const int page = __shfl_sync(0xffffffffu, pg, c - c0);
+          if (page == -1 || j_pre == kStages) {
+            go = false;
+          } else {
+            issue_tma(j_pre, page, v.h, c);
+            ++j_pre;
+          }
+        }
+        if (go && v.i + 1 < i_end) v.next(s_pref);
+        else go = false;
+      }
+      pdl_wait();
+    }
+    // pass 2: every chunk in order -- the queries at the start of each (sequence, head) run,
+    // the K/V of the chunks pass 1 did not fetch; page lookups one item ahead
+    int j = 0, r = -1;
+    bool failed = false;
+    int pg = lookup(w);
+    Walk wn = w;
+    bool has_next = w.i + 1 < i_end;
+    int pg_next = -1;
+    if (has_next) {
+      wn.next(s_pref);
+      pg_next = lookup(wn);
+    }
+    while (true) {
+      if (w.i == i_begin || w.s == 0) {
+        ++r;
+        if (!issue_q(r, w.b, w.h)) {
+          failed = true;
+          break;
+        }
+      }
+      const int c0 = kSuper * w.s, c1 = min(c0 + kSuper, chunks_live(s_p0[w.b], R));
+      for (int c = c0; c < c1; ++c, ++j) {
+        if (j < j_pre) continue;
+        const int st = j % kStages;
+        if (!__all_sync(0xffffffffu, mbar_wait(&empty[st], ((j / kStages) & 1) ^ 1u, s_abort))) {
+          failed = true;
+          break;
+        }
+        const int page = __shfl_sync(0xffffffffu, pg, c - c0);
+        if (page == -1) issue_gather(st, w.b, w.h, c);
+        else issue_tma(st, page, w.h, c);
+      }
+      if (failed || !has_next) break;
+      w = wn;
+      pg = pg_next;
+      has_next = w.i + 1 < i_end;
+      if (has_next) {
+        wn.next(s_pref);
+        pg_next = lookup(wn);
+      }
+    }
+    if (failed) {
+      if (lane == 0) *s_abort = 1;
+      perr |= ERR_WAIT_TIMEOUT;
+    }
+    // let every copy still in flight land before the CTA's shared memory is released
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    if (lane == 0) {
+      volatile int never = 0;
+      const int issued = max(j, j_pre);
+      for (int jj = max(0, issued - kStages); jj < issued; ++jj)
+        mbar_wait(&full[jj % kStages], static_cast<uint32_t>(jj / kStages) & 1u, &never, 100000000ull);
+    }
+    perr = __reduce_or_sync(0xffffffffu, perr);
+    if (lane == 0 && perr) atomicOr(a.err, perr);
+    return;
   }
 
-  // Q^T fragments (B operand of S^T = K Q^T), the same for every chunk
-  const uint32_t qbase = smem_u32(sQ);
-  uint32_t qf[8][2];
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks) ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), qf[ks]);
-
-  const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));   // log2(e) / sqrt(hd)
+  // -------------------------------------------------------------------- consumer warps
+  if (a.prewait) pdl_wait();
+  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3, ri = lane & 7;
   const int qa = 2 * t4, qb = 2 * t4 + 1;                    // the two queries of this lane
-  float* part = a.part + (static_cast<size_t>(b) * kH + h) * ((a.n_chunks + kSuper - 1) / kSuper) * R * kPartStride;
-  float M_a = -INFINITY, M_b = -INFINITY, L_a = 0.f, L_b = 0.f;
-  float O[2][4], Ol[2][4];   // hi and lo parts of the unnormalised output, dims 32 warp + 16 j
-  int consumed = 0;          // TMA chunks waited for
-  bool aborted = false;
-  for (int i = 0; i < n; ++i) {
-    const int c = chunk_of(i);
-    const int st = i % kStages;
-    uint8_t* stage = stages + st * kStageBytes;
-    if (c % kSuper == 0 || i == 0) {
-      M_a = M_b = -INFINITY;
-      L_a = L_b = 0.f;
+  const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(kHD));   // log2(e) / sqrt(hd)
+  Walk w;
+  w.seek(s_pref, B, i_begin);
+  int j = 0, r = -1, run_items = 0;
+  bool ok = true;            // false once a wait has run out: the rest is walked without compute
+  uint32_t qf[8][2];         // Q^T fragments (B operand of S^T = K Q^T) of the current run
+  while (true) {
+    if (w.i == i_begin || w.s == 0) {
+      ++r;
+      run_items = 0;
+      const int qs = r & 1;
+      if (ok && !__all_sync(0xffffffffu, mbar_wait(&qfull[qs], (r >> 1) & 1, s_abort))) ok = false;
+      const uint32_t qbase = smem_u32(sQ + qs * kQBytes);
 #pragma unroll
-      for (int j = 0; j < 2; ++j)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) O[j][e] = Ol[j][e] = 0.f;
+      for (int ks = 0; ks < 8; ++ks) ldsm_x2(qbase + swz(ri, 2 * ks + (mi & 1)), qf[ks]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&qempty[qs]);
     }
-    if (i < n_tma) {
-      const bool ok = mbar_wait(&full[st], static_cast<uint32_t>(i / kStages) & 1u, &s_abort);
-      if (__syncthreads_or(!ok)) {
-        aborted = true;
-        break;
+    const int b = w.b, h = w.h;
+    const int p0 = s_p0[b];
+    const int c0 = kSuper * w.s, c1 = min(c0 + kSuper, chunks_live(p0, R));
+    float M_a = -INFINITY, M_b = -INFINITY, L_a = 0.f, L_b = 0.f;
+    float O[2][4], Ol[2][4];   // hi and lo parts of the unnormalised output, dims 32 warp + 16 j
+#pragma unroll
+    for (int jj = 0; jj < 2; ++jj)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) O[jj][e] = Ol[jj][e] = 0.f;
+    for (int c = c0; c < c1; ++c, ++j) {
+      const int st = j % kStages;
+      if (ok && !__all_sync(0xffffffffu, mbar_wait(&full[st], (j / kStages) & 1, s_abort))) {
+        ok = false;
+        if (lane == 0) {
+          *s_abort = 1;
+          atomicOr(a.err, ERR_WAIT_TIMEOUT);
+        }
       }
-      consumed = i + 1;
-    } else {
-      gather_chunk(a, b, h, slot, sl, last, c, stage);
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-      __syncthreads();
-    }
-    const uint32_t kbase = smem_u32(stage);
-    const uint32_t vbase = kbase + kTileBytes;
-
-    // S^T[key][query] = K Q^T over four 16-key tiles, 8 k-steps of 16 dims: even and odd
-    // k-steps in separate accumulators (eight independent MMA chains), added at the end
-    float s[4][4], s1[4][4];
+      if (ok) {
+        const uint32_t kbase = smem_u32(stages + st * kStageBytes);
+        const uint32_t vbase = kbase + kTileBytes;
+        // S^T[key][query] = K Q^T over four 16-key tiles, 8 k-steps of 16 dims: even and odd
+        // k-steps in separate accumulators (eight independent MMA chains), added at the end
+        float s[4][4], s1[4][4];
 #pragma unroll
-    for (int kt = 0; kt < 4; ++kt)
+        for (int kt = 0; kt < 4; ++kt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) s[kt][e] = s1[kt][e] = 0.f;
+          for (int e = 0; e < 4; ++e) s[kt][e] = s1[kt][e] = 0.f;
 #pragma unroll
-    for (int ks = 0; ks < 8; ks += 2) {
+        for (int ks = 0; ks < 8; ks += 2) {
 #pragma unroll
-      for (int kt = 0; kt < 4; ++kt) {
-        uint32_t ak[4], ak1[4];
-        ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + (mi >> 1)), ak);
-        ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + 2 + (mi >> 1)), ak1);
-        mma_bf16_16816(s[kt], ak, qf[ks]);
-        mma_bf16_16816(s1[kt], ak1, qf[ks + 1]);
+          for (int kt = 0; kt < 4; ++kt) {
+            uint32_t ak[4], ak1[4];
+            ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + (mi >> 1)), ak);
+            ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + 2 + (mi >> 1)), ak1);
+            mma_bf16_16816(s[kt], ak, qf[ks]);
+            mma_bf16_16816(s1[kt], ak1, qf[ks + 1]);
+          }
+        }
+#pragma unroll
+        for (int kt = 0; kt < 4; ++kt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) s[kt][e] += s1[kt][e];
+        // visibility, chunk max per query (lanes sharing t4 hold the same two queries)
+        const int kb = c * kCH;
+        float m_a = -INFINITY, m_b = -INFINITY;
+#pragma unroll
+        for (int kt = 0; kt < 4; ++kt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int key = kb + 16 * kt + g + ((e >> 1) ? 8 : 0);
+            const int q = (e & 1) ? qb : qa;
+            const float x = (q < R && key <= p0 + q) ? s[kt][e] * scale : -INFINITY;
+            s[kt][e] = x;
+            if (e & 1) m_b = fmaxf(m_b, x);
+            else m_a = fmaxf(m_a, x);
+          }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          m_a = fmaxf(m_a, __shfl_xor_sync(0xffffffffu, m_a, o));
+          m_b = fmaxf(m_b, __shfl_xor_sync(0xffffffffu, m_b, o));
+        }
+        const float Mn_a = fmaxf(M_a, m_a), Mn_b = fmaxf(M_b, m_b);
+        const float al_a = (M_a == -INFINITY) ? 0.f : exp2f(M_a - Mn_a);
+        const float al_b = (M_b == -INFINITY) ? 0.f : exp2f(M_b - Mn_b);
+        M_a = Mn_a;
+        M_b = Mn_b;
+        // p = 2^(x - M) (exact zeros where masked), row sums, and P^T as bf16 hi + lo fragments
+        float l_a = 0.f, l_b = 0.f;
+        uint32_t ph[4][2], pl[4][2];
+#pragma unroll
+        for (int kt = 0; kt < 4; ++kt) {
+          float p[4], lo[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float Mq = (e & 1) ? M_b : M_a;
+            p[e] = (s[kt][e] == -INFINITY) ? 0.f : exp2f(s[kt][e] - Mq);
+            if (e & 1) l_b += p[e];
+            else l_a += p[e];
+            lo[e] = p[e] - __bfloat162float(__float2bfloat16(p[e]));
+          }
+          ph[kt][0] = movmatrix_t(pack_bf16(p[0], p[1]));     // keys 16kt+0..7
+          ph[kt][1] = movmatrix_t(pack_bf16(p[2], p[3]));     // keys 16kt+8..15
+          pl[kt][0] = movmatrix_t(pack_bf16(lo[0], lo[1]));
+          pl[kt][1] = movmatrix_t(pack_bf16(lo[2], lo[3]));
+        }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          l_a += __shfl_xor_sync(0xffffffffu, l_a, o);
+          l_b += __shfl_xor_sync(0xffffffffu, l_b, o);
+        }
+        L_a = L_a * al_a + l_a;
+        L_b = L_b * al_b + l_b;
+        // O^T[dim][query] = al * O^T + V^T P^T for this warp's two 16-dim tiles (dims
+        // 32w..32w+31), 4 k-steps of 16 keys; hi and lo products in separate accumulators
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          O[jj][0] *= al_a;
+          O[jj][1] *= al_b;
+          O[jj][2] *= al_a;
+          O[jj][3] *= al_b;
+          Ol[jj][0] *= al_a;
+          Ol[jj][1] *= al_b;
+          Ol[jj][2] *= al_a;
+          Ol[jj][3] *= al_b;
+        }
+#pragma unroll
+        for (int kt = 0; kt < 4; ++kt) {
+#pragma unroll
+          for (int jj = 0; jj < 2; ++jj) {
+            uint32_t av[4];
+            ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * (2 * warp + jj) + (mi & 1)), av);
+            mma_bf16_16816(O[jj], av, ph[kt]);
+            mma_bf16_16816(Ol[jj], av, pl[kt]);
+          }
+        }
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);   // this warp is done with the stage
     }
+    // end of the super-chunk: its (M, L, O) per query (each warp its 32 dims)
+    {
+      float* ps = a.part + ((static_cast<size_t>(b) * kH + h) * n_super + w.s) * R * kPartStride;
 #pragma unroll
-    for (int kt = 0; kt < 4; ++kt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) s[kt][e] += s1[kt][e];
-    // visibility, chunk max per query (lanes sharing t4 hold the same two queries)
-    const int kb = c * kCH;
-    float m_a = -INFINITY, m_b = -INFINITY;
-#pragma unroll
-    for (int kt = 0; kt < 4; ++kt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = kb + 16 * kt + g + ((e >> 1) ? 8 : 0);
-        const int q = (e & 1) ? qb : qa;
-        const float x = (q < R && key <= p0 + q) ? s[kt][e] * scale : -INFINITY;
-        s[kt][e] = x;
-        if (e & 1) m_b = fmaxf(m_b, x);
-        else m_a = fmaxf(m_a, x);
-      }
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) {
-      m_a = fmaxf(m_a, __shfl_xor_sync(0xffffffffu, m_a, o));
-      m_b = fmaxf(m_b, __shfl_xor_sync(0xffffffffu, m_b, o));
-    }
-    const float Mn_a = fmaxf(M_a, m_a), Mn_b = fmaxf(M_b, m_b);
-    const float al_a = (M_a == -INFINITY) ? 0.f : exp2f(M_a - Mn_a);
-    const float al_b = (M_b == -INFINITY) ? 0.f : exp2f(M_b - Mn_b);
-    M_a = Mn_a;
-    M_b = Mn_b;
-    // p = 2^(x - M) (exact zeros where masked), row sums, and P^T as bf16 hi + lo fragments
-    float l_a = 0.f, l_b = 0.f;
-    uint32_t ph[4][2], pl[4][2];
-#pragma unroll
-    for (int kt = 0; kt < 4; ++kt) {
-      float p[4], lo[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float Mq = (e & 1) ? M_b : M_a;
-        p[e] = (s[kt][e] == -INFINITY) ? 0.f : exp2f(s[kt][e] - Mq);
-        if (e & 1) l_b += p[e];
-        else l_a += p[e];
-        lo[e] = p[e] - __bfloat162float(__float2bfloat16(p[e]));
-      }
-      ph[kt][0] = movmatrix_t(pack_bf16(p[0], p[1]));     // keys 16kt+0..7
-      ph[kt][1] = movmatrix_t(pack_bf16(p[2], p[3]));     // keys 16kt+8..15
-      pl[kt][0] = movmatrix_t(pack_bf16(lo[0], lo[1]));
-      pl[kt][1] = movmatrix_t(pack_bf16(lo[2], lo[3]));
-    }
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) {
-      l_a += __shfl_xor_sync(0xffffffffu, l_a, o);
-      l_b += __shfl_xor_sync(0xffffffffu, l_b, o);
-    }
-    L_a = L_a * al_a + l_a;
-    L_b = L_b * al_b + l_b;
-    // O^T[dim][query] = al * O^T + V^T P^T for this warp's two 16-dim tiles (dims 32w..32w+31),
-    // 4 k-steps of 16 keys; hi and lo products in separate accumulators, summed per super-chunk
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      O[j][0] *= al_a;
-      O[j][1] *= al_b;
-      O[j][2] *= al_a;
-      O[j][3] *= al_b;
-      Ol[j][0] *= al_a;
-      Ol[j][1] *= al_b;
-      Ol[j][2] *= al_a;
-      Ol[j][3] *= al_b;
-    }
-#pragma unroll
-    for (int kt = 0; kt < 4; ++kt) {
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        uint32_t av[4];
-        ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * (2 * warp + j) + (mi & 1)), av);
-        mma_bf16_16816(O[j], av, ph[kt]);
-        mma_bf16_16816(Ol[j], av, pl[kt]);
-      }
-    }
-    __syncthreads();   // every warp is done with this stage
-    if (tid == 0 && i + kStages < n_tma) issue(i + kStages);
-
-    // end of a super-chunk: its (M, L, O) per query (each warp its 32 dims)
-    if ((c + 1) % kSuper == 0 || c + 1 == n_live) {
-      float* ps = part + static_cast<size_t>(c / kSuper) * R * kPartStride;
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int d = 16 * (2 * warp + j) + g;
+      for (int jj = 0; jj < 2; ++jj) {
+        const int d = 16 * (2 * warp + jj) + g;
         if (qa < R) {
-          ps[qa * kPartStride + d] = O[j][0] + Ol[j][0];
-          ps[qa * kPartStride + d + 8] = O[j][2] + Ol[j][2];
+          ps[qa * kPartStride + d] = O[jj][0] + Ol[jj][0];
+          ps[qa * kPartStride + d + 8] = O[jj][2] + Ol[jj][2];
         }
         if (qb < R) {
-          ps[qb * kPartStride + d] = O[j][1] + Ol[j][1];
-          ps[qb * kPartStride + d + 8] = O[j][3] + Ol[j][3];
+          ps[qb * kPartStride + d] = O[jj][1] + Ol[jj][1];
+          ps[qb * kPartStride + d + 8] = O[jj][3] + Ol[jj][3];
         }
       }
       if (warp == 0 && g == 0) {
@@ -464,61 +640,51 @@ __global__ void __launch_bounds__(kAttnThreads) attn_chunk_kernel(const __grid_c
         }
       }
     }
-  }
-  if (aborted) {
-    // a stage wait ran out: flag it and let the copies still in flight land, then take the
-    // ticket as usual so that the counters stay consistent (the merged result is invalid)
-    if (tid == 0) {
-      atomicOr(a.err, ERR_WAIT_TIMEOUT);
-      const int issued = min(n_tma, consumed + kStages);
-      int never = 0;
-      for (int i = consumed; i < issued; ++i)
-        mbar_wait(&full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, &never, 100000000ull);
+    ++run_items;
+    const bool more = w.i + 1 < i_end;
+    if (!more || w.s == w.nsup - 1) {
+      // this CTA's super-chunks of (b, h) are written: count them; the CTA that completes the
+      // count merges every super-chunk of (b, h)
+      __threadfence();
+      named_bar_sync(1, kConsumers);
+      if (tid == 0) {
+        int* ticket = a.tickets + b * kH + h;
+        const int old = atomicAdd(ticket, run_items);
+        const int last = (old + run_items == w.nsup) ? 1 : 0;
+        if (last) *ticket = 0;
+        s_flag[1] = last;
+      }
+      named_bar_sync(1, kConsumers);
+      if (s_flag[1]) {
+        __threadfence();
+        merge_seq_head(a, b, h, R, p0, n_super, s_mrg, tid);
+      }
     }
-    __syncthreads();
-  }
-
-  // the CTA that finishes last for (sequence, head) merges every query
-  __threadfence();
-  __syncthreads();
-  const int n_busy = min(n_units, n_sup_live);   // CTAs of this (sequence, head) with work
-  if (tid == 0) {
-    int* ticket = a.tickets + b * kH + h;
-    const int old = atomicAdd(ticket, 1);
-    s_last = (old == n_busy - 1) ? 1 : 0;
-    if (s_last) *ticket = 0;
-  }
-  __syncthreads();
-  if (s_last) {
-    __threadfence();
-    merge_all(a, b, h, R, p0, (n_live + kSuper - 1) / kSuper, reinterpret_cast<float*>(stages));
+    if (!more) break;
+    w.next(s_pref);
   }
 }
 
 cudaError_t attention_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(attn_chunk_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, attn_smem(2));
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_chunk_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, attn_smem(3));
-  return e;
+  return cudaFuncSetAttribute(attn_kernel<kAttnStages>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(attn_smem(kAttnStages, 2048)));
 }
 
 cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
-  // At most `unit` super-chunks per CTA: enough CTAs for about two waves of two per SM over the
-  // largest context the pools allow.  Pure scheduling: the arithmetic of every super-chunk and
-  // of the merge is the same for any assignment.
+  // As many CTAs as fit at once (three per SM, at most one per item).  Pure scheduling: the
+  // arithmetic of every super-chunk and of the merge is the same for any grid.
   AttnArgs a = a_in;
-  const int n_super = (a.n_chunks + kSuper - 1) / kSuper;
-  const long long target = 4ll * num_sms();
-  const long long per_unit = static_cast<long long>(B) * kH;
-  int unit = static_cast<int>((per_unit * n_super + target - 1) / target);
-  if (unit < 1) unit = 1;
-  if (unit > kUnitMaxSuper) unit = kUnitMaxSuper;
-  a.unit = unit;
-  const int n_units = (n_super + unit - 1) / unit;
-  const long long ctas = static_cast<long long>(n_units) * kH * B;
-  if (ctas <= 6ll * num_sms())
-    return launch_pdl(attn_chunk_kernel<2>, dim3(n_units, kH, B), dim3(kAttnThreads), attn_smem(2), s, a);
-  return launch_pdl(attn_chunk_kernel<3>, dim3(n_units, kH, B), dim3(kAttnThreads), attn_smem(3), s, a);
+  a.B = B;
+  const size_t smem = attn_smem(kAttnStages, B);
+  int per_sm = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_kernel<kAttnStages>, kAttnThreads, smem);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) per_sm = 1;
+  const long long most = static_cast<long long>(B) * kH * ((a.n_chunks + kSuper - 1) / kSuper);
+  long long grid = static_cast<long long>(per_sm) * num_sms();
+  if (grid > most) grid = most;
+  if (grid < 1) grid = 1;
+  return launch_pdl(attn_kernel<kAttnStages>, dim3(static_cast<unsigned>(grid)), dim3(kAttnThreads), smem, s, a);
 }
 
 }  // namespace fm

@@ -148,9 +148,13 @@ struct AttnArgs {
   const bf16* stage;           // keys at positions >= seq_len[slot]: staged row (pos - seq_len)
   long long stage_seq_stride, stage_row_stride, stage_kv_stride;
   float* part;                 // [B][H][ceil(n_chunks / 4)][R][132] super-chunk partials
-  int* tickets;                // [B][H] chunk counters, zero between launches
-  int n_chunks;
-  int unit;                    // chunks per CTA (set by attention_launch)
+  int* tickets;                // [B][H] super-chunk counters, zero between launches
+  int n_chunks;                // most chunks a sequence may span (pool capacity + staged rows)
+  int B;                       // sequences of this launch (set by attention_launch)
+  // Set when no kernel of the same graph writes the pages, the block table, the slots or the
+  // lengths (the verify step): the K/V of the first committed chunks is then fetched before
+  // the wait for the previous kernel.
+  int prewait;
   bf16* out;                   // [B*R][H*hd]
   int out_row_stride_seq;      // rows of out per sequence (R)
   int* err;

@@ -708,6 +708,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       a.out = ctx->attn_out;
       a.out_row_stride_seq = R;
       a.err = ctx->d_err;
+      a.prewait = 1;   // pages, block table, slots and lengths change only in accept_commit / seq_reset
       LAUNCH(SPEC_K_ATTN, 1, attention_launch(a, B, s));
     }
     // O-proj + residual
