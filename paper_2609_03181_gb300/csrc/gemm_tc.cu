@@ -100,6 +100,11 @@ __device__ __forceinline__ void epi_pre(const GemmArgs& a, const Item& it, int r
   }
 }
 
+// Rotate-half RoPE of the pair (x_i, x_{i+64}) with (cos, sin) = f, rounded the same way in
+// every epilogue: lo' = x_i cos - x_{i+64} sin, hi' = x_{i+64} cos + x_i sin.
+__device__ __forceinline__ float rope_lo(float lo, float hi, float2 f) { return __fmaf_rn(lo, f.x, -__fmul_rn(hi, f.y)); }
+__device__ __forceinline__ float rope_hi(float hi, float lo, float2 f) { return __fmaf_rn(hi, f.x, __fmul_rn(lo, f.y)); }
+
 // QKV with RoPE (q and k tiles): the cos/sin rows of a chunk's 16 positions, fetched by all
 // 128 epilogue threads as 16-byte pieces (rope_load, issued a chunk ahead) and put into one of
 // two shared buffers (rope_store) before the barrier that precedes their use.
@@ -201,7 +206,7 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) {
         const float2 f = cs[jj * 64];
-        v[jj] = (row < 64) ? (v[jj] * f.x - partner[jj] * f.y) : (v[jj] * f.x + partner[jj] * f.y);
+        v[jj] = (row < 64) ? rope_lo(v[jj], partner[jj], f) : rope_hi(v[jj], partner[jj], f);
       }
     }
 #pragma unroll
@@ -260,25 +265,32 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
 // Cluster split-K reduction, run by the 128 epilogue threads of every CTA of the cluster after
 // the first cluster barrier: CTA `rank` takes chunks rank, rank + S, ..., adds the S partial
 // tiles of each (read from the cluster's shared memory) in split order -- the same sums as the
-// other schedules -- and runs the epilogue on them.
+// other schedules -- and runs the epilogue on them.  The epilogue operands of its first chunk
+// (`first`, and its RoPE factors in rope buffer 0) were fetched while the MMAs ran.  The CTA
+// arrives on the cluster barrier as soon as its last read of another CTA's shared memory is
+// done; the caller waits on it before the CTA exits.
 template <int EPI>
-__device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem& esm, uint32_t part_saddr, int row) {
+__device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem& esm, uint32_t part_saddr, int row,
+                                               const EpiPre& first) {
   Item it;
   get_item(a, blockIdx.x, it);
   const int S = a.cluster;
   const int rank = static_cast<int>(cluster_ctarank());
   const int nchunks = (it.rows + 15) >> 4;
   const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
+  if (rank >= nchunks) cluster_arrive();
   int k = 0;
   for (int c = rank; c < nchunks; c += S, ++k) {
-    if (rope) {
-      RopeRegs rr;
-      rope_load(a, it, c * 16, esm, rr);
-      rope_store(esm, k & 1, rr);
-      named_bar_sync(1, 128);
+    EpiPre cur = first;
+    if (k > 0) {
+      if (rope) {
+        RopeRegs rr;
+        rope_load(a, it, c * 16, esm, rr);
+        rope_store(esm, k & 1, rr);
+        named_bar_sync(1, 128);
+      }
+      epi_pre<EPI>(a, it, row, c * 16, esm, cur);
     }
-    EpiPre cur;
-    epi_pre<EPI>(a, it, row, c * 16, esm, cur);
     float v[16];
 #pragma unroll
     for (int hf = 0; hf < 2; ++hf) {
@@ -307,6 +319,7 @@ __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem&
         v[4 * q4 + 3] = t.w;
       }
     }
+    if (c + S >= nchunks) cluster_arrive();   // no more reads of the other CTAs' partial tiles
     epi_post<EPI>(a, it, row, c * 16, v, cur, esm, k & 1);
   }
 }
@@ -331,6 +344,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   int* s_vote = const_cast<int*>(s_abort) + 1;   // [4]
   int* s_last = s_vote + 4;
   EpiSmem esm;
+  EpiPre first_pre;   // cluster split-K: the epilogue operands of the first chunk this CTA reduces
   esm.xchg = reinterpret_cast<float*>(smem + C::STAGES * (C::A_BYTES + C::B_BYTES) + 256);
   esm.am_val = esm.xchg + C::XCHG_FLOATS;
   esm.am_idx = reinterpret_cast<int*>(esm.am_val + 128);
@@ -526,17 +540,20 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       get_item(a, i, it);
       const int acc = local % nbuf;
       const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
-      // the item's metadata, RoPE factors and first old residuals are fetched while its MMAs run
+      // the item's metadata, RoPE factors and first old residuals are fetched while its MMAs
+      // run (in a cluster, those of the first chunk this CTA reduces)
       stage_meta<EPI>(a, it, esm);
       const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
+      const int c_first = (a.cluster > 1) ? static_cast<int>(cluster_ctarank()) : 0;
       RopeRegs rr;
       if (rope) {
-        rope_load(a, it, 0, esm, rr);
+        rope_load(a, it, c_first * 16, esm, rr);
         rope_store(esm, 0, rr);
         named_bar_sync(1, 128);
       }
       EpiPre cur, nxt;
-      epi_pre<EPI>(a, it, row, 0, esm, cur);
+      epi_pre<EPI>(a, it, row, c_first * 16, esm, cur);
+      first_pre = cur;
       bool ok = mbar_wait(&tfull[acc], acc_ph, s_abort);
       ok = __all_sync(0xffffffffu, ok);
       if (lane == 0) s_vote[ew] = ok ? 1 : 0;
@@ -702,8 +719,9 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
 
   if (a.cluster > 1) {
     cluster_sync_all();   // every split's partial tile is in its CTA's shared memory
-    if (warp >= 2) cluster_reduce<EPI>(a, esm, smem_u32(smA), (warp & 3) * 32 + lane);
-    cluster_sync_all();   // no CTA leaves while the others still read its shared memory
+    if (warp >= 2) cluster_reduce<EPI>(a, esm, smem_u32(smA), (warp & 3) * 32 + lane, first_pre);
+    else cluster_arrive();
+    cluster_wait();       // no CTA leaves while the others still read its shared memory
   }
   tc_fence_before();
   __syncthreads();
@@ -837,13 +855,43 @@ int num_sms() {
   return n;
 }
 
+// Most clusters of s CTAs of the dense GEMM kernel (one CTA per SM) resident at once.
+static int max_resident_clusters(int s) {
+  static int cache[kMaxSplit + 1] = {};
+  if (cache[s] == 0) {
+    cudaFuncSetAttribute(gemm_tc_kernel<64, EPI_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<64>::SMEM_BYTES);
+    cudaFuncSetAttribute(gemm_tc_kernel<64, EPI_F32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(s * num_sms()));
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = Cfg<64>::SMEM_BYTES;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = static_cast<unsigned>(s);
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<64, EPI_F32>, &cfg) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = 1;
+    }
+    cache[s] = n;
+  }
+  return cache[s];
+}
+
 int dense_split_k(int N, int K) {
-  // about 64 CTAs per dense matrix, at least 4 k-chunks (32 KB of weights) per split
+  // Splits per weight tile: about one CTA per SM over the whole matrix, at least two k-chunks
+  // (16 KB of weights) per split, at most kMaxSplit, and no more than lets every tile's cluster
+  // of splits be resident at once.  A function of the shape (and the GPU) only.
   const int n_tiles = (N + 127) / 128;
   const int kc = K / 64;
-  int s = (64 + n_tiles - 1) / n_tiles;
-  if (s > kc / 4) s = kc / 4;
+  int s = num_sms() / n_tiles;
+  if (s > kc / 2) s = kc / 2;
   if (s > kMaxSplit) s = kMaxSplit;
+  while (s > 1 && n_tiles > max_resident_clusters(s)) --s;
   if (s < 1) s = 1;
   return s;
 }

@@ -52,7 +52,7 @@ constexpr int kAttnChunk = 64;            // split-KV chunk (keys), fixed by abs
 constexpr int kAttnSuper = 4;             // chunks per attention super-chunk (one partial each)
 constexpr int kAttnPartStride = 132;      // floats per (super-chunk, query) partial: O[128], M, L, pad
 constexpr int kMaxR = 8;                  // K_max + 1 <= 8 candidate rows per sequence
-constexpr int kMaxSplit = 6;              // split-K ways of a dense GEMM
+constexpr int kMaxSplit = 8;              // split-K ways of a dense GEMM (a portable cluster)
 
 // ------------------------------------------------------------------------- GEMM engine
 enum EpiKind : int {
