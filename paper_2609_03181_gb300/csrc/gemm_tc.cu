@@ -22,11 +22,14 @@
 
 namespace fm {
 
-template <int NMAX>
+// NMAX: most activation rows of a tile; ST: pipeline stages (8 for the long weight streams, 4
+// for the short per-split streams of the dense cluster schedule, which leaves room on the SM
+// for the CTAs of the next kernel to start early).
+template <int NMAX, int ST = (NMAX <= 64) ? 8 : 4>
 struct Cfg {
   static constexpr int A_BYTES = 128 * 128;            // 128 rows x 64 bf16
   static constexpr int B_BYTES = NMAX * 128;           // NMAX rows x 64 bf16
-  static constexpr int STAGES = (NMAX <= 64) ? 8 : 4;
+  static constexpr int STAGES = ST;
   static constexpr int TMEM_COLS = 2 * NMAX;           // two accumulator buffers
   static constexpr int XCHG_FLOATS = 128 * 17;
   static constexpr int AM_BYTES = 128 * 8;             // argmax partials of 8 row groups x 16 columns
@@ -35,6 +38,8 @@ struct Cfg {
   static constexpr int SMEM_BYTES =
       1024 + STAGES * (A_BYTES + B_BYTES) + 256 + XCHG_FLOATS * 4 + AM_BYTES + META_BYTES + ROPE_BYTES;
 };
+
+constexpr int kShallowStages = 4;   // stages of the dense cluster schedule
 
 struct Item {
   int e, n_tile, b_row, out_row, rows, split, box_log;
@@ -325,9 +330,9 @@ __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem&
 }
 
 // ------------------------------------------------------------------ kernel
-template <int NMAX, int EPI>
+template <int NMAX, int EPI, int ST>
 __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
-  using C = Cfg<NMAX>;
+  using C = Cfg<NMAX, ST>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t base_u32 = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
@@ -747,18 +752,18 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-template <int NMAX, int EPI>
+template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES>
 cudaError_t set_smem_attr() {
-  return cudaFuncSetAttribute(gemm_tc_kernel<NMAX, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              Cfg<NMAX>::SMEM_BYTES);
+  return cudaFuncSetAttribute(gemm_tc_kernel<NMAX, EPI, ST>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              Cfg<NMAX, ST>::SMEM_BYTES);
 }
 
-template <int NMAX, int EPI>
+template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES>
 cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(192);
-  cfg.dynamicSmemBytes = Cfg<NMAX>::SMEM_BYTES;
+  cfg.dynamicSmemBytes = Cfg<NMAX, ST>::SMEM_BYTES;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int n = 0;
@@ -776,7 +781,7 @@ cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   }
   cfg.attrs = attr;
   cfg.numAttrs = n;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI>, a);
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI, ST>, a);
 }
 }  // namespace
 
@@ -840,6 +845,10 @@ cudaError_t gemm_prepare() {
   FM_ATTR(EPI_SCATTER)
   FM_ATTR(EPI_ARGMAX)
 #undef FM_ATTR
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, kShallowStages>();
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_RESID, kShallowStages>();
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_QKV, kShallowStages>();
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_SWIGLU, kShallowStages>();
   num_sms();
   return e;
 }
@@ -855,16 +864,15 @@ int num_sms() {
   return n;
 }
 
-// Most clusters of s CTAs of the dense GEMM kernel (one CTA per SM) resident at once.
+// Most clusters of s CTAs of the dense cluster GEMM kernel (one CTA per SM) resident at once.
 static int max_resident_clusters(int s) {
   static int cache[kMaxSplit + 1] = {};
   if (cache[s] == 0) {
-    cudaFuncSetAttribute(gemm_tc_kernel<64, EPI_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<64>::SMEM_BYTES);
-    cudaFuncSetAttribute(gemm_tc_kernel<64, EPI_F32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+    set_smem_attr<64, EPI_F32, kShallowStages>();
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(s * num_sms()));
     cfg.blockDim = dim3(192);
-    cfg.dynamicSmemBytes = Cfg<64>::SMEM_BYTES;
+    cfg.dynamicSmemBytes = Cfg<64, kShallowStages>::SMEM_BYTES;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
     attr.val.clusterDim.x = static_cast<unsigned>(s);
@@ -873,7 +881,7 @@ static int max_resident_clusters(int s) {
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<64, EPI_F32>, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<64, EPI_F32, kShallowStages>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = 1;
     }
@@ -898,6 +906,20 @@ int dense_split_k(int N, int K) {
 
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   if (grid <= 0) return cudaSuccess;
+  if (a.cluster > 1 && nmax <= 64) {   // the dense cluster schedule: short per-split streams
+    switch (epi) {
+      case EPI_F32:
+        return launch_one<64, EPI_F32, kShallowStages>(a, grid, s, pdl);
+      case EPI_RESID:
+        return launch_one<64, EPI_RESID, kShallowStages>(a, grid, s, pdl);
+      case EPI_QKV:
+        return launch_one<64, EPI_QKV, kShallowStages>(a, grid, s, pdl);
+      case EPI_SWIGLU:
+        return launch_one<64, EPI_SWIGLU, kShallowStages>(a, grid, s, pdl);
+      default:
+        return cudaErrorInvalidValue;
+    }
+  }
 #define FM_CASE(E)                                                                      \
   case E:                                                                               \
     return nmax <= 64 ? launch_one<64, E>(a, grid, s, pdl) : launch_one<256, E>(a, grid, s, pdl);
