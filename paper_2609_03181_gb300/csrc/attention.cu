@@ -49,8 +49,11 @@ constexpr int kStageBytes = 2 * kTileBytes;      // K and V of a chunk: 32 KB
 constexpr int kQBytes = kMaxR * kHD * 2;         // the queries of one (sequence, head): 2 KB
 // Chunks in flight per CTA: two stages keep a CTA at 64 KB of shared memory and 128 registers
 // a thread, three CTAs per SM (192 KB in flight per SM, as three stages at two CTAs would) --
-// more CTAs, so that a small launch spreads over more of them.
+// more CTAs, so that a launch spreads over more of them.  Launches over one or two sequences
+// (at most a few items per SM) take four stages, one CTA per SM: a super-chunk's four chunks
+// are then all fetched before the wait for the previous kernel.
 constexpr int kAttnStages = 2;
+constexpr int kAttnStagesSmall = 4;
 constexpr int kConsumers = 128;                  // four warps, each owning 32 of the 128 dims
 constexpr int kAttnThreads = kConsumers + 32;    // plus the producer warp
 constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
@@ -204,7 +207,7 @@ __device__ __forceinline__ void merge_seq_head(const AttnArgs& a, int b, int h, 
 }
 
 template <int kStages>
-__global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 2) attn_kernel(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ uint8_t asmem_raw[];
   const uint32_t raw_u32 = smem_u32(asmem_raw);
   uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [S][K 16 KB | V 16 KB]
@@ -666,25 +669,35 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 2) attn_kerne
 }
 
 cudaError_t attention_prepare() {
-  return cudaFuncSetAttribute(attn_kernel<kAttnStages>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(attn_smem(kAttnStages, 2048)));
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<kAttnStages>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(attn_smem(kAttnStages, 2048)));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_kernel<kAttnStagesSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(attn_smem(kAttnStagesSmall, 2048)));
+  return e;
 }
 
-cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
-  // As many CTAs as fit at once (three per SM, at most one per item).  Pure scheduling: the
-  // arithmetic of every super-chunk and of the merge is the same for any grid.
-  AttnArgs a = a_in;
-  a.B = B;
-  const size_t smem = attn_smem(kAttnStages, B);
+template <int kStages>
+static cudaError_t attention_launch_s(const AttnArgs& a, int B, cudaStream_t s) {
+  const size_t smem = attn_smem(kStages, B);
   int per_sm = 0;
-  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_kernel<kAttnStages>, kAttnThreads, smem);
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_kernel<kStages>, kAttnThreads, smem);
   if (e != cudaSuccess) return e;
   if (per_sm < 1) per_sm = 1;
   const long long most = static_cast<long long>(B) * kH * ((a.n_chunks + kSuper - 1) / kSuper);
   long long grid = static_cast<long long>(per_sm) * num_sms();
   if (grid > most) grid = most;
   if (grid < 1) grid = 1;
-  return launch_pdl(attn_kernel<kAttnStages>, dim3(static_cast<unsigned>(grid)), dim3(kAttnThreads), smem, s, a);
+  return launch_pdl(attn_kernel<kStages>, dim3(static_cast<unsigned>(grid)), dim3(kAttnThreads), smem, s, a);
+}
+
+cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
+  // As many CTAs as fit at once (at most one per item).  Pure scheduling: the arithmetic of
+  // every super-chunk and of the merge is the same for any grid and stage count.
+  AttnArgs a = a_in;
+  a.B = B;
+  if (B <= 2) return attention_launch_s<kAttnStagesSmall>(a, B, s);
+  return attention_launch_s<kAttnStages>(a, B, s);
 }
 
 }  // namespace fm
