@@ -421,8 +421,8 @@ def run_fastmtp(args):
     peak, peak_kind = measured_peaks()
     L = shape.n_layers
     steps = args.steps
-    touched = counted["experts_touched"] / max(1, counted["launches"]["permute"])     # per layer, incl. shared
-    rows = counted["expert_rows"] / max(1, counted["launches"]["permute"])
+    touched = counted["experts_touched"] / max(1, counted["launches"]["router"])     # per layer, incl. shared
+    rows = counted["expert_rows"] / max(1, counted["launches"]["router"])
     d, I = shape.hidden, shape.expert_inter
     cls_bytes = {
         "expert_gate_up": touched * 2 * I * d * 2 + rows * d * 2 + rows * I * 2,
@@ -557,7 +557,7 @@ def run_sweep(args):
                     lens = ctx + 1 + torch.cumsum(h, 0) - h          # committed length seen by each verify
                     ctx_mean = float(lens[args.warmup:].mean())
                     tok = float(h[args.warmup:].sum())
-                    touched = counted["experts_touched"] / max(1, counted["launches"]["permute"])
+                    touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
                     vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
                     load = cnt / cnt.mean(-1, keepdim=True)
                     out = {"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K,

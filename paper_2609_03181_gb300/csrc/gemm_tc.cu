@@ -43,21 +43,34 @@ constexpr int kShallowStages = 4;   // stages of the dense cluster schedule
 
 struct Item {
   int e, n_tile, b_row, out_row, rows, split, box_log;
+  int grow;   // grouped: first row of the item within its expert
 };
 
-__device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it) {
-  if (a.items != nullptr) {
-    const int4 v = a.items[i];
-    it.e = v.x & 0xFFFF;
-    it.n_tile = v.x >> 16;
-    it.b_row = v.y;
-    it.out_row = v.z;
-    it.rows = v.w;
+// Per-expert tables of a grouped launch in shared memory, built by every CTA from the counts:
+// grp[e] first item of expert e (grp[66] = items), grp[67 + e] its rows.
+constexpr int kGrpItem = 0, kGrpCnt = kE + kShared + 1;
+
+__device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it, const int* grp) {
+  if (a.grp_cnt != nullptr) {
+    int lo = 0, hi = kE + kShared - 1;   // the last expert whose first item is <= i has items
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (grp[kGrpItem + mid] <= i) lo = mid;
+      else hi = mid - 1;
+    }
+    const int j = i - grp[kGrpItem + lo], m = j / a.grp_tiles;
+    it.e = lo;
+    it.n_tile = j - m * a.grp_tiles;
+    it.grow = kExpertTileRows * m;
+    it.rows = min(kExpertTileRows, grp[kGrpCnt + lo] - it.grow);
+    it.out_row = lo * a.map_stride + it.grow;
+    it.b_row = (a.grp_b_direct && lo >= a.n_routed) ? it.grow : it.out_row;
     it.split = 0;
     int bl = 0;
     while ((16 << bl) < it.rows) ++bl;
     it.box_log = bl;
   } else {
+    it.grow = 0;
     const int mt = i % a.m_tiles;
     const int t = i / a.m_tiles;
     const int ns = a.seq_split ? 1 : a.split_k;   // in-CTA splits: one item covers every split
@@ -153,8 +166,14 @@ __device__ __forceinline__ void stage_meta(const GemmArgs& a, const Item& it, co
         sm.s_pos[r] = a.pos[it.out_row + r];
         sm.s_off[r] = a.kv_rowoff[it.out_row + r];
       } else {
-        sm.s_pos[r] = a.sorted_tok[it.out_row + r];
-        sm.s_aux[r] = a.sorted_slot[it.out_row + r];
+        if (it.e < a.n_routed) {
+          const int v = a.rowmap[static_cast<size_t>(it.e) * a.map_stride + it.grow + r];
+          sm.s_pos[r] = v >> 3;
+          sm.s_aux[r] = v & 7;
+        } else {   // shared expert j: every token in order, slot top_k + j
+          sm.s_pos[r] = it.grow + r;
+          sm.s_aux[r] = kTopK + it.e - a.n_routed;
+        }
       }
     }
     named_bar_sync(1, 128);
@@ -278,7 +297,7 @@ template <int EPI>
 __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem& esm, uint32_t part_saddr, int row,
                                                const EpiPre& first) {
   Item it;
-  get_item(a, blockIdx.x, it);
+  get_item(a, blockIdx.x, it, nullptr);
   const int S = a.cluster;
   const int rank = static_cast<int>(cluster_ctarank());
   const int nchunks = (it.rows + 15) >> 4;
@@ -396,9 +415,53 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   // Dense launches know their items from the arguments: the producer streams its first weight
   // tiles (never written by earlier kernels) before it waits for the previous kernel; every
   // other thread waits before its first global access.
-  const bool dense = (a.items == nullptr);
+  const bool dense = (a.grp_cnt == nullptr);
   if (!(dense && warp == 0 && lane == 0)) pdl_wait();
-  const int n_items = dense ? a.n_items : *a.n_items_dev;
+  // grouped launches: the per-expert tables (in the RoPE buffer, which only QKV uses)
+  int* grp = reinterpret_cast<int*>(esm.rope);
+  int n_items = a.n_items;
+  if (!dense) {
+    if (threadIdx.x < 32) {   // three experts per lane, prefix sums by warp scan
+      int c[3], ni[3], sc = 0, si = 0, touched = 0;
+#pragma unroll
+      for (int k = 0; k < 3; ++k) {
+        const int e = 3 * static_cast<int>(threadIdx.x) + k;
+        c[k] = (e < kE + kShared) ? ((e < a.n_routed) ? a.grp_cnt[e] : a.grp_T) : 0;
+        ni[k] = (c[k] + kExpertTileRows - 1) / kExpertTileRows * a.grp_tiles;
+        sc += c[k];
+        si += ni[k];
+        touched += (c[k] > 0) ? 1 : 0;
+      }
+      int ic = sc, ii = si;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int yc = __shfl_up_sync(0xffffffffu, ic, o), yi = __shfl_up_sync(0xffffffffu, ii, o);
+        if (static_cast<int>(threadIdx.x) >= o) {
+          ic += yc;
+          ii += yi;
+        }
+      }
+      int ri = ii - si;
+#pragma unroll
+      for (int k = 0; k < 3; ++k) {
+        const int e = 3 * static_cast<int>(threadIdx.x) + k;
+        if (e < kE + kShared) {
+          grp[kGrpCnt + e] = c[k];
+          grp[kGrpItem + e] = ri;
+        }
+        ri += ni[k];
+      }
+      if (threadIdx.x == 31) grp[kGrpItem + kE + kShared] = ii;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) touched += __shfl_xor_sync(0xffffffffu, touched, o);
+      if (a.expert_ctr != nullptr && blockIdx.x == 0 && threadIdx.x == 31) {
+        atomicAdd(&a.expert_ctr[0], static_cast<unsigned long long>(touched));
+        atomicAdd(&a.expert_ctr[1], static_cast<unsigned long long>(ic));
+      }
+    }
+    __syncthreads();
+    n_items = grp[kGrpItem + kE + kShared];
+  }
   const int kc_total = a.K / 64;
 
   if (warp == 0) {
@@ -411,8 +474,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       bool waited = !dense;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x) {
         Item it;
-        get_item(a, i, it);
-        const int src = (a.items != nullptr && it.e >= a.n_routed) ? 1 : 0;
+        get_item(a, i, it, grp);
+        const int src = (!dense && it.e >= a.n_routed) ? 1 : 0;
         const int el = it.e - (src ? a.n_routed : 0);
         const CUtensorMap* amap = &a.a_map[src];
         const CUtensorMap* bmap = &a.b_map[src][it.box_log];
@@ -485,7 +548,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       bool failed = false;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x, ++local) {
         Item it;
-        get_item(a, i, it);
+        get_item(a, i, it, grp);
         const int acc = local % nbuf;
         const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
         if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, s_abort)) {
@@ -542,7 +605,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     int local = 0;
     for (int i = blockIdx.x; i < n_items; i += gridDim.x, ++local) {
       Item it;
-      get_item(a, i, it);
+      get_item(a, i, it, grp);
       const int acc = local % nbuf;
       const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
       // the item's metadata, RoPE factors and first old residuals are fetched while its MMAs

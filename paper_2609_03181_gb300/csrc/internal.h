@@ -66,7 +66,7 @@ enum EpiKind : int {
 
 // One work item: weight tile x activation rows.  x = expert | n_tile << 16, y = TMA row of
 // the activation source, z = output row (row index of the epilogue), w = number of rows.
-// Dense launches generate items implicitly; grouped launches read them from a device list.
+// Dense launches generate items from the shape; grouped launches from the per-expert row counts.
 struct GemmArgs {
   CUtensorMap a_map[2];        // weights: [0] main / routed experts, [1] shared experts
   CUtensorMap b_map[2][5];     // activations: [source][box height 16,32,64,128,256]
@@ -81,8 +81,16 @@ struct GemmArgs {
                                // its own TMEM accumulator (64-row boxes), no partials in memory
   int cluster;                 // dense, split_k > 1, one item per CTA: the split_k CTAs of a tile
                                // are a cluster and add their partials through shared memory
-  const int4* items;           // grouped: device item list
-  const int* n_items_dev;      //          and its length
+  // Grouped launches (grp_cnt != NULL): the work is every (expert, 64-row tile, weight tile),
+  // experts in order, routed experts e < n_routed with grp_cnt[e] rows, then the shared ones
+  // with grp_T rows each; expert e's rows are rows e * map_stride + 0.. of its input and output.
+  const int* grp_cnt;          // [n_routed] rows of each routed expert
+  int grp_T;                   // rows of each shared expert (the step's tokens)
+  int grp_tiles;               // weight tiles per expert
+  int grp_b_direct;            // shared experts read activation rows 0..T-1 directly
+  const int* rowmap;           // SCATTER: [n_routed][map_stride] (token << 3 | rank) of each row
+  int map_stride;
+  unsigned long long* expert_ctr;   // if set, CTA 0 adds (experts with rows, rows) of the launch
   int n_items;                 // dense: number of items
   int M;                       // dense: activation rows
   int m_tiles, box_log;        // dense: row tiles of 16 << box_log rows
@@ -93,7 +101,7 @@ struct GemmArgs {
   bf16* q_out; bf16* kv_base; const long long* kv_rowoff;    // QKV (q stored bf16)
   long long head_stride, v_off; const int* pos; const float2* rope; int max_pos;
   bf16* act; int ld_act;                                      // SWIGLU
-  float* y; const int* sorted_tok; const int* sorted_slot;    // SCATTER
+  float* y;                                                   // SCATTER: [T][8 slots][d]
   // ARGMAX: am_key[row] = max over tiles of (ordered logit << 32 | ~token) (atomicMax; zero =
   // empty).  fin_B > 0: the last CTA (ticket am_done) decodes the tokens of fin_B x fin_R rows,
   // computes the greedy accept lengths and clears the keys.
@@ -164,17 +172,18 @@ cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s);
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
-                              int* err, cudaStream_t s);
+                              int* err, int* zero, int n_zero, cudaStream_t s);
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
 // Router (+ expert grouping by the last CTA) and the permute row gather.
 struct RouteArgs {
   const float* h; const bf16* gain; float eps; const bf16* wr; const float* bias;
   bf16* xn; int* idx; float* gate; int* err; int T;
-  int* dst_row; int* sorted_tok; int* sorted_slot; int4* items_gu; int4* items_dn; int* n_items; int* counts;
-  unsigned long long* expert_ctr; int* ticket;
+  int* counts;     // [64] rows routed to each expert so far (zero before the layer's router)
+  int* rowmap;     // [64][map_stride] per expert: (token << 3 | rank) of each of its rows
+  bf16* x_sorted;  // [64][map_stride][d] per expert: its input rows (the rounded xn rows)
+  int map_stride;  // >= T
 };
 cudaError_t router_launch(const RouteArgs& a, cudaStream_t s);
-cudaError_t permute_launch(const int* dst_row, int T, const bf16* xn, bf16* x_sorted, cudaStream_t s);
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
                            bf16* out, cudaStream_t s);
 cudaError_t commit_launch(int B, int R, int stage_R, int Bmax, const int* slots, const int* m_ws, const int* vtok_ws,

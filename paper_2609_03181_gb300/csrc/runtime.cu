@@ -67,8 +67,8 @@ struct spec_ctx {
   CUtensorMap lm{}, eh{}, mqkv{}, mwo{}, mgu{}, mdn{};
   ActMaps a_xn{}, a_attn{}, a_xs{}, a_act{}, a_b{}, a_dcat{}, a_dxn{}, a_dattn{}, a_dact{}, a_u{};
 
-  int Bmax = 0, Rmax = 0, Tmax = 0, n_chunks = 0, lm_tiles = 0, dstage_rows = 0;
-  size_t max_items = 0, sk_floats = 0;
+  int Bmax = 0, Rmax = 0, Tmax = 0, Tcap = 0, n_chunks = 0, lm_tiles = 0, dstage_rows = 0;
+  size_t sk_floats = 0;
 
   // workspace (one allocation)
   void* ws = nullptr;
@@ -80,18 +80,12 @@ struct spec_ctx {
   float* attn_part = nullptr;
   int* attn_tickets = nullptr;
   int* commit_tickets = nullptr;
-  int* route_ticket = nullptr;
-  int* dst_row = nullptr;       // [Tmax * top_k] expert-sorted row of each (token, slot) pair
+  int* rowmap = nullptr;        // [n_experts][Tmax] (token << 3 | rank) of each routed expert row
   bf16* attn_out = nullptr;
   int* route_idx = nullptr;
   float* route_gate = nullptr;
   int* counts = nullptr;
   bf16* x_sorted = nullptr;
-  int* sorted_tok = nullptr;
-  int* sorted_slot = nullptr;
-  int4* items_gu = nullptr;
-  int4* items_dn = nullptr;
-  int* n_items = nullptr;
   bf16* act = nullptr;
   float* y = nullptr;
   bf16* b_ws = nullptr;
@@ -412,7 +406,6 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ctx->n_chunks = (c.max_pages_per_seq * c.page_size + Rmax + kAttnChunk - 1) / kAttnChunk;
   ctx->lm_tiles = (c.vocab + 127) / 128;
   ctx->dstage_rows = c.K_max > 1 ? c.K_max - 1 : 1;
-  ctx->max_items = static_cast<size_t>(kE + kShared + (Tmax * kSlots) / kExpertTileRows + 4) * (kI / 64);
   {
     // split-K partials: per split, a tile's rows are padded to the row box (< 2 * rows + 16)
     const int shapes[][2] = {{3 * kD, kD}, {kD, kD}, {kD, 2 * kD}, {kD, kId}, {2 * kId, kD}};
@@ -439,19 +432,14 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
                            Rmax * kAttnPartStride);
   add(&ctx->attn_tickets, sizeof(int) * Bmax * kH);
   add(&ctx->commit_tickets, sizeof(int) * Bmax);
-  add(&ctx->route_ticket, sizeof(int));
-  add(&ctx->dst_row, sizeof(int) * Tmax * kTopK);
+  ctx->Tcap = (Tmax + kExpertTileRows - 1) / kExpertTileRows * kExpertTileRows;
+  add(&ctx->rowmap, sizeof(int) * kE * ctx->Tcap);
   add(&ctx->attn_out, sizeof(bf16) * Tmax * d);
   add(&ctx->route_idx, sizeof(int) * L * Tmax * kTopK);
   add(&ctx->route_gate, sizeof(float) * L * Tmax * kTopK);
   add(&ctx->counts, sizeof(int) * L * kE);
-  add(&ctx->x_sorted, sizeof(bf16) * Tmax * kTopK * d);
-  add(&ctx->sorted_tok, sizeof(int) * Tmax * kSlots);
-  add(&ctx->sorted_slot, sizeof(int) * Tmax * kSlots);
-  add(&ctx->items_gu, sizeof(int4) * ctx->max_items);
-  add(&ctx->items_dn, sizeof(int4) * ctx->max_items);
-  add(&ctx->n_items, sizeof(int) * 2);
-  add(&ctx->act, sizeof(bf16) * Tmax * kSlots * kI);
+  add(&ctx->x_sorted, sizeof(bf16) * kE * ctx->Tcap * d);
+  add(&ctx->act, sizeof(bf16) * (kE + kShared) * ctx->Tcap * kI);
   add(&ctx->y, sizeof(float) * Tmax * kSlots * d);
   add(&ctx->b_ws, sizeof(bf16) * Tmax * d);
   add(&ctx->am_key, sizeof(unsigned long long) * Tmax);
@@ -538,8 +526,8 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ok = ok && encode_map_2d(&ctx->mdn, w->mtp_w_down, kId, kD, 128, &e);
   ok = ok && encode_act_maps(ctx->a_xn.m, ctx->xn, kD, Tmax, &e);
   ok = ok && encode_act_maps(ctx->a_attn.m, ctx->attn_out, kD, Tmax, &e);
-  ok = ok && encode_act_maps(ctx->a_xs.m, ctx->x_sorted, kD, static_cast<uint64_t>(Tmax) * kTopK, &e);
-  ok = ok && encode_act_maps(ctx->a_act.m, ctx->act, kI, static_cast<uint64_t>(Tmax) * kSlots, &e);
+  ok = ok && encode_act_maps(ctx->a_xs.m, ctx->x_sorted, kD, static_cast<uint64_t>(kE) * ctx->Tcap, &e);
+  ok = ok && encode_act_maps(ctx->a_act.m, ctx->act, kI, static_cast<uint64_t>(kE + kShared) * ctx->Tcap, &e);
   ok = ok && encode_act_maps(ctx->a_b.m, ctx->b_ws, kD, Tmax, &e);
   ok = ok && encode_act_maps(ctx->a_dcat.m, ctx->dcat, 2 * kD, Tmax, &e);
   ok = ok && encode_act_maps(ctx->a_dxn.m, ctx->dxn, kD, Tmax, &e);
@@ -663,7 +651,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   CK(cudaMemcpyAsync(ctx->cand_ws, cand, sizeof(int) * T, cudaMemcpyDeviceToDevice, s));
   LAUNCH(SPEC_K_EMBED, 1, embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
                        c.vocab, static_cast<const bf16*>(ctx->layers[0].attn_norm), eps, ctx->h, ctx->xn, ctx->pos,
-                       ctx->kv_rowoff, ctx->Rmax, ctx->Bmax, ctx->d_err, s));
+                       ctx->kv_rowoff, ctx->Rmax, ctx->Bmax, ctx->d_err, ctx->counts, L * kE, s));
   const int nmax_grouped = kExpertTileRows;
   for (int l = 0; l < L; ++l) {
     const spec_layer_weights& W = ctx->layers[l];
@@ -732,18 +720,12 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       ra.gate = rgate;
       ra.err = ctx->d_err;
       ra.T = T;
-      ra.dst_row = ctx->dst_row;
-      ra.sorted_tok = ctx->sorted_tok;
-      ra.sorted_slot = ctx->sorted_slot;
-      ra.items_gu = ctx->items_gu;
-      ra.items_dn = ctx->items_dn;
-      ra.n_items = ctx->n_items;
       ra.counts = ctx->counts + l * kE;
-      ra.expert_ctr = ctx->d_expert_ctr;
-      ra.ticket = ctx->route_ticket;
+      ra.rowmap = ctx->rowmap;
+      ra.x_sorted = ctx->x_sorted;
+      ra.map_stride = ctx->Tcap;
       LAUNCH(SPEC_K_ROUTER, 1, router_launch(ra, s));
     }
-    LAUNCH(SPEC_K_PERMUTE, 1, permute_launch(ctx->dst_row, T, ctx->xn, ctx->x_sorted, s));
     // routed + shared experts: gate/up + SwiGLU
     {
       GemmArgs g = base_args(ctx);
@@ -759,8 +741,12 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.paired = 1;
       g.half_rows = kI;
       g.n_routed = kE;
-      g.items = ctx->items_gu;
-      g.n_items_dev = ctx->n_items;
+      g.grp_cnt = ctx->counts + l * kE;
+      g.grp_T = T;
+      g.grp_tiles = 2 * kI / 128;
+      g.grp_b_direct = 1;   // shared experts read the normalised rows directly
+      g.map_stride = ctx->Tcap;
+      g.expert_ctr = ctx->d_expert_ctr;
       g.act = ctx->act;
       g.ld_act = kI;
       LAUNCH(SPEC_K_EXPERT_GU, 1, gemm_launch(EPI_SWIGLU, nmax_grouped, g, num_sms(), s));
@@ -778,11 +764,12 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.K = kI;
       g.a3d = 1;
       g.n_routed = kE;
-      g.items = ctx->items_dn;
-      g.n_items_dev = ctx->n_items + 1;
+      g.grp_cnt = ctx->counts + l * kE;
+      g.grp_T = T;
+      g.grp_tiles = kD / 128;
+      g.rowmap = ctx->rowmap;
+      g.map_stride = ctx->Tcap;
       g.y = ctx->y;
-      g.sorted_tok = ctx->sorted_tok;
-      g.sorted_slot = ctx->sorted_slot;
       LAUNCH(SPEC_K_EXPERT_DN, 1, gemm_launch(EPI_SCATTER, nmax_grouped, g, num_sms(), s));
     }
     const bf16* next_gain =

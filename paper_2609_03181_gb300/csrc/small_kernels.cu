@@ -1,5 +1,5 @@
 // Latency-bound kernels of the FastMTP step: embedding + RMSNorm, RMSNorm, router
-// (norm, logits, softmax, top-6), token permute/scatter by expert, MoE combine (+ the next
+// (norm, logits, softmax, top-6, per-expert row lists and input rows), MoE combine (+ the next
 // RMSNorm), the KV commit, and the glue of the draft chain.  Every reduction runs in a fixed
 // order, so a row's result never depends on the other rows of the batch.
 #include <math.h>
@@ -48,9 +48,12 @@ __device__ __forceinline__ void norm_row_store(const float (&x)[10], const bf16*
 __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R, const int* slots, const int* pending,
                                                          const int* seq_len, const bf16* embed, int vocab,
                                                          const bf16* gain, float eps, float* h, bf16* xn, int* pos,
-                                                         long long* kv_rowoff, int stage_R, int n_slots, int* err) {
+                                                         long long* kv_rowoff, int stage_R, int n_slots, int* err,
+                                                         int* zero, int n_zero) {
   pdl_trigger();
   pdl_wait();
+  if (blockIdx.x == 0)   // the step's per-expert row counters start from zero
+    for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
   __shared__ float red[4];
   const int row = blockIdx.x, b = row / R, r = row % R;
   const int slot = slots[b];
@@ -80,9 +83,9 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
-                              int* err, cudaStream_t s) {
+                              int* err, int* zero, int n_zero, cudaStream_t s) {
   return launch_pdl(embed_norm_kernel, dim3(B * R), dim3(128), 0, s, cand, R, slots, pending, seq_len, embed, vocab, gain,
-                    eps, h, xn, pos, kv_rowoff, stage_R, n_slots, err);
+                    eps, h, xn, pos, kv_rowoff, stage_R, n_slots, err, zero, n_zero);
 }
 
 // ---------------------------------------------------------------- RMSNorm
@@ -102,207 +105,116 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
   return launch_pdl(rmsnorm_kernel, dim3(rows), dim3(128), 0, s, x, gain, eps, out);
 }
 
-// ---------------------------------------------------------------- router + expert grouping
-// RR rows per CTA: 1 for small batches (latency), 4 above 128 rows (the 64 x 1280 router
-// matrix is then read once per four rows).  Per row:
-// RMSNorm of the residual row -> xn (bf16, also the experts' input); logits of the 64 experts
-// from the bf16 row, fp32 softmax, top-6 by probability (lower id on ties).  Every row's
-// arithmetic is the same whatever rows share its CTA.
-//
-// Then the CTA that finishes last (atomic ticket, no wait) groups the (token, slot) pairs of
-// the layer by expert: routed rows of expert e take act rows offs[e] .. offs[e+1]-1 in token
-// order (rank from a per-expert token bitmap and its prefix popcounts); the two shared experts
-// follow with all T tokens each.  It writes the destination row of every pair, the sorted
-// token/slot lists, the GEMM work lists (row tiles of at most 64 rows, so every grouped launch
-// runs the deep 8-stage weight pipeline) and the expert counters.
-constexpr int kRouterRows = 4;
+// ---------------------------------------------------------------- router
+// kRouteCtaRows token rows per CTA, in the first rows of a 16-row MMA tile (the router matrix
+// is read from L2 once per CTA; more CTAs spread the copies of the selected rows).  Per row: RMSNorm of the residual row -> xn (bf16, also the experts' input); the 64 logits of the
+// rounded row on bf16 tensor cores (mma.sync m16n8k16, fp32 accumulation; warp w computes
+// experts 8w..8w+7 of all 16 rows, each lane streaming 16-byte pieces of its expert's row);
+// fp32 softmax; top-6 by probability (lower id on ties).  Each selected (token, rank, expert)
+// takes the next row of its expert with one atomic add on the layer's per-expert counter,
+// records (token << 3 | rank) in that row of the expert's list and copies the rounded row to
+// that row of the expert's input region (map_stride rows per expert), so neither a grouping
+// pass nor a row gather follows.  A row's arithmetic is the same whatever rows share its CTA,
+// and a (token, expert) row's result does not depend on its position among the expert's rows.
+constexpr int kRouteRows = 16;      // rows of the MMA tile
+constexpr int kRouteCtaRows = 4;    // token rows of a CTA
+constexpr int kRouteStride = kD + 32;   // bf16 per staged row: rows 64 bytes apart in the banks
 constexpr int kMaxT = 2048;
-constexpr int kMaxW = kMaxT / 32;
 
-__device__ __forceinline__ void group_by_expert(const RouteArgs& a, int* gsm) {
-  const int T = a.T, W = (T + 31) / 32, T6 = T * kTopK, tid = threadIdx.x;
-  int* s_idx = gsm;                       // [T*6]
-  unsigned* bits = reinterpret_cast<unsigned*>(s_idx + T6);   // [64][W]
-  int* pre = reinterpret_cast<int*>(bits + kE * W);          // [64][W]
-  int* cnt = pre + kE * W;                // [66]
-  int* offs = cnt + kE + kShared;         // [67]
-  int* ibase = offs + kE + kShared + 1;   // [67] gate_up item offsets
-  int* dbase = ibase + kE + kShared + 1;  // [67]
-  for (int p = tid; p < T6; p += blockDim.x) s_idx[p] = __ldcg(a.idx + p);
-  for (int p = tid; p < kE * W; p += blockDim.x) bits[p] = 0u;
-  __syncthreads();
-  for (int p = tid; p < T6; p += blockDim.x) {
-    const int t = p / kTopK, e = s_idx[p];
-    atomicOr(&bits[e * W + (t >> 5)], 1u << (t & 31));
-  }
-  __syncthreads();
-  if (tid < kE) {
-    int run = 0;
-    for (int w = 0; w < W; ++w) {
-      pre[tid * W + w] = run;
-      run += __popc(bits[tid * W + w]);
-    }
-    cnt[tid] = run;
-  } else if (tid < kE + kShared) {
-    cnt[tid] = T;
-  }
-  __syncthreads();
-  if (tid < 32) {
-    // exclusive prefix sums over the 66 experts (three per lane, lanes in order)
-    int c3[3], m3[3];
-    int sc = 0, sm = 0;
-#pragma unroll
-    for (int k = 0; k < 3; ++k) {
-      const int e = tid * 3 + k;
-      c3[k] = (e < kE + kShared) ? cnt[e] : 0;
-      m3[k] = (c3[k] + kExpertTileRows - 1) / kExpertTileRows;
-      sc += c3[k];
-      sm += m3[k];
-    }
-    int ic = sc, im = sm;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int xc = __shfl_up_sync(0xffffffffu, ic, o), xm = __shfl_up_sync(0xffffffffu, im, o);
-      if (tid >= o) {
-        ic += xc;
-        im += xm;
-      }
-    }
-    int rc = ic - sc, rm = im - sm;   // exclusive
-#pragma unroll
-    for (int k = 0; k < 3; ++k) {
-      const int e = tid * 3 + k;
-      if (e <= kE + kShared) {
-        offs[e] = rc;
-        ibase[e] = rm * (kI / 64);
-        dbase[e] = rm * (kD / 128);
-      }
-      rc += c3[k];
-      rm += m3[k];
-    }
-    if (tid == 31) {
-      a.n_items[0] = im * (kI / 64);
-      a.n_items[1] = im * (kD / 128);
-    }
-  }
-  __syncthreads();
-  for (int p = tid; p < T6; p += blockDim.x) {
-    const int t = p / kTopK, sl = p % kTopK, e = s_idx[p];
-    const int dst = offs[e] + pre[e * W + (t >> 5)] + __popc(bits[e * W + (t >> 5)] & ((1u << (t & 31)) - 1u));
-    a.dst_row[p] = dst;
-    a.sorted_tok[dst] = t;
-    a.sorted_slot[dst] = sl;
-  }
-  for (int p = tid; p < kShared * T; p += blockDim.x) {
-    const int j = p / T, t = p % T;
-    a.sorted_tok[offs[kE + j] + t] = t;
-    a.sorted_slot[offs[kE + j] + t] = kTopK + j;
-  }
-  if (tid < kE + kShared) {
-    const int e = tid, n = cnt[e];
-    if (e < kE) a.counts[e] = n;
-    if (n > 0) {
-      atomicAdd(&a.expert_ctr[0], 1ull);
-      atomicAdd(&a.expert_ctr[1], static_cast<unsigned long long>(n));
-    }
-    const int mt = (n + kExpertTileRows - 1) / kExpertTileRows;
-    for (int m = 0; m < mt; ++m) {
-      const int rows = min(kExpertTileRows, n - kExpertTileRows * m);
-      const int out_row = offs[e] + kExpertTileRows * m;
-      const int b_row_gu = (e < kE) ? out_row : kExpertTileRows * m;   // shared experts read xn rows directly
-      for (int nt = 0; nt < kI / 64; ++nt)
-        a.items_gu[ibase[e] + m * (kI / 64) + nt] = make_int4(e | (nt << 16), b_row_gu, out_row, rows);
-      for (int nt = 0; nt < kD / 128; ++nt)
-        a.items_dn[dbase[e] + m * (kD / 128) + nt] = make_int4(e | (nt << 16), out_row, out_row, rows);
-    }
-  }
-}
-
-template <int RR>
 __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ RouteArgs a) {
   pdl_trigger();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // the first four experts of this warp's eight: router weights are never written by earlier
-  // kernels, so their loads go out before the wait for the previous kernel
-  uint4 raw[4][5];
-  auto load_group = [&](int e0) {
+  __shared__ __align__(16) bf16 xs[kRouteRows * kRouteStride];   // the rounded rows
+  __shared__ float lg[kRouteRows][kE];                           // logits, then probabilities
+  __shared__ int dst[kRouteRows][kTopK];                         // input row of each selection
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
+  // The router matrix is never written by earlier kernels: most of this lane's share of its
+  // expert's row (expert 8 warp + g, columns 32 c + 8 t4 .. + 7) is loaded before the wait, the
+  // rest after the norm.
+  constexpr int kSteps = kD / 32, kEarly = 32;
+  const uint4* wrow = reinterpret_cast<const uint4*>(a.wr + static_cast<size_t>(warp * 8 + g) * kD) + t4;
+  uint4 wq[kSteps];
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
-#pragma unroll
-      for (int c = 0; c < 5; ++c)
-        raw[q][c] = *reinterpret_cast<const uint4*>(a.wr + static_cast<size_t>(e0 + q) * kD + c * 256 + lane * 8);
-  };
-  load_group(warp * 8);
+  for (int c = 0; c < kEarly; ++c) wq[c] = wrow[4 * c];
   pdl_wait();
-  constexpr int NT = 256, EPT = kD / NT;
-  __shared__ float red[NT / 32][RR];
-  __shared__ __align__(16) float xs[RR][kD];
-  __shared__ float lg[RR][kE];
-  __shared__ float sp[RR][kE];
-  __shared__ int s_last;
-  extern __shared__ int gsm[];
-  const int t0 = blockIdx.x * RR;
-  const int nr = min(RR, a.T - t0);
+  const int t0 = blockIdx.x * kRouteCtaRows;
+  const int nr = min(kRouteCtaRows, a.T - t0);
+  // RMSNorm: warp w takes rows w and w + 8; a lane sums its 40 squares of a row in order, then
+  // a warp tree
   {
-    float v[RR][EPT];
-    float ss[RR];
+    uint2 gq[kD / 128];   // gain (bf16), lane's columns 4 (lane + 32 k) .. + 3
 #pragma unroll
-    for (int r = 0; r < RR; ++r) {
+    for (int k = 0; k < kD / 128; ++k) gq[k] = *reinterpret_cast<const uint2*>(a.gain + 4 * (lane + 32 * k));
 #pragma unroll
-      for (int k = 0; k < EPT; ++k) v[r][k] = (r < nr) ? a.h[static_cast<size_t>(t0 + r) * kD + threadIdx.x + NT * k] : 0.f;
-      ss[r] = 0.f;
+    for (int h2 = 0; h2 < 2; ++h2) {
+      const int r = warp + 8 * h2;
+      bf16* xr = xs + r * kRouteStride;
+      const float4* hr = reinterpret_cast<const float4*>(a.h + static_cast<size_t>(t0 + min(r, nr - 1)) * kD);
+      float4 v[kD / 128];
 #pragma unroll
-      for (int k = 0; k < EPT; ++k) ss[r] += v[r][k] * v[r][k];
-      ss[r] = warp_sum(ss[r]);
-    }
-    if (lane == 0)
+      for (int k = 0; k < kD / 128; ++k) v[k] = hr[lane + 32 * k];
+      float ss = 0.f;
 #pragma unroll
-      for (int r = 0; r < RR; ++r) red[warp][r] = ss[r];
-    __syncthreads();
-#pragma unroll
-    for (int r = 0; r < RR; ++r) {
-      if (r >= nr) break;
-      float tot = red[0][r];
-#pragma unroll
-      for (int w = 1; w < NT / 32; ++w) tot += red[w][r];
-      const float inv = rsqrtf(tot / kD + a.eps);
+      for (int k = 0; k < kD / 128; ++k) ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
+      ss = warp_sum(ss);
+      const float inv = rsqrtf(ss / kD + a.eps);
       bf16* xo = a.xn + static_cast<size_t>(t0 + r) * kD;
 #pragma unroll
-      for (int k = 0; k < EPT; ++k) {
-        const int i = threadIdx.x + NT * k;
-        const bf16 rb = __float2bfloat16(v[r][k] * inv * __bfloat162float(a.gain[i]));
-        xo[i] = rb;
-        xs[r][i] = __bfloat162float(rb);   // the rounded row, as the experts see it
+      for (int k = 0; k < kD / 128; ++k) {
+        const int i = 4 * (lane + 32 * k);
+        const __nv_bfloat162 g01 = *reinterpret_cast<const __nv_bfloat162*>(&gq[k].x);
+        const __nv_bfloat162 g23 = *reinterpret_cast<const __nv_bfloat162*>(&gq[k].y);
+        __align__(8) bf16 o4[4];
+        o4[0] = __float2bfloat16(v[k].x * inv * __low2float(g01));
+        o4[1] = __float2bfloat16(v[k].y * inv * __high2float(g01));
+        o4[2] = __float2bfloat16(v[k].z * inv * __low2float(g23));
+        o4[3] = __float2bfloat16(v[k].w * inv * __high2float(g23));
+        if (r < nr) *reinterpret_cast<uint2*>(xo + i) = *reinterpret_cast<const uint2*>(o4);
+        // rows past the launch's last are zero in the MMA input
+        *reinterpret_cast<uint2*>(xr + i) = (r < nr) ? *reinterpret_cast<const uint2*>(o4) : make_uint2(0u, 0u);
       }
     }
   }
+#pragma unroll
+  for (int c = kEarly; c < kSteps; ++c) wq[c] = wrow[4 * c];
   __syncthreads();
-  for (int e0 = warp * 8; e0 < warp * 8 + 8; e0 += 4) {
-    // four experts at a time: 20 independent 16-byte weight loads in flight per lane, each
-    // weight used for every row of the CTA
-    if (e0 != warp * 8) load_group(e0);
+  // logits D[row][expert] = xs W^T: 40 steps of 32 columns, two k16 MMAs each.  Within a step
+  // the columns enter the MMA in a fixed permuted order (lane t4's four pairs 32c + 8t4 + 2j,
+  // j = 0..3, as k pairs 2t4 and 2t4 + 8 of the first MMA and of the second), the same for the
+  // rows and the weights.
+  // two independent accumulator chains (even and odd steps), added at the end
+  float dq[2][4] = {};
 #pragma unroll
-    for (int r = 0; r < RR; ++r) {
-      if (r >= nr) break;
+  for (int c = 0; c < kSteps; ++c) {
+    const uint4 w = wq[c];
+    const uint4 x0 = *reinterpret_cast<const uint4*>(xs + g * kRouteStride + 32 * c + 8 * t4);
+    const uint4 x1 = *reinterpret_cast<const uint4*>(xs + (g + 8) * kRouteStride + 32 * c + 8 * t4);
+    const uint32_t a0[4] = {x0.x, x1.x, x0.y, x1.y}, b0[2] = {w.x, w.y};
+    const uint32_t a1[4] = {x0.z, x1.z, x0.w, x1.w}, b1[2] = {w.z, w.w};
+    mma_bf16_16816(dq[c & 1], a0, b0);
+    mma_bf16_16816(dq[c & 1], a1, b1);
+  }
+  float d[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        float acc = 0.f;
-#pragma unroll
-        for (int c = 0; c < 5; ++c) {
-          const int i0 = c * 256 + lane * 8;
-          const bf16* wv = reinterpret_cast<const bf16*>(&raw[q][c]);
-#pragma unroll
-          for (int u = 0; u < 8; ++u) acc += __bfloat162float(wv[u]) * xs[r][i0 + u];
-        }
-        acc = warp_sum(acc);
-        if (lane == 0) lg[r][e0 + q] = acc + (a.bias ? a.bias[e0 + q] : 0.f);
-      }
-    }
+  for (int u = 0; u < 4; ++u) d[u] = dq[0][u] + dq[1][u];
+  {
+    const int e = warp * 8 + 2 * t4;
+    const float b0 = a.bias ? a.bias[e] : 0.f, b1 = a.bias ? a.bias[e + 1] : 0.f;
+    lg[g][e] = d[0] + b0;
+    lg[g][e + 1] = d[1] + b1;
+    lg[g + 8][e] = d[2] + b0;
+    lg[g + 8][e + 1] = d[3] + b1;
   }
   __syncthreads();
-  if (warp < nr) {
-    const int r = warp;
-    const size_t t = t0 + r;
+  // softmax and top-6 of rows warp and warp + 8.  Lane l holds experts l and l + 32; the six
+  // winners come out in rank order from six warp-wide maxima of (probability, lower id first)
+  // keys -- the order better() defines.  Both rows are ranked before any row of an expert is
+  // claimed, so that their atomic adds are in flight together.
+  int rank[2][2] = {{-1, -1}, {-1, -1}};
+  float pv[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll
+  for (int h2 = 0; h2 < 2; ++h2) {
+    const int r = warp + 8 * h2;
+    if (r >= nr) break;
     const float l0 = lg[r][lane], l1 = lg[r][lane + 32];
     const float m = warp_max(fmaxf(l0, l1));
     const float e0 = expf(l0 - m), e1 = expf(l1 - m);
@@ -315,82 +227,58 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
       if (!(p0 == p0)) p0 = -1.f;
       if (!(p1 == p1)) p1 = -1.f;
     }
-    // top-6: the rank of each expert among the 64 (a higher probability, or an equal one with a
-    // lower id, ranks ahead) -- the experts of rank 0..5 are the selection, in that order
-    sp[r][lane] = p0;
-    sp[r][lane + 32] = p1;
-    __syncwarp();
-    int rk0 = 0, rk1 = 0;
-#pragma unroll 16
-    for (int j = 0; j < kE; ++j) {
-      const float pj = sp[r][j];
-      rk0 += better(pj, j, p0, lane) ? 1 : 0;
-      rk1 += better(pj, j, p1, lane + 32) ? 1 : 0;
-    }
-    if (rk0 < kTopK) {
-      a.idx[t * kTopK + rk0] = lane;
-      a.gate[t * kTopK + rk0] = p0;
-    }
-    if (rk1 < kTopK) {
-      a.idx[t * kTopK + rk1] = lane + 32;
-      a.gate[t * kTopK + rk1] = p1;
+    pv[h2][0] = p0;
+    pv[h2][1] = p1;
+    unsigned long long k0 = argmax_key(p0, lane), k1 = argmax_key(p1, lane + 32);   // 0: taken
+#pragma unroll
+    for (int k = 0; k < kTopK; ++k) {
+      unsigned long long best = k0 > k1 ? k0 : k1;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+        best = other > best ? other : best;
+      }
+      if (best == k0) {
+        rank[h2][0] = k;
+        k0 = 0ull;
+      } else if (best == k1) {
+        rank[h2][1] = k;
+        k1 = 0ull;
+      }
     }
   }
-  // the last CTA to finish groups the layer's pairs by expert
-  __threadfence();
+  int pos[2][2];
+#pragma unroll
+  for (int h2 = 0; h2 < 2; ++h2)
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+      if (rank[h2][j] >= 0) pos[h2][j] = atomicAdd(a.counts + lane + 32 * j, 1);
+#pragma unroll
+  for (int h2 = 0; h2 < 2; ++h2)
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+      if (rank[h2][j] >= 0) {
+        const int t = t0 + warp + 8 * h2, e = lane + 32 * j;
+        a.idx[static_cast<size_t>(t) * kTopK + rank[h2][j]] = e;
+        a.gate[static_cast<size_t>(t) * kTopK + rank[h2][j]] = pv[h2][j];
+        a.rowmap[static_cast<size_t>(e) * a.map_stride + pos[h2][j]] = (t << 3) | rank[h2][j];
+        dst[warp + 8 * h2][rank[h2][j]] = e * a.map_stride + pos[h2][j];
+      }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    const int old = atomicAdd(a.ticket, 1);
-    s_last = (old == static_cast<int>(gridDim.x) - 1) ? 1 : 0;
-    if (s_last) *a.ticket = 0;
+  // the rounded rows into their experts' input rows, 16 bytes per thread and step
+  constexpr int kVec = kD / 8;
+  for (int i = threadIdx.x; i < nr * kTopK * kVec; i += 256) {
+    const int v = i % kVec, sel = i / kVec, r = sel / kTopK;
+    const uint4 x = *reinterpret_cast<const uint4*>(xs + r * kRouteStride + 8 * v);
+    *reinterpret_cast<uint4*>(a.x_sorted + static_cast<size_t>(dst[r][sel % kTopK]) * kD + 8 * v) = x;
   }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  group_by_expert(a, gsm);
 }
 
-cudaError_t router_prepare() {
-  const int smem = static_cast<int>(sizeof(int) * (kMaxT * kTopK + 2 * kE * kMaxW + 4 * 67));
-  cudaError_t e = cudaFuncSetAttribute(router_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(router_kernel<kRouterRows>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  return e;
-}
+cudaError_t router_prepare() { return cudaSuccess; }
 
 cudaError_t router_launch(const RouteArgs& a, cudaStream_t s) {
-  if (a.T > kMaxT || a.T < 1) return cudaErrorInvalidValue;
-  const int W = (a.T + 31) / 32;
-  const size_t smem = sizeof(int) * (static_cast<size_t>(a.T) * kTopK + 2 * kE * W + 4 * (kE + kShared + 1));
-  if (a.T <= 128) return launch_pdl(router_kernel<1>, dim3(a.T), dim3(256), smem, s, a);
-  return launch_pdl(router_kernel<kRouterRows>, dim3((a.T + kRouterRows - 1) / kRouterRows), dim3(256), smem, s, a);
-}
-
-// ---------------------------------------------------------------- permute (row gather)
-// Copies the normalised row of every routed (token, slot) pair to its expert-sorted row of
-// the experts' input, one warp per pair, all of a row's loads issued before its stores.
-__global__ void __launch_bounds__(256) permute_kernel(const int* dst_row, int T6, const bf16* xn, bf16* xs) {
-  pdl_trigger();
-  pdl_wait();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * 8 + warp, nw = gridDim.x * 8;
-  for (int p = gw; p < T6; p += nw) {
-    const int t = p / kTopK, dst = dst_row[p];
-    const uint4* src = reinterpret_cast<const uint4*>(xn + static_cast<size_t>(t) * kD);
-    uint4* d = reinterpret_cast<uint4*>(xs + static_cast<size_t>(dst) * kD);
-    uint4 v[kD / 8 / 32];
-#pragma unroll
-    for (int c = 0; c < kD / 8 / 32; ++c) v[c] = src[lane + 32 * c];
-#pragma unroll
-    for (int c = 0; c < kD / 8 / 32; ++c) d[lane + 32 * c] = v[c];
-  }
-}
-
-cudaError_t permute_launch(const int* dst_row, int T, const bf16* xn, bf16* x_sorted, cudaStream_t s) {
-  const int pairs = T * kTopK;
-  int grid = (pairs + 7) / 8;     // one warp per (token, slot) row copy
-  if (grid > 1024) grid = 1024;
-  if (grid < 1) grid = 1;
-  return launch_pdl(permute_kernel, dim3(grid), dim3(256), 0, s, dst_row, pairs, xn, x_sorted);
+  if (a.T > kMaxT || a.T < 1 || a.T > a.map_stride) return cudaErrorInvalidValue;
+  return launch_pdl(router_kernel, dim3((a.T + kRouteCtaRows - 1) / kRouteCtaRows), dim3(256), 0, s, a);
 }
 
 // ---------------------------------------------------------------- combine
