@@ -197,8 +197,10 @@ spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, in
  * the stream and fills *out:
  *   launches[c], ms[c]  kernel launches and summed event time of class c (SPEC_K_*);
  *   experts_touched     routed + shared experts with at least one row, summed over the
- *                       grouped-GEMM launches (the expert weight bytes actually read);
- *   expert_rows         (token, expert) rows processed by those launches. */
+ *                       grouped gate/up launches (the expert weight bytes actually read);
+ *   expert_rows         (token, expert) rows processed by those launches.
+ * SPEC_K_PERMUTE stays in the numbering but no longer launches: the router writes each
+ * expert's input rows itself. */
 enum { SPEC_K_EMBED = 0, SPEC_K_QKV = 1, SPEC_K_ATTN = 2, SPEC_K_OPROJ = 3, SPEC_K_ROUTER = 4,
        SPEC_K_PERMUTE = 5, SPEC_K_EXPERT_GU = 6, SPEC_K_EXPERT_DN = 7, SPEC_K_COMBINE = 8,
        SPEC_K_LMHEAD = 9, SPEC_K_ARGMAX = 10, SPEC_K_COMMIT = 11, SPEC_K_DRAFT_GEMM = 12,
