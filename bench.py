@@ -429,6 +429,8 @@ def run_fastmtp(args):
         "expert_down": touched * d * I * 2 + rows * I * 2 + rows * d * 4,
         "lm_head": shape.vocab * d * 2.0,
     }
+    if counted["launches"]["expert_down"] == 0:   # gate/up and down run as one launch per layer
+        cls_bytes["expert_gate_up"] += cls_bytes["expert_down"]
     gemm_ms = {k: prof["ms"][k] for k in ("expert_gate_up", "expert_down", "qkv", "oproj", "lm_head",
                                           "attention", "draft_gemm")}
     dom = max(("expert_gate_up", "expert_down", "lm_head"), key=lambda k: prof["ms"][k])

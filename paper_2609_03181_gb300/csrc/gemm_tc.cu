@@ -44,27 +44,38 @@ constexpr int kShallowStages = 4;   // stages of the dense cluster schedule
 struct Item {
   int e, n_tile, b_row, out_row, rows, split, box_log;
   int grow;   // grouped: first row of the item within its expert
+  int phase;  // EPI_MOE: 0 gate/up item, 1 down item
 };
 
 // Per-expert tables of a grouped launch in shared memory, built by every CTA from the counts:
-// grp[e] first item of expert e (grp[66] = items), grp[67 + e] its rows.
-constexpr int kGrpItem = 0, kGrpCnt = kE + kShared + 1;
+// grp[e] first item of expert e (grp[66] = items), grp[67 + e] its rows, and for EPI_MOE
+// grp[134 + e] the first down item of expert e counted from the first down item.
+constexpr int kGrpItem = 0, kGrpCnt = kE + kShared + 1, kGrpDn = 2 * (kE + kShared + 1);
 
-__device__ __forceinline__ void get_item(const GemmArgs& a, int i, Item& it, const int* grp) {
+__device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, int i, Item& it, const int* grp) {
+  it.phase = 0;
   if (a.grp_cnt != nullptr) {
+    const int* pre = grp + kGrpItem;
+    const GemmArgs* P = &a;
+    if (i >= grp[kGrpItem + kE + kShared]) {   // past the gate/up items: an EPI_MOE down item
+      i -= grp[kGrpItem + kE + kShared];
+      pre = grp + kGrpDn;
+      P = &a2;
+      it.phase = 1;
+    }
     int lo = 0, hi = kE + kShared - 1;   // the last expert whose first item is <= i has items
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (grp[kGrpItem + mid] <= i) lo = mid;
+      if (pre[mid] <= i) lo = mid;
       else hi = mid - 1;
     }
-    const int j = i - grp[kGrpItem + lo], m = j / a.grp_tiles;
+    const int j = i - pre[lo], m = j / P->grp_tiles;
     it.e = lo;
-    it.n_tile = j - m * a.grp_tiles;
+    it.n_tile = j - m * P->grp_tiles;
     it.grow = kExpertTileRows * m;
     it.rows = min(kExpertTileRows, grp[kGrpCnt + lo] - it.grow);
     it.out_row = lo * a.map_stride + it.grow;
-    it.b_row = (a.grp_b_direct && lo >= a.n_routed) ? it.grow : it.out_row;
+    it.b_row = (P->grp_b_direct && lo >= a.n_routed) ? it.grow : it.out_row;
     it.split = 0;
     int bl = 0;
     while ((16 << bl) < it.rows) ++bl;
@@ -297,7 +308,7 @@ template <int EPI>
 __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem& esm, uint32_t part_saddr, int row,
                                                const EpiPre& first) {
   Item it;
-  get_item(a, blockIdx.x, it, nullptr);
+  get_item(a, a, blockIdx.x, it, nullptr);
   const int S = a.cluster;
   const int rank = static_cast<int>(cluster_ctarank());
   const int nchunks = (it.rows + 15) >> 4;
@@ -350,7 +361,8 @@ __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem&
 
 // ------------------------------------------------------------------ kernel
 template <int NMAX, int EPI, int ST>
-__global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
+__global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a,
+                                                         const __grid_constant__ GemmArgs a2) {
   using C = Cfg<NMAX, ST>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t base_u32 = smem_u32(smem_raw);
@@ -422,36 +434,46 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   int n_items = a.n_items;
   if (!dense) {
     if (threadIdx.x < 32) {   // three experts per lane, prefix sums by warp scan
-      int c[3], ni[3], sc = 0, si = 0, touched = 0;
+      int c[3], ni[3], nd[3], sc = 0, si = 0, sd = 0, touched = 0;
 #pragma unroll
       for (int k = 0; k < 3; ++k) {
         const int e = 3 * static_cast<int>(threadIdx.x) + k;
         c[k] = (e < kE + kShared) ? ((e < a.n_routed) ? a.grp_cnt[e] : a.grp_T) : 0;
-        ni[k] = (c[k] + kExpertTileRows - 1) / kExpertTileRows * a.grp_tiles;
+        const int mt = (c[k] + kExpertTileRows - 1) / kExpertTileRows;
+        ni[k] = mt * a.grp_tiles;
+        nd[k] = (EPI == EPI_MOE) ? mt * a2.grp_tiles : 0;
         sc += c[k];
         si += ni[k];
+        sd += nd[k];
         touched += (c[k] > 0) ? 1 : 0;
       }
-      int ic = sc, ii = si;
+      int ic = sc, ii = si, id = sd;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int yc = __shfl_up_sync(0xffffffffu, ic, o), yi = __shfl_up_sync(0xffffffffu, ii, o);
+        const int yd = __shfl_up_sync(0xffffffffu, id, o);
         if (static_cast<int>(threadIdx.x) >= o) {
           ic += yc;
           ii += yi;
+          id += yd;
         }
       }
-      int ri = ii - si;
+      int ri = ii - si, rd = id - sd;
 #pragma unroll
       for (int k = 0; k < 3; ++k) {
         const int e = 3 * static_cast<int>(threadIdx.x) + k;
         if (e < kE + kShared) {
           grp[kGrpCnt + e] = c[k];
           grp[kGrpItem + e] = ri;
+          grp[kGrpDn + e] = rd;
         }
         ri += ni[k];
+        rd += nd[k];
       }
-      if (threadIdx.x == 31) grp[kGrpItem + kE + kShared] = ii;
+      if (threadIdx.x == 31) {
+        grp[kGrpItem + kE + kShared] = ii;
+        grp[kGrpDn + kE + kShared] = id;
+      }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) touched += __shfl_xor_sync(0xffffffffu, touched, o);
       if (a.expert_ctr != nullptr && blockIdx.x == 0 && threadIdx.x == 31) {
@@ -460,9 +482,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       }
     }
     __syncthreads();
-    n_items = grp[kGrpItem + kE + kShared];
+    n_items = grp[kGrpItem + kE + kShared] + ((EPI == EPI_MOE) ? grp[kGrpDn + kE + kShared] : 0);
   }
-  const int kc_total = a.K / 64;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
@@ -474,33 +495,52 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       bool waited = !dense;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x) {
         Item it;
-        get_item(a, i, it, grp);
+        get_item(a, a2, i, it, grp);
+        const GemmArgs& P = it.phase ? a2 : a;   // the item's operands (EPI_MOE down items: a2)
+        const int kc_total = P.K / 64;
         const int src = (!dense && it.e >= a.n_routed) ? 1 : 0;
         const int el = it.e - (src ? a.n_routed : 0);
-        const CUtensorMap* amap = &a.a_map[src];
-        const CUtensorMap* bmap = &a.b_map[src][it.box_log];
+        const CUtensorMap* amap = &P.a_map[src];
+        const CUtensorMap* bmap = &P.b_map[src][it.box_log];
         const uint32_t bytes = C::A_BYTES + (16u << it.box_log) * 128u;
         const int kc0 = a.seq_split ? 0 : it.split * kc_total / a.split_k;
         const int kc1 = a.seq_split ? kc_total : (it.split + 1) * kc_total / a.split_k;
         auto load_a = [&](int st, int kc) {
           uint8_t* sa = smA + st * C::A_BYTES;
           const int k = kc * 64;
-          if (a.paired) {
+          if (P.paired) {
             const int r0 = it.n_tile * 64;
-            if (a.a3d) {
+            if (P.a3d) {
               tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
-              tma_load_3d(sa + 8192, amap, &full[st], k, a.half_rows + r0, el, pol_w);
+              tma_load_3d(sa + 8192, amap, &full[st], k, P.half_rows + r0, el, pol_w);
             } else {
               tma_load_2d(sa, amap, &full[st], k, r0, pol_w);
-              tma_load_2d(sa + 8192, amap, &full[st], k, a.half_rows + r0, pol_w);
+              tma_load_2d(sa + 8192, amap, &full[st], k, P.half_rows + r0, pol_w);
             }
           } else {
             const int r0 = it.n_tile * 128;
-            if (a.a3d) tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
+            if (P.a3d) tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
             else tma_load_2d(sa, amap, &full[st], k, r0, pol_w);
           }
         };
         int kc = kc0;
+        if (EPI == EPI_MOE && it.phase == 1) {
+          // a down item reads the SwiGLU rows of its (expert, row tile): wait until all gate/up
+          // tiles of them are stored (they come earlier in the item order, so they always end)
+          const int* d = a.dep + it.e * a.dep_stride + it.grow / kExpertTileRows;
+          if (ld_acquire_gpu(d) < a.grp_tiles) {
+            const uint64_t t0 = globaltimer();
+            while (ld_acquire_gpu(d) < a.grp_tiles) {
+              if (*s_abort || globaltimer() - t0 > kWaitLimitNs) {
+                failed = true;
+                break;
+              }
+              __nanosleep(64);
+            }
+            if (failed) break;
+          }
+          fence_proxy_async_global();   // the rows were stored by other CTAs' generic stores
+        }
         if (!waited) {
           // first item: the stages are all free (g == 0); weights first, activations after the wait
           const int npre = min(C::STAGES, kc1 - kc0);
@@ -548,7 +588,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       bool failed = false;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x, ++local) {
         Item it;
-        get_item(a, i, it, grp);
+        get_item(a, a2, i, it, grp);
+        const int kc_total = (it.phase ? a2.K : a.K) / 64;
         const int acc = local % nbuf;
         const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
         if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, s_abort)) {
@@ -605,12 +646,16 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     int local = 0;
     for (int i = blockIdx.x; i < n_items; i += gridDim.x, ++local) {
       Item it;
-      get_item(a, i, it, grp);
+      get_item(a, a2, i, it, grp);
       const int acc = local % nbuf;
       const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
       // the item's metadata, RoPE factors and first old residuals are fetched while its MMAs
       // run (in a cluster, those of the first chunk this CTA reduces)
-      stage_meta<EPI>(a, it, esm);
+      if constexpr (EPI == EPI_MOE) {
+        if (it.phase) stage_meta<EPI_SCATTER>(a2, it, esm);
+      } else {
+        stage_meta<EPI>(a, it, esm);
+      }
       const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
       const int c_first = (a.cluster > 1) ? static_cast<int>(cluster_ctarank()) : 0;
       RopeRegs rr;
@@ -651,12 +696,24 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
 #pragma unroll
             for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
           }
-          epi_post<EPI>(a, it, row, c * 16, v, cur, esm, c & 1);
+          if constexpr (EPI == EPI_MOE) {
+            if (it.phase) epi_post<EPI_SCATTER>(a2, it, row, c * 16, v, cur, esm, c & 1);
+            else epi_post<EPI_SWIGLU>(a, it, row, c * 16, v, cur, esm, c & 1);
+          } else {
+            epi_post<EPI>(a, it, row, c * 16, v, cur, esm, c & 1);
+          }
           cur = nxt;
           if (rope && c + 1 < nchunks) {
             rope_store(esm, (c + 1) & 1, rr);
             named_bar_sync(1, 128);
           }
+        }
+        if (EPI == EPI_MOE && it.phase == 0) {
+          // this gate/up tile's SwiGLU rows are stored: count it for the down items of (e, m)
+          fence_proxy_async_global();
+          __threadfence();
+          named_bar_sync(1, 128);
+          if (threadIdx.x == 64) atomicAdd(a.dep + it.e * a.dep_stride + it.grow / kExpertTileRows, 1);
         }
         tc_fence_before();
         __syncwarp();
@@ -844,7 +901,7 @@ cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   }
   cfg.attrs = attr;
   cfg.numAttrs = n;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI, ST>, a);
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI, ST>, a, a);
 }
 }  // namespace
 
@@ -908,6 +965,7 @@ cudaError_t gemm_prepare() {
   FM_ATTR(EPI_SCATTER)
   FM_ATTR(EPI_ARGMAX)
 #undef FM_ATTR
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, kShallowStages>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_RESID, kShallowStages>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_QKV, kShallowStages>();
@@ -965,6 +1023,24 @@ int dense_split_k(int N, int K) {
   while (s > 1 && n_tiles > max_resident_clusters(s)) --s;
   if (s < 1) s = 1;
   return s;
+}
+
+cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream_t s) {
+  // one persistent CTA per SM; its down items wait on gate/up tiles of other CTAs, so the
+  // launch is cooperative (every CTA resident at once)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(num_sms());
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = Cfg<64>::SMEM_BYTES;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<64, EPI_MOE, Cfg<64>::STAGES>, gate_up, down);
 }
 
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {

@@ -61,7 +61,8 @@ enum EpiKind : int {
   EPI_QKV = 2,      // RoPE on q/k, q -> fp32 buffer, k/v -> bf16 cache rows
   EPI_SWIGLU = 3,   // tile = 64 gate rows + 64 up rows -> bf16 silu(g)*u
   EPI_SCATTER = 4,  // expert down: out row (token, slot) from the sorted index
-  EPI_ARGMAX = 5    // running (max, argmax) of each column in a packed key (LM head)
+  EPI_ARGMAX = 5,   // running (max, argmax) of each column in a packed key (LM head)
+  EPI_MOE = 6       // grouped gate/up (SWIGLU) items, then the down (SCATTER) items, one launch
 };
 
 // One work item: weight tile x activation rows.  x = expert | n_tile << 16, y = TMA row of
@@ -91,6 +92,12 @@ struct GemmArgs {
   const int* rowmap;           // SCATTER: [n_routed][map_stride] (token << 3 | rank) of each row
   int map_stride;
   unsigned long long* expert_ctr;   // if set, CTA 0 adds (experts with rows, rows) of the launch
+  // EPI_MOE: this struct describes the gate/up items, a second one (the kernel's second
+  // argument) the down items.  The gate/up epilogue of (expert e, row tile m) adds one to
+  // dep[e * dep_stride + m] after its SwiGLU rows are stored; a down item of (e, m) waits until
+  // all grp_tiles gate/up tiles of (e, m) have.
+  int* dep;
+  int dep_stride;
   int n_items;                 // dense: number of items
   int M;                       // dense: activation rows
   int m_tiles, box_log;        // dense: row tiles of 16 << box_log rows
@@ -123,6 +130,8 @@ bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, u
 // pdl = false launches without programmatic serialization (for streams whose earlier kernels
 // may still be writing the weights).
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl = true);
+// The routed + shared experts' gate/up and down in one cooperative launch (EPI_MOE).
+cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream_t s);
 int num_sms();
 // Sets the message spec_last_error(NULL) returns in this thread.
 void set_thread_error(const std::string& msg);
@@ -172,7 +181,7 @@ cudaError_t attention_launch(const AttnArgs& a, int B, cudaStream_t s);
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
-                              int* err, int* zero, int n_zero, cudaStream_t s);
+                              int* err, int* zero, int n_zero, int* zero2, int n_zero2, cudaStream_t s);
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
 // Router (+ expert grouping by the last CTA) and the permute row gather.
 struct RouteArgs {

@@ -85,6 +85,8 @@ struct spec_ctx {
   int* route_idx = nullptr;
   float* route_gate = nullptr;
   int* counts = nullptr;
+  int* moe_dep = nullptr;       // [L][n_experts + n_shared][dep_stride] gate/up tiles done per row tile
+  int dep_stride = 0;
   bf16* x_sorted = nullptr;
   bf16* act = nullptr;
   float* y = nullptr;
@@ -438,6 +440,8 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->route_idx, sizeof(int) * L * Tmax * kTopK);
   add(&ctx->route_gate, sizeof(float) * L * Tmax * kTopK);
   add(&ctx->counts, sizeof(int) * L * kE);
+  ctx->dep_stride = ctx->Tcap / kExpertTileRows;
+  add(&ctx->moe_dep, sizeof(int) * L * (kE + kShared) * ctx->dep_stride);
   add(&ctx->x_sorted, sizeof(bf16) * kE * ctx->Tcap * d);
   add(&ctx->act, sizeof(bf16) * (kE + kShared) * ctx->Tcap * kI);
   add(&ctx->y, sizeof(float) * Tmax * kSlots * d);
@@ -651,8 +655,8 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
   CK(cudaMemcpyAsync(ctx->cand_ws, cand, sizeof(int) * T, cudaMemcpyDeviceToDevice, s));
   LAUNCH(SPEC_K_EMBED, 1, embed_norm_launch(ctx->cand_ws, B, R, slots, ctx->pending, ctx->seq_len, static_cast<const bf16*>(ctx->w.embed),
                        c.vocab, static_cast<const bf16*>(ctx->layers[0].attn_norm), eps, ctx->h, ctx->xn, ctx->pos,
-                       ctx->kv_rowoff, ctx->Rmax, ctx->Bmax, ctx->d_err, ctx->counts, L * kE, s));
-  const int nmax_grouped = kExpertTileRows;
+                       ctx->kv_rowoff, ctx->Rmax, ctx->Bmax, ctx->d_err, ctx->counts, L * kE, ctx->moe_dep,
+                       L * (kE + kShared) * ctx->dep_stride, s));
   for (int l = 0; l < L; ++l) {
     const spec_layer_weights& W = ctx->layers[l];
     const LayerMaps& M = ctx->lmaps[l];
@@ -726,7 +730,8 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       ra.map_stride = ctx->Tcap;
       LAUNCH(SPEC_K_ROUTER, 1, router_launch(ra, s));
     }
-    // routed + shared experts: gate/up + SwiGLU
+    // routed + shared experts: gate/up + SwiGLU, then down scattered to (token, slot), in one
+    // cooperative launch (a down tile starts as soon as the gate/up tiles of its rows are done)
     {
       GemmArgs g = base_args(ctx);
       g.a_map[0] = M.gu_routed;
@@ -749,28 +754,26 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.expert_ctr = ctx->d_expert_ctr;
       g.act = ctx->act;
       g.ld_act = kI;
-      LAUNCH(SPEC_K_EXPERT_GU, 1, gemm_launch(EPI_SWIGLU, nmax_grouped, g, num_sms(), s));
-    }
-    // routed + shared experts: down, scattered to (token, slot)
-    {
-      GemmArgs g = base_args(ctx);
-      g.a_map[0] = M.dn_routed;
-      g.a_map[1] = M.dn_shared;
+      g.dep = ctx->moe_dep + static_cast<size_t>(l) * (kE + kShared) * ctx->dep_stride;
+      g.dep_stride = ctx->dep_stride;
+      GemmArgs d = base_args(ctx);
+      d.a_map[0] = M.dn_routed;
+      d.a_map[1] = M.dn_shared;
       for (int b = 0; b < 5; ++b) {
-        g.b_map[0][b] = ctx->a_act.m[b];
-        g.b_map[1][b] = ctx->a_act.m[b];
+        d.b_map[0][b] = ctx->a_act.m[b];
+        d.b_map[1][b] = ctx->a_act.m[b];
       }
-      g.N = kD;
-      g.K = kI;
-      g.a3d = 1;
-      g.n_routed = kE;
-      g.grp_cnt = ctx->counts + l * kE;
-      g.grp_T = T;
-      g.grp_tiles = kD / 128;
-      g.rowmap = ctx->rowmap;
-      g.map_stride = ctx->Tcap;
-      g.y = ctx->y;
-      LAUNCH(SPEC_K_EXPERT_DN, 1, gemm_launch(EPI_SCATTER, nmax_grouped, g, num_sms(), s));
+      d.N = kD;
+      d.K = kI;
+      d.a3d = 1;
+      d.n_routed = kE;
+      d.grp_cnt = ctx->counts + l * kE;
+      d.grp_T = T;
+      d.grp_tiles = kD / 128;
+      d.rowmap = ctx->rowmap;
+      d.map_stride = ctx->Tcap;
+      d.y = ctx->y;
+      LAUNCH(SPEC_K_EXPERT_GU, 1, moe_launch(g, d, s));
     }
     const bf16* next_gain =
         static_cast<const bf16*>(l + 1 < L ? ctx->layers[l + 1].attn_norm : ctx->w.final_norm);

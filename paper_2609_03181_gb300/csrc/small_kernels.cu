@@ -49,11 +49,13 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
                                                          const int* seq_len, const bf16* embed, int vocab,
                                                          const bf16* gain, float eps, float* h, bf16* xn, int* pos,
                                                          long long* kv_rowoff, int stage_R, int n_slots, int* err,
-                                                         int* zero, int n_zero) {
+                                                         int* zero, int n_zero, int* zero2, int n_zero2) {
   pdl_trigger();
   pdl_wait();
-  if (blockIdx.x == 0)   // the step's per-expert row counters start from zero
+  if (blockIdx.x == 0) {   // the step's per-expert row counters and tile counters start from zero
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
+    for (int i = threadIdx.x; i < n_zero2; i += blockDim.x) zero2[i] = 0;
+  }
   __shared__ float red[4];
   const int row = blockIdx.x, b = row / R, r = row % R;
   const int slot = slots[b];
@@ -83,9 +85,9 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
-                              int* err, int* zero, int n_zero, cudaStream_t s) {
+                              int* err, int* zero, int n_zero, int* zero2, int n_zero2, cudaStream_t s) {
   return launch_pdl(embed_norm_kernel, dim3(B * R), dim3(128), 0, s, cand, R, slots, pending, seq_len, embed, vocab, gain,
-                    eps, h, xn, pos, kv_rowoff, stage_R, n_slots, err, zero, n_zero);
+                    eps, h, xn, pos, kv_rowoff, stage_R, n_slots, err, zero, n_zero, zero2, n_zero2);
 }
 
 // ---------------------------------------------------------------- RMSNorm
