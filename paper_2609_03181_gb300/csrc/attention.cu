@@ -61,8 +61,9 @@ constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, que
 // Shared memory of a CTA of a launch over B sequences: 1 KB alignment slack, the stages, two
 // query slots, the barriers, the merge scratch and flags, and the per-sequence tables (first
 // query position, slot, item prefix).
+constexpr int kXchgBytes = 4 * 32 * 16 + 2 * 4 * kMaxR * 4;   // P fragments of the 4 key tiles, max / sum partials
 constexpr size_t attn_smem(int stages, int B) {
-  return 1024 + stages * kStageBytes + 2 * kQBytes + (2 * stages + 4) * 8 + (2 * kMaxR + 8) * 4 +
+  return 1024 + stages * kStageBytes + 2 * kQBytes + kXchgBytes + (2 * stages + 4) * 8 + (2 * kMaxR + 8) * 4 +
          (3 * static_cast<size_t>(B) + 1) * 4;
 }
 
@@ -205,7 +206,10 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
   const uint32_t raw_u32 = smem_u32(asmem_raw);
   uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [S][K 16 KB | V 16 KB]
   uint8_t* sQ = stages + kStages * kStageBytes;                             // [2][8 queries][128] bf16
-  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + 2 * kQBytes);           // [S] chunk landed
+  uint4* sP = reinterpret_cast<uint4*>(sQ + 2 * kQBytes);                  // [4 key tiles][32 lanes] P^T frags
+  float* s_cmax = reinterpret_cast<float*>(sP + 4 * 32);                    // [4 warps][8 queries] chunk max
+  float* s_csum = s_cmax + 4 * kMaxR;                                       // [4 warps][8 queries] chunk sum
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_csum + 4 * kMaxR);         // [S] chunk landed
   uint64_t* empty = full + kStages;                                         // [S] chunk consumed
   uint64_t* qfull = empty + kStages;                                        // [2] queries landed
   uint64_t* qempty = qfull + 2;                                             // [2] queries loaded
@@ -508,81 +512,79 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
           atomicOr(a.err, ERR_WAIT_TIMEOUT);
         }
       }
-      if (ok) {
+      {
+        // Warp w scores the chunk's keys 16w..16w+15 (S^T = K Q^T over 8 k-steps of 16 dims,
+        // even and odd k-steps in separate accumulators, added at the end); the chunk's max and
+        // sum per query and its P^T fragments (bf16 hi + lo) go through shared memory, so that
+        // each warp can then multiply all 64 keys of V^T for its 32 output dims.  Waits and
+        // barriers run even after a wait has run out (then on stale data) so that the four
+        // warps always meet at the same barriers.
         const uint32_t kbase = smem_u32(stages + st * kStageBytes);
         const uint32_t vbase = kbase + kTileBytes;
-        // S^T[key][query] = K Q^T over four 16-key tiles, 8 k-steps of 16 dims: even and odd
-        // k-steps in separate accumulators (eight independent MMA chains), added at the end
-        float s[4][4], s1[4][4];
-#pragma unroll
-        for (int kt = 0; kt < 4; ++kt)
-#pragma unroll
-          for (int e = 0; e < 4; ++e) s[kt][e] = s1[kt][e] = 0.f;
+        float sc[4] = {0.f, 0.f, 0.f, 0.f}, sc1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int ks = 0; ks < 8; ks += 2) {
-#pragma unroll
-          for (int kt = 0; kt < 4; ++kt) {
-            uint32_t ak[4], ak1[4];
-            ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + (mi >> 1)), ak);
-            ldsm_x4(kbase + swt(16 * kt + ri + ((mi & 1) ? 8 : 0), 2 * ks + 2 + (mi >> 1)), ak1);
-            mma_bf16_16816(s[kt], ak, qf[ks]);
-            mma_bf16_16816(s1[kt], ak1, qf[ks + 1]);
-          }
+          uint32_t ak[4], ak1[4];
+          ldsm_x4(kbase + swt(16 * warp + ri + ((mi & 1) ? 8 : 0), 2 * ks + (mi >> 1)), ak);
+          ldsm_x4(kbase + swt(16 * warp + ri + ((mi & 1) ? 8 : 0), 2 * ks + 2 + (mi >> 1)), ak1);
+          mma_bf16_16816(sc, ak, qf[ks]);
+          mma_bf16_16816(sc1, ak1, qf[ks + 1]);
         }
-#pragma unroll
-        for (int kt = 0; kt < 4; ++kt)
-#pragma unroll
-          for (int e = 0; e < 4; ++e) s[kt][e] += s1[kt][e];
-        // visibility, chunk max per query (lanes sharing t4 hold the same two queries)
-        const int kb = c * kCH;
+        // visibility and this warp's max per query (lanes sharing t4 hold the same two queries)
+        const int kb = c * kCH + 16 * warp;
         float m_a = -INFINITY, m_b = -INFINITY;
 #pragma unroll
-        for (int kt = 0; kt < 4; ++kt)
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int key = kb + 16 * kt + g + ((e >> 1) ? 8 : 0);
-            const int q = (e & 1) ? qb : qa;
-            const float x = (q < R && key <= p0 + q) ? s[kt][e] * scale : -INFINITY;
-            s[kt][e] = x;
-            if (e & 1) m_b = fmaxf(m_b, x);
-            else m_a = fmaxf(m_a, x);
-          }
+        for (int e = 0; e < 4; ++e) {
+          const int key = kb + g + ((e >> 1) ? 8 : 0);
+          const int q = (e & 1) ? qb : qa;
+          const float x = (q < R && key <= p0 + q) ? (sc[e] + sc1[e]) * scale : -INFINITY;
+          sc[e] = x;
+          if (e & 1) m_b = fmaxf(m_b, x);
+          else m_a = fmaxf(m_a, x);
+        }
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) {
           m_a = fmaxf(m_a, __shfl_xor_sync(0xffffffffu, m_a, o));
           m_b = fmaxf(m_b, __shfl_xor_sync(0xffffffffu, m_b, o));
         }
+        if (g == 0) {
+          s_cmax[warp * kMaxR + qa] = m_a;
+          s_cmax[warp * kMaxR + qb] = m_b;
+        }
+        named_bar_sync(2, kConsumers);
+        m_a = fmaxf(fmaxf(s_cmax[qa], s_cmax[kMaxR + qa]), fmaxf(s_cmax[2 * kMaxR + qa], s_cmax[3 * kMaxR + qa]));
+        m_b = fmaxf(fmaxf(s_cmax[qb], s_cmax[kMaxR + qb]), fmaxf(s_cmax[2 * kMaxR + qb], s_cmax[3 * kMaxR + qb]));
         const float Mn_a = fmaxf(M_a, m_a), Mn_b = fmaxf(M_b, m_b);
         const float al_a = (M_a == -INFINITY) ? 0.f : exp2f(M_a - Mn_a);
         const float al_b = (M_b == -INFINITY) ? 0.f : exp2f(M_b - Mn_b);
         M_a = Mn_a;
         M_b = Mn_b;
-        // p = 2^(x - M) (exact zeros where masked), row sums, and P^T as bf16 hi + lo fragments
-        float l_a = 0.f, l_b = 0.f;
-        uint32_t ph[4][2], pl[4][2];
+        // p = 2^(x - M) (exact zeros where masked), this warp's sums, and its P^T fragments
+        float l_a = 0.f, l_b = 0.f, p[4], lo[4];
 #pragma unroll
-        for (int kt = 0; kt < 4; ++kt) {
-          float p[4], lo[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float Mq = (e & 1) ? M_b : M_a;
-            p[e] = (s[kt][e] == -INFINITY) ? 0.f : exp2f(s[kt][e] - Mq);
-            if (e & 1) l_b += p[e];
-            else l_a += p[e];
-            lo[e] = p[e] - __bfloat162float(__float2bfloat16(p[e]));
-          }
-          ph[kt][0] = movmatrix_t(pack_bf16(p[0], p[1]));     // keys 16kt+0..7
-          ph[kt][1] = movmatrix_t(pack_bf16(p[2], p[3]));     // keys 16kt+8..15
-          pl[kt][0] = movmatrix_t(pack_bf16(lo[0], lo[1]));
-          pl[kt][1] = movmatrix_t(pack_bf16(lo[2], lo[3]));
+        for (int e = 0; e < 4; ++e) {
+          const float Mq = (e & 1) ? M_b : M_a;
+          p[e] = (sc[e] == -INFINITY) ? 0.f : exp2f(sc[e] - Mq);
+          if (e & 1) l_b += p[e];
+          else l_a += p[e];
+          lo[e] = p[e] - __bfloat162float(__float2bfloat16(p[e]));
         }
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) {
           l_a += __shfl_xor_sync(0xffffffffu, l_a, o);
           l_b += __shfl_xor_sync(0xffffffffu, l_b, o);
         }
-        L_a = L_a * al_a + l_a;
-        L_b = L_b * al_b + l_b;
+        if (g == 0) {
+          s_csum[warp * kMaxR + qa] = l_a;
+          s_csum[warp * kMaxR + qb] = l_b;
+        }
+        sP[warp * 32 + lane] = make_uint4(movmatrix_t(pack_bf16(p[0], p[1])),    // keys 16w+0..7
+                                          movmatrix_t(pack_bf16(p[2], p[3])),    // keys 16w+8..15
+                                          movmatrix_t(pack_bf16(lo[0], lo[1])),
+                                          movmatrix_t(pack_bf16(lo[2], lo[3])));
+        named_bar_sync(2, kConsumers);
+        L_a = L_a * al_a + (((s_csum[qa] + s_csum[kMaxR + qa]) + s_csum[2 * kMaxR + qa]) + s_csum[3 * kMaxR + qa]);
+        L_b = L_b * al_b + (((s_csum[qb] + s_csum[kMaxR + qb]) + s_csum[2 * kMaxR + qb]) + s_csum[3 * kMaxR + qb]);
         // O^T[dim][query] = al * O^T + V^T P^T for this warp's two 16-dim tiles (dims
         // 32w..32w+31), 4 k-steps of 16 keys; hi and lo products in separate accumulators
 #pragma unroll
@@ -598,12 +600,14 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
         }
 #pragma unroll
         for (int kt = 0; kt < 4; ++kt) {
+          const uint4 pf = sP[kt * 32 + lane];
+          const uint32_t ph[2] = {pf.x, pf.y}, pl[2] = {pf.z, pf.w};
 #pragma unroll
           for (int jj = 0; jj < 2; ++jj) {
             uint32_t av[4];
             ldsm_x4_t(vbase + swt(16 * kt + ri + ((mi >> 1) ? 8 : 0), 2 * (2 * warp + jj) + (mi & 1)), av);
-            mma_bf16_16816(O[jj], av, ph[kt]);
-            mma_bf16_16816(Ol[jj], av, pl[kt]);
+            mma_bf16_16816(O[jj], av, ph);
+            mma_bf16_16816(Ol[jj], av, pl);
           }
         }
       }
