@@ -644,10 +644,11 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
     const bool more = w.i + 1 < i_end;
     if (!more || w.s == w.nsup - 1) {
       // this CTA's super-chunks of (b, h) are written: count them; the CTA that completes the
-      // count merges every super-chunk of (b, h)
-      __threadfence();
+      // count merges every super-chunk of (b, h).  The barrier orders the four warps' partial
+      // stores before thread 0's device-scope fence and count (fences are cumulative).
       named_bar_sync(1, kConsumers);
       if (tid == 0) {
+        __threadfence();
         int* ticket = a.tickets + b * kH + h;
         const int old = atomicAdd(ticket, run_items);
         const int last = (old + run_items == w.nsup) ? 1 : 0;
