@@ -16,13 +16,13 @@ from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, ind
 pytestmark = pytest.mark.gpu
 
 
-def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None):
+def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=None):
     """One verify_step + accept_commit of len(ctx_lens) sequences on the GPU; the sequences in
     `check` (default: all) are compared with the oracle, the others get uniform random drafts and
     only fill the batch.  Returns (tokens compared, tokens skipped below the margin)."""
     B = len(ctx_lens)
     check = list(range(B)) if check is None else list(check)
-    vw = S.verifier_weights(shape, seed, gain_std=gain_std)
+    vw = S.verifier_weights(shape, seed, gain_std=gain_std, zipf_s=zipf_s)
     dw = S.draft_weights(shape, seed, gain_std=gain_std)
     model = O.Verifier(vw)
     kvs, dkvs = seq_prefixes(shape, seed, ctx_lens)
@@ -143,3 +143,12 @@ def test_verify_max_batch_256():
     shape = S.ModelShape(n_layers=1, vocab=4096)
     ctx = [int(c) for c in S.integers(9, "ctx", 256, 1, 160)]
     run_verify_case(shape, 9, ctx, K=3, check=range(3, 256, 16))
+
+
+def test_verify_zipf_hot_experts():
+    """Zipf-skewed routing (router bias -1.2 ln(rank)): the hottest experts take most of the 192
+    candidate rows, so their gate/up and down tiles span several 64-row tiles and every down
+    tile waits on the gate/up tiles of its own rows; 8 of the 48 sequences are checked."""
+    shape = S.ModelShape(n_layers=2, vocab=4096)
+    ctx = [int(c) for c in S.integers(11, "ctx", 48, 1, 300)]
+    run_verify_case(shape, 11, ctx, K=3, check=range(0, 48, 6), zipf_s=1.2)
