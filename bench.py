@@ -429,22 +429,24 @@ def run_fastmtp(args):
         "expert_down": touched * d * I * 2 + rows * I * 2 + rows * d * 4,
         "lm_head": shape.vocab * d * 2.0,
     }
-    if counted["launches"]["expert_down"] == 0:   # gate/up and down run as one launch per layer
+    fused = counted["launches"]["expert_down"] == 0   # gate/up and down run as one launch per layer
+    if fused:
         cls_bytes["expert_gate_up"] += cls_bytes["expert_down"]
     gemm_ms = {k: prof["ms"][k] for k in ("expert_gate_up", "expert_down", "qkv", "oproj", "lm_head",
                                           "attention", "draft_gemm")}
     dom = max(("expert_gate_up", "expert_down", "lm_head"), key=lambda k: prof["ms"][k])
     dur_ms = prof["ms"][dom] / max(1, prof["launches"][dom])
     achieved = cls_bytes[dom] / (dur_ms / 1000.0) / 1e9
+    label = "experts" if (fused and dom == "expert_gate_up") else dom
     traffic = None
     tpath = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if os.path.exists(tpath):
         tj = json.load(open(tpath))
         src = open(os.path.join(ROOT, "paper_2609_03181_gb300", "csrc", "gemm_tc.cu"), "rb").read()
-        if tj.get("kernel_class") == dom and tj.get("gemm_tc_sha256") == hashlib.sha256(src).hexdigest():
+        if tj.get("kernel_class") == label and tj.get("gemm_tc_sha256") == hashlib.sha256(src).hexdigest():
             traffic = tj.get("dram_bytes_per_launch")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                "traffic": traffic, "kernel": dom, "algorithmic_bytes_per_launch": cls_bytes[dom],
+                "traffic": traffic, "kernel": label, "algorithmic_bytes_per_launch": cls_bytes[dom],
                 "avg_launch_ms": dur_ms, "peak_source": peak_kind}
     routed_touched = touched - shape.n_shared
     vbytes = algorithmic_bytes(shape, B, K, statistics.mean(ctx) + (args.warmup + steps / 2) * 2, routed_touched)
