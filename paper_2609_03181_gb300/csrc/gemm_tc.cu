@@ -426,9 +426,11 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
 
   // Dense launches know their items from the arguments: the producer streams its first weight
   // tiles (never written by earlier kernels) before it waits for the previous kernel; every
-  // other thread waits before its first global access.
+  // other thread waits before its first global access.  The producer's warp skips this wait
+  // as a whole: its other lanes read nothing an earlier kernel writes, and a blocking wait on
+  // them would hold the producer lane too, so the weights would only be requested after it.
   const bool dense = (a.grp_cnt == nullptr);
-  if (!(dense && warp == 0 && lane == 0)) pdl_wait();
+  if (!(dense && warp == 0)) pdl_wait();
   // grouped launches: the per-expert tables (in the RoPE buffer, which only QKV uses)
   int* grp = reinterpret_cast<int*>(esm.rope);
   int n_items = a.n_items;
