@@ -65,7 +65,7 @@ def parse():
     p.add_argument("--sweep", action="store_true", help="run the (batch, context, K, router) grid")
     p.add_argument("--sweep-batch", default="1,4,16,64,256")
     p.add_argument("--sweep-ctx", default="1024,4096,8192")
-    p.add_argument("--sweep-k", default="1,2,3")
+    p.add_argument("--sweep-k", default="0,1,2,3", help="draft depths; 0 = greedy decoding, the speedup baseline")
     p.add_argument("--sweep-router", default="uniform,zipf")
     return p.parse_args()
 
@@ -488,6 +488,7 @@ def run_sweep(args):
 
     import synth_inputs as S
     from paper_2609_03181_gb300 import fastmtp as F
+    from paper_2609_03181_gb300 import metrics as M
 
     batches = [int(x) for x in args.sweep_batch.split(",")]
     ctxs = [int(x) for x in args.sweep_ctx.split(",")]
@@ -522,6 +523,7 @@ def run_sweep(args):
                 slots = torch.arange(B, dtype=torch.int32, device=dev)
                 c0 = torch.tensor([[p] for p in pend], dtype=torch.int32, device=dev)
                 v0 = torch.empty(B, 1, dtype=torch.int32, device=dev)
+                ar_tok_s = None   # greedy autoregressive (K=0) throughput of this (router, ctx, B)
                 for K in Ks:
                     for b in range(B):
                         eng.reset_seq(b, ctx, eng.block_table(b), pend[b])
@@ -537,16 +539,20 @@ def run_sweep(args):
                         eng.verify_step(slots, c0, v0, acc)
                         eng.accept_commit(slots, v0, acc)
                     eng.sync()
+                    # K=0 is plain greedy decoding: no draft step; each verify takes the token the
+                    # previous commit wrote (two buffers, alternating)
+                    ar_bufs = [v0, torch.empty_like(v0)]
                     with torch.cuda.stream(stream):
                         for i in range(n_all):
                             if i == args.warmup:
                                 eng.profile(2)
                             ev[i][0].record(stream)
-                            eng.draft_step(slots, K, cand)
+                            if K > 0:
+                                eng.draft_step(slots, K, cand)
                             ev[i][1].record(stream)
-                            eng.verify_step(slots, cand, vt, acc)
+                            eng.verify_step(slots, cand if K > 0 else ar_bufs[i % 2], vt, acc)
                             ev[i][2].record(stream)
-                            eng.accept_commit(slots, com, hist[i])
+                            eng.accept_commit(slots, com if K > 0 else ar_bufs[(i + 1) % 2], hist[i])
                             ev[i][3].record(stream)
                     eng.sync()
                     counted = eng.profile_read()
@@ -564,8 +570,11 @@ def run_sweep(args):
                     touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
                     vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
                     load = cnt / cnt.mean(-1, keepdim=True)
+                    tok_s = tok / (ms_step * args.steps / 1000.0)
+                    if K == 0:
+                        ar_tok_s = tok_s
                     out = {"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K,
-                           "tokens_per_s": tok / (ms_step * args.steps / 1000.0), "ms_step": ms_step,
+                           "tokens_per_s": tok_s, "ms_step": ms_step,
                            "ms_step_mean": statistics.mean(ev[i][0].elapsed_time(ev[i][3]) for i in timed),
                            "ms_draft": ms_draft, "ms_verify": ms_verify, "ms_commit": ms(2, 3),
                            "tau": tok / (args.steps * B),
@@ -576,6 +585,10 @@ def run_sweep(args):
                            "expert_load_max_over_mean": float(load.max(-1).values.mean()),
                            "expert_share_top1": float((cnt.max(-1).values / cnt.sum(-1)).mean()),
                            "steps": args.steps, "warmup": args.warmup}
+                    if ar_tok_s is not None:
+                        # the paper's speedup over greedy decoding and step cost c = tau / S
+                        sp = M.speedup_vs_ar(tok_s, ar_tok_s, out["tau"])
+                        out["speedup_vs_ar"], out["step_cost_c"] = sp["S"], sp["c"]
                     print(json.dumps(out), flush=True)
         eng.close()
         del eng

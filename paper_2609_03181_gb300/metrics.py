@@ -5,7 +5,9 @@
 * acceptance rate: the position-averaged (tau - 1) / k;
 * a_d: probability that draft depth d is accepted given that all shallower depths were;
 * c = tau / S: cost of one speculative step in units of one autoregressive step;
-* the fixed per-step overhead implied by c: t_AR * (c - 1).
+* the fixed per-step overhead implied by c: t_AR * (c - 1);
+* S = throughput at depth k over greedy decoding (k = 0) of the same setting, and the depth
+  that maximises it (the paper's k trade-off: tau grows with k, and so does c).
 """
 from __future__ import annotations
 
@@ -27,6 +29,21 @@ def acceptance_rate(tau: float, k: int) -> float:
 
 def step_cost(tau: float, speedup: float) -> float:
     return tau / speedup
+
+
+def speedup_vs_ar(tok_s: float, ar_tok_s: float, tau: float) -> Dict[str, float]:
+    """S = tok_s / ar_tok_s (committed tokens per second at depth k over greedy decoding of the
+    same batch and context) and the step cost c = tau / S it implies."""
+    S = tok_s / ar_tok_s
+    return {"S": S, "c": step_cost(tau, S)}
+
+
+def best_depth(tok_s_by_k: Dict[int, float]) -> Dict[str, float]:
+    """The draft depth with the highest throughput among the measured ones (k = 0 is greedy
+    decoding and must be present), and its speedup S over k = 0.  Ties go to the smaller depth."""
+    ar = tok_s_by_k[0]
+    k = min(tok_s_by_k, key=lambda d: (-tok_s_by_k[d], d))
+    return {"k": k, "S": tok_s_by_k[k] / ar}
 
 
 def fixed_overhead(t_ar: float, c: float) -> float:

@@ -45,3 +45,28 @@ def test_from_accept_hist():
     assert st["a_d"] == [3 / 4, 2 / 3, 1 / 2]
     assert abs(M.tau_from_conditional(st["a_d"]) - st["tau"]) < 1e-12
     assert M.from_accept_hist([0, 0, 0])["steps"] == 0
+
+
+@pytest.mark.parametrize("mode,k_best", [("eager", 3), ("graph", 1)])
+def test_best_depth_follows_the_table(mode, k_best):
+    # the table's own throughputs: eager decoding gains most at k=3, CUDA-graph decoding at k=1
+    # (the fixed per-step overhead weighs more once the autoregressive step is fast)
+    row = T[mode]
+    by_k = {0: row["ar_tok_s"], **{k: t for k, t in zip(row["k"], row["tok_s"])}}
+    best = M.best_depth(by_k)
+    assert best["k"] == k_best
+    assert abs(best["S"] - row["S"][row["k"].index(k_best)]) <= 0.006
+
+
+@pytest.mark.parametrize("mode", ["eager", "graph"])
+def test_speedup_vs_ar_reproduces_S_and_c(mode):
+    row = T[mode]
+    for i in range(len(row["k"])):
+        sp = M.speedup_vs_ar(row["tok_s"][i], row["ar_tok_s"], row["tau"][i])
+        assert abs(sp["S"] - row["S"][i]) <= 0.006
+        assert abs(sp["c"] - row["c"][i]) <= 0.015
+
+
+def test_best_depth_ties_and_greedy():
+    assert M.best_depth({0: 10.0, 1: 9.0, 2: 8.0}) == {"k": 0, "S": 1.0}
+    assert M.best_depth({0: 10.0, 1: 20.0, 2: 20.0})["k"] == 1
