@@ -13,12 +13,15 @@ whole job over all GPUs.  Prints one JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl fastmtp|reference]
   python bench.py --sweep [--sweep-batch 1,4,16,64,256] [--sweep-ctx 1024,4096,8192]
-                  [--sweep-k 1,2,3] [--sweep-router uniform,zipf]
+                  [--sweep-k 0,1,2,3] [--sweep-router uniform,zipf]
+  python bench.py --trace [--batch B --ctx-lo C --ctx-hi C]
 
 `--impl reference` times the fp64 CPU oracle on a bounded sample of the same workload (the
 method's only other implementation here); under torchrun only rank 0 runs it.  `--sweep`
 measures the step at every (batch, context, K, router) point of the verify-throughput grid,
-one JSON line per point (one GPU).
+one JSON line per point (one GPU); K = 0 is greedy decoding, the baseline of the speedup S.
+`--trace` prints the device timeline of one step (every launch and the breakdown of a verify
+layer) from the FASTMTP_TRACE=1 build of the library; it is not a timing run.
 """
 from __future__ import annotations
 
@@ -63,6 +66,9 @@ def parse():
     p.add_argument("--device-kv", action="store_true",
                    help="draw the KV prefixes on the GPU (PyTorch's generator) instead of the host Philox stream")
     p.add_argument("--sweep", action="store_true", help="run the (batch, context, K, router) grid")
+    p.add_argument("--trace", action="store_true",
+                   help="device timeline of one step (builds the FASTMTP_TRACE=1 library): every launch "
+                        "and the per-kernel breakdown of a verify layer, as JSON lines")
     p.add_argument("--sweep-batch", default="1,4,16,64,256")
     p.add_argument("--sweep-ctx", default="1024,4096,8192")
     p.add_argument("--sweep-k", default="0,1,2,3", help="draft depths; 0 = greedy decoding, the speedup baseline")
@@ -597,8 +603,68 @@ def run_sweep(args):
     print(json.dumps({"sweep_clocks": clk}), flush=True)
 
 
+def run_trace(args):
+    """One graph-replayed step (draft + verify + commit) of the bench workload, traced per CTA by
+    the FASTMTP_TRACE=1 build of the library (entry, wait return and exit times).  Not a timing
+    run: the records add a few atomics and stores per CTA.  Prints every launch, then the mean
+    verify-layer breakdown (ready -> done per kernel and the hand-over gaps), as JSON lines."""
+    os.environ["FASTMTP_TRACE"] = "1"   # read when the build module is first imported
+    import torch
+
+    from paper_2609_03181_gb300 import fastmtp as F
+    from paper_2609_03181_gb300 import trace as TR
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    shape, vw, dw, ctx, pend, kvs, dkvs = workload(args, 0)
+    B, K = args.batch, args.K
+    stream = torch.cuda.Stream(dev)
+    eng = F.Engine(vw, dw, max_batch=B, K_max=K, max_ctx=max(ctx) + (args.warmup + 4) * (K + 1) + 8, page_size=64,
+                   device=str(dev), stream=stream)
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    acc = torch.empty(B, dtype=torch.int32, device=dev)
+    com = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    ncom = torch.empty(B, dtype=torch.int32, device=dev)
+    for b in range(B):
+        eng.load_prefix(b, kvs[b], dkvs[b], pend[b])
+    c0 = torch.tensor([[p] for p in pend], dtype=torch.int32, device=dev)
+    v0 = torch.empty(B, 1, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize(dev)
+
+    def step():
+        eng.draft_step(slots, K, cand)
+        eng.verify_step(slots, cand, vt, acc)
+        eng.accept_commit(slots, com, ncom)
+
+    with torch.cuda.stream(stream):
+        eng.verify_step(slots, c0, v0, acc)
+        eng.accept_commit(slots, v0, acc)
+        for _ in range(max(1, args.warmup)):
+            step()
+    eng.sync()
+    F.trace_read(reset=True)   # drop the warm-up records
+    with torch.cuda.stream(stream):
+        step()
+    eng.sync()
+    recs = F.trace_read(reset=True)
+    ls = TR.launches(recs)
+    for g in ls:
+        print(json.dumps({"launch": g["name"], "kid": g["kid"], "grid": [g["grid_x"], g["grid_y"]], "ctas": g["ctas"],
+                          "entry_us": g["entry"], "ready_us": g["ready"], "done_us": g["done"]}), flush=True)
+    layers = TR.verify_layers(ls)
+    print(json.dumps({"trace": True, "batch": B, "K": K, "ctx": [args.ctx_lo, args.ctx_hi], "layers": args.layers,
+                      "records": int(len(recs)), "launches": len(ls), "verify_layers": len(layers),
+                      "verify_layer_us": TR.layer_breakdown(layers)}), flush=True)
+    eng.close()
+
+
 def main():
     args = parse()
+    if args.trace:
+        run_trace(args)
+        return
     if args.sweep:
         run_sweep(args)
     elif args.impl == "reference":

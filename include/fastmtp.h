@@ -214,6 +214,23 @@ typedef struct spec_profile_t {
 spec_status spec_profile(spec_ctx* ctx, int32_t mode);
 spec_status spec_profile_read(spec_ctx* ctx, spec_profile_t* out);
 
+/* Device timeline for measurement (no counterpart in the paper; it backs the per-kernel time
+ * breakdown of the step).  A library built with FASTMTP_TRACE=1 (a separate build, see the
+ * package's build script) records, for thread 0 of every CTA of every kernel, the global timer at
+ * entry, when its first wait for the previous kernel returns and, for the GEMM, attention, router
+ * and combine kernels, at exit.  spec_trace_read waits for the device, copies up to `cap`
+ * records to `host_records` (host memory, 4 x uint64 each: signature, block index, t_a, t_b;
+ * signature = kernel id << 48 | gridDim.x << 32 | gridDim.y << 16 | blockDim.x, bit 63 set on
+ * exit records, whose t_a is the exit time; other records carry entry time and wait-return
+ * time in nanoseconds), stores the count in *n_records and, if `reset`, empties the device
+ * buffers (65,536 records per kernel source file; later records are dropped).  Kernel ids:
+ * 1 + GEMM epilogue (1 plain fp32, 2 residual, 3 QKV, 4 SwiGLU, 5 scatter, 6 argmax, 7 fused
+ * experts), 16 attention, 17 router, 18 combine, 19 embedding, 20 RMSNorm, 21 commit, 22-24
+ * draft glue.  Errors: SPEC_EINVAL for a NULL n_records, cap < 0, a NULL buffer with cap > 0,
+ * or a library built without the timeline (then *n_records = 0); SPEC_ECUDA if a copy fails.
+ * Messages via spec_last_error(NULL). */
+spec_status spec_trace_read(void* host_records, int32_t cap, int32_t reset, int32_t* n_records);
+
 /* Y = X W^T like spec_gemm_bf16, computed split-K, for callers that cannot allocate device
  * memory: code running while a stream is captured into a CUDA graph (an allocation there is
  * rejected or breaks the capture), runtimes that give out device memory only from their own

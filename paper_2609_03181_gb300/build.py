@@ -1,6 +1,10 @@
 """Builds the CUDA library libfastmtp.so in-tree (paper_2609_03181_gb300/_lib/) with nvcc for
 sm_103a.  Translation units compile in parallel; the result is reused while the sources, the
-header and the flags are unchanged."""
+header and the flags are unchanged.
+
+With FASTMTP_TRACE=1 in the environment the build defines FM_TRACE (the per-CTA device
+timeline read by spec_trace_read) and goes to paper_2609_03181_gb300/_lib_trace/ instead, so the
+normal library is left as it is."""
 from __future__ import annotations
 
 import hashlib
@@ -13,11 +17,12 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
-LIBDIR = os.path.join(PKG, "_lib")
+TRACE = os.environ.get("FASTMTP_TRACE", "0") not in ("", "0")
+LIBDIR = os.path.join(PKG, "_lib_trace" if TRACE else "_lib")
 LIB = os.path.join(LIBDIR, "libfastmtp.so")
 SOURCES = ["gemm_tc.cu", "attention.cu", "small_kernels.cu", "runtime.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE]
+FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE] + (["-DFM_TRACE"] if TRACE else [])
 
 
 def _nvcc() -> str:

@@ -219,7 +219,7 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
   int* s_p0 = s_flag + 8;                                                   // [B] first query position
   int* s_slot = s_p0 + a.B;                                                 // [B] slot
   int* s_pref = s_slot + a.B;                                               // [B + 1] first item
-  pdl_trigger();
+  pdl_trigger(kTrAttn);
   if (!a.prewait) pdl_wait();
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -664,6 +664,7 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
     if (!more) break;
     w.next(s_pref);
   }
+  trace_exit();
 }
 
 cudaError_t attention_prepare() {
@@ -697,5 +698,9 @@ cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
   if (B <= 2) return attention_launch_s<kAttnStagesSmall>(a, B, s);
   return attention_launch_s<kAttnStages>(a, B, s);
 }
+
+#ifdef FM_TRACE
+FM_TRACE_READER(trace_read_attn)
+#endif
 
 }  // namespace fm

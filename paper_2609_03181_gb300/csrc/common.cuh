@@ -216,10 +216,96 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
          | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
 }
 
+// ---------------------------------------------------------------- device timeline (FM_TRACE)
+// A library built with FM_TRACE (build.py: FASTMTP_TRACE=1) records for thread 0 of every CTA
+// the global timer at kernel entry (pdl_trigger), when its first wait for the previous kernel
+// returns (pdl_wait) and, for the main kernels, at exit (trace_exit).  A record is four 64-bit
+// words {signature, block, t_a, t_b}, appended at an atomically claimed index to a buffer of
+// this translation unit; spec_trace_read collects the buffers.  signature = kernel id << 48 |
+// gridDim.x << 32 | gridDim.y << 16 | blockDim.x, bit 63 set on exit records (t_a = exit time);
+// entry/wait records carry t_a = entry, t_b = wait return.  Records past the buffer's capacity
+// are dropped.  Builds without FM_TRACE compile all of it out.
+enum TraceKernel : int {
+  kTrGemm = 1,   // + the GEMM epilogue (EPI_*)
+  kTrAttn = 16,
+  kTrRouter = 17,
+  kTrCombine = 18,
+  kTrEmbed = 19,
+  kTrNorm = 20,
+  kTrCommit = 21,
+  kTrDraftPrep = 22,
+  kTrGather = 23,
+  kTrDraftNext = 24,
+};
+#ifdef FM_TRACE
+constexpr unsigned kTraceCap = 1u << 16;
+static __device__ unsigned long long g_trace[kTraceCap][4];
+static __device__ unsigned int g_trace_n;
+__device__ __forceinline__ unsigned long long* trace_slot() {
+  __shared__ unsigned long long slot[2];   // entry time (0 once recorded), kernel id
+  return slot;
+}
+__device__ __forceinline__ bool trace_lead() { return threadIdx.x == 0 && threadIdx.y == 0 && threadIdx.z == 0; }
+__device__ __forceinline__ unsigned long long trace_sig(unsigned long long kid) {
+  return (kid << 48) | (static_cast<unsigned long long>(gridDim.x) << 32) |
+         (static_cast<unsigned long long>(gridDim.y) << 16) | blockDim.x;
+}
+__device__ __forceinline__ void trace_put(unsigned long long sig, unsigned long long t_a, unsigned long long t_b) {
+  const unsigned n = atomicAdd(&g_trace_n, 1u);
+  if (n < kTraceCap) {
+    g_trace[n][0] = sig;
+    g_trace[n][1] = blockIdx.x + 65536ull * blockIdx.y;
+    g_trace[n][2] = t_a;
+    g_trace[n][3] = t_b;
+  }
+}
+// Host side: copies up to `cap` records of this translation unit to `host`, returns how many,
+// and clears the buffer if `reset`.
+#define FM_TRACE_READER(name)                                                                   \
+  int name(unsigned long long* host, int cap, bool reset) {                                    \
+    unsigned n = 0;                                                                             \
+    if (cudaMemcpyFromSymbol(&n, g_trace_n, sizeof(n)) != cudaSuccess) return -1;              \
+    if (n > kTraceCap) n = kTraceCap;                                                           \
+    if (static_cast<int>(n) > cap) n = static_cast<unsigned>(cap);                              \
+    if (n > 0 && cudaMemcpyFromSymbol(host, g_trace, n * 4 * sizeof(unsigned long long)) != cudaSuccess) \
+      return -1;                                                                                \
+    if (reset) {                                                                                \
+      const unsigned z = 0;                                                                     \
+      if (cudaMemcpyToSymbol(g_trace_n, &z, sizeof(z)) != cudaSuccess) return -1;               \
+    }                                                                                           \
+    return static_cast<int>(n);                                                                 \
+  }
+#endif
+
 // Programmatic dependent launch: let the next kernel in the stream be scheduled now, and wait
-// until every earlier kernel has completed and its memory is visible.
-__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// until every earlier kernel has completed and its memory is visible.  `kid` names the kernel
+// in the device timeline of FM_TRACE builds.
+__device__ __forceinline__ void pdl_trigger(int kid) {
+#ifdef FM_TRACE
+  if (trace_lead()) {
+    trace_slot()[0] = globaltimer();
+    trace_slot()[1] = static_cast<unsigned long long>(kid);
+  }
+#else
+  (void)kid;
+#endif
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+#ifdef FM_TRACE
+  if (trace_lead() && trace_slot()[0] != 0ull) {
+    trace_put(trace_sig(trace_slot()[1]), trace_slot()[0], globaltimer());
+    trace_slot()[0] = 0ull;
+  }
+#endif
+}
+// Exit record of the device timeline (thread 0 of the CTA; FM_TRACE builds only).
+__device__ __forceinline__ void trace_exit() {
+#ifdef FM_TRACE
+  if (trace_lead()) trace_put(trace_sig(trace_slot()[1]) | (1ull << 63), globaltimer(), 0ull);
+#endif
+}
 
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");

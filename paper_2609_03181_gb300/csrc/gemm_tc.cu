@@ -391,7 +391,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  pdl_trigger();
+  pdl_trigger(kTrGemm + EPI);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -857,6 +857,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     tc_fence_after();
     tmem_dealloc(tmem_base, tmem_cols);
   }
+  trace_exit();
 }
 
 // ------------------------------------------------------------------ host side
@@ -1076,5 +1077,9 @@ cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStre
   }
 #undef FM_CASE
 }
+
+#ifdef FM_TRACE
+FM_TRACE_READER(trace_read_gemm)
+#endif
 
 }  // namespace fm

@@ -135,6 +135,13 @@ cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream
 int num_sms();
 // Sets the message spec_last_error(NULL) returns in this thread.
 void set_thread_error(const std::string& msg);
+#ifdef FM_TRACE
+// Device-timeline buffers of the three kernel translation units (FM_TRACE builds): copy up to
+// `cap` records (4 x u64 each) to host memory, return the count (-1 on a CUDA error).
+int trace_read_gemm(unsigned long long* host, int cap, bool reset);
+int trace_read_attn(unsigned long long* host, int cap, bool reset);
+int trace_read_small(unsigned long long* host, int cap, bool reset);
+#endif
 // Kernel attributes (dynamic shared memory limits) set once, before any launch or capture.
 cudaError_t gemm_prepare();
 cudaError_t attention_prepare();

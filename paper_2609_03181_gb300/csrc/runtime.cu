@@ -981,6 +981,26 @@ extern "C" spec_status spec_sync(spec_ctx* ctx) {
   return SPEC_OK;
 }
 
+extern "C" spec_status spec_trace_read(void* host_records, int32_t cap, int32_t reset, int32_t* n_records) {
+  if (n_records == nullptr || cap < 0 || (cap > 0 && host_records == nullptr))
+    return fail(nullptr, SPEC_EINVAL, "spec_trace_read: n_records NULL, cap < 0 or NULL buffer");
+  *n_records = 0;
+#ifdef FM_TRACE
+  unsigned long long* out = static_cast<unsigned long long*>(host_records);
+  int n = 0;
+  for (auto rd : {fm::trace_read_gemm, fm::trace_read_attn, fm::trace_read_small}) {
+    const int got = rd(out + 4 * static_cast<size_t>(n), cap - n, reset != 0);
+    if (got < 0) return fail(nullptr, SPEC_ECUDA, "spec_trace_read: copy of the trace buffers failed");
+    n += got;
+  }
+  *n_records = n;
+  return SPEC_OK;
+#else
+  (void)reset;
+  return fail(nullptr, SPEC_EINVAL, "spec_trace_read: the library was built without the device timeline (FASTMTP_TRACE=1)");
+#endif
+}
+
 extern "C" spec_status spec_profile(spec_ctx* ctx, int32_t mode) {
   if (ctx == nullptr) return fail(nullptr, SPEC_EINVAL, "ctx is NULL");
   if (mode < 0 || mode > 2) return fail(ctx, SPEC_EINVAL, "mode must be 0, 1 or 2");

@@ -50,7 +50,7 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
                                                          const bf16* gain, float eps, float* h, bf16* xn, int* pos,
                                                          long long* kv_rowoff, int stage_R, int n_slots, int* err,
                                                          int* zero, int n_zero, int* zero2, int n_zero2) {
-  pdl_trigger();
+  pdl_trigger(kTrEmbed);
   pdl_wait();
   if (blockIdx.x == 0) {   // the step's per-expert row counters and tile counters start from zero
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
@@ -92,7 +92,7 @@ cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, c
 
 // ---------------------------------------------------------------- RMSNorm
 __global__ void __launch_bounds__(128) rmsnorm_kernel(const float* x, const bf16* gain, float eps, bf16* out) {
-  pdl_trigger();
+  pdl_trigger(kTrNorm);
   pdl_wait();
   __shared__ float red[4];
   const size_t row = blockIdx.x;
@@ -124,7 +124,7 @@ constexpr int kRouteStride = kD + 32;   // bf16 per staged row: rows 64 bytes ap
 constexpr int kMaxT = 2048;
 
 __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ RouteArgs a) {
-  pdl_trigger();
+  pdl_trigger(kTrRouter);
   __shared__ __align__(16) bf16 xs[kRouteRows * kRouteStride];   // the rounded rows
   __shared__ float lg[kRouteRows][kE];                           // logits, then probabilities
   __shared__ int dst[kRouteRows][kTopK];                         // input row of each selection
@@ -274,6 +274,7 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
     const uint4 x = *reinterpret_cast<const uint4*>(xs + r * kRouteStride + 8 * v);
     *reinterpret_cast<uint4*>(a.x_sorted + static_cast<size_t>(dst[r][sel % kTopK]) * kD + 8 * v) = x;
   }
+  trace_exit();
 }
 
 cudaError_t router_prepare() { return cudaSuccess; }
@@ -287,7 +288,7 @@ cudaError_t router_launch(const RouteArgs& a, cudaStream_t s) {
 // h += sum_{s<6} gate_s * y_s + y_shared0 + y_shared1 (fixed slot order), then RMSNorm -> out.
 __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, const float* gate, const bf16* gain,
                                                       float eps, bf16* out) {
-  pdl_trigger();
+  pdl_trigger(kTrCombine);
   pdl_wait();
   constexpr int NT = 256, EPT = kD / NT;
   __shared__ float red[NT / 32];
@@ -314,6 +315,7 @@ __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, 
     h[t * kD + threadIdx.x + NT * k] = x[k];
   }
   norm_row_store_t<NT>(x, gain, eps, out + t * kD, red);
+  trace_exit();
 }
 
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,
@@ -334,7 +336,7 @@ __global__ void __launch_bounds__(256) commit_kernel(int R, int stage_R, int Bma
                                                      int max_pages, int* seq_len, int* pending, const bf16* b_ws,
                                                      bf16* draft_b, int* draft_tok, int* draft_n, int* committed,
                                                      int* n_committed, int* tickets, int* err) {
-  pdl_trigger();
+  pdl_trigger(kTrCommit);
   pdl_wait();
   __shared__ int s_last;
   const int b = blockIdx.x, l = blockIdx.y, slot = slots[b];
@@ -430,7 +432,7 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
                                                          int* pos, long long* kv_rowoff, int* last_row, int page_size,
                                                          const int* block_table, int max_pages, int n_pages, int* cand,
                                                          int cand_ld, int n_slots, int* err) {
-  pdl_trigger();
+  pdl_trigger(kTrDraftPrep);
   pdl_wait();
   __shared__ float red[4];
   const int b = blockIdx.x / R, i = blockIdx.x % R, row = blockIdx.x;
@@ -496,7 +498,7 @@ cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len
 }
 
 __global__ void gather_rows_kernel(const float* src, const int* rows, float* dst) {
-  pdl_trigger();
+  pdl_trigger(kTrGather);
   pdl_wait();
   const int b = blockIdx.x;
   const float4* s = reinterpret_cast<const float4*>(src + static_cast<size_t>(rows[b]) * kD);
@@ -518,7 +520,7 @@ __global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_
                                                          const bf16* enorm, const bf16* hnorm, float eps, bf16* dcat,
                                                          int* pos, long long* kv_rowoff, long long dstage_seq_stride,
                                                          int* cand, int cand_ld) {
-  pdl_trigger();
+  pdl_trigger(kTrDraftNext);
   pdl_wait();
   __shared__ float red[4];
   __shared__ int s_tok;
@@ -561,5 +563,9 @@ cudaError_t draft_next_launch(unsigned long long* am_key, int vocab, int* err, i
   return launch_pdl(draft_next_kernel, dim3(B), dim3(128), 0, s, am_key, vocab, err, k, K, slots, n_slots, seq_len, u, embed, enorm, hnorm,
                     eps, dcat, pos, kv_rowoff, dstage_seq_stride, cand, cand_ld);
 }
+
+#ifdef FM_TRACE
+FM_TRACE_READER(trace_read_small)
+#endif
 
 }  // namespace fm

@@ -20,8 +20,8 @@ WS_B, WS_ROUTE_IDX, WS_ROUTE_GATE, WS_EXPERT_CNT, WS_DRAFT_U, WS_HIDDEN = range(
 # Public entry points, in the order include/fastmtp.h declares them.
 ENTRY_POINTS = ["spec_init", "spec_seq_reset", "spec_seq_set_draft_rows", "draft_step", "verify_step",
                 "accept_commit", "spec_sync", "spec_seq_state", "spec_read_workspace", "spec_gemm_bf16",
-                "spec_profile", "spec_profile_read", "spec_gemm_bf16_noalloc", "spec_destroy",
-                "spec_last_error"]
+                "spec_profile", "spec_profile_read", "spec_trace_read", "spec_gemm_bf16_noalloc",
+                "spec_destroy", "spec_last_error"]
 KERNEL_CLASSES = ["embed", "qkv", "attention", "oproj", "router", "permute", "expert_gate_up", "expert_down",
                   "combine", "lm_head", "argmax", "commit", "draft_gemm", "draft_misc"]
 
@@ -82,6 +82,7 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
         "spec_gemm_bf16": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
         "spec_profile": (ctypes.c_int, [P, I32]),
         "spec_profile_read": (ctypes.c_int, [P, ctypes.POINTER(SpecProfile)]),
+        "spec_trace_read": (ctypes.c_int, [P, I32, I32, ctypes.POINTER(I32)]),
         "spec_gemm_bf16_noalloc": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
         "spec_destroy": (None, [P]),
         "spec_last_error": (ctypes.c_char_p, [P]),
@@ -115,6 +116,20 @@ def gemm_bf16(X: torch.Tensor, W: torch.Tensor, stream: Optional[torch.cuda.Stre
     if st != SPEC_OK:
         raise FastMTPError(st, lib.spec_last_error(None).decode())
     return Y
+
+
+def trace_read(reset: bool = True, cap: int = 3 << 16):
+    """The device-timeline records of a FASTMTP_TRACE=1 build (spec_trace_read) as a uint64
+    numpy array [n][4]: signature, block, t_a, t_b (see include/fastmtp.h)."""
+    import numpy as np
+
+    lib = load_library()
+    buf = np.zeros((cap, 4), dtype=np.uint64)
+    n = ctypes.c_int32(0)
+    st = lib.spec_trace_read(buf.ctypes.data, cap, 1 if reset else 0, ctypes.byref(n))
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+    return buf[: n.value].copy()
 
 
 def gemm_bf16_noalloc(X: torch.Tensor, W: torch.Tensor, Y: torch.Tensor,
