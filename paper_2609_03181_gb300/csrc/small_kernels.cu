@@ -137,20 +137,25 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
   uint4 wq[kSteps];
 #pragma unroll
   for (int c = 0; c < kEarly; ++c) wq[c] = wrow[4 * c];
+  uint2 gq[kD / 128];   // norm gain (bf16, also a weight), lane's columns 4 (lane + 32 k) .. + 3
+#pragma unroll
+  for (int k = 0; k < kD / 128; ++k) gq[k] = *reinterpret_cast<const uint2*>(a.gain + 4 * (lane + 32 * k));
   pdl_wait();
   const int t0 = blockIdx.x * kRouteCtaRows;
   const int nr = min(kRouteCtaRows, a.T - t0);
-  // RMSNorm: warp w takes rows w and w + 8; a lane sums its 40 squares of a row in order, then
-  // a warp tree
+  // RMSNorm: warp w takes rows w and w + 8 of the 16-row MMA tile, of which the first nr are
+  // token rows and the rest zeros; a lane sums its 40 squares of a row in order, then a warp tree
   {
-    uint2 gq[kD / 128];   // gain (bf16), lane's columns 4 (lane + 32 k) .. + 3
-#pragma unroll
-    for (int k = 0; k < kD / 128; ++k) gq[k] = *reinterpret_cast<const uint2*>(a.gain + 4 * (lane + 32 * k));
 #pragma unroll
     for (int h2 = 0; h2 < 2; ++h2) {
       const int r = warp + 8 * h2;
       bf16* xr = xs + r * kRouteStride;
-      const float4* hr = reinterpret_cast<const float4*>(a.h + static_cast<size_t>(t0 + min(r, nr - 1)) * kD);
+      if (r >= nr) {   // a padding row of the MMA tile (warp-uniform): zeros, no load
+#pragma unroll
+        for (int k = 0; k < kD / 128; ++k) *reinterpret_cast<uint2*>(xr + 4 * (lane + 32 * k)) = make_uint2(0u, 0u);
+        continue;
+      }
+      const float4* hr = reinterpret_cast<const float4*>(a.h + static_cast<size_t>(t0 + r) * kD);
       float4 v[kD / 128];
 #pragma unroll
       for (int k = 0; k < kD / 128; ++k) v[k] = hr[lane + 32 * k];
@@ -170,9 +175,8 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
         o4[1] = __float2bfloat16(v[k].y * inv * __high2float(g01));
         o4[2] = __float2bfloat16(v[k].z * inv * __low2float(g23));
         o4[3] = __float2bfloat16(v[k].w * inv * __high2float(g23));
-        if (r < nr) *reinterpret_cast<uint2*>(xo + i) = *reinterpret_cast<const uint2*>(o4);
-        // rows past the launch's last are zero in the MMA input
-        *reinterpret_cast<uint2*>(xr + i) = (r < nr) ? *reinterpret_cast<const uint2*>(o4) : make_uint2(0u, 0u);
+        *reinterpret_cast<uint2*>(xo + i) = *reinterpret_cast<const uint2*>(o4);
+        *reinterpret_cast<uint2*>(xr + i) = *reinterpret_cast<const uint2*>(o4);
       }
     }
   }
