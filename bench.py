@@ -69,6 +69,7 @@ def parse():
     p.add_argument("--trace", action="store_true",
                    help="device timeline of one step (builds the FASTMTP_TRACE=1 library): every launch "
                         "and the per-kernel breakdown of a verify layer, as JSON lines")
+    p.add_argument("--trace-out", default="", help="with --trace: also save the raw records (.npy, uint64 [n][4])")
     p.add_argument("--sweep-batch", default="1,4,16,64,256")
     p.add_argument("--sweep-ctx", default="1024,4096,8192")
     p.add_argument("--sweep-k", default="0,1,2,3", help="draft depths; 0 = greedy decoding, the speedup baseline")
@@ -649,6 +650,9 @@ def run_trace(args):
         step()
     eng.sync()
     recs = F.trace_read(reset=True)
+    if args.trace_out:
+        import numpy as np
+        np.save(args.trace_out, recs)
     ls = TR.launches(recs)
     for g in ls:
         print(json.dumps({"launch": g["name"], "kid": g["kid"], "grid": [g["grid_x"], g["grid_y"]], "ctas": g["ctas"],

@@ -2,6 +2,12 @@
 (entry, wait return, exit; include/fastmtp.h) to launches and the time breakdown of one verify
 layer.
 
+Grouping: a kernel is launched only after every CTA of the previous kernel has entered (each
+triggers its dependents at entry), so no other kernel's CTA enters between two CTA entries of
+one launch; the records of one kernel are split into launches exactly where another kernel's
+entry falls between two of theirs.  This holds for launches that run in several waves, whose
+late CTAs enter long after the first ones.
+
 A launch's `ready` time is the first wait return of its CTAs (the moment the previous kernel's
 results are visible to it), its `done` time the last exit record of its CTAs.  The layer
 breakdown gives, for each kernel of a verify layer, ready -> done and the hand-over from the
@@ -21,7 +27,6 @@ KERNEL_NAMES = {1: "gemm_f32", 2: "gemm_resid", 3: "gemm_qkv", 4: "gemm_swiglu",
                 24: "draft_next"}
 # the kernels of one verify layer, in launch order (QKV, attention, O-proj, router, experts, combine)
 VERIFY_LAYER = (3, 16, 2, 17, 7, 18)
-GAP_NS = 3000   # wait returns of one launch lie closer together than this
 
 
 def _sig_fields(sig: int) -> Dict[str, int]:
@@ -29,7 +34,7 @@ def _sig_fields(sig: int) -> Dict[str, int]:
             "block": sig & 0xFFFF}
 
 
-def launches(records: np.ndarray, gap_ns: int = GAP_NS) -> List[Dict[str, object]]:
+def launches(records: np.ndarray) -> List[Dict[str, object]]:
     """Groups the records into launches, in the order their inputs became ready.  Times are in
     microseconds from the first entry of the trace."""
     r = np.asarray(records, dtype=np.uint64).reshape(-1, 4)
@@ -39,13 +44,20 @@ def launches(records: np.ndarray, gap_ns: int = GAP_NS) -> List[Dict[str, object
     is_exit = np.array([int(s) & EXIT_BIT != 0 for s in sig], dtype=bool)
     base = np.array([int(s) & ~EXIT_BIT for s in sig], dtype=object)
     t0 = int(r[~is_exit, 2].min()) if (~is_exit).any() else int(r[:, 2].min())
+    entries = r[~is_exit, 2].astype(np.int64)
+    entry_sig = base[~is_exit]
     out = []
-    for s in sorted(set(base[~is_exit])):
+    for s in sorted(set(entry_sig)):
         m = (base == s) & ~is_exit
         rows = r[m]
-        rows = rows[np.argsort(rows[:, 3].astype(np.int64), kind="stable")]
-        tb = rows[:, 3].astype(np.int64)
-        cuts = [0] + [i for i in range(1, len(tb)) if tb[i] - tb[i - 1] > gap_ns] + [len(tb)]
+        rows = rows[np.argsort(rows[:, 2].astype(np.int64), kind="stable")]
+        ta = rows[:, 2].astype(np.int64)
+        others = np.sort(entries[entry_sig != s])
+        # a cut between consecutive entries of this kernel if another kernel's entry lies
+        # strictly between them
+        lo = np.searchsorted(others, ta[:-1], side="right")
+        hi = np.searchsorted(others, ta[1:], side="left")
+        cuts = [0] + [i + 1 for i in np.nonzero(hi > lo)[0].tolist()] + [len(ta)]
         ex = np.sort(r[(base == s) & is_exit][:, 2].astype(np.int64))
         groups = []
         for j in range(len(cuts) - 1):

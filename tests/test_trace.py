@@ -52,6 +52,30 @@ def test_verify_layers_and_breakdown():
     assert abs(b["layer"] - 56.4) < 1e-9
 
 
+def test_launch_in_two_waves_stays_one_launch():
+    # 152 CTAs enter at once, 104 more only as the first ones leave (their waits return at entry,
+    # far from the first wave's); a second kernel enters after the last of them
+    recs = []
+    for c in range(256):
+        t_in = 1_000 if c < 152 else 20_000 + 100 * c
+        recs.append([sig(17, 256, 256), c, t_in, max(t_in, 5_000)])
+    for c in range(4):
+        recs.append([sig(7, 152, 192), c, 60_000 + c, 61_000])
+    ls = TR.launches(np.array(recs, dtype=np.uint64))
+    assert [(g["name"], g["ctas"]) for g in ls] == [("router", 256), ("experts", 4)]
+
+
+def test_same_kernel_split_only_by_another_kernels_entry():
+    recs = []
+    for c in range(3):
+        recs.append([sig(20, 3, 128), c, 1_000 + c, 2_000])        # RMSNorm launch 1
+    recs.append([sig(1, 10, 192), 0, 2_500, 3_000])                # a GEMM in between
+    for c in range(3):
+        recs.append([sig(20, 3, 128), c, 2_600 + c, 4_000])        # RMSNorm launch 2, 1.6 us later
+    ls = TR.launches(np.array(recs, dtype=np.uint64))
+    assert [(g["name"], g["ctas"]) for g in ls] == [("rmsnorm", 3), ("gemm_f32", 1), ("rmsnorm", 3)]
+
+
 def test_empty_trace():
     assert TR.launches(np.zeros((0, 4), dtype=np.uint64)) == []
     assert TR.verify_layers([]) == []
