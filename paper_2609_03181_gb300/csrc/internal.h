@@ -190,7 +190,8 @@ cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, c
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
                               int* err, int* zero, int n_zero, int* zero2, int n_zero2, cudaStream_t s);
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
-// Router (+ expert grouping by the last CTA) and the permute row gather.
+// Router: RMSNorm, logits, softmax, top-6; each selection claims the next row of its expert
+// (atomic add on counts) and copies the token's rounded row into the expert's input region.
 struct RouteArgs {
   const float* h; const bf16* gain; float eps; const bf16* wr; const float* bias;
   bf16* xn; int* idx; float* gate; int* err; int T;

@@ -48,3 +48,16 @@ def test_host_side_validation_without_gpu():
     assert lib.accept_commit(None, 1, None, None, None) == F.SPEC_EINVAL
     assert lib.spec_gemm_bf16(None, None, None, 1, 1, 64, None) == F.SPEC_EINVAL
     lib.spec_destroy(None)
+
+
+def test_trace_read_without_the_timeline_build():
+    # the normal build has no device timeline: spec_trace_read says so (no CUDA call), after its
+    # argument checks
+    lib = F.load_library()
+    n = ctypes.c_int32(7)
+    assert lib.spec_trace_read(None, 0, 1, None) == F.SPEC_EINVAL
+    assert lib.spec_trace_read(None, 4, 1, ctypes.byref(n)) == F.SPEC_EINVAL   # NULL buffer with cap > 0
+    assert lib.spec_trace_read(None, -1, 1, ctypes.byref(n)) == F.SPEC_EINVAL
+    buf = (ctypes.c_uint64 * 8)()
+    assert lib.spec_trace_read(buf, 2, 1, ctypes.byref(n)) == F.SPEC_EINVAL
+    assert n.value == 0 and b"FASTMTP_TRACE" in lib.spec_last_error(None)
