@@ -11,7 +11,9 @@
 """
 from __future__ import annotations
 
-from typing import Dict, Sequence
+import json
+import math
+from typing import Dict, Iterable, Sequence, Tuple
 
 
 def tau_from_conditional(a: Sequence[float]) -> float:
@@ -44,6 +46,38 @@ def best_depth(tok_s_by_k: Dict[int, float]) -> Dict[str, float]:
     ar = tok_s_by_k[0]
     k = min(tok_s_by_k, key=lambda d: (-tok_s_by_k[d], d))
     return {"k": k, "S": tok_s_by_k[k] / ar}
+
+
+class DepthPolicy:
+    """Draft depth by batch size and context length, from measured throughputs: for every
+    measured (batch, context) the depth with the highest committed tokens/s (best_depth); a
+    query takes the nearest measured point, by log2 distance in batch first, then in context.
+    Built from the JSON lines of `bench.py --sweep` (one router mode) or from a table
+    {(batch, ctx): {K: tok_s}} that includes K = 0."""
+
+    def __init__(self, table: Dict[Tuple[int, int], Dict[int, float]]):
+        self.best = {key: best_depth(by_k)["k"] for key, by_k in table.items() if 0 in by_k}
+        if not self.best:
+            raise ValueError("no measured point has the greedy (K = 0) baseline")
+
+    @classmethod
+    def from_sweep_lines(cls, lines: Iterable[str], router: str = "uniform") -> "DepthPolicy":
+        table: Dict[Tuple[int, int], Dict[int, float]] = {}
+        for line in lines:
+            line = line.strip()
+            if not line:
+                continue
+            d = json.loads(line)
+            if not d.get("sweep") or d.get("router") != router:
+                continue
+            table.setdefault((int(d["batch"]), int(d["ctx"])), {})[int(d["K"])] = float(d["tokens_per_s"])
+        return cls(table)
+
+    def choose(self, batch: int, ctx: int) -> int:
+        def dist(key):
+            b, c = key
+            return (abs(math.log2(b) - math.log2(max(1, batch))), abs(math.log2(c) - math.log2(max(1, ctx))), b, c)
+        return self.best[min(self.best, key=dist)]
 
 
 def fixed_overhead(t_ar: float, c: float) -> float:

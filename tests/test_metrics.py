@@ -70,3 +70,33 @@ def test_speedup_vs_ar_reproduces_S_and_c(mode):
 def test_best_depth_ties_and_greedy():
     assert M.best_depth({0: 10.0, 1: 9.0, 2: 8.0}) == {"k": 0, "S": 1.0}
     assert M.best_depth({0: 10.0, 1: 20.0, 2: 20.0})["k"] == 1
+
+
+def _line(router, B, ctx, K, tok_s):
+    return json.dumps({"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K, "tokens_per_s": tok_s})
+
+
+def test_depth_policy_from_sweep_lines():
+    lines = [_line("uniform", 1, 1024, 0, 100.0), _line("uniform", 1, 1024, 2, 160.0), _line("uniform", 1, 1024, 3, 150.0),
+             _line("uniform", 64, 1024, 0, 100.0), _line("uniform", 64, 1024, 3, 190.0),
+             _line("uniform", 64, 8192, 0, 100.0), _line("uniform", 64, 8192, 1, 120.0),
+             _line("zipf", 1, 1024, 0, 100.0), _line("zipf", 1, 1024, 1, 300.0), json.dumps({"sweep_clocks": {}})]
+    pol = M.DepthPolicy.from_sweep_lines(lines)
+    assert pol.choose(1, 1024) == 2
+    assert pol.choose(2, 900) == 2           # nearest batch in log2 is 1
+    assert pol.choose(48, 1000) == 3         # batch 64, context 1024
+    assert pol.choose(64, 6000) == 1         # batch 64, nearer context 8192
+    assert M.DepthPolicy.from_sweep_lines(lines, router="zipf").choose(1, 1) == 1
+
+
+def test_depth_policy_on_the_papers_table():
+    # batch 1 only: eager decoding takes k = 3, CUDA-graph decoding k = 1 (the table's own S)
+    for mode, k in (("eager", 3), ("graph", 1)):
+        row = T[mode]
+        pol = M.DepthPolicy({(1, 1): {0: row["ar_tok_s"], **dict(zip(row["k"], row["tok_s"]))}})
+        assert pol.choose(1, 4096) == k
+
+
+def test_depth_policy_needs_the_greedy_baseline():
+    with pytest.raises(ValueError):
+        M.DepthPolicy({(1, 1024): {1: 10.0, 2: 12.0}})
