@@ -47,17 +47,19 @@ FALLBACK_HBM_GBS = 6800.0
 
 
 def parse():
+    import synth_inputs as S
+    c1, c4 = S.CONFIGS["cfg1"], S.CONFIGS["cfg4"]
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", default="fastmtp", choices=["fastmtp", "reference"])
-    p.add_argument("--batch", type=int, default=8)
-    p.add_argument("--K", type=int, default=3)
-    p.add_argument("--ctx-lo", type=int, default=768)
-    p.add_argument("--ctx-hi", type=int, default=1024)
-    p.add_argument("--layers", type=int, default=12)
-    p.add_argument("--seed", type=int, default=1)
+    p.add_argument("--batch", type=int, default=c1.batch)
+    p.add_argument("--K", type=int, default=c1.K)
+    p.add_argument("--ctx-lo", type=int, default=c1.ctx_lo)
+    p.add_argument("--ctx-hi", type=int, default=c1.ctx_hi)
+    p.add_argument("--layers", type=int, default=c1.n_layers)
+    p.add_argument("--seed", type=int, default=c1.seed)
     p.add_argument("--cpu-budget-s", type=float, default=20.0, help="CPU seconds of the oracle sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
@@ -70,10 +72,11 @@ def parse():
                    help="device timeline of one step (builds the FASTMTP_TRACE=1 library): every launch "
                         "and the per-kernel breakdown of a verify layer, as JSON lines")
     p.add_argument("--trace-out", default="", help="with --trace: also save the raw records (.npy, uint64 [n][4])")
-    p.add_argument("--sweep-batch", default="1,4,16,64,256")
-    p.add_argument("--sweep-ctx", default="1024,4096,8192")
-    p.add_argument("--sweep-k", default="0,1,2,3", help="draft depths; 0 = greedy decoding, the speedup baseline")
-    p.add_argument("--sweep-router", default="uniform,zipf")
+    p.add_argument("--sweep-batch", default=",".join(map(str, c4.grid["batch"])))
+    p.add_argument("--sweep-ctx", default=",".join(map(str, c4.grid["ctx"])))
+    p.add_argument("--sweep-k", default=",".join(map(str, c4.grid["K"])),
+                   help="draft depths; 0 = greedy decoding, the speedup baseline")
+    p.add_argument("--sweep-router", default=",".join(c4.grid["router"]))
     return p.parse_args()
 
 
