@@ -48,7 +48,7 @@ FALLBACK_HBM_GBS = 6800.0
 
 def parse():
     import synth_inputs as S
-    c1, c4 = S.CONFIGS["cfg1"], S.CONFIGS["cfg4"]
+    c1, c4 = S.WORKLOADS["verify_12l_b8_ctx768_1024"], S.WORKLOADS["sweep_12l_b1_256_ctx1024_8192"]
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=20)

@@ -50,7 +50,7 @@ class ModelShape:
 
 @dataclass(frozen=True)
 class Workload:
-    """One of the five workload configurations (cfg0..cfg4): sizes, seeds and the input recipe
+    """One of the five workloads of the verify/draft step: sizes, seeds and the input recipe
     only.  ctx is the committed context range U[ctx_lo, ctx_hi] per sequence (the first
     `visual` positions stand in for the page's visual tokens); `draft_only` runs the draft block
     alone; `gen_tokens` is the number of committed tokens a loop workload generates; `grid`
@@ -69,17 +69,17 @@ class Workload:
     grid: Optional[dict] = None
 
 
-# The five workload configurations of the verify/draft step (seeded, synthetic).
-CONFIGS = {
-    "cfg0": Workload("one decoder layer, verify step", n_layers=1, batch=1, K=3, ctx_lo=512, ctx_hi=512,
+# The five workloads of the verify/draft step (seeded, synthetic), named by what they are.
+WORKLOADS = {
+    "one_layer_b1_ctx512": Workload("one decoder layer, verify step", n_layers=1, batch=1, K=3, ctx_lo=512, ctx_hi=512,
                      seed=0, p_match=0.7),
-    "cfg1": Workload("12-layer verifier, verify step", n_layers=12, batch=8, K=3, ctx_lo=768, ctx_hi=1024,
+    "verify_12l_b8_ctx768_1024": Workload("12-layer verifier, verify step", n_layers=12, batch=8, K=3, ctx_lo=768, ctx_hi=1024,
                      seed=1, visual=256),
-    "cfg2": Workload("draft block alone", n_layers=0, batch=32, K=3, ctx_lo=2048, ctx_hi=2048, seed=2,
+    "draft_block_b32_ctx2048": Workload("draft block alone", n_layers=0, batch=32, K=3, ctx_lo=2048, ctx_hi=2048, seed=2,
                      draft_only=True),
-    "cfg3": Workload("speculative decode loop, verifier + draft block", n_layers=12, batch=64, K=3,
+    "loop_12l_b64_ctx1024_4096": Workload("speculative decode loop, verifier + draft block", n_layers=12, batch=64, K=3,
                      ctx_lo=1024, ctx_hi=4096, seed=3, gen_tokens=512),
-    "cfg4": Workload("verify-throughput sweep", n_layers=12, batch=256, K=3, ctx_lo=1024, ctx_hi=8192, seed=4,
+    "sweep_12l_b1_256_ctx1024_8192": Workload("verify-throughput sweep", n_layers=12, batch=256, K=3, ctx_lo=1024, ctx_hi=8192, seed=4,
                      grid={"batch": (1, 4, 16, 64, 256), "ctx": (1024, 4096, 8192), "K": (0, 1, 2, 3),
                            "router": ("uniform", "zipf"), "zipf_s": 1.2, "seeds": (4, 5, 6, 7, 8)}),
 }

@@ -67,7 +67,7 @@ def run_draft_case(B, ctx, K, seed, vocab=129280):
     return checked, skipped
 
 
-def test_draft_block_cfg2():
+def test_draft_block_b32_ctx2048():
     run_draft_case(B=32, ctx=2048, K=3, seed=2)
 
 

@@ -66,7 +66,7 @@ def decode(eng, slots, pend, K_step):
     return out, (torch.stack(ms).cpu().numpy() if ms else np.zeros(0))
 
 
-def test_cfg3_speculative_equals_greedy_at_scale():
+def test_speculative_equals_greedy_b64_512_tokens():
     shape = S.ModelShape()
     vw, dw, _ = S.successor_weights(shape, SEED, 7.0)
     ctx = [int(c) for c in S.integers(SEED, "ctx", B, 1024, 4096)]

@@ -119,7 +119,7 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
     return int(sure.sum()), int((~sure).sum())
 
 
-def test_verify_one_layer_cfg0():
+def test_verify_one_layer_b1_ctx512():
     shape = S.ModelShape(n_layers=1)
     run_verify_case(shape, 0, [512], K=3)
 
@@ -130,7 +130,7 @@ def test_verify_ragged_small_contexts():
     run_verify_case(shape, 5, [0, 1, 63, 64, 129, 200], K=2)
 
 
-def test_verify_twelve_layers_cfg1():
+def test_verify_twelve_layers_b8_ctx768_1024():
     shape = S.ModelShape()
     ctx = [int(c) for c in S.integers(1, "ctx", 8, 768, 1024)]
     run_verify_case(shape, 1, ctx, K=3, gain_std=0.0)

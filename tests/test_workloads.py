@@ -1,28 +1,33 @@
-"""The workload presets (synth_inputs.CONFIGS) and bench.py's defaults agree: the bench's step
-is cfg1 and its sweep grid cfg4."""
+"""The workload presets (synth_inputs.WORKLOADS) and bench.py's defaults agree: the bench's
+step is the 12-layer B=8 verify workload and its sweep grid the sweep workload's axes."""
 import sys
 
 import synth_inputs as S
 
+STEP, SWEEP = "verify_12l_b8_ctx768_1024", "sweep_12l_b1_256_ctx1024_8192"
 
-def test_bench_defaults_are_cfg1_and_cfg4(monkeypatch):
+
+def test_bench_defaults_are_the_step_and_sweep_workloads(monkeypatch):
     monkeypatch.setattr(sys, "argv", ["bench.py"])
     import bench
     a = bench.parse()
-    c1, c4 = S.CONFIGS["cfg1"], S.CONFIGS["cfg4"]
-    assert (a.batch, a.K, a.ctx_lo, a.ctx_hi, a.layers, a.seed) == (c1.batch, c1.K, c1.ctx_lo, c1.ctx_hi,
-                                                                   c1.n_layers, c1.seed)
-    assert [int(x) for x in a.sweep_batch.split(",")] == list(c4.grid["batch"])
-    assert [int(x) for x in a.sweep_ctx.split(",")] == list(c4.grid["ctx"])
-    assert [int(x) for x in a.sweep_k.split(",")] == list(c4.grid["K"])
-    assert a.sweep_router.split(",") == list(c4.grid["router"])
+    st, sw = S.WORKLOADS[STEP], S.WORKLOADS[SWEEP]
+    assert (a.batch, a.K, a.ctx_lo, a.ctx_hi, a.layers, a.seed) == (st.batch, st.K, st.ctx_lo, st.ctx_hi,
+                                                                   st.n_layers, st.seed)
+    assert [int(x) for x in a.sweep_batch.split(",")] == list(sw.grid["batch"])
+    assert [int(x) for x in a.sweep_ctx.split(",")] == list(sw.grid["ctx"])
+    assert [int(x) for x in a.sweep_k.split(",")] == list(sw.grid["K"])
+    assert a.sweep_router.split(",") == list(sw.grid["router"])
 
 
 def test_presets_are_consistent():
-    assert sorted(S.CONFIGS) == ["cfg0", "cfg1", "cfg2", "cfg3", "cfg4"]
-    for name, w in S.CONFIGS.items():
+    assert len(S.WORKLOADS) == 5
+    for name, w in S.WORKLOADS.items():
         assert 1 <= w.batch <= 256 and 1 <= w.K <= 7 and 1 <= w.ctx_lo <= w.ctx_hi
         assert w.ctx_hi + w.K + 1 <= S.ModelShape().max_position
         assert w.draft_only == (w.n_layers == 0)
-    assert S.CONFIGS["cfg4"].grid["K"][0] == 0          # the greedy baseline of the speedup
-    assert S.CONFIGS["cfg3"].gen_tokens == 512
+        # the name carries the batch and the context range
+        assert f"_b{w.batch}_" in name or f"_b1_{w.batch}_" in name, name
+        assert f"ctx{w.ctx_lo}" in name, name
+    assert S.WORKLOADS[SWEEP].grid["K"][0] == 0          # the greedy baseline of the speedup
+    assert S.WORKLOADS["loop_12l_b64_ctx1024_4096"].gen_tokens == 512
