@@ -1,4 +1,4 @@
-"""End-to-end speculative greedy decoding at the benchmark spec's loop size: the 12-layer MoE
+"""End-to-end speculative greedy decoding at serving scale: the 12-layer MoE
 verifier plus the FastMTP draft block, batch 64, prompt contexts U[1024, 4096], 512 generated
 tokens per sequence, acceptance-tuned weights (successor map, beta/alpha = 7).  The committed
 streams must equal plain greedy decoding token for token (Sec. 3.1: lossless), with drafts
