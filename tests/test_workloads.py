@@ -31,3 +31,17 @@ def test_presets_are_consistent():
         assert f"ctx{w.ctx_lo}" in name, name
     assert S.WORKLOADS[SWEEP].grid["K"][0] == 0          # the greedy baseline of the speedup
     assert S.WORKLOADS["loop_12l_b64_ctx1024_4096"].gen_tokens == 512
+
+
+def test_verify_bytes_match_the_derived_roofline_table():
+    """bench.algorithmic_bytes (the numerator of every verify roofline fraction) against byte
+    counts worked out by hand from the model's shapes (K=3; routed experts touched per layer
+    under uniform routing, 64 (1 - (58/64)^T)): 2.44 GB at B=1, ctx 1024 (20.8 experts); 6.15 GB
+    at B=8, ctx ~896 (61.3); 22.1 GB at B=64, ctx 4096 (64); 134.9 GB at B=256, ctx 8192 (64),
+    each to three digits."""
+    import bench
+    sh = S.ModelShape()
+    for B, ctx, experts, gb in ((1, 1024, 20.8, 2.44), (8, 896, 61.3, 6.15), (64, 4096, 64, 22.1),
+                                (256, 8192, 64, 134.9)):
+        got = bench.algorithmic_bytes(sh, B, 3, ctx, experts) / 1e9
+        assert abs(got - gb) <= 0.006 * gb, (B, got, gb)
