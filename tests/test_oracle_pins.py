@@ -218,6 +218,52 @@ def test_moe_is_invariant_to_expert_relabelling():
     assert torch.allclose(_moe_once(model, x)[0], y0, atol=1e-12)
 
 
+# ----------------------------------------------------------------------------- greedy argmax
+
+def test_argmax_with_gap_hand_values():
+    """v_r = argmax of each row, the lowest id among equal maxima (the reading for ties), and the
+    margin top-1 minus top-2 taken on the row's own values (0 for a tie).  Expected numbers are
+    written out by hand, not produced by another argmax."""
+    logits = torch.tensor([
+        [1.0, 3.0, 3.0, 2.0],            # tie of ids 1 and 2 at the maximum -> 1, margin 0
+        [5.0, 1.0, 4.5, -2.0],           # clear maximum at id 0, runner-up 4.5 -> margin 0.5
+        [-1.0, -1.0, -1.0, -1.0],        # all equal -> id 0, margin 0
+        [0.25, 0.75, 0.5, 0.75 - 2.0 ** -20],   # near tie resolved by value -> id 1, margin 2^-20
+        [-7.0, -3.0, -3.5, -9.0],        # negative values -> id 1, margin 0.5
+        [2.0, 0.0, 0.0, 2.0],            # tie of the first and the last id -> 0, margin 0
+    ], dtype=F64)
+    v, gap = O.argmax_with_gap(logits)
+    assert v.tolist() == [1, 0, 0, 1, 1, 0]
+    assert gap.tolist() == [0.0, 0.5, 0.0, 2.0 ** -20, 0.5, 0.0]
+
+
+def test_verify_argmax_tie_goes_to_lower_token():
+    """Through verify(): with every layer the identity (zero W_o and down projections) the state
+    is b = N_o(E[x]); making W_lm rows 29 and 7 equal to a scaled copy of b puts both ids at
+    the exact maximum, and the verifier must answer 7 with margin 0; with row 29 scaled up by
+    2^-7 it must answer 29."""
+    model = tiny_model(12)
+    for lw in model.w.layers:
+        lw.wo = torch.zeros_like(lw.wo)
+        lw.w_down = torch.zeros_like(lw.w_down)
+        lw.shared_down = torch.zeros_like(lw.shared_down)
+    caches = tiny_caches(TINY, 12, 1, 3, 3)
+    x = caches[0].pending
+    b = F.rms_norm(model.w.embed[x].to(F64), (TINY.hidden,), model.w.final_norm.to(F64), eps=TINY.rms_eps)
+    row = (b * 4).to(torch.bfloat16)     # logit ~4 |b|^2 >> every random row's logit
+    lm = model.w.lm_head.clone()
+    lm[7] = row
+    lm[29] = row
+    model.w.lm_head = lm
+    model._lm = None
+    out = O.verify(model, caches, [[x]], rb=False)
+    assert int(out.v[0, 0]) == 7 and float(out.v_gap[0, 0]) == 0.0
+    lm[29] = (row.to(F64) * (1 + 2 ** -7)).to(torch.bfloat16)
+    model._lm = None
+    out = O.verify(model, caches, [[x]], rb=False)
+    assert int(out.v[0, 0]) == 29 and float(out.v_gap[0, 0]) > 0.0
+
+
 # ----------------------------------------------------------------------------- acceptance
 
 @pytest.mark.parametrize("K", [1, 2, 3, 4])
@@ -394,6 +440,69 @@ def test_draft_chain_follows_the_diagonal():
     for b, c in enumerate(caches):
         y = c.pending
         assert out.tokens[b] == [int(sigma[y]), int(sigma[sigma[y]]), int(sigma[sigma[sigma[y]]])]
+
+
+def test_deep_draft_depths_attend_to_tentative_rows():
+    """Closed form in which the draft block's attention matters at every depth: W_k = 0 and a
+    zero key prefix make every score 0, so attention is the plain mean of the value rows the
+    query may see; W_down = 0 makes the FFN add nothing.  Depth k at row p = j + k - 1 must see
+    the committed rows 0..j, the tentative rows j+1..p-1 written by the shallower depths of the
+    same chain, and its own row p (Sec. 3.1, Fig. "FastMTP state-shift alignment").  The chain is
+    recomputed here with library primitives only and compared state by state; a chain that
+    dropped the tentative rows is shown to differ."""
+    model = tiny_model(14)
+    dr = _tiny_drafter(14, model)
+    H, hd, d = TINY.n_heads, TINY.head_dim, TINY.hidden
+    wqkv = dr.dw.wqkv.clone()
+    wqkv[H * hd:2 * H * hd] = 0
+    dr.dw.wqkv = wqkv
+    dr.dw.w_down = torch.zeros_like(dr.dw.w_down)
+    caches = tiny_caches(TINY, 14, 2, 4, 7)
+    dcs = []
+    for b, c in enumerate(caches):
+        kv = S.draft_kv_prefix(14, b, c.ctx, H, hd).clone()
+        kv[0] = 0                                     # committed keys: zero
+        dcs.append(O.DraftCache.from_prefix(kv))
+    vprefix = [dc.v.clone() for dc in dcs]
+    vo = O.verify(model, caches, [[c.pending] for c in caches], rb=False)
+    O.commit(caches, vo, [[c.pending] for c in caches], dcs)
+    rows_b = [dc.rows_b.clone() for dc in dcs]
+    rows_t = [list(dc.rows_tok) for dc in dcs]
+    K = 4
+    out = O.draft(dr, dcs, K, rb=False)
+
+    eps = TINY.rms_eps
+    rn = lambda x, g: F.rms_norm(x, (d,), g.to(F64), eps=eps)
+    E, W = model.w.embed.to(F64), model.w.lm_head.to(F64)
+    Pm, Wv, Wo = dr.dw.eh_proj.to(F64), dr.dw.wqkv.to(F64)[2 * H * hd:], dr.dw.wo.to(F64)
+
+    def z_of(tok, a):
+        return F.linear(torch.cat([rn(E[tok], dr.dw.enorm), rn(a, dr.dw.hnorm)]), Pm)
+
+    def v_of(z):
+        return F.linear(rn(z, dr.dw.attn_norm), Wv)
+
+    for b in range(2):
+        vrows = list(vprefix[b].reshape(-1, H * hd))
+        for a, tok in zip(rows_b[b], rows_t[b]):      # committed rows keep their base states
+            z = z_of(tok, a.to(F64))
+            vrows.append(v_of(z))
+        n_committed = len(vrows)
+        u_alt = None
+        for k in range(K):
+            if k > 0:
+                z = z_of(tok, u)
+                vrows.append(v_of(z))                 # row p of depth k+1 (tentative)
+            mean_v = torch.stack(vrows).mean(0)       # uniform weights over rows 0..p
+            u = rn(z + F.linear(mean_v, Wo), model.w.final_norm)
+            assert torch.allclose(out.u[b][k], u, atol=1e-10, rtol=0), (b, k)
+            if k == 2:
+                # the same depth without the tentative row of depth 2: must be different
+                seen = vrows[:n_committed] + vrows[-1:]
+                u_alt = rn(z + F.linear(torch.stack(seen).mean(0), Wo), model.w.final_norm)
+            tok = int(F.linear(u, W).argmax())
+            assert tok == out.tokens[b][k], (b, k)
+        assert not torch.allclose(u_alt, out.u[b][2], atol=1e-6)
 
 
 def test_draft_cache_tracks_committed_length_and_base_states():
