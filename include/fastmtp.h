@@ -162,7 +162,11 @@ spec_status accept_commit(spec_ctx* ctx, int32_t B, const int32_t* slots, int32_
 
 /* Waits for the context's stream and reports the device guard flag: SPEC_OK, or
  * SPEC_EDEVICE with the flag bits in spec_last_error (the flag is then cleared).  Also
- * SPEC_ECUDA if the stream reports an error. */
+ * SPEC_ECUDA if the stream reports an error.
+ * With ctx NULL: waits for the whole current device (cudaDeviceSynchronize) and reports the
+ * guard flags of the context-free entry points spec_gemm_bf16 and spec_gemm_bf16_noalloc on
+ * that device (1 = a pipeline wait ran out and the tiles it covers were left unwritten), with
+ * the bits in spec_last_error(NULL); the flags are then cleared.  Allocates nothing. */
 spec_status spec_sync(spec_ctx* ctx);
 
 /* Reads one slot's state (synchronous): committed KV length and pending token. */
@@ -239,12 +243,17 @@ spec_status spec_trace_read(void* host_records, int32_t cap, int32_t reset, int3
  * tickets live in a fixed file-scope device array of 4 MiB + 4 KiB that every GPU loading the
  * library holds until the process exits; the call allocates and frees nothing.  The first call
  * on a device looks the array up on that device (it must be current) and should come before
- * any stream capture.  Every call shares the array and leaves its last contents there; the
- * call clears the tickets it uses before its kernel runs.  Calls whose kernels overlap on the
- * GPU race on the array: keep them on one stream.  Limits: n_tiles * m_tiles * splits * rows
- * box * 128 floats <= 2^20 (e.g. M <= 64 with N <= 4096 at K = 1280); larger problems get
- * SPEC_EINVAL with the reason in spec_last_error(NULL).  Same argument rules and errors as
- * spec_gemm_bf16 otherwise; asynchronous on `stream`. */
+ * any stream capture; host threads may make first calls concurrently (the lookup is locked).
+ * Every call shares the array and leaves its last contents there; the call clears the tickets
+ * it uses before its kernel runs.  Calls whose kernels overlap on the GPU race on the array:
+ * keep them on one stream.  Splits: min(SM count / ceil(N/128), Kdim/128, 8), at least 1.
+ * Limits: ceil(N/128) * ceil(M/box) * splits * box * 128 floats <= 2^20, box the row tile
+ * (16, 32, 64, 128 or 256: the smallest power of two >= min(M, 256), at least 16); e.g. M <= 64
+ * with N <= 4096 at Kdim = 1280, or M = 256 with N <= 512 on a 152-SM GPU.  Larger problems get
+ * SPEC_EINVAL with the reason in spec_last_error(NULL).  Device-side faults (a pipeline wait
+ * that ran out) are not returned by this call, which does not wait for its kernel: they set a
+ * guard flag that spec_sync(NULL) reports.  Same argument rules and errors as spec_gemm_bf16
+ * otherwise; asynchronous on `stream`. */
 spec_status spec_gemm_bf16_noalloc(const void* X, const void* W, float* Y, int32_t M, int32_t N,
                                    int32_t Kdim, void* stream);
 

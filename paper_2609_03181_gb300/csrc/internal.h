@@ -135,6 +135,9 @@ cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream
 int num_sms();
 // Sets the message spec_last_error(NULL) returns in this thread.
 void set_thread_error(const std::string& msg);
+// Reads and clears the device guard flag of spec_gemm_bf16_noalloc's kernels on the current
+// device (0 if that entry point never ran there); the caller has synchronised the device.
+cudaError_t noalloc_take_flag(int* flag);
 #ifdef FM_TRACE
 // Device-timeline buffers of the three kernel translation units (FM_TRACE builds): copy up to
 // `cap` records (4 x u64 each) to host memory, return the count (-1 on a CUDA error).

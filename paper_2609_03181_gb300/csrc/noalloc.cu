@@ -9,6 +9,8 @@
 // file-scope device array, so the call allocates nothing.  The caller still passes X, W and Y.
 #include <string.h>
 
+#include <atomic>
+#include <mutex>
 #include <string>
 
 #include "../../include/fastmtp.h"
@@ -27,13 +29,18 @@ static __device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchFloats];
 static __device__ __align__(256) int g_noalloc_tickets[kNoAllocTickets];
 static __device__ int g_noalloc_err;
 
+// Device addresses of the arrays, per device.  `ready` is published with release order after
+// the pointers are written and read with acquire order, and the first lookup on a device runs
+// under a lock, so host threads making their first calls at the same time each see either no
+// entry (and wait for the lock) or a complete one.
 struct DevPtrs {
-  bool ready = false;
+  std::atomic<bool> ready{false};
   float* scratch = nullptr;
   int* tickets = nullptr;
   int* err = nullptr;
 };
 DevPtrs g_dev[64];
+std::mutex g_dev_lock;
 
 spec_status fail(spec_status s, const std::string& m) {
   set_thread_error(m);   // reported by spec_last_error(NULL)
@@ -48,17 +55,37 @@ spec_status device_ptrs(DevPtrs** out) {
   if (e != cudaSuccess) return fail(SPEC_ECUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
   if (dev < 0 || dev >= 64) return fail(SPEC_EINVAL, "device index above 63");
   DevPtrs& p = g_dev[dev];
-  if (!p.ready) {
-    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&p.scratch), g_noalloc_scratch);
-    if (e == cudaSuccess) e = cudaGetSymbolAddress(reinterpret_cast<void**>(&p.tickets), g_noalloc_tickets);
-    if (e == cudaSuccess) e = cudaGetSymbolAddress(reinterpret_cast<void**>(&p.err), g_noalloc_err);
-    if (e == cudaSuccess) e = gemm_prepare();
-    if (e != cudaSuccess)
-      return fail(SPEC_ECUDA, std::string("scratch symbol lookup: ") + cudaGetErrorString(e));
-    p.ready = true;
+  if (!p.ready.load(std::memory_order_acquire)) {
+    std::lock_guard<std::mutex> hold(g_dev_lock);
+    if (!p.ready.load(std::memory_order_relaxed)) {
+      float* scratch = nullptr;
+      int* tickets = nullptr;
+      int* err = nullptr;
+      e = cudaGetSymbolAddress(reinterpret_cast<void**>(&scratch), g_noalloc_scratch);
+      if (e == cudaSuccess) e = cudaGetSymbolAddress(reinterpret_cast<void**>(&tickets), g_noalloc_tickets);
+      if (e == cudaSuccess) e = cudaGetSymbolAddress(reinterpret_cast<void**>(&err), g_noalloc_err);
+      if (e == cudaSuccess) e = gemm_prepare();
+      if (e != cudaSuccess)
+        return fail(SPEC_ECUDA, std::string("scratch symbol lookup: ") + cudaGetErrorString(e));
+      p.scratch = scratch;
+      p.tickets = tickets;
+      p.err = err;
+      p.ready.store(true, std::memory_order_release);
+    }
   }
   *out = &p;
   return SPEC_OK;
+}
+
+// Split count: a function of the SM count, N and K only (about one CTA per SM over the weight
+// tiles, at least two 64-wide k-chunks per split, at most kMaxSplit), so the shapes that fit the
+// fixed scratch do not depend on any occupancy query.
+int noalloc_split_k(int N, int K) {
+  const int n_tiles = (N + 127) / 128;
+  int s = num_sms() / n_tiles;
+  if (s > (K / 64) / 2) s = (K / 64) / 2;
+  if (s > kMaxSplit) s = kMaxSplit;
+  return s < 1 ? 1 : s;
 }
 
 }  // namespace
@@ -81,7 +108,7 @@ extern "C" spec_status spec_gemm_bf16_noalloc(const void* X, const void* W, floa
   const int box = 16 << bl;
   g.m_tiles = (M + box - 1) / box;
   g.n_tiles = (N + 127) / 128;
-  g.split_k = dense_split_k(N, Kdim);
+  g.split_k = noalloc_split_k(N, Kdim);
   g.n_items = g.n_tiles * g.split_k * g.m_tiles;
   const size_t need = static_cast<size_t>(g.n_tiles) * g.m_tiles * g.split_k * box * 128;
   if (need > kNoAllocScratchFloats || g.n_tiles * g.m_tiles > kNoAllocTickets)
@@ -107,4 +134,19 @@ extern "C" spec_status spec_gemm_bf16_noalloc(const void* X, const void* W, floa
   ce = gemm_launch(EPI_F32, box <= 64 ? 64 : 256, g, grid, s, false);
   if (ce != cudaSuccess) return fail(SPEC_ECUDA, std::string("launch: ") + cudaGetErrorString(ce));
   return SPEC_OK;
+}
+
+// The guard flag of this entry point's kernels on the current device (0 if it never ran there),
+// cleared after reading.  Called by spec_sync(NULL) after it has waited for the device.
+cudaError_t fm::noalloc_take_flag(int* flag) {
+  *flag = 0;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= 64 || !g_dev[dev].ready.load(std::memory_order_acquire)) return e;
+  e = cudaMemcpyFromSymbol(flag, g_noalloc_err, sizeof(int));
+  if (e == cudaSuccess && *flag != 0) {
+    const int zero = 0;
+    e = cudaMemcpyToSymbol(g_noalloc_err, &zero, sizeof(int));
+  }
+  return e;
 }

@@ -965,8 +965,33 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
 }
 
 // ============================================================================ sync / introspection
+namespace {
+__device__ int g_gemm_err;   // guard flag of spec_gemm_bf16's kernels
+}
+
+// spec_sync(NULL): waits for the current device and reports the guard flags of the
+// context-free entry points spec_gemm_bf16 and spec_gemm_bf16_noalloc.
+static spec_status sync_device_flags() {
+  spec_ctx* ctx = nullptr;
+  CK(cudaDeviceSynchronize());
+  int gemm_flag = 0, na_flag = 0;
+  CK(cudaMemcpyFromSymbol(&gemm_flag, g_gemm_err, sizeof(int)));
+  if (gemm_flag != 0) {
+    const int zero = 0;
+    CK(cudaMemcpyToSymbol(g_gemm_err, &zero, sizeof(int)));
+  }
+  CK(noalloc_take_flag(&na_flag));
+  if (gemm_flag != 0 || na_flag != 0) {
+    char buf[256];
+    snprintf(buf, sizeof(buf), "device guard flag: spec_gemm_bf16 0x%x, spec_gemm_bf16_noalloc 0x%x (1 wait timeout, "
+             "32 position)", gemm_flag, na_flag);
+    return fail(nullptr, SPEC_EDEVICE, buf);
+  }
+  return SPEC_OK;
+}
+
 extern "C" spec_status spec_sync(spec_ctx* ctx) {
-  if (ctx == nullptr) return fail(nullptr, SPEC_EINVAL, "ctx is NULL");
+  if (ctx == nullptr) return sync_device_flags();
   CK(cudaStreamSynchronize(ctx->stream));
   int flag = 0;
   CK(cudaMemcpy(&flag, ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost));
@@ -1066,9 +1091,6 @@ extern "C" spec_status spec_read_workspace(spec_ctx* ctx, int32_t id, void* dst,
 }
 
 // ============================================================================ standalone GEMM
-namespace {
-__device__ int g_gemm_err;
-}
 
 extern "C" spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, int32_t N, int32_t Kdim,
                                       void* stream) {

@@ -146,6 +146,15 @@ def gemm_bf16_noalloc(X: torch.Tensor, W: torch.Tensor, Y: torch.Tensor,
     return Y
 
 
+def device_sync() -> None:
+    """spec_sync(NULL): waits for the current device and raises FastMTPError (SPEC_EDEVICE) if a
+    kernel of spec_gemm_bf16 or spec_gemm_bf16_noalloc set its guard flag since the last check."""
+    lib = load_library()
+    st = lib.spec_sync(None)
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+
+
 class Engine:
     """A spec_ctx with device copies of the verifier and draft weights and the two KV pools.
 
