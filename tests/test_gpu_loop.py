@@ -10,7 +10,7 @@ import torch
 import oracle as O
 import synth_inputs as S
 from paper_2609_03181_gb300 import fastmtp as F
-from tests.gpu_util import GAP
+from tests.gpu_util import GAP, REL_TOL, argmax_margin, rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -98,26 +98,54 @@ def test_speculative_with_draft_head_equals_greedy(setup):
     assert all(0 <= m <= K for m in ms)
 
 
-def test_greedy_matches_oracle_greedy(setup):
-    """Token i of a stream is compared while every decision leading to it was unique at steps
-    0..i: oracle router margins (6th vs 7th expert probability) above 3e-4 and argmax margins
-    above 2e-2 logits.  Two bf16 layers leave ~0.15% rms state noise here: router-probability
-    noise ~2e-5 and logit-difference noise ~1.5e-3, so both margins are over 10 sigma."""
+def test_greedy_matches_oracle_greedy(succ):
+    """Greedy decoding on the GPU (K = 0, one token per step) against the oracle's greedy
+    decoding, 12 tokens of each of the 4 sequences, on the acceptance-tuned weights (their
+    greedy decisions have logit margins of ~10^3, so a chain is not cut short by random near-ties
+    the way N(0, 0.02) weights cut it, whose margins are ~0.1 against a state-noise margin of
+    ~0.05).  Token i is compared while the oracle's top-1 minus top-2 logit margin at that
+    position exceeds 8 standard deviations of the logit noise the measured state difference
+    implies (at least 1e-3); a sequence's comparison ends at its first token below that margin.
+    The state b of every compared position is within 2e-2."""
+    setup = succ
     reset(setup)
-    n = 6
-    greedy, _ = run_loop(setup, n, 0)
+    n = 12
+    eng = setup["eng"]
+    dev = torch.device("cuda")
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    toks, bgpu = [[] for _ in range(B)], [[] for _ in range(B)]
+    for i in range(n):
+        cand = torch.tensor([[eng.seq_state(b)[1]] for b in range(B)], dtype=torch.int32, device=dev)
+        vt = torch.empty(B, 1, dtype=torch.int32, device=dev)
+        acc = torch.empty(B, dtype=torch.int32, device=dev)
+        eng.verify_step(slots, cand, vt, acc)
+        brows = eng.read_workspace(F.WS_B, (B, SHAPE.hidden), torch.bfloat16)
+        com = torch.empty(B, 1, dtype=torch.int32, device=dev)
+        nc = torch.empty(B, dtype=torch.int32, device=dev)
+        eng.accept_commit(slots, com, nc)
+        eng.sync()
+        for b in range(B):
+            toks[b].append(int(com[b, 0]))
+            bgpu[b].append(brows[b])
     model = O.Verifier(setup["vw"])
-    compared = 0
-    for b in range(B):
-        cache = O.SeqCache.from_prefix(setup["kvs"][b], setup["pend"][b])
-        for i in range(n):
-            vo = O.verify(model, [cache], [[cache.pending]], rb=True)
-            if float(vo.v_gap[0, 0]) <= 2e-2 or min(float(g.min()) for g in vo.route_gap) <= 3e-4:
-                break
-            assert greedy[b][i] == int(vo.v[0, 0]), (b, i)
+    caches = [O.SeqCache.from_prefix(setup["kvs"][b], setup["pend"][b]) for b in range(B)]
+    compared, alive = 0, [True] * B
+    for i in range(n):
+        cand = [[c.pending] for c in caches]
+        vo = O.verify(model, caches, cand, rb=True)
+        for b in range(B):
+            if not alive[b]:
+                continue
+            assert rel_err(bgpu[b][i], vo.b[b, 0]) < REL_TOL, (b, i)
+            margin = argmax_margin(setup["vw"].lm_head, bgpu[b][i][None], vo.b[b, 0][None])[0]
+            if float(vo.v_gap[b, 0]) <= margin:
+                alive[b] = False
+                continue
+            assert toks[b][i] == int(vo.v[b, 0]), (b, i)
             compared += 1
-            O.commit([cache], vo, [[cache.pending]])
-    assert compared >= 1
+        O.commit(caches, vo, cand)
+    print(f"[parity] 2-layer greedy stream vs oracle greedy: {compared} of {n * B} tokens compared")
+    assert compared >= 40
 
 
 def test_batch_invariance_alone_vs_in_batch(setup):
@@ -166,12 +194,14 @@ def test_speculative_with_accepting_draft_head_equals_greedy(succ):
 
 
 def test_rows_identical_across_gemm_schedules():
-    """Batch invariance across the two dense-GEMM schedules: with few rows every split of K runs
-    in its own CTA (partials reduced through memory), from 128 rows on one CTA runs all splits of
-    a tile into separate TMEM accumulators.  Sequence 0 verified alone (4 rows) and as row 0 of
-    a batch of 40 (160 rows), then drafted alone (4 depth-1 rows) and in the batch (160 rows):
-    the b rows, verifier tokens, draft states u and draft tokens are bit-identical."""
-    seed, Bb = 31, 40
+    """Batch invariance across the GEMM schedules: with few rows every split of a dense K runs
+    in its own CTA of a cluster (partials reduced through shared memory), from 128 rows on one
+    CTA runs all splits of a tile into separate TMEM accumulators, and from 512 candidate rows
+    the expert launch groups rows in 256-row tiles instead of 64-row ones.  Sequence 0 verified
+    alone (4 rows), as row 0 of a batch of 40 (160 rows) and of a batch of 128 (512 rows), then
+    drafted alone and in each batch: the b rows, verifier tokens, draft states u and draft
+    tokens are bit-identical."""
+    seed, Bb = 31, 128
     vw = S.verifier_weights(SHAPE, seed, gain_std=0.1)
     dw = S.draft_weights(SHAPE, seed, gain_std=0.1)
     ctx = [int(c) for c in S.integers(seed, "ctx", Bb, 30, 120)]
@@ -181,7 +211,7 @@ def test_rows_identical_across_gemm_schedules():
     eng = F.Engine(vw, dw, max_batch=Bb, K_max=K, max_ctx=max(ctx) + 16, page_size=64)
     dev = torch.device("cuda")
     res = []
-    for bsz in (1, Bb):
+    for bsz in (1, 40, Bb):
         for b in range(bsz):
             eng.load_prefix(b, kvs[b], dkvs[b], pend[b])
         slots = torch.arange(bsz, dtype=torch.int32, device=dev)
@@ -199,5 +229,6 @@ def test_rows_identical_across_gemm_schedules():
         eng.sync()
         res.append((bst[: K + 1].clone(), vt[0].cpu().clone(), u[:, 0].clone(), dcand[0].cpu().clone()))
     eng.close()
-    for x, y in zip(res[0], res[1]):
-        assert torch.equal(x, y)
+    for other in res[1:]:
+        for x, y in zip(res[0], other):
+            assert torch.equal(x, y)

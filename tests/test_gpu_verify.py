@@ -16,10 +16,13 @@ from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, ind
 pytestmark = pytest.mark.gpu
 
 
-def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=None):
+def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=None, rb=True, min_keep=None):
     """One verify_step + accept_commit of len(ctx_lens) sequences on the GPU; the sequences in
-    `check` (default: all) are compared with the oracle, the others get uniform random drafts and
-    only fill the batch.  Returns (tokens compared, tokens skipped below the margin)."""
+    `check` (default: all) are compared with the oracle (storage-rounding mode if `rb`, else the
+    plain fp64 definition), the others get uniform random drafts and only fill the batch.
+    `min_keep` is the least number of checked rows that must stay comparable through every layer
+    (default: all of them when fewer than four sequences are checked, else all but two
+    sequences' rows).  Prints the comparison counts and returns them."""
     B = len(ctx_lens)
     check = list(range(B)) if check is None else list(check)
     vw = S.verifier_weights(shape, seed, gain_std=gain_std, zipf_s=zipf_s)
@@ -33,7 +36,7 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
     cand = [[int(pend[b])] + [int(t) for t in other[b]] for b in range(B)]
     for j, b in enumerate(check):
         cand[b] = cand_chk[j]
-    ref = O.verify(model, caches, cand_chk, rb=True)
+    ref = O.verify(model, caches, cand_chk, rb=rb, keep_hidden=True)
 
     eng = F.Engine(vw, dw, max_batch=B, K_max=max(K, 3), max_ctx=max(ctx_lens) + 8, page_size=64)
     for b in range(B):
@@ -56,24 +59,52 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
     # whose expert set differs below the margin (a legitimate near-tie) leaves the comparison of
     # hidden states from then on, together with the later candidates of its sequence (they
     # attend to its K/V); such rows are counted.
+    # Per layer, the router probabilities of the selected experts of every row still comparable
+    # (its selections and those of the earlier rows of its sequence equal so far) are a check of
+    # the layer's hidden state: within 2e-2 of the oracle's, relative to the row's largest.
+    gate_gpu = eng.read_workspace(F.WS_ROUTE_GATE, (shape.n_layers, eng.max_batch * (eng.K_max + 1), shape.top_k),
+                                  torch.float32)
     diverged = np.zeros(T, dtype=bool)
+    near_ties = 0
+    div_per_layer = []
     for l in range(shape.n_layers):
-        g = np.sort(ridx[l, rows].numpy(), -1)
+        gi = ridx[l, rows].numpy()
+        g = np.sort(gi, -1)
         r = np.sort(ref.route_idx[l].numpy(), -1)
         live = ~diverged
         n_ok, n_skip, n_bad = index_parity(g[live], r[live], ref.route_gap[l].numpy()[live])
+        near_ties += n_skip
         assert n_bad == 0, f"layer {l}: {n_bad} router mismatches over {n_ok} rows"
+        same = live & ~(g != r).any(-1)
+        for i in np.nonzero(same)[0]:
+            og = np.argsort(gi[i])
+            orf = np.argsort(ref.route_idx[l][i].numpy())
+            e = rel_err(gate_gpu[l, rows[i]][og], ref.route_gate[l][i][orf])
+            assert e < REL_TOL, f"layer {l} row {i}: router probability rel err {e:.3g}"
         differ = (g != r).any(-1) & ~diverged
+        div_per_layer.append(int(differ.sum()))
         for row in np.nonzero(differ)[0]:
             seq = row // R
             diverged[row:(seq + 1) * R] = True
     keep = ~diverged
     errs = [rel_err(b_gpu[i], ref.b.reshape(T, -1)[i]) for i in range(T)]
-    # bf16 storage decorrelates GPU and oracle rounding decisions within a few layers (about 1%
-    # hidden-state noise), so deep stacks lose rows to near-ties; a quarter must remain
-    assert keep.sum() >= T // 4, f"only {keep.sum()} of {T} rows comparable"
+    # bf16 storage decorrelates GPU and oracle rounding decisions over many layers (about 1%
+    # hidden-state noise at 12 layers), so a router near-tie can resolve differently; such a row
+    # and the later rows of its sequence leave the comparison (counted and printed)
+    # default floor: every row when one to three sequences are checked, else all but the rows of
+    # two sequences
+    need = (T if len(check) < 4 else T - 2 * R) if min_keep is None else min_keep
+    print(f"[parity] layers {shape.n_layers}, rows {T}, comparable through every layer {int(keep.sum())}, "
+          f"router near-ties skipped {near_ties}, rows leaving per layer {div_per_layer}")
+    assert keep.sum() >= need, f"only {keep.sum()} of {T} rows comparable (need {need})"
     assert max(e for e, k in zip(errs, keep) if k) < REL_TOL, (
         f"b rel err per row {['%.3g' % e for e in errs]}, diverged rows {np.nonzero(diverged)[0].tolist()}")
+    # the fp32 residual stream after the last layer, row by row
+    h_gpu = eng.read_workspace(F.WS_HIDDEN, (B * R, shape.hidden), torch.float32)[rows]
+    h_ref = ref.hidden[-1]
+    for i in np.nonzero(keep)[0]:
+        e = rel_err(h_gpu[i], h_ref[i])
+        assert e < REL_TOL, f"row {i}: residual stream rel err {e:.3g}"
 
     # verifier tokens: exact where the oracle's logit margin exceeds the noise the measured state
     # difference implies (at least 1e-3); accept lengths where all of a sequence's tokens are
@@ -116,12 +147,24 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
                 assert rel_err(k_gpu, ref.new_k[j][l][r]) < REL_TOL
                 assert rel_err(v_gpu, ref.new_v[j][l][r]) < REL_TOL
     eng.close()
-    return int(sure.sum()), int((~sure).sum())
+    print(f"[parity] verifier tokens compared {int(sure.sum())}, below the margin {int((~sure).sum())}")
+    return {"rows": T, "kept": int(keep.sum()), "near_ties": near_ties, "tokens": int(sure.sum()),
+            "tokens_skipped": int((~sure).sum())}
 
 
 def test_verify_one_layer_b1_ctx512():
     shape = S.ModelShape(n_layers=1)
     run_verify_case(shape, 0, [512], K=3)
+
+
+def test_verify_one_layer_against_plain_definition():
+    """The same one-layer step against the oracle without storage rounding (rb=False: fp64
+    everywhere between the bf16 weights and inputs), so that a precision shortcut the rounding
+    mode happened to copy would still show: b and the committed K/V within 2e-2, routing and
+    tokens exact above the margins."""
+    shape = S.ModelShape(n_layers=1)
+    run_verify_case(shape, 0, [512], K=3, rb=False)
+    run_verify_case(S.ModelShape(n_layers=2, vocab=4096), 5, [0, 63, 200, 777], K=3, rb=False)
 
 
 def test_verify_ragged_small_contexts():
@@ -133,7 +176,7 @@ def test_verify_ragged_small_contexts():
 def test_verify_twelve_layers_b8_ctx768_1024():
     shape = S.ModelShape()
     ctx = [int(c) for c in S.integers(1, "ctx", 8, 768, 1024)]
-    run_verify_case(shape, 1, ctx, K=3, gain_std=0.0)
+    run_verify_case(shape, 1, ctx, K=3, gain_std=0.0, min_keep=16)
 
 
 def test_verify_max_batch_256():
