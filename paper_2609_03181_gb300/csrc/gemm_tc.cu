@@ -72,8 +72,8 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, 
     const int j = i - pre[lo], m = j / P->grp_tiles;
     it.e = lo;
     it.n_tile = j - m * P->grp_tiles;
-    it.grow = kExpertTileRows * m;
-    it.rows = min(kExpertTileRows, grp[kGrpCnt + lo] - it.grow);
+    it.grow = a.grp_rows * m;
+    it.rows = min(a.grp_rows, grp[kGrpCnt + lo] - it.grow);
     it.out_row = lo * a.map_stride + it.grow;
     it.b_row = (P->grp_b_direct && lo >= a.n_routed) ? it.grow : it.out_row;
     it.split = 0;
@@ -441,7 +441,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       for (int k = 0; k < 3; ++k) {
         const int e = 3 * static_cast<int>(threadIdx.x) + k;
         c[k] = (e < kE + kShared) ? ((e < a.n_routed) ? a.grp_cnt[e] : a.grp_T) : 0;
-        const int mt = (c[k] + kExpertTileRows - 1) / kExpertTileRows;
+        const int mt = (c[k] + a.grp_rows - 1) / a.grp_rows;
         ni[k] = mt * a.grp_tiles;
         nd[k] = (EPI == EPI_MOE) ? mt * a2.grp_tiles : 0;
         sc += c[k];
@@ -529,7 +529,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         if (EPI == EPI_MOE && it.phase == 1) {
           // a down item reads the SwiGLU rows of its (expert, row tile): wait until all gate/up
           // tiles of them are stored (they come earlier in the item order, so they always end)
-          const int* d = a.dep + it.e * a.dep_stride + it.grow / kExpertTileRows;
+          const int* d = a.dep + it.e * a.dep_stride + it.grow / a.grp_rows;
           if (ld_acquire_gpu(d) < a.grp_tiles) {
             const uint64_t t0 = globaltimer();
             while (ld_acquire_gpu(d) < a.grp_tiles) {
@@ -715,7 +715,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           fence_proxy_async_global();
           __threadfence();
           named_bar_sync(1, 128);
-          if (threadIdx.x == 64) atomicAdd(a.dep + it.e * a.dep_stride + it.grow / kExpertTileRows, 1);
+          if (threadIdx.x == 64) atomicAdd(a.dep + it.e * a.dep_stride + it.grow / a.grp_rows, 1);
         }
         tc_fence_before();
         __syncwarp();
@@ -969,6 +969,7 @@ cudaError_t gemm_prepare() {
   FM_ATTR(EPI_ARGMAX)
 #undef FM_ATTR
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE>();
+  if (e == cudaSuccess) e = set_smem_attr<256, EPI_MOE>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, kShallowStages>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_RESID, kShallowStages>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_QKV, kShallowStages>();
@@ -1030,11 +1031,15 @@ int dense_split_k(int N, int K) {
 
 cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream_t s) {
   // one persistent CTA per SM; its down items wait on gate/up tiles of other CTAs, so the
-  // launch is cooperative (every CTA resident at once)
+  // launch is cooperative (every CTA resident at once).  Items of up to 64 rows run the
+  // 8-stage 64-column kernel, items of up to 256 rows the 4-stage 256-column kernel.
+  const bool large = gate_up.grp_rows > kExpertTileRows;
+  if (gate_up.grp_rows != down.grp_rows || (gate_up.grp_rows != kExpertTileRows && gate_up.grp_rows != kExpertTileRowsLarge))
+    return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(num_sms());
   cfg.blockDim = dim3(192);
-  cfg.dynamicSmemBytes = Cfg<64>::SMEM_BYTES;
+  cfg.dynamicSmemBytes = large ? Cfg<256>::SMEM_BYTES : Cfg<64>::SMEM_BYTES;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
@@ -1043,6 +1048,7 @@ cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
+  if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<256, EPI_MOE, Cfg<256>::STAGES>, gate_up, down);
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<64, EPI_MOE, Cfg<64>::STAGES>, gate_up, down);
 }
 

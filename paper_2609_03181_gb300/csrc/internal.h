@@ -89,6 +89,7 @@ struct GemmArgs {
   int grp_T;                   // rows of each shared expert (the step's tokens)
   int grp_tiles;               // weight tiles per expert
   int grp_b_direct;            // shared experts read activation rows 0..T-1 directly
+  int grp_rows;                // row tile of the grouped items: kExpertTileRows or kExpertTileRowsLarge
   const int* rowmap;           // SCATTER: [n_routed][map_stride] (token << 3 | rank) of each row
   int map_stride;
   unsigned long long* expert_ctr;   // if set, CTA 0 adds (experts with rows, rows) of the launch
@@ -155,8 +156,13 @@ cudaError_t router_prepare();
 // a tile are computed by one CTA (GemmArgs::seq_split) instead of one CTA each.
 int dense_split_k(int N, int K);
 constexpr int kSeqSplitRows = 128;
-// Row tile of the grouped expert launches (work-list items cover at most this many rows).
+// Row tile of the grouped expert launches (work-list items cover at most this many rows): 64
+// rows (the 8-stage, 64-column kernel) below kExpertLargeFromRows candidate rows, 256 rows (the
+// 4-stage, 256-column kernel, each weight tile read once per 256 rows) from there on.  The tile
+// height only groups rows into items; every row's sums are the same at either height.
 constexpr int kExpertTileRows = 64;
+constexpr int kExpertTileRowsLarge = 256;
+constexpr int kExpertLargeFromRows = 512;
 
 // ------------------------------------------------------------------------- other kernels
 struct AttnArgs {

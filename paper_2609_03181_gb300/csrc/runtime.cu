@@ -750,6 +750,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.grp_T = T;
       g.grp_tiles = 2 * kI / 128;
       g.grp_b_direct = 1;   // shared experts read the normalised rows directly
+      g.grp_rows = (T >= kExpertLargeFromRows) ? kExpertTileRowsLarge : kExpertTileRows;
       g.map_stride = ctx->Tcap;
       g.expert_ctr = ctx->d_expert_ctr;
       g.act = ctx->act;
@@ -770,6 +771,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       d.grp_cnt = ctx->counts + l * kE;
       d.grp_T = T;
       d.grp_tiles = kD / 128;
+      d.grp_rows = g.grp_rows;
       d.rowmap = ctx->rowmap;
       d.map_stride = ctx->Tcap;
       d.y = ctx->y;
