@@ -63,6 +63,8 @@ def parse():
     p.add_argument("--cpu-budget-s", type=float, default=20.0, help="CPU seconds of the oracle sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-points", action="store_true",
+                   help="skip the B=1/64/256 points of the metric's batch range (ctx 1024, K=3)")
     p.add_argument("--weights", default="successor", choices=["successor", "random"],
                    help="successor: acceptance-tuned seeded weights (tau ~2.7); random: N(0,0.02) everywhere")
     p.add_argument("--device-kv", action="store_true",
@@ -162,6 +164,18 @@ def algorithmic_bytes(shape, B, K, ctx_mean, experts_touched_routed_per_layer):
     kv_tok = 2 * H * hd * 2
     per_layer = attn_w + router_w + shared_w + expert_w * experts_touched_routed_per_layer
     return L * per_layer + 2 * V * d + B * ctx_mean * L * kv_tok + T * L * kv_tok + T * d * 2
+
+
+def draft_algorithmic_bytes(shape, B, K, ctx_mean, rows_new):
+    """Bytes one draft step must move: per depth the projection P, the block B_theta's four
+    matrices and the tied LM head (each read once), and the draft cache rows every sequence's
+    query attends to; plus the K/V rows the depth-1 pass commits and the embedding rows read."""
+    d, H, hd, Id, V = shape.hidden, shape.n_heads, shape.head_dim, shape.draft_inter, shape.vocab
+    P = 2 * d * 2 * d
+    block = 2 * (3 * H * hd * d + d * H * hd + 2 * Id * d + d * Id)
+    lm = 2 * V * d
+    kv_row = 2 * H * hd * 2
+    return K * (P + block + lm) + K * B * ctx_mean * kv_row + rows_new * kv_row + (rows_new + B * K) * d * 2
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -287,6 +301,91 @@ def run_reference(args):
 
 
 # ----------------------------------------------------------------------------- GPU leg
+POINT_BATCHES = (1, 64, 256)
+POINT_CTX = 1024
+
+
+def run_points(args, shape, vw, dw, dev, peak, peak_kind):
+    """The metric's batch range on the same weights: uniform routing, K = 3, committed contexts
+    of exactly 1024 tokens (N(0,1) KV drawn on the device), B = 1, 64 and 256 on one engine.
+    Per point: one K=0 step, `warmup` steps, then timed steps (50 at B = 1, whose acceptance
+    varies most from step to step; `steps` otherwise) with an event pair around each phase;
+    per-step medians.  Returns one object per point."""
+    import torch
+
+    from paper_2609_03181_gb300 import fastmtp as F
+
+    K, L = 3, shape.n_layers
+    n_steps = {b: (max(args.steps, 50) if b == 1 else args.steps) for b in POINT_BATCHES}
+    grow = (args.warmup + max(n_steps.values()) + 2) * (K + 1)
+    Bmax = max(POINT_BATCHES)
+    stream = torch.cuda.Stream(dev)
+    eng = F.Engine(vw, dw, max_batch=Bmax, K_max=K, max_ctx=POINT_CTX + grow, page_size=64, device=str(dev),
+                   stream=stream)
+    g = torch.Generator(device=dev)
+    g.manual_seed(4)
+    for l in range(L):
+        eng.kv_pool[l].normal_(generator=g)
+    eng.dkv_pool.normal_(generator=g)
+    torch.cuda.synchronize(dev)
+    out = []
+    for bi, B in enumerate(POINT_BATCHES):
+        import synth_inputs as S
+        pend = [int(t) for t in S.integers(40 + bi, "pending", B, 0, shape.vocab - 1)]
+        for b in range(B):
+            eng.reset_seq(b, POINT_CTX, eng.block_table(b), pend[b])
+        slots = torch.arange(B, dtype=torch.int32, device=dev)
+        c0 = torch.tensor([[p] for p in pend], dtype=torch.int32, device=dev)
+        v0 = torch.empty(B, 1, dtype=torch.int32, device=dev)
+        acc = torch.empty(B, dtype=torch.int32, device=dev)
+        cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+        vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+        com = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+        n_all = args.warmup + n_steps[B]
+        hist = torch.zeros(n_all, B, dtype=torch.int32, device=dev)
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_all)]
+        torch.cuda.synchronize(dev)
+        with torch.cuda.stream(stream):
+            eng.verify_step(slots, c0, v0, acc)
+            eng.accept_commit(slots, v0, acc)
+            for i in range(n_all):
+                if i == args.warmup:
+                    eng.profile(2)
+                ev[i][0].record(stream)
+                eng.draft_step(slots, K, cand)
+                ev[i][1].record(stream)
+                eng.verify_step(slots, cand, vt, acc)
+                ev[i][2].record(stream)
+                eng.accept_commit(slots, com, hist[i])
+                ev[i][3].record(stream)
+        eng.sync()
+        counted = eng.profile_read()
+        eng.profile(0)
+        timed = range(args.warmup, n_all)
+        med = lambda a, b: statistics.median(ev[i][a].elapsed_time(ev[i][b]) for i in timed)
+        ms_step, ms_draft, ms_verify = med(0, 3), med(0, 1), med(1, 2)
+        h = hist.double().cpu()
+        lens = POINT_CTX + 1 + torch.cumsum(h, 0) - h
+        ctx_mean = float(lens[args.warmup:].mean())
+        tok = float(h[args.warmup:].sum())
+        nt = n_steps[B]
+        touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
+        vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
+        dbytes = draft_algorithmic_bytes(shape, B, K, ctx_mean, tok / nt)
+        out.append({"batch": B, "ctx": POINT_CTX, "K": K, "router": "uniform", "steps": nt,
+                    "tokens_per_s": tok / (ms_step * nt / 1000.0), "ms_step": ms_step, "ms_draft": ms_draft,
+                    "ms_verify": ms_verify, "tau": tok / (nt * B),
+                    "verify_roofline": {"frac": vbytes / ms_verify / 1e6 / peak,
+                                        "achieved_gbs": vbytes / ms_verify / 1e6, "bytes": vbytes},
+                    "draft_roofline": {"frac": dbytes / ms_draft / 1e6 / peak,
+                                       "achieved_gbs": dbytes / ms_draft / 1e6, "bytes": dbytes},
+                    "experts_touched_per_layer": touched, "peak_gbs": peak, "peak_source": peak_kind})
+    eng.close()
+    del eng
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_fastmtp(args):
     import torch
     import torch.distributed as dist
@@ -421,6 +520,12 @@ def run_fastmtp(args):
         e2e = {"value": tok / dt, "unit": "tokens/s", "h2d_bytes_per_step": B * 4,
                "d2h_bytes_per_step": B * (K + 1) * 4 + B * 4}
     eng.close()
+    del eng
+    torch.cuda.empty_cache()
+    points = None
+    if not args.no_points and world == 1:
+        pk, pkind = measured_peaks()
+        points = run_points(args, shape, vw, dw, dev, pk, pkind)
 
     if rank != 0:
         if world > 1:
@@ -457,10 +562,14 @@ def run_fastmtp(args):
             traffic = tj.get("dram_bytes_per_launch")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": traffic, "kernel": label, "algorithmic_bytes_per_launch": cls_bytes[dom],
-                "avg_launch_ms": dur_ms, "peak_source": peak_kind}
+                "avg_launch_ms": dur_ms, "avg_launch_timing": "serialised replay (event pair per launch)",
+                "peak_source": peak_kind}
     routed_touched = touched - shape.n_shared
     vbytes = algorithmic_bytes(shape, B, K, statistics.mean(ctx) + (args.warmup + steps / 2) * 2, routed_touched)
     v_ach = vbytes / (ms_verify / 1000.0) / 1e9
+    ctx_run = statistics.mean(ctx) + (args.warmup + steps / 2) * 2
+    dbytes = draft_algorithmic_bytes(shape, B, K, ctx_run, accepted / steps)
+    d_ach = dbytes / (ms_draft / 1000.0) / 1e9
     launches_total = sum(counted["launches"].values())
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
@@ -472,8 +581,14 @@ def run_fastmtp(args):
         "roofline": roofline,
         "verify_roofline": {"bound": "hbm", "achieved": v_ach, "peak": peak, "unit": "GB/s", "frac": v_ach / peak,
                             "algorithmic_bytes": vbytes, "ms": ms_verify},
+        "draft_roofline": {"bound": "hbm", "achieved": d_ach, "peak": peak, "unit": "GB/s", "frac": d_ach / peak,
+                           "algorithmic_bytes": dbytes, "ms": ms_draft},
         "phase_ms": {"draft": ms_draft, "verify": ms_verify, "commit": ms_commit},
         "kernel_ms_per_step": {k: v / steps for k, v in prof["ms"].items()},
+        "kernel_ms_timing": ("serialised: a separate replay of the same steps with a CUDA event pair around "
+                             "every launch group, which removes the programmatic-dependent-launch overlap "
+                             "between kernels (sums exceed ms_per_step; roofline.avg_launch_ms is from it)"),
+        "sweep_points": points,
         "tau": accepted / (steps * B), "accept_hist_m": m_hist,
         "experts_touched_per_layer": touched,
         "gpu_launches": launches_total,
