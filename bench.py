@@ -372,7 +372,8 @@ def run_points(args, shape, vw, dw, dev, peak, peak_kind):
         touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
         vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
         dbytes = draft_algorithmic_bytes(shape, B, K, ctx_mean, tok / nt)
-        out.append({"batch": B, "ctx": POINT_CTX, "K": K, "router": "uniform", "steps": nt,
+        out.append({"batch": B, "ctx": POINT_CTX, "K": K, "K_policy": F.choose_depth(B, POINT_CTX),
+                    "router": "uniform", "steps": nt,
                     "tokens_per_s": tok / (ms_step * nt / 1000.0), "ms_step": ms_step, "ms_draft": ms_draft,
                     "ms_verify": ms_verify, "tau": tok / (nt * B),
                     "verify_roofline": {"frac": vbytes / ms_verify / 1e6 / peak,
@@ -624,7 +625,8 @@ def run_sweep(args):
     peak, peak_kind = measured_peaks()
     shape = S.ModelShape(n_layers=args.layers)
     Bmax, Kmax = max(batches), max(Ks)
-    grow = (args.warmup + args.steps + 2) * (Kmax + 1)
+    steps_for = lambda B: max(args.steps, 50) if B == 1 else args.steps   # B=1 acceptance varies most
+    grow = (args.warmup + steps_for(1) + 2) * (Kmax + 1)
     clocks = ClockSampler(0)
     clocks.start()
     for router in routers:
@@ -649,6 +651,8 @@ def run_sweep(args):
                 c0 = torch.tensor([[p] for p in pend], dtype=torch.int32, device=dev)
                 v0 = torch.empty(B, 1, dtype=torch.int32, device=dev)
                 ar_tok_s = None   # greedy autoregressive (K=0) throughput of this (router, ctx, B)
+                n_steps = steps_for(B)
+                by_k = {}
                 for K in Ks:
                     for b in range(B):
                         eng.reset_seq(b, ctx, eng.block_table(b), pend[b])
@@ -656,7 +660,7 @@ def run_sweep(args):
                     cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
                     vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
                     com = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
-                    n_all = args.warmup + args.steps
+                    n_all = args.warmup + n_steps
                     hist = torch.zeros(n_all, B, dtype=torch.int32, device=dev)
                     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_all)]
                     torch.cuda.synchronize(dev)
@@ -695,26 +699,34 @@ def run_sweep(args):
                     touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
                     vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
                     load = cnt / cnt.mean(-1, keepdim=True)
-                    tok_s = tok / (ms_step * args.steps / 1000.0)
+                    tok_s = tok / (ms_step * n_steps / 1000.0)
                     if K == 0:
                         ar_tok_s = tok_s
                     out = {"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K,
                            "tokens_per_s": tok_s, "ms_step": ms_step,
                            "ms_step_mean": statistics.mean(ev[i][0].elapsed_time(ev[i][3]) for i in timed),
                            "ms_draft": ms_draft, "ms_verify": ms_verify, "ms_commit": ms(2, 3),
-                           "tau": tok / (args.steps * B),
+                           "tau": tok / (n_steps * B),
                            "verify_roofline": {"bytes": vbytes, "achieved_gbs": vbytes / ms_verify / 1e6,
                                                "peak": peak, "peak_source": peak_kind,
                                                "frac": vbytes / ms_verify / 1e6 / peak},
                            "experts_touched_per_layer": touched,
                            "expert_load_max_over_mean": float(load.max(-1).values.mean()),
                            "expert_share_top1": float((cnt.max(-1).values / cnt.sum(-1)).mean()),
-                           "steps": args.steps, "warmup": args.warmup}
+                           "steps": n_steps, "warmup": args.warmup}
                     if ar_tok_s is not None:
                         # the paper's speedup over greedy decoding and step cost c = tau / S
                         sp = M.speedup_vs_ar(tok_s, ar_tok_s, out["tau"])
                         out["speedup_vs_ar"], out["step_cost_c"] = sp["S"], sp["c"]
                     print(json.dumps(out), flush=True)
+                    by_k[K] = tok_s
+                if 0 in by_k:
+                    # the depth the packaged table's policy picks for this point, beside the best
+                    # depth measured here
+                    best = M.best_depth(by_k)
+                    print(json.dumps({"sweep_best": True, "router": router, "batch": B, "ctx": ctx,
+                                      "K_best_measured": best["k"], "S_best": best["S"],
+                                      "K_policy": F.choose_depth(B, ctx)}), flush=True)
         eng.close()
         del eng
         torch.cuda.empty_cache()

@@ -146,6 +146,17 @@ def gemm_bf16_noalloc(X: torch.Tensor, W: torch.Tensor, Y: torch.Tensor,
     return Y
 
 
+def choose_depth(batch: int, ctx: int, table: Optional[dict] = None) -> int:
+    """Draft depth K for a step of `batch` sequences at committed context `ctx`: the depth with
+    the highest measured committed tokens/s at the nearest measured (batch, context) point of
+    the draft-depth table (the packaged GB300 table unless `table` is given); 0 means plain
+    greedy decoding.  Host-side only: no library call."""
+    from . import depth_table as _dt
+    from . import metrics as _m
+    pol = _m.DepthPolicy.from_table(table if table is not None else _dt.load_packaged())
+    return pol.choose(int(batch), int(ctx))
+
+
 def device_sync() -> None:
     """spec_sync(NULL): waits for the current device and raises FastMTPError (SPEC_EDEVICE) if a
     kernel of spec_gemm_bf16 or spec_gemm_bf16_noalloc set its guard flag since the last check."""

@@ -73,6 +73,14 @@ class DepthPolicy:
             table.setdefault((int(d["batch"]), int(d["ctx"])), {})[int(d["K"])] = float(d["tokens_per_s"])
         return cls(table)
 
+    @classmethod
+    def from_table(cls, table: dict) -> "DepthPolicy":
+        """From the packaged table format (depth_table.py): {"points": [{"batch": b, "ctx": c,
+        "tokens_per_s": {"0": t0, "1": t1, ...}}, ...]}."""
+        t = {(int(p["batch"]), int(p["ctx"])): {int(k): float(v) for k, v in p["tokens_per_s"].items()}
+             for p in table["points"]}
+        return cls(t)
+
     def choose(self, batch: int, ctx: int) -> int:
         def dist(key):
             b, c = key

@@ -100,3 +100,33 @@ def test_depth_policy_on_the_papers_table():
 def test_depth_policy_needs_the_greedy_baseline():
     with pytest.raises(ValueError):
         M.DepthPolicy({(1, 1024): {1: 10.0, 2: 12.0}})
+
+
+def test_packaged_depth_table_policy():
+    """The library's packaged draft-depth table (a GB300 sweep): at every measured (batch, context)
+    choose_depth returns the depth with the highest measured tokens/s there (computed here from
+    the table's numbers), and an unmeasured point takes its nearest measured neighbour."""
+    from paper_2609_03181_gb300 import depth_table as DT
+    from paper_2609_03181_gb300 import fastmtp as FM
+    t = DT.load_packaged()
+    assert t["router"] == "uniform" and len(t["points"]) >= 10
+    for p in t["points"]:
+        tok = {int(k): v for k, v in p["tokens_per_s"].items()}
+        assert 0 in tok
+        best = max(sorted(tok), key=lambda k: tok[k])          # first maximum: the smaller depth
+        assert FM.choose_depth(p["batch"], p["ctx"]) == best, p
+    pts = {(p["batch"], p["ctx"]) for p in t["points"]}
+    assert (3, 1100) not in pts
+    b_near = min({b for b, _ in pts}, key=lambda b: abs(__import__("math").log2(b) - __import__("math").log2(3)))
+    c_near = min({c for b, c in pts if b == b_near}, key=lambda c: abs(__import__("math").log2(c) - __import__("math").log2(1100)))
+    assert FM.choose_depth(3, 1100) == FM.choose_depth(b_near, c_near)
+
+
+def test_depth_table_from_sweep_lines():
+    from paper_2609_03181_gb300 import depth_table as DT
+    lines = [_line("uniform", 4, 1024, 0, 100.0), _line("uniform", 4, 1024, 1, 150.0), _line("zipf", 4, 1024, 1, 9.0),
+             json.dumps({"sweep_clocks": {"sm_mhz": 2070.0}}), "not json"]
+    t = DT.build_table(lines, "uniform", "test")
+    assert t["points"] == [{"batch": 4, "ctx": 1024, "tokens_per_s": {"0": 100.0, "1": 150.0}, "steps": {"0": 0, "1": 0}}]
+    assert t["clocks"] == {"sm_mhz": 2070.0}
+    assert M.DepthPolicy.from_table(t).choose(4, 1024) == 1
