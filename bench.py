@@ -70,6 +70,8 @@ def parse():
     p.add_argument("--device-kv", action="store_true",
                    help="draw the KV prefixes on the GPU (PyTorch's generator) instead of the host Philox stream")
     p.add_argument("--sweep", action="store_true", help="run the (batch, context, K, router) grid")
+    p.add_argument("--objective", action="store_true",
+                   help="time only the draft-head training objective (64 rows, K=3, full vocabulary)")
     p.add_argument("--trace", action="store_true",
                    help="device timeline of one step (builds the FASTMTP_TRACE=1 library): every launch "
                         "and the per-kernel breakdown of a verify layer, as JSON lines")
@@ -387,6 +389,55 @@ def run_points(args, shape, vw, dw, dev, peak, peak_kind):
     return out
 
 
+LOSS_ROWS, LOSS_K = 64, 3
+
+
+def run_loss_point(args, shape, dev, peak, peak_kind, iters=20):
+    """The draft-head objective (spec_draft_loss) over 64 rows and K = 3 depths with the full
+    129,280-token LM head: W_lm (331 MB, larger than L2) streamed once per call.  CUDA events
+    around `iters` back-to-back calls after 3 warm-up calls; roofline = max(bytes / HBM peak,
+    FLOPs / bf16 peak) against the measured time."""
+    import torch
+
+    import synth_inputs as S
+    from paper_2609_03181_gb300 import fastmtp as F
+
+    R, K, V, d = LOSS_ROWS, LOSS_K, shape.vocab, shape.hidden
+    u = S.normal(77, "loss.u", (K, R, d), 1.0).to(dev)
+    b = S.normal(77, "loss.b", (R, d), 1.0).to(dev)
+    W = S.normal(77, "loss.w", (V, d), 0.02).to(dev)
+    tgt = torch.from_numpy(S.integers(77, "loss.t", R, 0, V - 1).astype("int32")).to(dev)
+    ws = torch.empty(F.draft_loss_workspace_bytes(K, R, V), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(dev)
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            F.draft_loss(u, b, tgt, W, workspace=ws, stream=stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(iters):
+            out, _ = F.draft_loss(u, b, tgt, W, workspace=ws, stream=stream)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / iters
+    rows_packed = R * 4
+    byts = V * d * 2 + rows_packed * d * 2
+    flops = 2.0 * V * d * rows_packed
+    pk_tf = None
+    try:
+        pk_tf = float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["bf16_tflops"])
+    except Exception:
+        pk_tf = 1900.0
+    gbs = byts / ms / 1e6
+    tfs = flops / ms / 1e9
+    bound = "hbm" if byts / peak >= flops / (pk_tf * 1000.0) else "tensor"
+    return {"rows": R, "K": K, "vocab": V, "ms": ms, "achieved_gbs": gbs, "hbm_frac": gbs / peak,
+            "achieved_tflops": tfs, "tensor_frac": tfs / pk_tf, "bound": bound,
+            "frac": max(gbs / peak, tfs / pk_tf), "algorithmic_bytes": byts, "flops": flops,
+            "loss": float(out[0]), "peak_source": peak_kind,
+            "timing": "CUDA events around back-to-back calls (pack, GEMM + softmax statistics, fold, mean)"}
+
+
 def run_fastmtp(args):
     import torch
     import torch.distributed as dist
@@ -524,9 +575,11 @@ def run_fastmtp(args):
     del eng
     torch.cuda.empty_cache()
     points = None
+    loss_point = None
     if not args.no_points and world == 1:
         pk, pkind = measured_peaks()
         points = run_points(args, shape, vw, dw, dev, pk, pkind)
+        loss_point = run_loss_point(args, shape, dev, pk, pkind)
 
     if rank != 0:
         if world > 1:
@@ -590,6 +643,7 @@ def run_fastmtp(args):
                              "every launch group, which removes the programmatic-dependent-launch overlap "
                              "between kernels (sums exceed ms_per_step; roofline.avg_launch_ms is from it)"),
         "sweep_points": points,
+        "draft_objective": loss_point,
         "tau": accepted / (steps * B), "accept_hist_m": m_hist,
         "experts_touched_per_layer": touched,
         "gpu_launches": launches_total,
@@ -798,6 +852,14 @@ def main():
     args = parse()
     if args.trace:
         run_trace(args)
+        return
+    if args.objective:
+        import torch
+        import synth_inputs as S
+        torch.cuda.set_device(0)
+        pk, pkind = measured_peaks()
+        print(json.dumps({"draft_objective": run_loss_point(args, S.ModelShape(), torch.device("cuda", 0), pk, pkind)}),
+              flush=True)
         return
     if args.sweep:
         run_sweep(args)

@@ -164,8 +164,9 @@ spec_status accept_commit(spec_ctx* ctx, int32_t B, const int32_t* slots, int32_
  * SPEC_EDEVICE with the flag bits in spec_last_error (the flag is then cleared).  Also
  * SPEC_ECUDA if the stream reports an error.
  * With ctx NULL: waits for the whole current device (cudaDeviceSynchronize) and reports the
- * guard flags of the context-free entry points spec_gemm_bf16 and spec_gemm_bf16_noalloc on
- * that device (1 = a pipeline wait ran out and the tiles it covers were left unwritten), with
+ * guard flags of the context-free entry points spec_gemm_bf16, spec_gemm_bf16_noalloc and
+ * spec_draft_loss on that device (1 = a pipeline wait ran out and the tiles it covers were
+ * left unwritten), with
  * the bits in spec_last_error(NULL); the flags are then cleared.  Allocates nothing. */
 spec_status spec_sync(spec_ctx* ctx);
 
@@ -256,6 +257,35 @@ spec_status spec_trace_read(void* host_records, int32_t cap, int32_t reset, int3
  * otherwise; asynchronous on `stream`. */
 spec_status spec_gemm_bf16_noalloc(const void* X, const void* W, float* Y, int32_t M, int32_t N,
                                    int32_t Kdim, void* stream);
+
+/* Draft-head training objective (Sec. 5.6 "Draft-head objective": the CE, KL and MSE terms per
+ * recursive depth and their alpha-weighted sum).  For rows p = 0..n_rows-1 and depths
+ * k = 1..K (1 <= K <= 7):
+ *   CE_k  = mean_p -log softmax(W_lm u_p^(k))[x_{p+2}]
+ *   KL_k  = mean_p KL(Q_p || softmax(W_lm u_p^(k))),  Q_p = softmax(W_lm b_{p+1})
+ *   MSE_k = mean_p ||u_p^(k) - b_{p+1}||^2
+ *   L     = w_ce sum_k alpha_k CE_k + w_kl sum_k alpha_k KL_k + w_mse sum_k alpha_k MSE_k,
+ *           alpha_k = beta^(k-1) / sum_{r=1..K} beta^(r-1)   (the paper: beta 0.6, w 0.85/0.45/0.45)
+ * the means taken over the rows with valid[p] != 0.  Arguments (dev unless noted):
+ *   u        bf16 [K][n_rows][d]   draft states u_p^(k) (d = 1280, 16-byte aligned)
+ *   b_next   bf16 [n_rows][d]      verifier states b_{p+1} (the detached targets)
+ *   target   int32 [n_rows]        tokens x_{p+2}; an id outside [0, vocab) makes that row's CE NaN
+ *   valid    int32 [n_rows] or NULL (every row counted)
+ *   lm_head  bf16 [vocab][d]       the tied LM head (16-byte aligned)
+ *   out      fp32 [1 + 3K]         L, CE_1..CE_K, KL_1..KL_K, MSE_1..MSE_K
+ *   row_out  fp32 [K][n_rows][3] or NULL: per row (CE, KL, MSE), valid or not
+ *   workspace, workspace_bytes: caller-owned device memory (256-byte aligned) of at least the
+ *            size spec_draft_loss_workspace returns; the call allocates nothing.
+ * One pass over W_lm: the logits are reduced on chip to per-row softmax statistics and never
+ * written.  Asynchronous on `stream`; calls sharing a workspace must not overlap.  Device-side
+ * faults (a pipeline wait that ran out) set a guard flag that spec_sync(NULL) reports.
+ * Errors: SPEC_EINVAL (null pointer, sizes, alignment, workspace too small, beta <= 0 or a
+ * non-finite weight), SPEC_ECUDA. */
+spec_status spec_draft_loss_workspace(int32_t K, int32_t n_rows, int32_t vocab, size_t* bytes);
+spec_status spec_draft_loss(const void* u, const void* b_next, const int32_t* target, const int32_t* valid,
+                            const void* lm_head, int32_t K, int32_t n_rows, int32_t vocab, float beta,
+                            float w_ce, float w_kl, float w_mse, float* out, float* row_out,
+                            void* workspace, size_t workspace_bytes, void* stream);
 
 /* Frees the workspace.  Borrowed weights and pools are untouched.  NULL is ignored. */
 void spec_destroy(spec_ctx* ctx);

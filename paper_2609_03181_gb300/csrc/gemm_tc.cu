@@ -294,6 +294,53 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
       atomicMax(a.am_key + it.out_row + j0 + t, argmax_key(bv, it.n_tile * 128 + bi));
     }
     named_bar_sync(1, 128);
+  } else if constexpr (EPI == EPI_LOSS) {
+    // Softmax statistics of 16 activation rows over the tile's 128 vocabulary entries: thread
+    // (column j, group g) first takes vocabulary rows 16g..16g+15 of column j -- its max, its sum
+    // of exp(x - max) and, for a draft column, the KL cross term sum exp(q - max_q) (q - x)
+    // against the group's verifier column -- then 16 threads merge the 8 groups in order.
+    float* xchg = sm.xchg;
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
+    named_bar_sync(1, 128);
+    const int t = threadIdx.x - 64, j = t & 15, grp = t >> 4;
+    const int jq = j & ~(a.loss_G - 1);
+    const int nv = min(16, a.N - (it.n_tile * 128 + grp * 16));
+    float m = -INFINITY, mq = -INFINITY;
+    for (int r = 0; r < nv; ++r) {
+      m = fmaxf(m, xchg[(grp * 16 + r) * 17 + j]);
+      mq = fmaxf(mq, xchg[(grp * 16 + r) * 17 + jq]);
+    }
+    float Z = 0.f, A = 0.f;
+    for (int r = 0; r < nv; ++r) {
+      const float x = xchg[(grp * 16 + r) * 17 + j];
+      Z += expf(x - m);
+      if (j != jq) {
+        const float q = xchg[(grp * 16 + r) * 17 + jq];
+        A += expf(q - mq) * (q - x);
+      }
+    }
+    float4* sp = reinterpret_cast<float4*>(sm.rope);
+    sp[grp * 16 + j] = make_float4(m, Z, A, mq);
+    named_bar_sync(1, 128);
+    if (t < 16 && j0 + t < it.rows) {
+      float M = -INFINITY, MQ = -INFINITY;
+#pragma unroll
+      for (int g2 = 0; g2 < 8; ++g2) {
+        const float4 p = sp[g2 * 16 + t];
+        M = fmaxf(M, p.x);
+        MQ = fmaxf(MQ, p.w);
+      }
+      float Zs = 0.f, As = 0.f;
+#pragma unroll
+      for (int g2 = 0; g2 < 8; ++g2) {
+        const float4 p = sp[g2 * 16 + t];
+        if (p.x != -INFINITY) Zs += p.y * expf(p.x - M);
+        if (p.w != -INFINITY) As += p.z * expf(p.w - MQ);
+      }
+      a.loss_part[static_cast<size_t>(it.n_tile) * a.ldo + it.out_row + j0 + t] = make_float4(M, Zs, As, MQ);
+    }
+    named_bar_sync(1, 128);
   }
 }
 
@@ -967,6 +1014,7 @@ cudaError_t gemm_prepare() {
   FM_ATTR(EPI_SWIGLU)
   FM_ATTR(EPI_SCATTER)
   FM_ATTR(EPI_ARGMAX)
+  FM_ATTR(EPI_LOSS)
 #undef FM_ATTR
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE>();
   if (e == cudaSuccess) e = set_smem_attr<256, EPI_MOE>();
@@ -1078,6 +1126,7 @@ cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStre
     FM_CASE(EPI_SWIGLU)
     FM_CASE(EPI_SCATTER)
     FM_CASE(EPI_ARGMAX)
+    FM_CASE(EPI_LOSS)
     default:
       return cudaErrorInvalidValue;
   }

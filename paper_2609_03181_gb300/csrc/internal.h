@@ -62,7 +62,8 @@ enum EpiKind : int {
   EPI_SWIGLU = 3,   // tile = 64 gate rows + 64 up rows -> bf16 silu(g)*u
   EPI_SCATTER = 4,  // expert down: out row (token, slot) from the sorted index
   EPI_ARGMAX = 5,   // running (max, argmax) of each column in a packed key (LM head)
-  EPI_MOE = 6       // grouped gate/up (SWIGLU) items, then the down (SCATTER) items, one launch
+  EPI_MOE = 6,      // grouped gate/up (SWIGLU) items, then the down (SCATTER) items, one launch
+  EPI_LOSS = 7      // draft-head objective: per (vocab tile, activation row) softmax statistics
 };
 
 // One work item: weight tile x activation rows.  x = expert | n_tile << 16, y = TMA row of
@@ -116,6 +117,11 @@ struct GemmArgs {
   unsigned long long* am_key; int* am_done;
   int fin_B, fin_R; const int* fin_cand; int* fin_vtok_out; int* fin_vtok_ws; int* fin_accept_out; int* fin_m_ws;
   float* sk_ws; int* sk_tickets;                              // split-K partials / per-tile tickets
+  // LOSS: activation rows come in groups of loss_G (a power of two dividing 16): row 0 of a group
+  // is a verifier state b, rows 1.. are draft states u.  loss_part[tile * ldo + row] = (max, sum
+  // of exp(x - max), sum of exp(q - max_q) (q - x) with q the group's b-row logit, max_q), over
+  // the tile's vocabulary entries (entries >= N excluded).
+  float4* loss_part; int loss_G;
   int* err;
 };
 
@@ -139,6 +145,8 @@ void set_thread_error(const std::string& msg);
 // Reads and clears the device guard flag of spec_gemm_bf16_noalloc's kernels on the current
 // device (0 if that entry point never ran there); the caller has synchronised the device.
 cudaError_t noalloc_take_flag(int* flag);
+// The same for the GEMM of spec_draft_loss.
+cudaError_t loss_take_flag(int* flag);
 #ifdef FM_TRACE
 // Device-timeline buffers of the three kernel translation units (FM_TRACE builds): copy up to
 // `cap` records (4 x u64 each) to host memory, return the count (-1 on a CUDA error).

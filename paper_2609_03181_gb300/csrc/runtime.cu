@@ -972,7 +972,7 @@ __device__ int g_gemm_err;   // guard flag of spec_gemm_bf16's kernels
 }
 
 // spec_sync(NULL): waits for the current device and reports the guard flags of the
-// context-free entry points spec_gemm_bf16 and spec_gemm_bf16_noalloc.
+// context-free entry points spec_gemm_bf16, spec_gemm_bf16_noalloc and spec_draft_loss.
 static spec_status sync_device_flags() {
   spec_ctx* ctx = nullptr;
   CK(cudaDeviceSynchronize());
@@ -982,11 +982,13 @@ static spec_status sync_device_flags() {
     const int zero = 0;
     CK(cudaMemcpyToSymbol(g_gemm_err, &zero, sizeof(int)));
   }
+  int loss_flag = 0;
   CK(noalloc_take_flag(&na_flag));
-  if (gemm_flag != 0 || na_flag != 0) {
+  CK(loss_take_flag(&loss_flag));
+  if (gemm_flag != 0 || na_flag != 0 || loss_flag != 0) {
     char buf[256];
-    snprintf(buf, sizeof(buf), "device guard flag: spec_gemm_bf16 0x%x, spec_gemm_bf16_noalloc 0x%x (1 wait timeout, "
-             "32 position)", gemm_flag, na_flag);
+    snprintf(buf, sizeof(buf), "device guard flag: spec_gemm_bf16 0x%x, spec_gemm_bf16_noalloc 0x%x, spec_draft_loss "
+             "0x%x (1 wait timeout, 32 position)", gemm_flag, na_flag, loss_flag);
     return fail(nullptr, SPEC_EDEVICE, buf);
   }
   return SPEC_OK;

@@ -21,7 +21,7 @@ WS_B, WS_ROUTE_IDX, WS_ROUTE_GATE, WS_EXPERT_CNT, WS_DRAFT_U, WS_HIDDEN = range(
 ENTRY_POINTS = ["spec_init", "spec_seq_reset", "spec_seq_set_draft_rows", "draft_step", "verify_step",
                 "accept_commit", "spec_sync", "spec_seq_state", "spec_read_workspace", "spec_gemm_bf16",
                 "spec_profile", "spec_profile_read", "spec_trace_read", "spec_gemm_bf16_noalloc",
-                "spec_destroy", "spec_last_error"]
+                "spec_draft_loss_workspace", "spec_draft_loss", "spec_destroy", "spec_last_error"]
 KERNEL_CLASSES = ["embed", "qkv", "attention", "oproj", "router", "permute", "expert_gate_up", "expert_down",
                   "combine", "lm_head", "argmax", "commit", "draft_gemm", "draft_misc"]
 
@@ -84,6 +84,9 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
         "spec_profile_read": (ctypes.c_int, [P, ctypes.POINTER(SpecProfile)]),
         "spec_trace_read": (ctypes.c_int, [P, I32, I32, ctypes.POINTER(I32)]),
         "spec_gemm_bf16_noalloc": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
+        "spec_draft_loss_workspace": (ctypes.c_int, [I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)]),
+        "spec_draft_loss": (ctypes.c_int, [P, P, P, P, P, I32, I32, I32, ctypes.c_float, ctypes.c_float,
+                                           ctypes.c_float, ctypes.c_float, P, P, P, ctypes.c_size_t, P]),
         "spec_destroy": (None, [P]),
         "spec_last_error": (ctypes.c_char_p, [P]),
     }
@@ -144,6 +147,44 @@ def gemm_bf16_noalloc(X: torch.Tensor, W: torch.Tensor, Y: torch.Tensor,
     if st != SPEC_OK:
         raise FastMTPError(st, lib.spec_last_error(None).decode())
     return Y
+
+
+def draft_loss_workspace_bytes(K: int, n_rows: int, vocab: int) -> int:
+    lib = load_library()
+    n = ctypes.c_size_t()
+    st = lib.spec_draft_loss_workspace(K, n_rows, vocab, ctypes.byref(n))
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+    return int(n.value)
+
+
+def draft_loss(u: torch.Tensor, b_next: torch.Tensor, target: torch.Tensor, lm_head: torch.Tensor,
+               valid: Optional[torch.Tensor] = None, beta: float = 0.6, weights=(0.85, 0.45, 0.45),
+               workspace: Optional[torch.Tensor] = None, stream: Optional[torch.cuda.Stream] = None):
+    """spec_draft_loss: the draft-head objective of K depths over n_rows rows.  u bf16 [K][R][d],
+    b_next bf16 [R][d], target int32 [R], lm_head bf16 [V][d], valid int32 [R] or None (CUDA
+    tensors).  Returns (out fp32 [1 + 3K] = L, CE_k, KL_k, MSE_k; rows fp32 [K][R][3])."""
+    lib = load_library()
+    K, R, d = u.shape
+    V = lm_head.shape[0]
+    need = draft_loss_workspace_bytes(K, R, V)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=u.device)
+    out = torch.empty(1 + 3 * K, dtype=torch.float32, device=u.device)
+    rows = torch.empty(K, R, 3, dtype=torch.float32, device=u.device)
+    for t in (u, b_next, lm_head):
+        assert t.dtype == torch.bfloat16 and t.is_contiguous() and t.is_cuda
+    assert target.dtype == torch.int32 and target.is_contiguous()
+    vp = None
+    if valid is not None:
+        assert valid.dtype == torch.int32 and valid.is_contiguous()
+        vp = valid.data_ptr()
+    st = lib.spec_draft_loss(u.data_ptr(), b_next.data_ptr(), target.data_ptr(), vp, lm_head.data_ptr(), K, R, V,
+                             float(beta), float(weights[0]), float(weights[1]), float(weights[2]), out.data_ptr(),
+                             rows.data_ptr(), workspace.data_ptr(), workspace.numel(), _stream_handle(stream))
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+    return out, rows
 
 
 def choose_depth(batch: int, ctx: int, table: Optional[dict] = None) -> int:
