@@ -400,9 +400,10 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
       while (go) {
         const int pg = lookup(v);
         const int c0 = kSuper * v.s, c1 = min(c0 + kSuper, chunks_live(s_p0[v.b], R));
+        const int safe = s_p0[v.b] - a.qoff - a.prewait_guard;   // keys below this are not written by this graph
         for (int c = c0; c < c1 && go; ++c) {
           const int page = __shfl_sync(0xffffffffu, pg, c - c0);
-          if (page == -1 || j_pre == kStages) {
+          if (page == -1 || j_pre == kStages || (c + 1) * kCH > safe) {
             go = false;
           } else {
             issue_tma(j_pre, page, v.h, c);

@@ -537,7 +537,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
-      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_w = a.a_keep ? l2_policy_evict_last() : l2_policy_evict_first();
       const uint64_t pol_x = l2_policy_evict_last();
       uint32_t g = 0;   // loads issued
       bool failed = false;

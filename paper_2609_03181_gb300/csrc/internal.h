@@ -122,6 +122,7 @@ struct GemmArgs {
   // of exp(x - max), sum of exp(q - max_q) (q - x) with q the group's b-row logit, max_q), over
   // the tile's vocabulary entries (entries >= N excluded).
   float4* loss_part; int loss_G;
+  int a_keep;                  // weight tiles loaded with the L2 evict-last policy (kept resident)
   int* err;
 };
 
@@ -196,6 +197,9 @@ struct AttnArgs {
   // lengths (the verify step): the K/V of the first committed chunks is then fetched before
   // the wait for the previous kernel.
   int prewait;
+  // With prewait: only chunks whose keys all sit below seq_len - prewait_guard are fetched before
+  // the wait (the draft step writes the draft pool's last K_max + 1 committed rows itself).
+  int prewait_guard;
   bf16* out;                   // [B*R][H*hd]
   int out_row_stride_seq;      // rows of out per sequence (R)
   int* err;
@@ -206,7 +210,6 @@ cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, c
                               const int* seq_len, const bf16* embed, int vocab, const bf16* gain, float eps,
                               float* h, bf16* xn, int* pos, long long* kv_rowoff, int stage_R, int n_slots,
                               int* err, int* zero, int n_zero, int* zero2, int n_zero2, cudaStream_t s);
-cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
 // Router: RMSNorm, logits, softmax, top-6; each selection claims the next row of its expert
 // (atomic add on counts) and copies the token's rounded row into the expert's input region.
 struct RouteArgs {
@@ -231,6 +234,7 @@ cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len
                               bf16* dcat, int* pos, long long* kv_rowoff, int* last_row, int page_size,
                               const int* block_table, int max_pages, int n_pages, int* cand, int cand_ld,
                               int n_slots, int* err, cudaStream_t s);
+cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s);
 cudaError_t gather_rows_launch(const float* src, const int* rows, int B, float* dst, cudaStream_t s);
 cudaError_t draft_next_launch(unsigned long long* am_key, int vocab, int* err, int B, int k, int K, const int* slots,
                               int n_slots, const int* seq_len, const bf16* u, const bf16* embed,

@@ -172,6 +172,15 @@ GemmArgs base_args(spec_ctx* ctx) {
   return g;
 }
 
+// A GemmArgs of a draft-block projection: the block's weights (54 MB with P) are loaded with the
+// L2 evict-last policy, so that they stay resident across the depths of a step while the LM
+// head streams through L2 with evict-first.
+GemmArgs draft_args(spec_ctx* ctx) {
+  GemmArgs g = base_args(ctx);
+  g.a_keep = 1;
+  return g;
+}
+
 int box_log_for(int rows) {
   int bl = 0;
   while ((16 << bl) < rows && bl < 4) ++bl;
@@ -849,14 +858,14 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
                        c.page_size, ctx->block_table, c.max_pages_per_seq, c.n_pages_total, cand, ld, ctx->Bmax,
                        ctx->d_err, s));
   {
-    GemmArgs g = base_args(ctx);
+    GemmArgs g = draft_args(ctx);
     g.out = ctx->z;
     g.ldo = kD;
     LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_F32, ctx->eh, ctx->a_dcat, kD, 2 * kD, T1, true));
   }
   LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->z, T1, static_cast<const bf16*>(ctx->w.mtp_attn_norm), eps, ctx->dxn, s));
   {
-    GemmArgs g = base_args(ctx);
+    GemmArgs g = draft_args(ctx);
     g.q_out = ctx->q;
     g.kv_base = ctx->dkv_pool;
     g.kv_rowoff = ctx->kv_rowoff;
@@ -869,12 +878,12 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
 
   for (int k = 1; k <= K; ++k) {
     if (k > 1) {
-      GemmArgs g = base_args(ctx);
+      GemmArgs g = draft_args(ctx);
       g.out = ctx->dres;
       g.ldo = kD;
       LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_F32, ctx->eh, ctx->a_dcat, kD, 2 * kD, B, true));
       LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.mtp_attn_norm), eps, ctx->dxn, s));
-      GemmArgs q = base_args(ctx);
+      GemmArgs q = draft_args(ctx);
       q.q_out = ctx->q;
       q.kv_base = ctx->dstage;
       q.kv_rowoff = ctx->kv_rowoff;
@@ -911,23 +920,27 @@ extern "C" spec_status draft_step(spec_ctx* ctx, int32_t B, int32_t K, const int
       a.out = ctx->dattn;
       a.out_row_stride_seq = 1;
       a.err = ctx->d_err;
+      // committed draft rows older than the last Rmax positions were written by earlier steps
+      // (draft_prep / accept_commit / seq_reset, other graphs): fetched before the wait
+      a.prewait = 1;
+      a.prewait_guard = ctx->Rmax;
       LAUNCH(SPEC_K_ATTN, 1, attention_launch(a, B, s));
     }
     {
-      GemmArgs g = base_args(ctx);
+      GemmArgs g = draft_args(ctx);
       g.out = ctx->dres;
       g.ldo = kD;
       LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_RESID, ctx->mwo, ctx->a_dattn, kD, kD, B, true));
     }
     LAUNCH(SPEC_K_DRAFT_MISC, 1, rmsnorm_launch(ctx->dres, B, static_cast<const bf16*>(ctx->w.mtp_ffn_norm), eps, ctx->dxn, s));
     {
-      GemmArgs g = base_args(ctx);
+      GemmArgs g = draft_args(ctx);
       g.act = ctx->dact;
       g.ld_act = kId;
       LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_SWIGLU, ctx->mgu, ctx->a_dxn, 2 * kId, kD, B, true, true, kId));
     }
     {
-      GemmArgs g = base_args(ctx);
+      GemmArgs g = draft_args(ctx);
       g.out = ctx->dres;
       g.ldo = kD;
       LAUNCH(SPEC_K_DRAFT_GEMM, 1, run_dense(ctx, g, EPI_RESID, ctx->mdn, ctx->a_dact, kD, kId, B, true));
