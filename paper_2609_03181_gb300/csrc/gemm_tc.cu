@@ -82,8 +82,10 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, 
     it.box_log = bl;
   } else {
     it.grow = 0;
-    const int mt = i % a.m_tiles;
-    const int t = i / a.m_tiles;
+    // items run through the activation tiles first, or (loss_G: the two operands swapped, A =
+    // activations) through the A tiles first, so that the CTAs reading one B tile run together
+    const int mt = a.loss_G ? i / a.n_tiles : i % a.m_tiles;
+    const int t = a.loss_G ? i % a.n_tiles : i / a.m_tiles;
     const int ns = a.seq_split ? 1 : a.split_k;   // in-CTA splits: one item covers every split
     it.split = t % ns;
     it.n_tile = t / ns;
@@ -294,54 +296,47 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
       atomicMax(a.am_key + it.out_row + j0 + t, argmax_key(bv, it.n_tile * 128 + bi));
     }
     named_bar_sync(1, 128);
-  } else if constexpr (EPI == EPI_LOSS) {
-    // Softmax statistics of 16 activation rows over the tile's 128 vocabulary entries: thread
-    // (column j, group g) first takes vocabulary rows 16g..16g+15 of column j -- its max, its sum
-    // of exp(x - max) and, for a draft column, the KL cross term sum exp(q - max_q) (q - x)
-    // against the group's verifier column -- then 16 threads merge the 8 groups in order.
-    float* xchg = sm.xchg;
-#pragma unroll
-    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
-    named_bar_sync(1, 128);
-    const int t = threadIdx.x - 64, j = t & 15, grp = t >> 4;
-    const int jq = j & ~(a.loss_G - 1);
-    const int nv = min(16, a.N - (it.n_tile * 128 + grp * 16));
-    float m = -INFINITY, mq = -INFINITY;
-    for (int r = 0; r < nv; ++r) {
-      m = fmaxf(m, xchg[(grp * 16 + r) * 17 + j]);
-      mq = fmaxf(mq, xchg[(grp * 16 + r) * 17 + jq]);
-    }
-    float Z = 0.f, A = 0.f;
-    for (int r = 0; r < nv; ++r) {
-      const float x = xchg[(grp * 16 + r) * 17 + j];
-      Z += expf(x - m);
-      if (j != jq) {
-        const float q = xchg[(grp * 16 + r) * 17 + jq];
-        A += expf(q - mq) * (q - x);
-      }
-    }
-    float4* sp = reinterpret_cast<float4*>(sm.rope);
-    sp[grp * 16 + j] = make_float4(m, Z, A, mq);
-    named_bar_sync(1, 128);
-    if (t < 16 && j0 + t < it.rows) {
-      float M = -INFINITY, MQ = -INFINITY;
-#pragma unroll
-      for (int g2 = 0; g2 < 8; ++g2) {
-        const float4 p = sp[g2 * 16 + t];
-        M = fmaxf(M, p.x);
-        MQ = fmaxf(MQ, p.w);
-      }
-      float Zs = 0.f, As = 0.f;
-#pragma unroll
-      for (int g2 = 0; g2 < 8; ++g2) {
-        const float4 p = sp[g2 * 16 + t];
-        if (p.x != -INFINITY) Zs += p.y * expf(p.x - M);
-        if (p.w != -INFINITY) As += p.z * expf(p.w - MQ);
-      }
-      a.loss_part[static_cast<size_t>(it.n_tile) * a.ldo + it.out_row + j0 + t] = make_float4(M, Zs, As, MQ);
-    }
-    named_bar_sync(1, 128);
   }
+}
+
+
+// Draft-head objective (EPI_LOSS): the operands are swapped for this launch -- A is the packed
+// activation matrix (tile row = activation row, one per epilogue thread), B a tile of 256
+// vocabulary rows of W_lm (the accumulator columns) -- so each thread folds its own row's logits
+// with an online softmax, chunk by chunk: running max m and sum z of exp(x - m), and for the KL
+// term the verifier logits q of its row group (lane (lane & ~(G-1)): row 0 of the group holds
+// b_{p+1}) with running max mq and a = sum exp(q - mq) (q - x).  No shared memory, no barrier.
+struct LossState {
+  float m, z, mq, a;
+};
+__device__ __forceinline__ void loss_chunk(const GemmArgs& a, const Item& it, int j0, const float (&v)[16], LossState& st) {
+  const int lane = threadIdx.x & 31;
+  const int src = lane & ~(a.loss_G - 1);
+  const int nv = min(16, it.rows - j0);   // valid vocabulary columns of this chunk
+  float q[16];
+#pragma unroll
+  for (int jj = 0; jj < 16; ++jj) q[jj] = __shfl_sync(0xffffffffu, v[jj], src);
+  if (nv <= 0) return;
+  float xm = -INFINITY, qm = -INFINITY;
+#pragma unroll
+  for (int jj = 0; jj < 16; ++jj)
+    if (jj < nv) {
+      xm = fmaxf(xm, v[jj]);
+      qm = fmaxf(qm, q[jj]);
+    }
+  const float m1 = fmaxf(st.m, xm), q1 = fmaxf(st.mq, qm);
+  float z = (st.m == -INFINITY) ? 0.f : st.z * __expf(st.m - m1);
+  float acc = (st.mq == -INFINITY) ? 0.f : st.a * __expf(st.mq - q1);
+#pragma unroll
+  for (int jj = 0; jj < 16; ++jj)
+    if (jj < nv) {
+      z += __expf(v[jj] - m1);
+      acc += __expf(q[jj] - q1) * (q[jj] - v[jj]);
+    }
+  st.m = m1;
+  st.z = z;
+  st.mq = q1;
+  st.a = acc;
 }
 
 // Cluster split-K reduction, run by the 128 epilogue threads of every CTA of the cluster after
@@ -538,7 +533,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
       const uint64_t pol_w = a.a_keep ? l2_policy_evict_last() : l2_policy_evict_first();
-      const uint64_t pol_x = l2_policy_evict_last();
+      // (operands swapped for the objective: the streamed W_lm tiles are the B side)
+      const uint64_t pol_x = a.loss_G ? l2_policy_evict_first() : l2_policy_evict_last();
       uint32_t g = 0;   // loads issued
       bool failed = false;
       bool waited = !dense;
@@ -731,6 +727,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * acc_stride;
       const int nchunks = (it.rows + 15) >> 4;
       float v[16];
+      LossState ls = {-INFINITY, 0.f, -INFINITY, 0.f};
       if (a.split_k == 1 || a.seq_split) {
         for (int c = 0; c < nchunks; ++c) {
           if (c + 1 < nchunks) {
@@ -748,6 +745,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           if constexpr (EPI == EPI_MOE) {
             if (it.phase) epi_post<EPI_SCATTER>(a2, it, row, c * 16, v, cur, esm, c & 1);
             else epi_post<EPI_SWIGLU>(a, it, row, c * 16, v, cur, esm, c & 1);
+          } else if constexpr (EPI == EPI_LOSS) {
+            loss_chunk(a, it, c * 16, v, ls);
           } else {
             epi_post<EPI>(a, it, row, c * 16, v, cur, esm, c & 1);
           }
@@ -756,6 +755,12 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
             rope_store(esm, (c + 1) & 1, rr);
             named_bar_sync(1, 128);
           }
+        }
+        if constexpr (EPI == EPI_LOSS) {
+          // this activation row's statistics over the item's vocabulary tile
+          const int arow = it.n_tile * 128 + row;
+          if (arow < a.N)
+            a.loss_part[static_cast<size_t>(it.out_row / 256) * a.ldo + arow] = make_float4(ls.m, ls.z, ls.a, ls.mq);
         }
         if (EPI == EPI_MOE && it.phase == 0) {
           // this gate/up tile's SwiGLU rows are stored: count it for the down items of (e, m)

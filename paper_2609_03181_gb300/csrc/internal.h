@@ -117,10 +117,12 @@ struct GemmArgs {
   unsigned long long* am_key; int* am_done;
   int fin_B, fin_R; const int* fin_cand; int* fin_vtok_out; int* fin_vtok_ws; int* fin_accept_out; int* fin_m_ws;
   float* sk_ws; int* sk_tickets;                              // split-K partials / per-tile tickets
-  // LOSS: activation rows come in groups of loss_G (a power of two dividing 16): row 0 of a group
-  // is a verifier state b, rows 1.. are draft states u.  loss_part[tile * ldo + row] = (max, sum
-  // of exp(x - max), sum of exp(q - max_q) (q - x) with q the group's b-row logit, max_q), over
-  // the tile's vocabulary entries (entries >= N excluded).
+  // LOSS (operands swapped: a_map = the packed activations, tiles of 128 rows, N their count;
+  // b_map = W_lm, 256-row vocabulary tiles, M the vocabulary size): activation rows come in
+  // groups of loss_G (a power of two, 2..8), row 0 of a group a verifier state b, rows 1.. draft
+  // states u.  loss_part[vocab tile * ldo + row] = (max, sum of exp(x - max), sum of
+  // exp(q - max_q) (q - x) with q the group's b-row logit, max_q) over the tile's vocabulary.
+  // loss_G != 0 also makes dense items run through the A tiles first.
   float4* loss_part; int loss_G;
   int a_keep;                  // weight tiles loaded with the L2 evict-last policy (kept resident)
   int* err;

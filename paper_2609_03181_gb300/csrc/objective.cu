@@ -7,11 +7,13 @@
 //
 // One pass over the tied LM head, logits never written: the rows [b_{p+1}; u_p^(1); ..; u_p^(K)]
 // of every p are packed into one activation matrix (groups of G = the power of two >= K+1 rows,
-// spare rows zero), the tcgen05 GEMM engine multiplies it with each 128-token vocabulary tile of
-// W_lm and its LOSS epilogue reduces the tile to per-row softmax statistics (max, sum of
-// exp(x - max), and the KL cross term sum exp(q - max_q) (q - x) against the row's verifier
-// logits q); a finishing kernel folds the tiles of each row in tile order, adds the target logit
-// (one dot product) and the squared distance, and a last kernel averages over the valid rows.
+// spare rows zero); the tcgen05 GEMM engine, with the activations as the 128-row A operand and a
+// 256-token vocabulary tile of W_lm as the B operand, leaves each activation row's logits in one
+// thread's TMEM lane, and its LOSS epilogue folds them into per-row softmax statistics (max, sum
+// of exp(x - max), and the KL cross term sum exp(q - max_q) (q - x) against the verifier logits
+// q of the row's group, taken from the group's first lane); a finishing kernel folds the tiles of
+// each row in tile order, adds the target logit (one dot product) and the squared distance, and a
+// last kernel averages over the valid rows.
 // KL(Q || P) = sum_v Q(v) (q_v - x_v) - lse(q) + lse(x), the sum being A / Z_q.
 #include <math.h>
 #include <string.h>
@@ -33,7 +35,7 @@ constexpr int kLossMaxRows = 1 << 16;   // packed activation rows (n_rows * G)
 static __device__ int g_loss_err;
 
 struct LossLayout {
-  int G, M, box_log, box, M_pad, m_tiles, n_tiles;
+  int G, M, M_pad, a_tiles, v_tiles;   // packed rows, padded to 128-row A tiles; 256-token vocabulary tiles
   size_t x_off, part_off, rows_off, total;
 };
 
@@ -44,16 +46,12 @@ LossLayout loss_layout(int K, int n_rows, int vocab) {
   L.G = 2;
   while (L.G < K + 1) L.G <<= 1;
   L.M = n_rows * L.G;
-  int bl = 0;
-  while ((16 << bl) < (L.M < 256 ? L.M : 256) && bl < 4) ++bl;
-  L.box_log = bl;
-  L.box = 16 << bl;
-  L.M_pad = (L.M + L.box - 1) / L.box * L.box;
-  L.m_tiles = L.M_pad / L.box;
-  L.n_tiles = (vocab + 127) / 128;
+  L.M_pad = (L.M + 127) / 128 * 128;
+  L.a_tiles = L.M_pad / 128;
+  L.v_tiles = (vocab + 255) / 256;
   L.x_off = 0;
   L.part_off = align256(static_cast<size_t>(L.M_pad) * kD * sizeof(bf16));
-  L.rows_off = L.part_off + align256(static_cast<size_t>(L.n_tiles) * L.M_pad * sizeof(float4));
+  L.rows_off = L.part_off + align256(static_cast<size_t>(L.v_tiles) * L.M_pad * sizeof(float4));
   L.total = L.rows_off + align256(static_cast<size_t>(K) * n_rows * 3 * sizeof(float));
   return L;
 }
@@ -252,18 +250,20 @@ extern "C" spec_status spec_draft_loss(const void* u, const void* b_next, const 
   GemmArgs g;
   memset(&g, 0, sizeof(g));
   std::string err;
-  if (!encode_map_2d(&g.a_map[0], lm_head, kD, vocab, 128, &err)) return fail(SPEC_EINVAL, err);
-  if (!encode_act_maps(g.b_map[0], X, kD, L.M_pad, &err)) return fail(SPEC_EINVAL, err);
+  // operands swapped: A = the packed activation rows (128-row tiles), B = W_lm (256-row boxes)
+  if (!encode_map_2d(&g.a_map[0], X, kD, L.M_pad, 128, &err)) return fail(SPEC_EINVAL, err);
+  if (!encode_act_maps(g.b_map[0], lm_head, kD, vocab, &err)) return fail(SPEC_EINVAL, err);
   g.n_routed = 1 << 30;
-  g.N = vocab;
+  g.N = L.M_pad;
   g.K = kD;
-  g.M = L.M_pad;
-  g.box_log = L.box_log;
-  g.m_tiles = L.m_tiles;
-  g.n_tiles = L.n_tiles;
+  g.M = vocab;
+  g.box_log = 4;
+  g.m_tiles = L.v_tiles;
+  g.n_tiles = L.a_tiles;
   g.split_k = 1;
-  g.n_items = L.n_tiles * L.m_tiles;
+  g.n_items = L.v_tiles * L.a_tiles;
   g.ldo = L.M_pad;
+  g.a_keep = 1;   // the packed rows are read once per vocabulary tile: keep them in L2
   g.loss_part = part;
   g.loss_G = L.G;
   g.err = g_err_ptr[dev];
@@ -280,10 +280,10 @@ extern "C" spec_status spec_draft_loss(const void* u, const void* b_next, const 
   e = cudaGetLastError();
   if (e == cudaSuccess) {
     const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
-    e = gemm_launch(EPI_LOSS, L.box <= 64 ? 64 : 256, g, grid, s, false);
+    e = gemm_launch(EPI_LOSS, 256, g, grid, s, false);
   }
   if (e == cudaSuccess) {
-    loss_finish_kernel<<<n_rows, 32 * (K + 1), 0, s>>>(part, L.M_pad, L.n_tiles, L.G, K, n_rows,
+    loss_finish_kernel<<<n_rows, 32 * (K + 1), 0, s>>>(part, L.M_pad, L.v_tiles, L.G, K, n_rows,
                                                       static_cast<const bf16*>(u), static_cast<const bf16*>(b_next),
                                                       target, static_cast<const bf16*>(lm_head), vocab, rows);
     e = cudaGetLastError();

@@ -56,8 +56,9 @@ def test_draft_loss_host_checks_without_gpu():
     assert lib.spec_draft_loss_workspace(0, 4, 100, ctypes.byref(n)) == F.SPEC_EINVAL and n.value == 0
     assert lib.spec_draft_loss_workspace(3, 64, 129280, None) == F.SPEC_EINVAL
     assert lib.spec_draft_loss_workspace(3, 64, 129280, ctypes.byref(n)) == F.SPEC_OK
-    # packed rows 64 x 4 = 256 bf16 rows of 1280, 1010 tiles x 256 rows of 16-byte partials, 3 x 64 x 3 floats
-    assert n.value == 256 * 1280 * 2 + 1010 * 256 * 16 + 2304   # each part a multiple of 256 bytes
+    # packed rows 64 x 4 = 256 bf16 rows of 1280, 505 vocabulary tiles of 256 x 256 rows of 16-byte
+    # partials, 3 x 64 x 3 floats; each part a multiple of 256 bytes
+    assert n.value == 256 * 1280 * 2 + 505 * 256 * 16 + 2304
     assert lib.spec_draft_loss(None, None, None, None, None, 3, 4, 100, ctypes.c_float(0.6), ctypes.c_float(0.85),
                                ctypes.c_float(0.45), ctypes.c_float(0.45), None, None, None, 0, None) == F.SPEC_EINVAL
     assert b"null" in lib.spec_last_error(None)
