@@ -32,6 +32,12 @@ the rotated queries and K/V that feed the attention products, attention outputs,
 activations, the states b and u); everything between those points stays fp64.  `rb=False` is
 the plain definition.
 
+fp8-expert variant (not in the paper; a precision option of this library): when a layer carries
+e4m3 expert weights with one fp32 scale per output row (synth_inputs.quantize_experts_fp8), the
+oracle dequantises them exactly (code value x scale, in fp64) and rounds the two tensors that enter
+the expert products, the normalised input rows and the SwiGLU activations, to e4m3 (ties to even,
+saturating at 448), where the bf16 path rounds the activations to bf16.
+
 Parity of absolute hidden-state values on random weights is pinned only through the special
 cases and invariants in tests/test_oracle_pins.py (closed forms, brute force, the identity
 draft block, losslessness); beyond those the values are parity unpinned.
@@ -48,7 +54,7 @@ import torch
 F64 = torch.float64
 
 __all__ = [
-    "round_bf16", "rms_norm", "rope", "attention", "silu", "swiglu", "router_topk",
+    "round_bf16", "round_e4m3", "decode_e4m3", "dequant_rows", "rms_norm", "rope", "attention", "silu", "swiglu", "router_topk",
     "argmax_with_gap", "accept_length", "SeqCache", "DraftCache", "Verifier", "Drafter",
     "VerifyOut", "DraftOut", "verify", "commit", "draft", "greedy_decode",
     "speculative_decode", "DecodeStats",
@@ -66,6 +72,38 @@ def round_bf16(x: torch.Tensor) -> torch.Tensor:
     m, e = np.frexp(a)                     # a = m * 2**e with 0.5 <= |m| < 1
     r = np.rint(m * 256.0) / 256.0         # keep 8 significant bits; rint ties to even
     return torch.from_numpy(np.ldexp(r, e)).reshape(x.shape)
+
+
+E4M3_MAX = 448.0
+
+
+def round_e4m3(x: torch.Tensor) -> torch.Tensor:
+    """Round to the nearest e4m3 value (1 sign, 4 exponent bits with bias 7, 3 mantissa bits, no
+    infinities), ties to even, saturating: |x| >= 448 gives +-448.  Normal values keep 4
+    significant bits (|x| >= 2^-6); below that the grid is the subnormal step 2^-9."""
+    a = np.clip(x.detach().to(F64).contiguous().numpy(), -E4M3_MAX, E4M3_MAX)
+    m, e = np.frexp(a)                                   # a = m * 2**e, 0.5 <= |m| < 1
+    normal = np.ldexp(np.rint(m * 16.0) / 16.0, e)       # 4 significant bits, rint ties to even
+    sub = np.rint(a / 2.0 ** -9) * 2.0 ** -9
+    r = np.where(np.abs(a) >= 2.0 ** -6, normal, sub)
+    return torch.from_numpy(np.clip(r, -E4M3_MAX, E4M3_MAX)).reshape(x.shape)
+
+
+def decode_e4m3(codes: torch.Tensor) -> torch.Tensor:
+    """Values of e4m3 byte codes (uint8): sign bit 7, exponent bits 6..3 (bias 7), mantissa bits
+    2..0; exponent 0 is subnormal, m * 2^-9."""
+    b = codes.to(torch.int64)
+    s = torch.where((b >> 7) & 1 == 1, -1.0, 1.0).to(F64)
+    e = (b >> 3) & 15
+    m = (b & 7).to(F64)
+    normal = (1.0 + m / 8.0) * torch.pow(torch.tensor(2.0, dtype=F64), (e - 7).to(F64))
+    sub = m * 2.0 ** -9
+    return s * torch.where(e == 0, sub, normal)
+
+
+def dequant_rows(codes: torch.Tensor, scale: torch.Tensor) -> torch.Tensor:
+    """fp8 weight matrix [.., rows, k] with one fp32 scale per row [.., rows]: values * scale."""
+    return decode_e4m3(codes) * f64(scale)[..., None]
 
 
 def _rb(x: torch.Tensor, on: bool) -> torch.Tensor:
@@ -124,13 +162,18 @@ def silu(x: torch.Tensor) -> torch.Tensor:
     return x / (1.0 + torch.exp(-x))
 
 
-def swiglu(x: torch.Tensor, w_gate_up: torch.Tensor, w_down: torch.Tensor, rb: bool) -> torch.Tensor:
-    """SwiGLU FFN: W_down (silu(W_gate x) * W_up x).  w_gate_up: [2I][d], gate rows first."""
+def swiglu(x: torch.Tensor, w_gate_up: torch.Tensor, w_down: torch.Tensor, rb: bool, fp8: bool = False) -> torch.Tensor:
+    """SwiGLU FFN: W_down (silu(W_gate x) * W_up x).  w_gate_up: [2I][d], gate rows first.
+
+    fp8=True is the fp8-expert variant (not in the paper): the weights given are the dequantised
+    e4m3 matrices, and the two tensors that enter the expert products -- the input rows and the
+    SwiGLU activations -- are rounded to e4m3 (instead of the activations to bf16)."""
     I = w_gate_up.shape[0] // 2
     wgu = f64(w_gate_up)
-    g = f64(x) @ wgu[:I].T
-    u = f64(x) @ wgu[I:].T
-    act = _rb(silu(g) * u, rb)
+    xi = round_e4m3(f64(x)) if fp8 else f64(x)
+    g = xi @ wgu[:I].T
+    u = xi @ wgu[I:].T
+    act = round_e4m3(silu(g) * u) if fp8 else _rb(silu(g) * u, rb)
     return act @ f64(w_down).T
 
 
@@ -255,15 +298,24 @@ def _moe(model: Verifier, lw, x: torch.Tensor, rb: bool):
     s = model.s
     idx, gates, _, gap = router_topk(x, lw.router, s.top_k, lw.router_bias)
     n = x.shape[0]
+    fp8 = getattr(lw, "w_gate_up_f8", None) is not None     # the fp8-expert variant
+    if fp8:
+        wgu = lambda e: dequant_rows(lw.w_gate_up_f8[e], lw.gate_up_scale[e])
+        wdn = lambda e: dequant_rows(lw.w_down_f8[e], lw.down_scale[e])
+        sgu = lambda j: dequant_rows(lw.shared_gate_up_f8[j], lw.shared_gate_up_scale[j])
+        sdn = lambda j: dequant_rows(lw.shared_down_f8[j], lw.shared_down_scale[j])
+    else:
+        wgu, wdn = (lambda e: lw.w_gate_up[e]), (lambda e: lw.w_down[e])
+        sgu, sdn = (lambda j: lw.shared_gate_up[j]), (lambda j: lw.shared_down[j])
     y_slot = torch.zeros(n, s.top_k, s.hidden, dtype=F64)
     for e in sorted(set(idx.flatten().tolist())):
         rows, slots = torch.nonzero(idx == e, as_tuple=True)
-        y_slot[rows, slots] = swiglu(x[rows], lw.w_gate_up[e], lw.w_down[e], rb)
+        y_slot[rows, slots] = swiglu(x[rows], wgu(e), wdn(e), rb, fp8)
     out = torch.zeros(n, s.hidden, dtype=F64)
     for k in range(s.top_k):
         out = out + gates[:, k:k + 1] * y_slot[:, k]
     for j in range(s.n_shared):
-        out = out + swiglu(x, lw.shared_gate_up[j], lw.shared_down[j], rb)
+        out = out + swiglu(x, sgu(j), sdn(j), rb, fp8)
     return out, idx, gates, gap
 
 

@@ -269,6 +269,34 @@ def successor_weights(shape: ModelShape, seed: int, beta_over_alpha: float, alph
     return vw, dw, pi
 
 
+def quantize_experts_fp8(vw: "VerifierWeights") -> "VerifierWeights":
+    """The fp8-expert variant of a verifier (input construction only): every routed and shared
+    expert matrix stored as e4m3 byte codes with one fp32 scale per output row, scale =
+    max |row| / 448, codes = the row divided by its scale rounded to the nearest e4m3 value (ties
+    to even, through PyTorch's float8_e4m3fn conversion).  Adds the fields w_gate_up_f8,
+    gate_up_scale, w_down_f8, down_scale, shared_gate_up_f8, shared_gate_up_scale,
+    shared_down_f8, shared_down_scale (uint8 codes, fp32 scales) to a copy of every layer; the
+    bf16 matrices stay as they were."""
+    import copy
+
+    def q(w):
+        wf = w.float()
+        sc = wf.abs().amax(-1).clamp_min(1e-30) / 448.0
+        codes = (wf / sc[..., None]).clamp(-448.0, 448.0).to(torch.float8_e4m3fn).view(torch.uint8)
+        return codes.contiguous(), sc.contiguous()
+
+    out = copy.copy(vw)
+    out.layers = []
+    for lw in vw.layers:
+        l2 = copy.copy(lw)
+        l2.w_gate_up_f8, l2.gate_up_scale = q(lw.w_gate_up)
+        l2.w_down_f8, l2.down_scale = q(lw.w_down)
+        l2.shared_gate_up_f8, l2.shared_gate_up_scale = q(lw.shared_gate_up)
+        l2.shared_down_f8, l2.shared_down_scale = q(lw.shared_down)
+        out.layers.append(l2)
+    return out
+
+
 def kv_prefix_device(seed: int, seq: int, n_layers: int, ctx: int, n_heads: int, head_dim: int,
                      device) -> torch.Tensor:
     """Like kv_prefix, drawn on `device` by PyTorch's seeded generator (a different stream from
