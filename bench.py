@@ -152,16 +152,16 @@ def job_totals(ms, tokens, world, device):
     return float(t.item()), int(n.item())
 
 
-def algorithmic_bytes(shape, B, K, ctx_mean, experts_touched_routed_per_layer):
+def algorithmic_bytes(shape, B, K, ctx_mean, experts_touched_routed_per_layer, fp8_experts=False):
     """Bytes the verify step must move: every weight matrix it reads once (routed experts counted
-    from the actual routing), the committed KV it reads, the candidate KV it writes and the
-    embedding rows."""
+    from the actual routing; e4m3 experts one byte per weight plus an fp32 scale per row), the
+    committed KV it reads, the candidate KV it writes and the embedding rows."""
     d, H, hd, I, E, L, V = (shape.hidden, shape.n_heads, shape.head_dim, shape.expert_inter, shape.n_experts,
                             shape.n_layers, shape.vocab)
     T = B * (K + 1)
     attn_w = 2 * (3 * H * hd * d + d * H * hd)
     router_w = 2 * E * d
-    expert_w = 2 * 3 * d * I
+    expert_w = (3 * d * I + 4 * (2 * I + d)) if fp8_experts else 2 * 3 * d * I
     shared_w = shape.n_shared * expert_w
     kv_tok = 2 * H * hd * 2
     per_layer = attn_w + router_w + shared_w + expert_w * experts_touched_routed_per_layer
@@ -389,6 +389,67 @@ def run_points(args, shape, vw, dw, dev, peak, peak_kind):
     return out
 
 
+def run_fp8_point(args, shape, vw, dw, ctx, pend, kvs, dkvs, dev, peak, peak_kind):
+    """The bench step (draft + verify + commit, B=8, K=3, the same inputs) with the fp8-expert
+    variant: expert matrices quantised to e4m3 with per-row scales (input construction on the
+    host), e4m3 expert products.  Event pairs around each phase, per-step medians."""
+    import torch
+
+    import synth_inputs as S
+    from paper_2609_03181_gb300 import fastmtp as F
+
+    B, K = args.batch, args.K
+    v8 = S.quantize_experts_fp8(vw)
+    n_all = args.warmup + args.steps
+    stream = torch.cuda.Stream(dev)
+    eng = F.Engine(v8, dw, max_batch=B, K_max=K, max_ctx=max(ctx) + (n_all + 4) * (K + 1) + 8, page_size=64,
+                   device=str(dev), stream=stream, expert_fp8=True)
+    for b in range(B):
+        eng.load_prefix(b, kvs[b], dkvs[b], pend[b])
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    c0 = torch.tensor([[p] for p in pend], dtype=torch.int32, device=dev)
+    v0 = torch.empty(B, 1, dtype=torch.int32, device=dev)
+    acc = torch.empty(B, dtype=torch.int32, device=dev)
+    cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    com = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    hist = torch.zeros(n_all, B, dtype=torch.int32, device=dev)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_all)]
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        eng.verify_step(slots, c0, v0, acc)
+        eng.accept_commit(slots, v0, acc)
+        for i in range(n_all):
+            if i == args.warmup:
+                eng.profile(2)
+            ev[i][0].record(stream)
+            eng.draft_step(slots, K, cand)
+            ev[i][1].record(stream)
+            eng.verify_step(slots, cand, vt, acc)
+            ev[i][2].record(stream)
+            eng.accept_commit(slots, com, hist[i])
+            ev[i][3].record(stream)
+    eng.sync()
+    counted = eng.profile_read()
+    eng.close()
+    del eng
+    torch.cuda.empty_cache()
+    timed = range(args.warmup, n_all)
+    med = lambda a, b: statistics.median(ev[i][a].elapsed_time(ev[i][b]) for i in timed)
+    ms_step, ms_verify = med(0, 3), med(1, 2)
+    h = hist.double().cpu()
+    tok = float(h[args.warmup:].sum())
+    touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
+    ctx_mean = statistics.mean(ctx) + (args.warmup + args.steps / 2) * 2
+    vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared, fp8_experts=True)
+    return {"variant": "fp8 experts: e4m3 expert matrices with a per-row fp32 scale, e4m3 expert inputs and "
+                       "activations (no counterpart in the paper)",
+            "batch": B, "K": K, "steps": args.steps, "tokens_per_s": tok / (ms_step * args.steps / 1000.0),
+            "ms_step": ms_step, "ms_verify": ms_verify, "ms_draft": med(0, 1), "tau": tok / (args.steps * B),
+            "verify_roofline": {"frac": vbytes / ms_verify / 1e6 / peak, "achieved_gbs": vbytes / ms_verify / 1e6,
+                                "bytes": vbytes, "peak_source": peak_kind}}
+
+
 LOSS_ROWS, LOSS_K = 64, 3
 
 
@@ -576,10 +637,12 @@ def run_fastmtp(args):
     torch.cuda.empty_cache()
     points = None
     loss_point = None
+    fp8_point = None
     if not args.no_points and world == 1:
         pk, pkind = measured_peaks()
         points = run_points(args, shape, vw, dw, dev, pk, pkind)
         loss_point = run_loss_point(args, shape, dev, pk, pkind)
+        fp8_point = run_fp8_point(args, shape, vw, dw, ctx, pend, kvs, dkvs, dev, pk, pkind)
 
     if rank != 0:
         if world > 1:
@@ -644,6 +707,7 @@ def run_fastmtp(args):
                              "between kernels (sums exceed ms_per_step; roofline.avg_launch_ms is from it)"),
         "sweep_points": points,
         "draft_objective": loss_point,
+        "fp8_experts": fp8_point,
         "tau": accepted / (steps * B), "accept_hist_m": m_hist,
         "experts_touched_per_layer": touched,
         "gpu_launches": launches_total,
@@ -679,7 +743,7 @@ def run_sweep(args):
     peak, peak_kind = measured_peaks()
     shape = S.ModelShape(n_layers=args.layers)
     Bmax, Kmax = max(batches), max(Ks)
-    steps_for = lambda B: max(args.steps, 50) if B == 1 else args.steps   # B=1 acceptance varies most
+    steps_for = lambda B: max(args.steps, 50) if B <= 4 else args.steps   # acceptance varies most at small B
     grow = (args.warmup + steps_for(1) + 2) * (Kmax + 1)
     clocks = ClockSampler(0)
     clocks.start()

@@ -72,6 +72,13 @@ typedef struct spec_config {
   int32_t K_max;              /* largest draft depth K, 0..7 */
   int32_t max_position;       /* RoPE table length (position limit, e.g. 32768) */
   float rms_eps, rope_theta;  /* 1e-6, 1e6 */
+  /* 0: bf16 expert weights (the paper's model).  1: fp8 experts, a precision option with no
+   * counterpart in the paper: the routed and shared expert matrices are e4m3 byte codes (1 sign,
+   * 4 exponent bits with bias 7, 3 mantissa bits) with one fp32 scale per output row (the
+   * *_scale pointers of spec_layer_weights), and the rows entering the expert products (the
+   * normalised token rows and the SwiGLU activations) are rounded to e4m3 (ties to even,
+   * saturating at 448); products in fp32 (tcgen05 kind::f8f6f4). */
+  int32_t expert_fp8;
 } spec_config;
 
 /* One verifier layer (all dev, bf16 unless noted). */
@@ -86,6 +93,13 @@ typedef struct spec_layer_weights {
   const void* shared_gate_up;  /* [n_shared][2I][d] */
   const void* shared_down;     /* [n_shared][d][I] */
   const float* router_bias;    /* fp32 [E] added to the router logits, or NULL */
+  /* expert_fp8 only (else ignored): fp32 scale of every row of w_gate_up [E][2I], w_down [E][d],
+   * shared_gate_up [n_shared][2I], shared_down [n_shared][d]; the four expert matrices above
+   * are then e4m3 codes (1 byte per element, same shapes). */
+  const float* gate_up_scale;
+  const float* down_scale;
+  const float* shared_gate_up_scale;
+  const float* shared_down_scale;
 } spec_layer_weights;
 
 /* All weights (dev, bf16).  E, N_o and W_lm are shared by the verifier and the draft head
@@ -192,6 +206,15 @@ spec_status spec_read_workspace(spec_ctx* ctx, int32_t id, void* dst, size_t byt
  * pointers 16-byte aligned.  Asynchronous on `stream`; needs no context.  Errors:
  * SPEC_EINVAL, SPEC_ECUDA. */
 spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, int32_t N,
+                           int32_t Kdim, void* stream);
+
+/* Dense e4m3 projection Y = (X W^T) * scale on the same tcgen05 engine as the fp8 experts
+ * (kind::f8f6f4): X dev e4m3 codes [M][Kdim], W dev e4m3 codes [N][Kdim] (1 sign, 4 exponent
+ * bits with bias 7, 3 mantissa bits), w_scale dev fp32 [N] (one per row of W), Y dev fp32
+ * [M][N]; Kdim a multiple of 128, both code pointers 16-byte aligned.  A precision option with
+ * no counterpart in the paper.  Asynchronous on `stream`; needs no context.  Errors:
+ * SPEC_EINVAL, SPEC_ECUDA; device-side faults via spec_sync(NULL). */
+spec_status spec_gemm_e4m3(const void* X, const void* W, const float* w_scale, float* Y, int32_t M, int32_t N,
                            int32_t Kdim, void* stream);
 
 /* Kernel-class timing for measurement.  spec_profile(ctx, mode): mode 1 zeroes the counters

@@ -14,6 +14,7 @@
 // order; split-K partials are reduced by the last-arriving CTA of a tile in split order (an
 // atomic ticket, no spin-wait).  Split counts depend on the matrix shape only, so a row's
 // result never depends on how many other rows share the launch.
+#include <cuda_fp8.h>
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -198,6 +199,11 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
                                          const EpiPre& p, const EpiSmem& sm, int rope_buf) {
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
     const int n = it.n_tile * 128 + row;
+    if (EPI == EPI_F32 && a.f8 && n < a.N) {   // e4m3 GEMM: each weight row's scale
+      const float sc = a.w_scale[0][n];
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) v[jj] *= sc;
+    }
     if (n < a.N) {
       float* base = a.out + static_cast<size_t>(it.out_row + j0) * a.ldo + n;
 #pragma unroll
@@ -206,14 +212,25 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
     }
   } else if constexpr (EPI == EPI_SCATTER) {
     const int n = it.n_tile * 128 + row;
+    float sc = 1.f;   // fp8 experts: the scale of output feature n's weight row
+    if (a.f8)
+      sc = ((it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
+                                : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows)[n];
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj)
       if (j0 + jj < it.rows)
-        a.y[(static_cast<size_t>(sm.s_pos[j0 + jj]) * kSlots + sm.s_aux[j0 + jj]) * kD + n] = v[jj];
+        a.y[(static_cast<size_t>(sm.s_pos[j0 + jj]) * kSlots + sm.s_aux[j0 + jj]) * kD + n] = v[jj] * sc;
   } else if constexpr (EPI == EPI_SWIGLU) {
     float* xchg = sm.xchg;
+    float sc = 1.f;   // fp8 experts: this weight row's scale (tile rows 0..63 gate, 64..127 up)
+    if (a.f8) {
+      const int wr = (row < 64) ? it.n_tile * 64 + row : a.half_rows + it.n_tile * 64 + (row - 64);
+      const float* ws = (it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
+                                            : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows;
+      sc = ws[wr];
+    }
 #pragma unroll
-    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
+    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj] * sc;
     named_bar_sync(1, 128);
     if (row < 64) {
       const int f = it.n_tile * 64 + row;
@@ -222,7 +239,10 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
         const int r = j0 + jj;
         if (r < it.rows) {
           const float u = xchg[(row + 64) * 17 + jj];
-          a.act[static_cast<size_t>(it.out_row + r) * a.ld_act + f] = __float2bfloat16(silu_f(v[jj]) * u);
+          const float y = silu_f(v[jj] * sc) * u;
+          const size_t at = static_cast<size_t>(it.out_row + r) * a.ld_act + f;
+          if (a.f8) a.act8[at] = __nv_cvt_float_to_fp8(y, __NV_SATFINITE, __NV_E4M3);
+          else a.act[at] = __float2bfloat16(y);
         }
       }
     }
@@ -542,7 +562,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         Item it;
         get_item(a, a2, i, it, grp);
         const GemmArgs& P = it.phase ? a2 : a;   // the item's operands (EPI_MOE down items: a2)
-        const int kc_total = P.K / 64;
+        const int kw = P.f8 ? 128 : 64;           // elements of a 128-byte k-chunk
+        const int kc_total = P.K / kw;
         const int src = (!dense && it.e >= a.n_routed) ? 1 : 0;
         const int el = it.e - (src ? a.n_routed : 0);
         const CUtensorMap* amap = &P.a_map[src];
@@ -552,7 +573,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         const int kc1 = a.seq_split ? kc_total : (it.split + 1) * kc_total / a.split_k;
         auto load_a = [&](int st, int kc) {
           uint8_t* sa = smA + st * C::A_BYTES;
-          const int k = kc * 64;
+          const int k = kc * kw;
           if (P.paired) {
             const int r0 = it.n_tile * 64;
             if (P.a3d) {
@@ -596,7 +617,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           pdl_wait();
           waited = true;
           for (int q = 0; q < npre; ++q)
-            tma_load_2d(smB + q * C::B_BYTES, bmap, &full[q], (kc0 + q) * 64, it.b_row, pol_x);
+            tma_load_2d(smB + q * C::B_BYTES, bmap, &full[q], (kc0 + q) * kw, it.b_row, pol_x);
           g = npre;
           kc = kc0 + npre;
         }
@@ -609,7 +630,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           }
           mbar_arrive_expect_tx(&full[st], bytes);
           load_a(st, kc);
-          tma_load_2d(smB + st * C::B_BYTES, bmap, &full[st], kc * 64, it.b_row, pol_x);
+          tma_load_2d(smB + st * C::B_BYTES, bmap, &full[st], kc * kw, it.b_row, pol_x);
         }
       }
       if (!waited) pdl_wait();
@@ -634,7 +655,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x, ++local) {
         Item it;
         get_item(a, a2, i, it, grp);
-        const int kc_total = (it.phase ? a2.K : a.K) / 64;
+        const bool f8 = (it.phase ? a2.f8 : a.f8) != 0;
+        const int kc_total = (it.phase ? a2.K : a.K) / (f8 ? 128 : 64);
         const int acc = local % nbuf;
         const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
         if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, s_abort)) {
@@ -642,7 +664,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           break;
         }
         tc_fence_after();
-        const uint32_t idesc = idesc_bf16(128, 16 << it.box_log);
+        const uint32_t idesc = f8 ? idesc_e4m3(128, 16 << it.box_log) : idesc_bf16(128, 16 << it.box_log);
         const int kc0 = a.seq_split ? 0 : it.split * kc_total / a.split_k;
         const int kc1 = a.seq_split ? kc_total : (it.split + 1) * kc_total / a.split_k;
         // with in-CTA splits, split sp accumulates k-chunks [sp*kc/S, (sp+1)*kc/S) into its own
@@ -664,9 +686,16 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           tc_fence_after();
           const uint64_t ad = sw128_kmajor_desc(smem_u32(smA + st * C::A_BYTES));
           const uint64_t bd = sw128_kmajor_desc(smem_u32(smB + st * C::B_BYTES));
+          // 4 MMAs per 128-byte k-chunk (K=16 bf16 or K=32 e4m3 each): +32 B in the swizzled row
+          if (f8) {
 #pragma unroll
-          for (int s = 0; s < 4; ++s)   // 4 x K=16 per 64-column chunk: +32 B in the swizzled row
-            tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+            for (int s = 0; s < 4; ++s)
+              tc_mma_e4m3(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+          } else {
+#pragma unroll
+            for (int s = 0; s < 4; ++s)
+              tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+          }
           tc_commit(&empty[st]);
         }
         if (failed) break;
@@ -961,17 +990,18 @@ cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
 }  // namespace
 
 bool encode_map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
-                   std::string* err) {
+                   std::string* err, int elem_bytes) {
   auto fn = get_encode();
   if (fn == nullptr) {
     *err = "cuTensorMapEncodeTiled not available from the driver";
     return false;
   }
   cuuint64_t dims[2] = {inner, rows};
-  cuuint64_t strides[1] = {inner * 2};
-  cuuint32_t box[2] = {64, box_rows};
+  cuuint64_t strides[1] = {inner * static_cast<cuuint64_t>(elem_bytes)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(128 / elem_bytes), box_rows};
   cuuint32_t es[2] = {1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+  const CUtensorMapDataType dt = elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  CUresult r = fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, es,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
@@ -982,17 +1012,19 @@ bool encode_map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t ro
 }
 
 bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t depth,
-                   uint32_t box_rows, std::string* err) {
+                   uint32_t box_rows, std::string* err, int elem_bytes) {
   auto fn = get_encode();
   if (fn == nullptr) {
     *err = "cuTensorMapEncodeTiled not available from the driver";
     return false;
   }
+  const cuuint64_t eb = static_cast<cuuint64_t>(elem_bytes);
   cuuint64_t dims[3] = {inner, rows, depth};
-  cuuint64_t strides[2] = {inner * 2, inner * rows * 2};
-  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint64_t strides[2] = {inner * eb, inner * rows * eb};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(128 / elem_bytes), box_rows, 1};
   cuuint32_t es[3] = {1, 1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+  const CUtensorMapDataType dt = elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  CUresult r = fn(m, dt, 3, const_cast<void*>(base), dims, strides, box, es,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
@@ -1002,9 +1034,10 @@ bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t ro
   return true;
 }
 
-bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err) {
+bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err,
+                     int elem_bytes) {
   for (int b = 0; b < 5; ++b)
-    if (!encode_map_2d(&maps[b], base, inner, rows, 16u << b, err)) return false;
+    if (!encode_map_2d(&maps[b], base, inner, rows, 16u << b, err, elem_bytes)) return false;
   return true;
 }
 

@@ -125,16 +125,26 @@ struct GemmArgs {
   // loss_G != 0 also makes dense items run through the A tiles first.
   float4* loss_part; int loss_G;
   int a_keep;                  // weight tiles loaded with the L2 evict-last policy (kept resident)
+  // fp8 experts: both operands e4m3 bytes (k-chunks of 128 elements, tcgen05 kind::f8f6f4); the
+  // SWIGLU / SCATTER epilogues multiply each weight row's accumulator by its fp32 scale
+  // (w_scale[0]: routed experts [E][scale_rows], w_scale[1]: shared experts), and SWIGLU writes
+  // its rows as e4m3 to act8.
+  int f8;
+  const float* w_scale[2];
+  int scale_rows;
+  uint8_t* act8;
   int* err;
 };
 
-// Encodes a 2-D or 3-D bf16 tensor map with the 128-byte swizzle (box inner dim 64).
+// Encodes a 2-D or 3-D tensor map with the 128-byte swizzle: bf16 elements (elem_bytes 2, box
+// inner dim 64) or e4m3 bytes (elem_bytes 1, box inner dim 128); `inner` counts elements.
 bool encode_map_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
-                   std::string* err);
+                   std::string* err, int elem_bytes = 2);
 bool encode_map_3d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t depth,
-                   uint32_t box_rows, std::string* err);
-// Fills b_map[src][*] for an activation buffer of `rows` x `inner` bf16.
-bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err);
+                   uint32_t box_rows, std::string* err, int elem_bytes = 2);
+// Fills b_map[src][*] for an activation buffer of `rows` x `inner` elements.
+bool encode_act_maps(CUtensorMap (&maps)[5], const void* base, uint64_t inner, uint64_t rows, std::string* err,
+                     int elem_bytes = 2);
 
 // Launches the persistent tcgen05 GEMM; nmax = 64 or 256 (largest row box of any item).
 // pdl = false launches without programmatic serialization (for streams whose earlier kernels
@@ -221,6 +231,10 @@ struct RouteArgs {
   int* rowmap;     // [64][map_stride] per expert: (token << 3 | rank) of each of its rows
   bf16* x_sorted;  // [64][map_stride][d] per expert: its input rows (the rounded xn rows)
   int map_stride;  // >= T
+  // fp8 experts (else NULL): the rows rounded to e4m3 -- every token row into xn8 [T][d] (the
+  // shared experts' input) and each selection into x_sorted8 [64][map_stride][d] instead of x_sorted
+  uint8_t* xn8;
+  uint8_t* x_sorted8;
 };
 cudaError_t router_launch(const RouteArgs& a, cudaStream_t s);
 cudaError_t combine_launch(float* h, const float* y, const float* gate, int T, const bf16* gain, float eps,

@@ -89,6 +89,12 @@ struct spec_ctx {
   int dep_stride = 0;
   bf16* x_sorted = nullptr;
   bf16* act = nullptr;
+  // fp8 experts: e4m3 copies of the expert inputs and SwiGLU activations (else NULL)
+  bool fp8 = false;
+  uint8_t* x_sorted8 = nullptr;   // [n_experts][Tcap][d]
+  uint8_t* xn8 = nullptr;         // [Tmax][d]
+  uint8_t* act8 = nullptr;        // [n_experts + n_shared][Tcap][I]
+  ActMaps a_xs8{}, a_xn8{}, a_act8{};
   float* y = nullptr;
   bf16* b_ws = nullptr;
   unsigned long long* am_key = nullptr;   // packed (logit, token) per row of the LM head
@@ -374,6 +380,7 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
     return fail(nullptr, SPEC_EINVAL, "config field out of range");
   if (c.max_batch * (c.K_max + 1) > 2048)
     return fail(nullptr, SPEC_EINVAL, "max_batch * (K_max + 1) must be <= 2048");
+  if (c.expert_fp8 != 0 && c.expert_fp8 != 1) return fail(nullptr, SPEC_EINVAL, "expert_fp8 must be 0 or 1");
   if (w->layers == nullptr || w->embed == nullptr || w->lm_head == nullptr || w->final_norm == nullptr ||
       w->enorm == nullptr || w->hnorm == nullptr || w->eh_proj == nullptr || w->mtp_attn_norm == nullptr ||
       w->mtp_wqkv == nullptr || w->mtp_wo == nullptr || w->mtp_ffn_norm == nullptr || w->mtp_w_gate_up == nullptr ||
@@ -385,6 +392,9 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
                         L.shared_gate_up, L.shared_down};
     for (const void* p : ps)
       if (p == nullptr || !aligned16(p)) return fail(nullptr, SPEC_EINVAL, "layer weight NULL or not 16-byte aligned");
+    if (c.expert_fp8 && (L.gate_up_scale == nullptr || L.down_scale == nullptr || L.shared_gate_up_scale == nullptr ||
+                         L.shared_down_scale == nullptr))
+      return fail(nullptr, SPEC_EINVAL, "expert_fp8: a layer's expert scales are NULL");
   }
   const void* top[] = {w->embed, w->lm_head, w->eh_proj, w->mtp_wqkv, w->mtp_wo, w->mtp_w_gate_up, w->mtp_w_down,
                        kv_pool, draft_kv_pool};
@@ -453,6 +463,12 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   add(&ctx->moe_dep, sizeof(int) * L * (kE + kShared) * ctx->dep_stride);
   add(&ctx->x_sorted, sizeof(bf16) * kE * ctx->Tcap * d);
   add(&ctx->act, sizeof(bf16) * (kE + kShared) * ctx->Tcap * kI);
+  ctx->fp8 = c.expert_fp8 != 0;
+  if (ctx->fp8) {
+    add(&ctx->x_sorted8, static_cast<size_t>(kE) * ctx->Tcap * d);
+    add(&ctx->xn8, static_cast<size_t>(Tmax) * d);
+    add(&ctx->act8, static_cast<size_t>(kE + kShared) * ctx->Tcap * kI);
+  }
   add(&ctx->y, sizeof(float) * Tmax * kSlots * d);
   add(&ctx->b_ws, sizeof(bf16) * Tmax * d);
   add(&ctx->am_key, sizeof(unsigned long long) * Tmax);
@@ -526,10 +542,11 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
     LayerMaps& m = ctx->lmaps[l];
     ok = ok && encode_map_2d(&m.wqkv, W.wqkv, kD, 3 * kD, 128, &e);
     ok = ok && encode_map_2d(&m.wo, W.wo, kD, kD, 128, &e);
-    ok = ok && encode_map_3d(&m.gu_routed, W.w_gate_up, kD, 2 * kI, kE, 64, &e);
-    ok = ok && encode_map_3d(&m.gu_shared, W.shared_gate_up, kD, 2 * kI, kShared, 64, &e);
-    ok = ok && encode_map_3d(&m.dn_routed, W.w_down, kI, kD, kE, 128, &e);
-    ok = ok && encode_map_3d(&m.dn_shared, W.shared_down, kI, kD, kShared, 128, &e);
+    const int eb = ctx->fp8 ? 1 : 2;   // expert matrices: e4m3 bytes or bf16
+    ok = ok && encode_map_3d(&m.gu_routed, W.w_gate_up, kD, 2 * kI, kE, 64, &e, eb);
+    ok = ok && encode_map_3d(&m.gu_shared, W.shared_gate_up, kD, 2 * kI, kShared, 64, &e, eb);
+    ok = ok && encode_map_3d(&m.dn_routed, W.w_down, kI, kD, kE, 128, &e, eb);
+    ok = ok && encode_map_3d(&m.dn_shared, W.shared_down, kI, kD, kShared, 128, &e, eb);
   }
   ok = ok && encode_map_2d(&ctx->lm, w->lm_head, kD, c.vocab, 128, &e);
   ok = ok && encode_map_2d(&ctx->eh, w->eh_proj, 2 * kD, kD, 128, &e);
@@ -540,6 +557,11 @@ extern "C" spec_status spec_init(const spec_config* cfg, const spec_weights* w, 
   ok = ok && encode_act_maps(ctx->a_xn.m, ctx->xn, kD, Tmax, &e);
   ok = ok && encode_act_maps(ctx->a_attn.m, ctx->attn_out, kD, Tmax, &e);
   ok = ok && encode_act_maps(ctx->a_xs.m, ctx->x_sorted, kD, static_cast<uint64_t>(kE) * ctx->Tcap, &e);
+  if (ctx->fp8) {
+    ok = ok && encode_act_maps(ctx->a_xs8.m, ctx->x_sorted8, kD, static_cast<uint64_t>(kE) * ctx->Tcap, &e, 1);
+    ok = ok && encode_act_maps(ctx->a_xn8.m, ctx->xn8, kD, Tmax, &e, 1);
+    ok = ok && encode_act_maps(ctx->a_act8.m, ctx->act8, kI, static_cast<uint64_t>(kE + kShared) * ctx->Tcap, &e, 1);
+  }
   ok = ok && encode_act_maps(ctx->a_act.m, ctx->act, kI, static_cast<uint64_t>(kE + kShared) * ctx->Tcap, &e);
   ok = ok && encode_act_maps(ctx->a_b.m, ctx->b_ws, kD, Tmax, &e);
   ok = ok && encode_act_maps(ctx->a_dcat.m, ctx->dcat, 2 * kD, Tmax, &e);
@@ -737,6 +759,8 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       ra.rowmap = ctx->rowmap;
       ra.x_sorted = ctx->x_sorted;
       ra.map_stride = ctx->Tcap;
+      ra.xn8 = ctx->xn8;               // NULL unless fp8 experts
+      ra.x_sorted8 = ctx->x_sorted8;
       LAUNCH(SPEC_K_ROUTER, 1, router_launch(ra, s));
     }
     // routed + shared experts: gate/up + SwiGLU, then down scattered to (token, slot), in one
@@ -746,8 +770,8 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.a_map[0] = M.gu_routed;
       g.a_map[1] = M.gu_shared;
       for (int b = 0; b < 5; ++b) {
-        g.b_map[0][b] = ctx->a_xs.m[b];
-        g.b_map[1][b] = ctx->a_xn.m[b];
+        g.b_map[0][b] = ctx->fp8 ? ctx->a_xs8.m[b] : ctx->a_xs.m[b];
+        g.b_map[1][b] = ctx->fp8 ? ctx->a_xn8.m[b] : ctx->a_xn.m[b];
       }
       g.N = 2 * kI;
       g.K = kD;
@@ -764,14 +788,21 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.expert_ctr = ctx->d_expert_ctr;
       g.act = ctx->act;
       g.ld_act = kI;
+      if (ctx->fp8) {
+        g.f8 = 1;
+        g.act8 = ctx->act8;
+        g.w_scale[0] = W.gate_up_scale;
+        g.w_scale[1] = W.shared_gate_up_scale;
+        g.scale_rows = 2 * kI;
+      }
       g.dep = ctx->moe_dep + static_cast<size_t>(l) * (kE + kShared) * ctx->dep_stride;
       g.dep_stride = ctx->dep_stride;
       GemmArgs d = base_args(ctx);
       d.a_map[0] = M.dn_routed;
       d.a_map[1] = M.dn_shared;
       for (int b = 0; b < 5; ++b) {
-        d.b_map[0][b] = ctx->a_act.m[b];
-        d.b_map[1][b] = ctx->a_act.m[b];
+        d.b_map[0][b] = ctx->fp8 ? ctx->a_act8.m[b] : ctx->a_act.m[b];
+        d.b_map[1][b] = d.b_map[0][b];
       }
       d.N = kD;
       d.K = kI;
@@ -784,6 +815,12 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       d.rowmap = ctx->rowmap;
       d.map_stride = ctx->Tcap;
       d.y = ctx->y;
+      if (ctx->fp8) {
+        d.f8 = 1;
+        d.w_scale[0] = W.down_scale;
+        d.w_scale[1] = W.shared_down_scale;
+        d.scale_rows = kD;
+      }
       LAUNCH(SPEC_K_EXPERT_GU, 1, moe_launch(g, d, s));
     }
     const bf16* next_gain =
@@ -1108,6 +1145,41 @@ extern "C" spec_status spec_read_workspace(spec_ctx* ctx, int32_t id, void* dst,
 }
 
 // ============================================================================ standalone GEMM
+extern "C" spec_status spec_gemm_e4m3(const void* X, const void* W, const float* w_scale, float* Y, int32_t M,
+                                      int32_t N, int32_t Kdim, void* stream) {
+  spec_ctx* ctx = nullptr;
+  if (X == nullptr || W == nullptr || w_scale == nullptr || Y == nullptr)
+    return fail(nullptr, SPEC_EINVAL, "null argument");
+  if (M < 1 || N < 1 || Kdim < 128 || Kdim % 128) return fail(nullptr, SPEC_EINVAL, "bad sizes (Kdim a multiple of 128)");
+  if (!aligned16(X) || !aligned16(W)) return fail(nullptr, SPEC_EINVAL, "X and W must be 16-byte aligned");
+  GemmArgs g;
+  memset(&g, 0, sizeof(g));
+  std::string e;
+  if (!encode_map_2d(&g.a_map[0], W, Kdim, N, 128, &e, 1)) return fail(nullptr, SPEC_EINVAL, e);
+  if (!encode_act_maps(g.b_map[0], X, Kdim, M, &e, 1)) return fail(nullptr, SPEC_EINVAL, e);
+  int* err = nullptr;
+  CK(gemm_prepare());
+  CK(cudaGetSymbolAddress(reinterpret_cast<void**>(&err), g_gemm_err));
+  g.err = err;
+  g.f8 = 1;
+  g.w_scale[0] = w_scale;
+  g.n_routed = 1 << 30;
+  g.N = N;
+  g.K = Kdim;
+  g.M = M;
+  g.box_log = box_log_for(M < 256 ? M : 256);
+  const int box = 16 << g.box_log;
+  g.m_tiles = (M + box - 1) / box;
+  g.n_tiles = (N + 127) / 128;
+  g.split_k = 1;
+  g.n_items = g.n_tiles * g.m_tiles;
+  g.out = Y;
+  g.ldo = N;
+  const int grid = g.n_items < num_sms() ? g.n_items : num_sms();
+  CK(gemm_launch(EPI_F32, box <= 64 ? 64 : 256, g, grid, static_cast<cudaStream_t>(stream), false));
+  return SPEC_OK;
+}
+
 
 extern "C" spec_status spec_gemm_bf16(const void* X, const void* W, float* Y, int32_t M, int32_t N, int32_t Kdim,
                                       void* stream) {

@@ -2,6 +2,7 @@
 // (norm, logits, softmax, top-6, per-expert row lists and input rows), MoE combine (+ the next
 // RMSNorm), the KV commit, and the glue of the draft chain.  Every reduction runs in a fixed
 // order, so a row's result never depends on the other rows of the batch.
+#include <cuda_fp8.h>
 #include <math.h>
 
 #include "common.cuh"
@@ -177,6 +178,14 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
         o4[3] = __float2bfloat16(v[k].w * inv * __high2float(g23));
         *reinterpret_cast<uint2*>(xo + i) = *reinterpret_cast<const uint2*>(o4);
         *reinterpret_cast<uint2*>(xr + i) = *reinterpret_cast<const uint2*>(o4);
+        if (a.xn8 != nullptr) {   // fp8 experts: the shared experts' input row, rounded to e4m3
+          uint32_t q = 0;
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            q |= static_cast<uint32_t>(__nv_cvt_float_to_fp8(__bfloat162float(o4[e]), __NV_SATFINITE, __NV_E4M3))
+                 << (8 * e);
+          *reinterpret_cast<uint32_t*>(a.xn8 + static_cast<size_t>(t0 + r) * kD + i) = q;
+        }
       }
     }
   }
@@ -271,12 +280,26 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
         dst[warp + 8 * h2][rank[h2][j]] = e * a.map_stride + pos[h2][j];
       }
   __syncthreads();
-  // the rounded rows into their experts' input rows, 16 bytes per thread and step
+  // the rounded rows into their experts' input rows, 8 elements per thread and step (16 bytes
+  // of bf16, or with fp8 experts 8 bytes of e4m3)
   constexpr int kVec = kD / 8;
   for (int i = threadIdx.x; i < nr * kTopK * kVec; i += 256) {
     const int v = i % kVec, sel = i / kVec, r = sel / kTopK;
     const uint4 x = *reinterpret_cast<const uint4*>(xs + r * kRouteStride + 8 * v);
-    *reinterpret_cast<uint4*>(a.x_sorted + static_cast<size_t>(dst[r][sel % kTopK]) * kD + 8 * v) = x;
+    const size_t row = static_cast<size_t>(dst[r][sel % kTopK]);
+    if (a.x_sorted8 != nullptr) {
+      const bf16* xe = reinterpret_cast<const bf16*>(&x);
+      uint32_t lo = 0, hi = 0;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        lo |= static_cast<uint32_t>(__nv_cvt_float_to_fp8(__bfloat162float(xe[e]), __NV_SATFINITE, __NV_E4M3)) << (8 * e);
+        hi |= static_cast<uint32_t>(__nv_cvt_float_to_fp8(__bfloat162float(xe[4 + e]), __NV_SATFINITE, __NV_E4M3))
+              << (8 * e);
+      }
+      *reinterpret_cast<uint2*>(a.x_sorted8 + row * kD + 8 * v) = make_uint2(lo, hi);
+    } else {
+      *reinterpret_cast<uint4*>(a.x_sorted + row * kD + 8 * v) = x;
+    }
   }
   trace_exit();
 }

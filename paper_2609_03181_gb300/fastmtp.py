@@ -20,7 +20,7 @@ WS_B, WS_ROUTE_IDX, WS_ROUTE_GATE, WS_EXPERT_CNT, WS_DRAFT_U, WS_HIDDEN = range(
 # Public entry points, in the order include/fastmtp.h declares them.
 ENTRY_POINTS = ["spec_init", "spec_seq_reset", "spec_seq_set_draft_rows", "draft_step", "verify_step",
                 "accept_commit", "spec_sync", "spec_seq_state", "spec_read_workspace", "spec_gemm_bf16",
-                "spec_profile", "spec_profile_read", "spec_trace_read", "spec_gemm_bf16_noalloc",
+                "spec_gemm_e4m3", "spec_profile", "spec_profile_read", "spec_trace_read", "spec_gemm_bf16_noalloc",
                 "spec_draft_loss_workspace", "spec_draft_loss", "spec_destroy", "spec_last_error"]
 KERNEL_CLASSES = ["embed", "qkv", "attention", "oproj", "router", "permute", "expert_gate_up", "expert_down",
                   "combine", "lm_head", "argmax", "commit", "draft_gemm", "draft_misc"]
@@ -30,13 +30,14 @@ class SpecConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "hidden", "n_heads", "head_dim", "n_layers", "n_experts", "top_k", "n_shared", "expert_inter",
         "draft_inter", "vocab", "page_size", "max_batch", "max_pages_per_seq", "n_pages_total", "K_max",
-        "max_position")] + [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+        "max_position")] + [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float),
+                             ("expert_fp8", ctypes.c_int32)]
 
 
 class SpecLayerWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in (
         "attn_norm", "wqkv", "wo", "moe_norm", "router", "w_gate_up", "w_down", "shared_gate_up",
-        "shared_down", "router_bias")]
+        "shared_down", "router_bias", "gate_up_scale", "down_scale", "shared_gate_up_scale", "shared_down_scale")]
 
 
 class SpecWeights(ctypes.Structure):
@@ -80,6 +81,7 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
         "spec_seq_state": (ctypes.c_int, [P, I32, ctypes.POINTER(I32), ctypes.POINTER(I32)]),
         "spec_read_workspace": (ctypes.c_int, [P, I32, P, ctypes.c_size_t]),
         "spec_gemm_bf16": (ctypes.c_int, [P, P, P, I32, I32, I32, P]),
+        "spec_gemm_e4m3": (ctypes.c_int, [P, P, P, P, I32, I32, I32, P]),
         "spec_profile": (ctypes.c_int, [P, I32]),
         "spec_profile_read": (ctypes.c_int, [P, ctypes.POINTER(SpecProfile)]),
         "spec_trace_read": (ctypes.c_int, [P, I32, I32, ctypes.POINTER(I32)]),
@@ -133,6 +135,21 @@ def trace_read(reset: bool = True, cap: int = 3 << 16):
     if st != SPEC_OK:
         raise FastMTPError(st, lib.spec_last_error(None).decode())
     return buf[: n.value].copy()
+
+
+def gemm_e4m3(X8: torch.Tensor, W8: torch.Tensor, w_scale: torch.Tensor,
+              stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Y = (X W^T) * w_scale through spec_gemm_e4m3 (X8 [M][K], W8 [N][K] uint8 e4m3 codes,
+    w_scale fp32 [N], CUDA tensors) -> fp32 [M][N]."""
+    lib = load_library()
+    M, K = X8.shape
+    N = W8.shape[0]
+    Y = torch.empty(M, N, dtype=torch.float32, device=X8.device)
+    st = lib.spec_gemm_e4m3(X8.data_ptr(), W8.data_ptr(), w_scale.data_ptr(), Y.data_ptr(), M, N, K,
+                            _stream_handle(stream))
+    if st != SPEC_OK:
+        raise FastMTPError(st, lib.spec_last_error(None).decode())
+    return Y
 
 
 def gemm_bf16_noalloc(X: torch.Tensor, W: torch.Tensor, Y: torch.Tensor,
@@ -214,7 +231,8 @@ class Engine:
     b*max_pages_per_seq .. (b+1)*max_pages_per_seq-1 of both pools."""
 
     def __init__(self, vw, dw, max_batch: int, K_max: int, max_ctx: int, page_size: int = 64,
-                 device: str = "cuda", stream: Optional[torch.cuda.Stream] = None, max_position: int = 32768):
+                 device: str = "cuda", stream: Optional[torch.cuda.Stream] = None, max_position: int = 32768,
+                 expert_fp8: bool = False):
         self.lib = load_library()
         if not torch.cuda.is_available():
             raise RuntimeError("FastMTP needs a CUDA GPU")
@@ -246,10 +264,20 @@ class Engine:
             L.wo = keep(lw.wo).data_ptr()
             L.moe_norm = keep(lw.moe_norm).data_ptr()
             L.router = keep(lw.router).data_ptr()
-            L.w_gate_up = keep(lw.w_gate_up).data_ptr()
-            L.w_down = keep(lw.w_down).data_ptr()
-            L.shared_gate_up = keep(lw.shared_gate_up).data_ptr()
-            L.shared_down = keep(lw.shared_down).data_ptr()
+            if expert_fp8:   # e4m3 codes with one fp32 scale per row (synth_inputs.quantize_experts_fp8)
+                L.w_gate_up = keep(lw.w_gate_up_f8).data_ptr()
+                L.w_down = keep(lw.w_down_f8).data_ptr()
+                L.shared_gate_up = keep(lw.shared_gate_up_f8).data_ptr()
+                L.shared_down = keep(lw.shared_down_f8).data_ptr()
+                L.gate_up_scale = keep(lw.gate_up_scale.float()).data_ptr()
+                L.down_scale = keep(lw.down_scale.float()).data_ptr()
+                L.shared_gate_up_scale = keep(lw.shared_gate_up_scale.float()).data_ptr()
+                L.shared_down_scale = keep(lw.shared_down_scale.float()).data_ptr()
+            else:
+                L.w_gate_up = keep(lw.w_gate_up).data_ptr()
+                L.w_down = keep(lw.w_down).data_ptr()
+                L.shared_gate_up = keep(lw.shared_gate_up).data_ptr()
+                L.shared_down = keep(lw.shared_down).data_ptr()
             L.router_bias = keep(lw.router_bias.float()).data_ptr() if lw.router_bias is not None else None
         w = SpecWeights()
         w.embed, w.lm_head, w.final_norm = self.embed.data_ptr(), self.lm_head.data_ptr(), final_norm.data_ptr()
@@ -267,7 +295,8 @@ class Engine:
                          top_k=s.top_k, n_shared=s.n_shared, expert_inter=s.expert_inter,
                          draft_inter=s.draft_inter, vocab=s.vocab, page_size=page_size, max_batch=max_batch,
                          max_pages_per_seq=self.max_pages, n_pages_total=self.n_pages, K_max=K_max,
-                         max_position=max_position, rms_eps=s.rms_eps, rope_theta=s.rope_theta)
+                         max_position=max_position, rms_eps=s.rms_eps, rope_theta=s.rope_theta,
+                         expert_fp8=1 if expert_fp8 else 0)
         self._cfg = cfg
         ctx = ctypes.c_void_p()
         torch.cuda.synchronize(self.device)

@@ -31,3 +31,20 @@ def test_gemm_rows_do_not_depend_on_batch():
     for i in (0, 17, 200):
         one = F.gemm_bf16(X[i:i + 1].contiguous(), W)
         assert torch.equal(one[0], full[i])
+
+
+@pytest.mark.parametrize("M,N,K", [(16, 256, 128), (16, 256, 1280), (64, 384, 4096), (200, 128, 896)])
+def test_gemm_e4m3_matches_fp64_product(M, N, K):
+    """spec_gemm_e4m3 (tcgen05 kind::f8f6f4) against the fp64 product of the decoded codes times
+    the row scales.  Codes of N(0, 1) values (no NaN codes)."""
+    import oracle as O
+    g = torch.Generator().manual_seed(M + N + K)
+    X8 = (torch.randn(M, K, generator=g) * 2).clamp(-448, 448).to(torch.float8_e4m3fn).view(torch.uint8)
+    W8 = torch.randn(N, K, generator=g).clamp(-448, 448).to(torch.float8_e4m3fn).view(torch.uint8)
+    sc = torch.rand(N, generator=g) + 0.5
+    Y = F.gemm_e4m3(X8.cuda(), W8.cuda(), sc.cuda())
+    F.device_sync()
+    ref = (O.decode_e4m3(X8) @ O.decode_e4m3(W8).T) * sc.double()
+    err = float((Y.double().cpu() - ref).abs().max() / ref.abs().max())
+    print(f"[e4m3 gemm] M={M} N={N} K={K}: relative error {err:.3g}")
+    assert err < 1e-4, f"relative error {err}"

@@ -16,16 +16,20 @@ from tests.gpu_util import REL_TOL, GAP, rel_err, seq_prefixes, make_drafts, ind
 pytestmark = pytest.mark.gpu
 
 
-def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=None, rb=True, min_keep=None):
+def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=None, rb=True, min_keep=None,
+                    fp8=False, rel_tol=REL_TOL):
     """One verify_step + accept_commit of len(ctx_lens) sequences on the GPU; the sequences in
     `check` (default: all) are compared with the oracle (storage-rounding mode if `rb`, else the
     plain fp64 definition), the others get uniform random drafts and only fill the batch.
+    `fp8` runs the fp8-expert variant on both sides; `rel_tol` replaces the 2e-2 rule for it.
     `min_keep` is the least number of checked rows that must stay comparable through every layer
     (default: all of them when fewer than four sequences are checked, else all but two
     sequences' rows).  Prints the comparison counts and returns them."""
     B = len(ctx_lens)
     check = list(range(B)) if check is None else list(check)
     vw = S.verifier_weights(shape, seed, gain_std=gain_std, zipf_s=zipf_s)
+    if fp8:   # the fp8-expert variant: e4m3 expert matrices with per-row scales, on both sides
+        vw = S.quantize_experts_fp8(vw)
     dw = S.draft_weights(shape, seed, gain_std=gain_std)
     model = O.Verifier(vw)
     kvs, dkvs = seq_prefixes(shape, seed, ctx_lens)
@@ -38,7 +42,7 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
         cand[b] = cand_chk[j]
     ref = O.verify(model, caches, cand_chk, rb=rb, keep_hidden=True)
 
-    eng = F.Engine(vw, dw, max_batch=B, K_max=max(K, 3), max_ctx=max(ctx_lens) + 8, page_size=64)
+    eng = F.Engine(vw, dw, max_batch=B, K_max=max(K, 3), max_ctx=max(ctx_lens) + 8, page_size=64, expert_fp8=fp8)
     for b in range(B):
         eng.load_prefix(b, kvs[b], dkvs[b], int(pend[b]))
     dev = torch.device("cuda")
@@ -80,7 +84,7 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
             og = np.argsort(gi[i])
             orf = np.argsort(ref.route_idx[l][i].numpy())
             e = rel_err(gate_gpu[l, rows[i]][og], ref.route_gate[l][i][orf])
-            assert e < REL_TOL, f"layer {l} row {i}: router probability rel err {e:.3g}"
+            assert e < rel_tol, f"layer {l} row {i}: router probability rel err {e:.3g}"
         differ = (g != r).any(-1) & ~diverged
         div_per_layer.append(int(differ.sum()))
         for row in np.nonzero(differ)[0]:
@@ -97,14 +101,14 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
     print(f"[parity] layers {shape.n_layers}, rows {T}, comparable through every layer {int(keep.sum())}, "
           f"router near-ties skipped {near_ties}, rows leaving per layer {div_per_layer}")
     assert keep.sum() >= need, f"only {keep.sum()} of {T} rows comparable (need {need})"
-    assert max(e for e, k in zip(errs, keep) if k) < REL_TOL, (
+    assert max(e for e, k in zip(errs, keep) if k) < rel_tol, (
         f"b rel err per row {['%.3g' % e for e in errs]}, diverged rows {np.nonzero(diverged)[0].tolist()}")
     # the fp32 residual stream after the last layer, row by row
     h_gpu = eng.read_workspace(F.WS_HIDDEN, (B * R, shape.hidden), torch.float32)[rows]
     h_ref = ref.hidden[-1]
     for i in np.nonzero(keep)[0]:
         e = rel_err(h_gpu[i], h_ref[i])
-        assert e < REL_TOL, f"row {i}: residual stream rel err {e:.3g}"
+        assert e < rel_tol, f"row {i}: residual stream rel err {e:.3g}"
 
     # verifier tokens: exact where the oracle's logit margin exceeds the noise the measured state
     # difference implies (at least 1e-3); accept lengths where all of a sequence's tokens are
@@ -144,8 +148,8 @@ def run_verify_case(shape, seed, ctx_lens, K, gain_std=0.1, check=None, zipf_s=N
                 page, off = bt[p // ps], p % ps
                 k_gpu = eng.kv_pool[l, page, 0, :, off, :].cpu()
                 v_gpu = eng.kv_pool[l, page, 1, :, off, :].cpu()
-                assert rel_err(k_gpu, ref.new_k[j][l][r]) < REL_TOL
-                assert rel_err(v_gpu, ref.new_v[j][l][r]) < REL_TOL
+                assert rel_err(k_gpu, ref.new_k[j][l][r]) < rel_tol
+                assert rel_err(v_gpu, ref.new_v[j][l][r]) < rel_tol
     eng.close()
     print(f"[parity] verifier tokens compared {int(sure.sum())}, below the margin {int((~sure).sum())}")
     return {"rows": T, "kept": int(keep.sum()), "near_ties": near_ties, "tokens": int(sure.sum()),
