@@ -53,6 +53,7 @@ struct Item {
 // grp[134 + e] the first down item of expert e counted from the first down item.
 constexpr int kGrpItem = 0, kGrpCnt = kE + kShared + 1, kGrpDn = 2 * (kE + kShared + 1);
 
+template <int EPI>
 __device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, int i, Item& it, const int* grp) {
   it.phase = 0;
   if (a.grp_cnt != nullptr) {
@@ -83,10 +84,11 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, 
     it.box_log = bl;
   } else {
     it.grow = 0;
-    // items run through the activation tiles first, or (loss_G: the two operands swapped, A =
+    // items run through the activation tiles first, or (EPI_LOSS: the two operands swapped, A =
     // activations) through the A tiles first, so that the CTAs reading one B tile run together
-    const int mt = a.loss_G ? i / a.n_tiles : i % a.m_tiles;
-    const int t = a.loss_G ? i % a.n_tiles : i / a.m_tiles;
+    constexpr bool swapped = (EPI == EPI_LOSS);
+    const int mt = swapped ? i / a.n_tiles : i % a.m_tiles;
+    const int t = swapped ? i % a.n_tiles : i / a.m_tiles;
     const int ns = a.seq_split ? 1 : a.split_k;   // in-CTA splits: one item covers every split
     it.split = t % ns;
     it.n_tile = t / ns;
@@ -194,12 +196,12 @@ __device__ __forceinline__ void stage_meta(const GemmArgs& a, const Item& it, co
   }
 }
 
-template <int EPI>
+template <int EPI, bool F8 = false>
 __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int row, int j0, float (&v)[16],
                                          const EpiPre& p, const EpiSmem& sm, int rope_buf) {
   if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
     const int n = it.n_tile * 128 + row;
-    if (EPI == EPI_F32 && a.f8 && n < a.N) {   // e4m3 GEMM: each weight row's scale
+    if (EPI == EPI_F32 && F8 && n < a.N) {   // e4m3 GEMM: each weight row's scale
       const float sc = a.w_scale[0][n];
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) v[jj] *= sc;
@@ -212,25 +214,28 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
     }
   } else if constexpr (EPI == EPI_SCATTER) {
     const int n = it.n_tile * 128 + row;
-    float sc = 1.f;   // fp8 experts: the scale of output feature n's weight row
-    if (a.f8)
-      sc = ((it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
-                                : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows)[n];
+    if constexpr (F8) {   // fp8 experts: the scale of output feature n's weight row
+      const float sc = ((it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
+                                            : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows)[n];
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) v[jj] *= sc;
+    }
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj)
       if (j0 + jj < it.rows)
-        a.y[(static_cast<size_t>(sm.s_pos[j0 + jj]) * kSlots + sm.s_aux[j0 + jj]) * kD + n] = v[jj] * sc;
+        a.y[(static_cast<size_t>(sm.s_pos[j0 + jj]) * kSlots + sm.s_aux[j0 + jj]) * kD + n] = v[jj];
   } else if constexpr (EPI == EPI_SWIGLU) {
     float* xchg = sm.xchg;
-    float sc = 1.f;   // fp8 experts: this weight row's scale (tile rows 0..63 gate, 64..127 up)
-    if (a.f8) {
+    if constexpr (F8) {   // fp8 experts: this weight row's scale (tile rows 0..63 gate, 64..127 up)
       const int wr = (row < 64) ? it.n_tile * 64 + row : a.half_rows + it.n_tile * 64 + (row - 64);
       const float* ws = (it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
                                             : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows;
-      sc = ws[wr];
+      const float sc = ws[wr];
+#pragma unroll
+      for (int jj = 0; jj < 16; ++jj) v[jj] *= sc;
     }
 #pragma unroll
-    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj] * sc;
+    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
     named_bar_sync(1, 128);
     if (row < 64) {
       const int f = it.n_tile * 64 + row;
@@ -239,10 +244,9 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
         const int r = j0 + jj;
         if (r < it.rows) {
           const float u = xchg[(row + 64) * 17 + jj];
-          const float y = silu_f(v[jj] * sc) * u;
           const size_t at = static_cast<size_t>(it.out_row + r) * a.ld_act + f;
-          if (a.f8) a.act8[at] = __nv_cvt_float_to_fp8(y, __NV_SATFINITE, __NV_E4M3);
-          else a.act[at] = __float2bfloat16(y);
+          if constexpr (F8) a.act8[at] = __nv_cvt_float_to_fp8(silu_f(v[jj]) * u, __NV_SATFINITE, __NV_E4M3);
+          else a.act[at] = __float2bfloat16(silu_f(v[jj]) * u);
         }
       }
     }
@@ -370,7 +374,7 @@ template <int EPI>
 __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem& esm, uint32_t part_saddr, int row,
                                                const EpiPre& first) {
   Item it;
-  get_item(a, a, blockIdx.x, it, nullptr);
+  get_item<EPI>(a, a, blockIdx.x, it, nullptr);
   const int S = a.cluster;
   const int rank = static_cast<int>(cluster_ctarank());
   const int nchunks = (it.rows + 15) >> 4;
@@ -422,7 +426,7 @@ __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem&
 }
 
 // ------------------------------------------------------------------ kernel
-template <int NMAX, int EPI, int ST>
+template <int NMAX, int EPI, int ST, bool F8 = false>
 __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a,
                                                          const __grid_constant__ GemmArgs a2) {
   using C = Cfg<NMAX, ST>;
@@ -554,15 +558,15 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     if (lane == 0) {
       const uint64_t pol_w = a.a_keep ? l2_policy_evict_last() : l2_policy_evict_first();
       // (operands swapped for the objective: the streamed W_lm tiles are the B side)
-      const uint64_t pol_x = a.loss_G ? l2_policy_evict_first() : l2_policy_evict_last();
+      const uint64_t pol_x = (EPI == EPI_LOSS) ? l2_policy_evict_first() : l2_policy_evict_last();
       uint32_t g = 0;   // loads issued
       bool failed = false;
       bool waited = !dense;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x) {
         Item it;
-        get_item(a, a2, i, it, grp);
+        get_item<EPI>(a, a2, i, it, grp);
         const GemmArgs& P = it.phase ? a2 : a;   // the item's operands (EPI_MOE down items: a2)
-        const int kw = P.f8 ? 128 : 64;           // elements of a 128-byte k-chunk
+        constexpr int kw = F8 ? 128 : 64;         // elements of a 128-byte k-chunk
         const int kc_total = P.K / kw;
         const int src = (!dense && it.e >= a.n_routed) ? 1 : 0;
         const int el = it.e - (src ? a.n_routed : 0);
@@ -654,9 +658,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       bool failed = false;
       for (int i = blockIdx.x; i < n_items && !failed; i += gridDim.x, ++local) {
         Item it;
-        get_item(a, a2, i, it, grp);
-        const bool f8 = (it.phase ? a2.f8 : a.f8) != 0;
-        const int kc_total = (it.phase ? a2.K : a.K) / (f8 ? 128 : 64);
+        get_item<EPI>(a, a2, i, it, grp);
+        const int kc_total = (it.phase ? a2.K : a.K) / (F8 ? 128 : 64);
         const int acc = local % nbuf;
         const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
         if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, s_abort)) {
@@ -664,7 +667,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           break;
         }
         tc_fence_after();
-        const uint32_t idesc = f8 ? idesc_e4m3(128, 16 << it.box_log) : idesc_bf16(128, 16 << it.box_log);
+        const uint32_t idesc = F8 ? idesc_e4m3(128, 16 << it.box_log) : idesc_bf16(128, 16 << it.box_log);
         const int kc0 = a.seq_split ? 0 : it.split * kc_total / a.split_k;
         const int kc1 = a.seq_split ? kc_total : (it.split + 1) * kc_total / a.split_k;
         // with in-CTA splits, split sp accumulates k-chunks [sp*kc/S, (sp+1)*kc/S) into its own
@@ -687,14 +690,10 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           const uint64_t ad = sw128_kmajor_desc(smem_u32(smA + st * C::A_BYTES));
           const uint64_t bd = sw128_kmajor_desc(smem_u32(smB + st * C::B_BYTES));
           // 4 MMAs per 128-byte k-chunk (K=16 bf16 or K=32 e4m3 each): +32 B in the swizzled row
-          if (f8) {
 #pragma unroll
-            for (int s = 0; s < 4; ++s)
-              tc_mma_e4m3(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
-          } else {
-#pragma unroll
-            for (int s = 0; s < 4; ++s)
-              tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+          for (int s = 0; s < 4; ++s) {
+            if constexpr (F8) tc_mma_e4m3(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+            else tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
           }
           tc_commit(&empty[st]);
         }
@@ -720,7 +719,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
     int local = 0;
     for (int i = blockIdx.x; i < n_items; i += gridDim.x, ++local) {
       Item it;
-      get_item(a, a2, i, it, grp);
+      get_item<EPI>(a, a2, i, it, grp);
       const int acc = local % nbuf;
       const uint32_t acc_ph = static_cast<uint32_t>(local / nbuf) & 1u;
       // the item's metadata, RoPE factors and first old residuals are fetched while its MMAs
@@ -772,12 +771,12 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
             for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
           }
           if constexpr (EPI == EPI_MOE) {
-            if (it.phase) epi_post<EPI_SCATTER>(a2, it, row, c * 16, v, cur, esm, c & 1);
-            else epi_post<EPI_SWIGLU>(a, it, row, c * 16, v, cur, esm, c & 1);
+            if (it.phase) epi_post<EPI_SCATTER, F8>(a2, it, row, c * 16, v, cur, esm, c & 1);
+            else epi_post<EPI_SWIGLU, F8>(a, it, row, c * 16, v, cur, esm, c & 1);
           } else if constexpr (EPI == EPI_LOSS) {
             loss_chunk(a, it, c * 16, v, ls);
           } else {
-            epi_post<EPI>(a, it, row, c * 16, v, cur, esm, c & 1);
+            epi_post<EPI, F8>(a, it, row, c * 16, v, cur, esm, c & 1);
           }
           cur = nxt;
           if (rope && c + 1 < nchunks) {
@@ -956,13 +955,13 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES>
+template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES, bool F8 = false>
 cudaError_t set_smem_attr() {
-  return cudaFuncSetAttribute(gemm_tc_kernel<NMAX, EPI, ST>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(gemm_tc_kernel<NMAX, EPI, ST, F8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               Cfg<NMAX, ST>::SMEM_BYTES);
 }
 
-template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES>
+template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES, bool F8 = false>
 cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
@@ -985,7 +984,7 @@ cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   }
   cfg.attrs = attr;
   cfg.numAttrs = n;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI, ST>, a, a);
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<NMAX, EPI, ST, F8>, a, a);
 }
 }  // namespace
 
@@ -1056,6 +1055,12 @@ cudaError_t gemm_prepare() {
 #undef FM_ATTR
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE>();
   if (e == cudaSuccess) e = set_smem_attr<256, EPI_MOE>();
+  // fp8 experts and the dense e4m3 GEMM: separate instantiations, so that the bf16 kernels carry
+  // no fp8 code
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE, Cfg<64>::STAGES, true>();
+  if (e == cudaSuccess) e = set_smem_attr<256, EPI_MOE, Cfg<256>::STAGES, true>();
+  if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, Cfg<64>::STAGES, true>();
+  if (e == cudaSuccess) e = set_smem_attr<256, EPI_F32, Cfg<256>::STAGES, true>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, kShallowStages>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_RESID, kShallowStages>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_QKV, kShallowStages>();
@@ -1134,12 +1139,21 @@ cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
+  if (gate_up.f8) {
+    if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<256, EPI_MOE, Cfg<256>::STAGES, true>, gate_up, down);
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<64, EPI_MOE, Cfg<64>::STAGES, true>, gate_up, down);
+  }
   if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<256, EPI_MOE, Cfg<256>::STAGES>, gate_up, down);
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<64, EPI_MOE, Cfg<64>::STAGES>, gate_up, down);
 }
 
 cudaError_t gemm_launch(int epi, int nmax, const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   if (grid <= 0) return cudaSuccess;
+  if (a.f8) {   // the dense e4m3 GEMM (plain fp32 output with row scales)
+    if (epi != EPI_F32 || a.cluster > 1 || a.split_k != 1) return cudaErrorInvalidValue;
+    return nmax <= 64 ? launch_one<64, EPI_F32, Cfg<64>::STAGES, true>(a, grid, s, pdl)
+                      : launch_one<256, EPI_F32, Cfg<256>::STAGES, true>(a, grid, s, pdl);
+  }
   if (a.cluster > 1 && nmax <= 64) {   // the dense cluster schedule: short per-split streams
     switch (epi) {
       case EPI_F32:
