@@ -70,6 +70,9 @@ def parse():
     p.add_argument("--device-kv", action="store_true",
                    help="draw the KV prefixes on the GPU (PyTorch's generator) instead of the host Philox stream")
     p.add_argument("--sweep", action="store_true", help="run the (batch, context, K, router) grid")
+    p.add_argument("--experts", default="bf16", choices=["bf16", "fp8"],
+                   help="fp8: the fp8-expert variant (e4m3 expert matrices with per-row scales) as the main "
+                        "workload; the default bf16 is the paper's model")
     p.add_argument("--objective", action="store_true",
                    help="time only the draft-head training objective (64 rows, K=3, full vocabulary)")
     p.add_argument("--trace", action="store_true",
@@ -125,6 +128,8 @@ def workload(args, rank=0):
     else:
         vw = S.verifier_weights(shape, seed)
         dw = S.draft_weights(shape, seed)
+    if getattr(args, "experts", "bf16") == "fp8":
+        vw = S.quantize_experts_fp8(vw)
     B = args.batch
     ctx, pend = sequence_inputs(args, shape, rank)
     sd = rank_seed(seed, rank)
@@ -523,7 +528,9 @@ def run_fastmtp(args):
     B, K = args.batch, args.K
     total_new = (args.warmup + args.steps) * (K + 1) * 2 + 2 * (K + 1) + 8
     stream = torch.cuda.Stream(dev)
+    fp8 = args.experts == "fp8"
     eng = F.Engine(vw, dw, max_batch=B, K_max=K, max_ctx=max(ctx) + total_new, page_size=64, device=str(dev),
+                   expert_fp8=fp8,
                    stream=stream)
     slots = torch.arange(B, dtype=torch.int32, device=dev)
     cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
@@ -638,11 +645,12 @@ def run_fastmtp(args):
     points = None
     loss_point = None
     fp8_point = None
-    if not args.no_points and world == 1:
+    if not args.no_points and world == 1 and not fp8:
         pk, pkind = measured_peaks()
         points = run_points(args, shape, vw, dw, dev, pk, pkind)
         loss_point = run_loss_point(args, shape, dev, pk, pkind)
-        fp8_point = run_fp8_point(args, shape, vw, dw, ctx, pend, kvs, dkvs, dev, pk, pkind)
+        if not fp8:
+            fp8_point = run_fp8_point(args, shape, vw, dw, ctx, pend, kvs, dkvs, dev, pk, pkind)
 
     if rank != 0:
         if world > 1:
@@ -656,9 +664,11 @@ def run_fastmtp(args):
     touched = counted["experts_touched"] / max(1, counted["launches"]["router"])     # per layer, incl. shared
     rows = counted["expert_rows"] / max(1, counted["launches"]["router"])
     d, I = shape.hidden, shape.expert_inter
+    eb = 1 if fp8 else 2   # bytes per expert weight and per expert input / activation element
+    sc = (4 * 2 * I, 4 * d) if fp8 else (0, 0)   # fp32 row scales of gate/up and down
     cls_bytes = {
-        "expert_gate_up": touched * 2 * I * d * 2 + rows * d * 2 + rows * I * 2,
-        "expert_down": touched * d * I * 2 + rows * I * 2 + rows * d * 4,
+        "expert_gate_up": touched * (2 * I * d * eb + sc[0]) + rows * d * eb + rows * I * eb,
+        "expert_down": touched * (d * I * eb + sc[1]) + rows * I * eb + rows * d * 4,
         "lm_head": shape.vocab * d * 2.0,
     }
     fused = counted["launches"]["expert_down"] == 0   # gate/up and down run as one launch per layer
@@ -682,7 +692,8 @@ def run_fastmtp(args):
                 "avg_launch_ms": dur_ms, "avg_launch_timing": "serialised replay (event pair per launch)",
                 "peak_source": peak_kind}
     routed_touched = touched - shape.n_shared
-    vbytes = algorithmic_bytes(shape, B, K, statistics.mean(ctx) + (args.warmup + steps / 2) * 2, routed_touched)
+    vbytes = algorithmic_bytes(shape, B, K, statistics.mean(ctx) + (args.warmup + steps / 2) * 2, routed_touched,
+                               fp8_experts=fp8)
     v_ach = vbytes / (ms_verify / 1000.0) / 1e9
     ctx_run = statistics.mean(ctx) + (args.warmup + steps / 2) * 2
     dbytes = draft_algorithmic_bytes(shape, B, K, ctx_run, accepted / steps)
@@ -693,7 +704,7 @@ def run_fastmtp(args):
         "warmup": args.warmup, "ms_per_step": ms_total / steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": data_desc(args),
         "config": {"workload": WORKLOAD, "batch": B, "K": K, "layers": L, "ctx": f"U[{args.ctx_lo},{args.ctx_hi}]",
-                   "weights": args.weights,
+                   "weights": args.weights, "experts": args.experts,
                    "l2": "inputs larger than L2: 6.3 GB of weights streamed per step", "parallelism": "replicas"},
         "roofline": roofline,
         "verify_roofline": {"bound": "hbm", "achieved": v_ach, "peak": peak, "unit": "GB/s", "frac": v_ach / peak,
