@@ -880,7 +880,7 @@ def run_trace(args):
     B, K = args.batch, args.K
     stream = torch.cuda.Stream(dev)
     eng = F.Engine(vw, dw, max_batch=B, K_max=K, max_ctx=max(ctx) + (args.warmup + 4) * (K + 1) + 8, page_size=64,
-                   device=str(dev), stream=stream)
+                   device=str(dev), stream=stream, expert_fp8=args.experts == "fp8")
     slots = torch.arange(B, dtype=torch.int32, device=dev)
     cand = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
     vt = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
@@ -918,7 +918,7 @@ def run_trace(args):
                           "entry_us": g["entry"], "ready_us": g["ready"], "done_us": g["done"]}), flush=True)
     layers = TR.verify_layers(ls)
     print(json.dumps({"trace": True, "batch": B, "K": K, "ctx": [args.ctx_lo, args.ctx_hi], "layers": args.layers,
-                      "records": int(len(recs)), "launches": len(ls), "verify_layers": len(layers),
+                      "experts": args.experts, "records": int(len(recs)), "launches": len(ls), "verify_layers": len(layers),
                       "verify_layer_us": TR.layer_breakdown(layers)}), flush=True)
     eng.close()
 
