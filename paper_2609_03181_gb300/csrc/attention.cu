@@ -9,7 +9,8 @@
 // Arithmetic (fixed by position, never by the launch shape): a super-chunk's chunks are
 // folded in chunk order by the online softmax (running max M, sum L and unnormalised output O
 // per query, rescaled by 2^(M_old - M_new) when the max grows); a query's result is the merge
-// of its super-chunks in order, O = sum_s w_s O_s / sum_s w_s L_s with w_s = 2^(M_s - max M).
+// of its super-chunks, O = sum_s w_s O_s / sum_s w_s L_s with w_s = 2^(M_s - max M), the
+// outputs added in position order and the sums over a fixed tree.
 // Scores K q^T and outputs V^T p^T run on bf16 tensor cores (mma.sync m16n8k16, fp32
 // accumulation, queries padded to 8); a score sums its even and its odd 16-dim steps
 // separately, then adds the two; p enters the product as two bf16 terms (hi + lo, about 16
@@ -59,11 +60,11 @@ constexpr int kAttnThreads = kConsumers + 32;    // plus the producer warp
 constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
 
 // Shared memory of a CTA of a launch over B sequences: 1 KB alignment slack, the stages, two
-// query slots, the barriers, the merge scratch and flags, and the per-sequence tables (first
-// query position, slot, item prefix).
+// query slots, the barriers, the flags, and the per-sequence tables (first query position,
+// slot, item prefix).
 constexpr int kXchgBytes = 4 * 32 * 16 + 2 * 4 * kMaxR * 4;   // P fragments of the 4 key tiles, max / sum partials
 constexpr size_t attn_smem(int stages, int B) {
-  return 1024 + stages * kStageBytes + 2 * kQBytes + kXchgBytes + (2 * stages + 4) * 8 + (2 * kMaxR + 8) * 4 +
+  return 1024 + stages * kStageBytes + 2 * kQBytes + kXchgBytes + (2 * stages + 4) * 8 + 8 * 4 +
          (3 * static_cast<size_t>(B) + 1) * 4;
 }
 
@@ -153,47 +154,72 @@ struct Walk {
 __device__ __forceinline__ int chunks_live(int p0, int R) { return (p0 + R - 1) / kCH + 1; }
 
 // Merge of the super-chunks of every query of (sequence b, head h), run by the 128 consumer
-// threads of the CTA that completed its count: query r combines super-chunks 0..floor(p_r/256)
-// in order.  Threads 0..R-1 find each query's max and weighted sum; warp w then writes queries
-// w, w + 4, each lane four dims.
-__device__ __forceinline__ void merge_seq_head(const AttnArgs& a, int b, int h, int R, int p0, int n_super,
-                                               float* s_mrg, int tid) {
+// threads of the CTA that completed its count: query r combines super-chunks 0..floor(p_r/256).
+// Warp w takes queries w, w + 4, each lane four output dims.  Every load a query needs is
+// issued before its first use (one round trip to L2 for up to 8 super-chunks): lane l holds the
+// maximum and the sum of super-chunk l (l + 32, ...), the maximum M is the warp's maximum, the
+// weighted sum L = sum_s w_s L_s is added per lane and then over a fixed tree of lanes, and the
+// output O = sum_s w_s O_s is added in position order, with w_s = 2^(M_s - M) taken from lane s
+// by a shuffle.  The order of every sum depends on the query's position only.
+__device__ __forceinline__ void merge_seq_head(const AttnArgs& a, int b, int h, int R, int p0, int n_super, int tid) {
   const int lane = tid & 31, warp = tid >> 5;
   const float* part = a.part + (static_cast<size_t>(b) * kH + h) * n_super * R * kPartStride;
-  if (tid < R) {
-    const int r = tid, lasts = (p0 + r) / (kCH * kSuper);
-    float M = -INFINITY;
-#pragma unroll 4
-    for (int s = 0; s <= lasts; ++s) M = fmaxf(M, __ldcg(part + (static_cast<size_t>(s) * R + r) * kPartStride + kHD));
-    float L = 0.f;
-#pragma unroll 4
-    for (int s = 0; s <= lasts; ++s) {
-      const float* pc = part + (static_cast<size_t>(s) * R + r) * kPartStride;
-      const float ms = __ldcg(pc + kHD);
-      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      L += __ldcg(pc + kHD + 1) * w;
-    }
-    s_mrg[r] = M;
-    s_mrg[kMaxR + r] = L;
-  }
-  named_bar_sync(1, kConsumers);
+  const size_t sst = static_cast<size_t>(R) * kPartStride;   // floats between super-chunks of a query
   const int d = lane * 4;
   for (int r = warp; r < R; r += kConsumers / 32) {
-    const int lasts = (p0 + r) / (kCH * kSuper);
-    const float M = s_mrg[r];
-    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-    for (int s = 0; s <= lasts; ++s) {
-      const float* pc = part + (static_cast<size_t>(s) * R + r) * kPartStride;
-      const float ms = __ldcg(pc + kHD);
-      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      const float4 x = __ldcg(reinterpret_cast<const float4*>(pc + d));
-      O.x += x.x * w;
-      O.y += x.y * w;
-      O.z += x.z * w;
-      O.w += x.w * w;
+    const int ns = (p0 + r) / (kCH * kSuper) + 1;
+    const float* pr = part + static_cast<size_t>(r) * kPartStride;
+    // the first group's statistics and the first eight outputs, all in flight together
+    float ms0 = -INFINITY, ls0 = 0.f;
+    if (lane < ns) {
+      ms0 = __ldcg(pr + lane * sst + kHD);
+      ls0 = __ldcg(pr + lane * sst + kHD + 1);
     }
-    const float inv = 1.f / s_mrg[kMaxR + r];
+    float4 x[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t)
+      if (t < ns) x[t] = __ldcg(reinterpret_cast<const float4*>(pr + t * sst + d));
+    float m = ms0;
+    for (int s = lane + 32; s < ns; s += 32) m = fmaxf(m, __ldcg(pr + s * sst + kHD));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    const float M = m;
+    float w0 = (ms0 == -INFINITY) ? 0.f : exp2f(ms0 - M);
+    float l = ls0 * w0;
+    for (int s = lane + 32; s < ns; s += 32) {
+      const float ms = __ldcg(pr + s * sst + kHD);
+      l += __ldcg(pr + s * sst + kHD + 1) * ((ms == -INFINITY) ? 0.f : exp2f(ms - M));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = 0; s0 < ns; s0 += 32) {
+      float w = w0;   // weight of super-chunk s0 + lane
+      if (s0 > 0) {
+        const int s = s0 + lane;
+        const float ms = (s < ns) ? __ldcg(pr + s * sst + kHD) : -INFINITY;
+        w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+      }
+      const int n = min(32, ns - s0);
+      for (int j = 0; j < n; j += 8) {
+        if (s0 > 0 || j > 0) {
+#pragma unroll
+          for (int t = 0; t < 8; ++t)
+            if (j + t < n) x[t] = __ldcg(reinterpret_cast<const float4*>(pr + (s0 + j + t) * sst + d));
+        }
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+          const float wt = __shfl_sync(0xffffffffu, w, (j + t) & 31);
+          if (j + t < n) {
+            O.x += x[t].x * wt;
+            O.y += x[t].y * wt;
+            O.z += x[t].z * wt;
+            O.w += x[t].w * wt;
+          }
+        }
+      }
+    }
+    const float inv = 1.f / l;
     bf16* o = a.out + (static_cast<size_t>(b) * a.out_row_stride_seq + r) * (kH * kHD) + h * kHD + d;
     *reinterpret_cast<__nv_bfloat162*>(o) = __floats2bfloat162_rn(O.x * inv, O.y * inv);
     *reinterpret_cast<__nv_bfloat162*>(o + 2) = __floats2bfloat162_rn(O.z * inv, O.w * inv);
@@ -213,8 +239,7 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
   uint64_t* empty = full + kStages;                                         // [S] chunk consumed
   uint64_t* qfull = empty + kStages;                                        // [2] queries landed
   uint64_t* qempty = qfull + 2;                                             // [2] queries loaded
-  float* s_mrg = reinterpret_cast<float*>(qempty + 2);                      // [2 * kMaxR] merge M, L
-  int* s_flag = reinterpret_cast<int*>(s_mrg + 2 * kMaxR);                  // abort, last, err, warp sums[5]
+  int* s_flag = reinterpret_cast<int*>(qempty + 2);                         // abort, last, err, warp sums[5]
   volatile int* s_abort = s_flag;
   int* s_p0 = s_flag + 8;                                                   // [B] first query position
   int* s_slot = s_p0 + a.B;                                                 // [B] slot
@@ -659,7 +684,7 @@ __global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kerne
       named_bar_sync(1, kConsumers);
       if (s_flag[1]) {
         __threadfence();
-        merge_seq_head(a, b, h, R, p0, n_super, s_mrg, tid);
+        merge_seq_head(a, b, h, R, p0, n_super, tid);
       }
     }
     if (!more) break;
