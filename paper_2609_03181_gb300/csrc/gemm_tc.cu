@@ -113,6 +113,7 @@ struct EpiPre {
 
 struct EpiSmem {
   float* xchg;
+  float* xchg2;       // SWIGLU: the second exchange buffer (in the RoPE region, past the grouped tables)
   float* am_val;
   int* am_idx;
   int* s_pos;         // QKV: position of each row of the item; SCATTER: token
@@ -225,7 +226,13 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
       if (j0 + jj < it.rows)
         a.y[(static_cast<size_t>(sm.s_pos[j0 + jj]) * kSlots + sm.s_aux[j0 + jj]) * kD + n] = v[jj];
   } else if constexpr (EPI == EPI_SWIGLU) {
-    float* xchg = sm.xchg;
+    // Tile rows 0..63 are gate features, 64..127 the up features of the same 64 outputs.  The
+    // gate thread of output p computes activation rows j0..j0+7 of it, the up thread rows
+    // j0+8..j0+15: each passes the other the 8 values it lacks through one of two exchange
+    // buffers (by chunk parity), so one barrier per chunk suffices: a buffer is written again
+    // two chunks later, after a barrier that every thread reaches only once it has read this
+    // chunk's values (between items, the barriers at the start of each item do the same).
+    float* xchg = (rope_buf & 1) ? sm.xchg2 : sm.xchg;
     if constexpr (F8) {   // fp8 experts: this weight row's scale (tile rows 0..63 gate, 64..127 up)
       const int wr = (row < 64) ? it.n_tile * 64 + row : a.half_rows + it.n_tile * 64 + (row - 64);
       const float* ws = (it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
@@ -234,23 +241,25 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
 #pragma unroll
       for (int jj = 0; jj < 16; ++jj) v[jj] *= sc;
     }
+    const int up = row >> 6, pr = row & 63, mine = up * 8;   // mine: first of this thread's 8 rows
 #pragma unroll
-    for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = v[jj];
+    for (int jj = 0; jj < 8; ++jj) xchg[row * 17 + (8 - mine) + jj] = up ? v[jj] : v[8 + jj];
     named_bar_sync(1, 128);
-    if (row < 64) {
-      const int f = it.n_tile * 64 + row;
+    const float* other = xchg + (row ^ 64) * 17 + mine;
+    const int f = it.n_tile * 64 + pr;
 #pragma unroll
-      for (int jj = 0; jj < 16; ++jj) {
-        const int r = j0 + jj;
-        if (r < it.rows) {
-          const float u = xchg[(row + 64) * 17 + jj];
-          const size_t at = static_cast<size_t>(it.out_row + r) * a.ld_act + f;
-          if constexpr (F8) a.act8[at] = __nv_cvt_float_to_fp8(silu_f(v[jj]) * u, __NV_SATFINITE, __NV_E4M3);
-          else a.act[at] = __float2bfloat16(silu_f(v[jj]) * u);
-        }
+    for (int jj = 0; jj < 8; ++jj) {
+      const int r = j0 + mine + jj;
+      const float o = other[jj];
+      const float own = up ? v[8 + jj] : v[jj];
+      const float g = up ? o : own;
+      const float u = up ? own : o;
+      if (r < it.rows) {
+        const size_t at = static_cast<size_t>(it.out_row + r) * a.ld_act + f;
+        if constexpr (F8) a.act8[at] = __nv_cvt_float_to_fp8(silu_f(g) * u, __NV_SATFINITE, __NV_E4M3);
+        else a.act[at] = __float2bfloat16(silu_f(g) * u);
       }
     }
-    named_bar_sync(1, 128);
   } else if constexpr (EPI == EPI_QKV) {
     const int which = it.n_tile / kH;   // 0 q, 1 k, 2 v
     const int head = it.n_tile % kH;
@@ -323,6 +332,46 @@ __device__ __forceinline__ void epi_post(const GemmArgs& a, const Item& it, int 
   }
 }
 
+
+// SwiGLU of two adjacent 16-column chunks (activation rows j0..j0+31) with one exchange: the
+// gate thread of output p computes rows j0..j0+15 of it, the up thread rows j0+16..j0+31; each
+// passes the other its 16 values of the other half through exchange buffer `buf` (alternating,
+// as in epi_post<EPI_SWIGLU>).  The same arithmetic per element as epi_post<EPI_SWIGLU>.
+template <bool F8>
+__device__ __forceinline__ void epi_swiglu32(const GemmArgs& a, const Item& it, int row, int j0, float (&v)[16],
+                                             float (&w)[16], const EpiSmem& sm, int buf) {
+  float* xchg = (buf & 1) ? sm.xchg2 : sm.xchg;
+  if constexpr (F8) {
+    const int wr = (row < 64) ? it.n_tile * 64 + row : a.half_rows + it.n_tile * 64 + (row - 64);
+    const float* ws = (it.e < a.n_routed) ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
+                                          : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows;
+    const float sc = ws[wr];
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      v[jj] *= sc;
+      w[jj] *= sc;
+    }
+  }
+  const int up = row >> 6, pr = row & 63;
+#pragma unroll
+  for (int jj = 0; jj < 16; ++jj) xchg[row * 17 + jj] = up ? v[jj] : w[jj];
+  named_bar_sync(1, 128);
+  const float* other = xchg + (row ^ 64) * 17;
+  const int f = it.n_tile * 64 + pr, r0 = j0 + up * 16;
+#pragma unroll
+  for (int jj = 0; jj < 16; ++jj) {
+    const int r = r0 + jj;
+    const float o = other[jj];
+    const float own = up ? w[jj] : v[jj];
+    const float g = up ? o : own;
+    const float u = up ? own : o;
+    if (r < it.rows) {
+      const size_t at = static_cast<size_t>(it.out_row + r) * a.ld_act + f;
+      if constexpr (F8) a.act8[at] = __nv_cvt_float_to_fp8(silu_f(g) * u, __NV_SATFINITE, __NV_E4M3);
+      else a.act[at] = __float2bfloat16(silu_f(g) * u);
+    }
+  }
+}
 
 // Draft-head objective (EPI_LOSS): the operands are swapped for this launch -- A is the packed
 // activation matrix (tile row = activation row, one per epilogue thread), B a tile of 256
@@ -454,6 +503,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   esm.s_pos = reinterpret_cast<int*>(esm.s_off + 256);
   esm.s_aux = esm.s_pos + 256;
   esm.rope = reinterpret_cast<float2*>(esm.s_aux + 256);
+  esm.xchg2 = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(esm.rope) + 1024);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -756,7 +806,27 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       const int nchunks = (it.rows + 15) >> 4;
       float v[16];
       LossState ls = {-INFINITY, 0.f, -INFINITY, 0.f};
-      if (a.split_k == 1 || a.seq_split) {
+      if (EPI == EPI_MOE && it.phase == 0) {
+        // gate/up items: two chunks per exchange
+        for (int c = 0, x = 0; c < nchunks; c += 2, ++x) {
+          if (c + 1 < nchunks) {
+            float w[16];
+            tc_ld16x2(tb + c * 16, tb + (c + 1) * 16, v, w);
+            epi_swiglu32<F8>(a, it, row, c * 16, v, w, esm, x & 1);
+          } else {
+            tc_ld16(tb + c * 16, v);
+            epi_post<EPI_SWIGLU, F8>(a, it, row, c * 16, v, cur, esm, x & 1);
+          }
+        }
+        tc_fence_before();   // the accumulator is read: the next item's MMAs may use it
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        // this gate/up tile's SwiGLU rows are stored: count it for the down items of (e, m)
+        fence_proxy_async_global();
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (threadIdx.x == 64) atomicAdd(a.dep + it.e * a.dep_stride + it.grow / a.grp_rows, 1);
+      } else if (a.split_k == 1 || a.seq_split) {
         for (int c = 0; c < nchunks; ++c) {
           if (c + 1 < nchunks) {
             epi_pre<EPI>(a, it, row, (c + 1) * 16, esm, nxt);
@@ -771,8 +841,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
             for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
           }
           if constexpr (EPI == EPI_MOE) {
-            if (it.phase) epi_post<EPI_SCATTER, F8>(a2, it, row, c * 16, v, cur, esm, c & 1);
-            else epi_post<EPI_SWIGLU, F8>(a, it, row, c * 16, v, cur, esm, c & 1);
+            epi_post<EPI_SCATTER, F8>(a2, it, row, c * 16, v, cur, esm, c & 1);   // down items
           } else if constexpr (EPI == EPI_LOSS) {
             loss_chunk(a, it, c * 16, v, ls);
           } else {
@@ -789,13 +858,6 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
           const int arow = it.n_tile * 128 + row;
           if (arow < a.N)
             a.loss_part[static_cast<size_t>(it.out_row / 256) * a.ldo + arow] = make_float4(ls.m, ls.z, ls.a, ls.mq);
-        }
-        if (EPI == EPI_MOE && it.phase == 0) {
-          // this gate/up tile's SwiGLU rows are stored: count it for the down items of (e, m)
-          fence_proxy_async_global();
-          __threadfence();
-          named_bar_sync(1, 128);
-          if (threadIdx.x == 64) atomicAdd(a.dep + it.e * a.dep_stride + it.grow / a.grp_rows, 1);
         }
         tc_fence_before();
         __syncwarp();
