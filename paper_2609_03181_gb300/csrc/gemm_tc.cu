@@ -26,12 +26,15 @@ namespace fm {
 // NMAX: most activation rows of a tile; ST: pipeline stages (8 for the long weight streams, 4
 // for the short per-split streams of the dense cluster schedule, which leaves room on the SM
 // for the CTAs of the next kernel to start early).
-template <int NMAX, int ST = (NMAX <= 64) ? 8 : 4>
+// DUAL (the expert launch's large-row items, NMAX = 128): every stage holds two 128-row weight
+// tiles multiplied by the same activation tile into two accumulators (gate and up features of
+// the same outputs, or two output tiles of the down projection).
+template <int NMAX, int ST = (NMAX <= 64) ? 8 : 4, bool DUAL = false>
 struct Cfg {
-  static constexpr int A_BYTES = 128 * 128;            // 128 rows x 64 bf16
+  static constexpr int A_BYTES = (DUAL ? 2 : 1) * 128 * 128;   // 128 rows x 64 bf16, per weight tile
   static constexpr int B_BYTES = NMAX * 128;           // NMAX rows x 64 bf16
   static constexpr int STAGES = ST;
-  static constexpr int TMEM_COLS = 2 * NMAX;           // two accumulator buffers
+  static constexpr int TMEM_COLS = (DUAL ? 4 : 2) * NMAX;   // two accumulator buffers (of two with DUAL)
   static constexpr int XCHG_FLOATS = 128 * 17;
   static constexpr int AM_BYTES = 128 * 8;             // argmax partials of 8 row groups x 16 columns
   static constexpr int META_BYTES = 256 * 16;          // per-row metadata of an item (QKV, SCATTER)
@@ -41,6 +44,10 @@ struct Cfg {
 };
 
 constexpr int kShallowStages = 4;   // stages of the dense cluster schedule
+
+// The configuration of an instantiation: the expert launch with 128-row items is the DUAL one.
+template <int NMAX, int EPI, int ST>
+using KCfg = Cfg<NMAX, ST, EPI == EPI_MOE && NMAX == 128>;
 
 struct Item {
   int e, n_tile, b_row, out_row, rows, split, box_log;
@@ -478,7 +485,8 @@ __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem&
 template <int NMAX, int EPI, int ST, bool F8 = false>
 __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a,
                                                          const __grid_constant__ GemmArgs a2) {
-  using C = Cfg<NMAX, ST>;
+  using C = KCfg<NMAX, EPI, ST>;
+  constexpr bool DUAL = (EPI == EPI_MOE && NMAX == 128);
   extern __shared__ uint8_t smem_raw[];
   const uint32_t base_u32 = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
@@ -530,7 +538,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   // groups of split_k x 64 columns
   const uint32_t tmem_cols = a.seq_split ? 512u : static_cast<uint32_t>(C::TMEM_COLS);
   const int nbuf = (a.seq_split && a.split_k > 4) ? 1 : 2;
-  const uint32_t acc_stride = a.seq_split ? static_cast<uint32_t>(a.split_k) * 64u : static_cast<uint32_t>(NMAX);
+  const uint32_t acc_stride =
+      a.seq_split ? static_cast<uint32_t>(a.split_k) * 64u : static_cast<uint32_t>((DUAL ? 2 : 1) * NMAX);
   if (warp == 1) {
     tmem_alloc(s_tmem, tmem_cols);
     tmem_relinquish();
@@ -628,6 +637,22 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         auto load_a = [&](int st, int kc) {
           uint8_t* sa = smA + st * C::A_BYTES;
           const int k = kc * kw;
+          if constexpr (DUAL) {
+            // two 128-row weight tiles: gate rows 128 t.. and up rows half_rows + 128 t.. (64-row
+            // boxes of the paired map), or down rows 256 t.. and 256 t + 128.. (128-row boxes)
+            if (P.paired) {
+              const int r0 = it.n_tile * 128;
+              tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
+              tma_load_3d(sa + 8192, amap, &full[st], k, r0 + 64, el, pol_w);
+              tma_load_3d(sa + 16384, amap, &full[st], k, P.half_rows + r0, el, pol_w);
+              tma_load_3d(sa + 16384 + 8192, amap, &full[st], k, P.half_rows + r0 + 64, el, pol_w);
+            } else {
+              const int r0 = it.n_tile * 256;
+              tma_load_3d(sa, amap, &full[st], k, r0, el, pol_w);
+              tma_load_3d(sa + 16384, amap, &full[st], k, r0 + 128, el, pol_w);
+            }
+            return;
+          }
           if (P.paired) {
             const int r0 = it.n_tile * 64;
             if (P.a3d) {
@@ -745,6 +770,16 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
             if constexpr (F8) tc_mma_e4m3(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
             else tc_mma_bf16(d_tmem, ad + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
           }
+          if constexpr (DUAL) {
+            // the second weight tile against the same activation tile, into the second accumulator
+            const uint64_t ad1 = sw128_kmajor_desc(smem_u32(smA + st * C::A_BYTES + 16384));
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+              if constexpr (F8)
+                tc_mma_e4m3(d_tmem + NMAX, ad1 + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+              else tc_mma_bf16(d_tmem + NMAX, ad1 + 2 * s, bd + 2 * s, idesc, (kc > sp_begin || s > 0) ? 1u : 0u);
+            }
+          }
           tc_commit(&empty[st]);
         }
         if (failed) break;
@@ -806,6 +841,79 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       const int nchunks = (it.rows + 15) >> 4;
       float v[16];
       LossState ls = {-INFINITY, 0.f, -INFINITY, 0.f};
+      if constexpr (DUAL) {
+        // 128-row items: accumulator 0 at tb, accumulator 1 at tb + NMAX (same lanes, same rows)
+        const bool routed = it.e < a.n_routed;
+        if (it.phase == 0) {
+          // gate feature f in accumulator 0, up feature f in accumulator 1: SwiGLU in registers
+          const int f = it.n_tile * 128 + row;
+          float sg = 1.f, su = 1.f;
+          if constexpr (F8) {
+            const float* ws = routed ? a.w_scale[0] + static_cast<size_t>(it.e) * a.scale_rows
+                                     : a.w_scale[1] + static_cast<size_t>(it.e - a.n_routed) * a.scale_rows;
+            sg = ws[f];
+            su = ws[a.half_rows + f];
+          }
+          for (int c = 0; c < nchunks; ++c) {
+            float g[16], u[16];
+            tc_ld16x2(tb + c * 16, tb + NMAX + c * 16, g, u);
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) {
+              const int r = c * 16 + jj;
+              if (r < it.rows) {
+                float gv = g[jj], uv = u[jj];
+                if constexpr (F8) {
+                  gv *= sg;
+                  uv *= su;
+                }
+                const size_t at = static_cast<size_t>(it.out_row + r) * a.ld_act + f;
+                if constexpr (F8) a.act8[at] = __nv_cvt_float_to_fp8(silu_f(gv) * uv, __NV_SATFINITE, __NV_E4M3);
+                else a.act[at] = __float2bfloat16(silu_f(gv) * uv);
+              }
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&tempty[acc]);
+          fence_proxy_async_global();   // the SwiGLU rows are stored: count the tile for (e, m)
+          __threadfence();
+          named_bar_sync(1, 128);
+          if (threadIdx.x == 64) atomicAdd(a.dep + it.e * a.dep_stride + it.grow / a.grp_rows, 1);
+        } else {
+          // output features n0 (accumulator 0) and n0 + 128 (accumulator 1), scattered to
+          // (token, slot)
+          const int n0 = it.n_tile * 256 + row;
+          float s0 = 1.f, s1 = 1.f;
+          if constexpr (F8) {
+            const float* ws = routed ? a2.w_scale[0] + static_cast<size_t>(it.e) * a2.scale_rows
+                                     : a2.w_scale[1] + static_cast<size_t>(it.e - a2.n_routed) * a2.scale_rows;
+            s0 = ws[n0];
+            s1 = ws[n0 + 128];
+          }
+          for (int c = 0; c < nchunks; ++c) {
+            float v0[16], v1[16];
+            tc_ld16x2(tb + c * 16, tb + NMAX + c * 16, v0, v1);
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) {
+              const int r = c * 16 + jj;
+              if (r < it.rows) {
+                float* dst = a2.y + (static_cast<size_t>(esm.s_pos[r]) * kSlots + esm.s_aux[r]) * kD + n0;
+                if constexpr (F8) {
+                  dst[0] = v0[jj] * s0;
+                  dst[128] = v1[jj] * s1;
+                } else {
+                  dst[0] = v0[jj];
+                  dst[128] = v1[jj];
+                }
+              }
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&tempty[acc]);
+        }
+        continue;
+      }
       if (EPI == EPI_MOE && it.phase == 0) {
         // gate/up items: two chunks per exchange
         for (int c = 0, x = 0; c < nchunks; c += 2, ++x) {
@@ -1020,7 +1128,7 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES, bool F8 = false>
 cudaError_t set_smem_attr() {
   return cudaFuncSetAttribute(gemm_tc_kernel<NMAX, EPI, ST, F8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              Cfg<NMAX, ST>::SMEM_BYTES);
+                              KCfg<NMAX, EPI, ST>::SMEM_BYTES);
 }
 
 template <int NMAX, int EPI, int ST = Cfg<NMAX>::STAGES, bool F8 = false>
@@ -1028,7 +1136,7 @@ cudaError_t launch_one(const GemmArgs& a, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(192);
-  cfg.dynamicSmemBytes = Cfg<NMAX, ST>::SMEM_BYTES;
+  cfg.dynamicSmemBytes = KCfg<NMAX, EPI, ST>::SMEM_BYTES;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int n = 0;
@@ -1116,11 +1224,11 @@ cudaError_t gemm_prepare() {
   FM_ATTR(EPI_LOSS)
 #undef FM_ATTR
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE>();
-  if (e == cudaSuccess) e = set_smem_attr<256, EPI_MOE>();
+  if (e == cudaSuccess) e = set_smem_attr<128, EPI_MOE, 4>();
   // fp8 experts and the dense e4m3 GEMM: separate instantiations, so that the bf16 kernels carry
   // no fp8 code
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_MOE, Cfg<64>::STAGES, true>();
-  if (e == cudaSuccess) e = set_smem_attr<256, EPI_MOE, Cfg<256>::STAGES, true>();
+  if (e == cudaSuccess) e = set_smem_attr<128, EPI_MOE, 4, true>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, Cfg<64>::STAGES, true>();
   if (e == cudaSuccess) e = set_smem_attr<256, EPI_F32, Cfg<256>::STAGES, true>();
   if (e == cudaSuccess) e = set_smem_attr<64, EPI_F32, kShallowStages>();
@@ -1185,14 +1293,14 @@ int dense_split_k(int N, int K) {
 cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream_t s) {
   // one persistent CTA per SM; its down items wait on gate/up tiles of other CTAs, so the
   // launch is cooperative (every CTA resident at once).  Items of up to 64 rows run the
-  // 8-stage 64-column kernel, items of up to 256 rows the 4-stage 256-column kernel.
+  // 8-stage 64-column kernel, items of up to 128 rows the 4-stage dual kernel.
   const bool large = gate_up.grp_rows > kExpertTileRows;
   if (gate_up.grp_rows != down.grp_rows || (gate_up.grp_rows != kExpertTileRows && gate_up.grp_rows != kExpertTileRowsLarge))
     return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(num_sms());
   cfg.blockDim = dim3(192);
-  cfg.dynamicSmemBytes = large ? Cfg<256>::SMEM_BYTES : Cfg<64>::SMEM_BYTES;
+  cfg.dynamicSmemBytes = large ? KCfg<128, EPI_MOE, 4>::SMEM_BYTES : Cfg<64>::SMEM_BYTES;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
@@ -1202,10 +1310,10 @@ cudaError_t moe_launch(const GemmArgs& gate_up, const GemmArgs& down, cudaStream
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   if (gate_up.f8) {
-    if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<256, EPI_MOE, Cfg<256>::STAGES, true>, gate_up, down);
+    if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<128, EPI_MOE, 4, true>, gate_up, down);
     return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<64, EPI_MOE, Cfg<64>::STAGES, true>, gate_up, down);
   }
-  if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<256, EPI_MOE, Cfg<256>::STAGES>, gate_up, down);
+  if (large) return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<128, EPI_MOE, 4>, gate_up, down);
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<64, EPI_MOE, Cfg<64>::STAGES>, gate_up, down);
 }
 

@@ -178,11 +178,14 @@ cudaError_t router_prepare();
 int dense_split_k(int N, int K);
 constexpr int kSeqSplitRows = 128;
 // Row tile of the grouped expert launches (work-list items cover at most this many rows): 64
-// rows (the 8-stage, 64-column kernel) below kExpertLargeFromRows candidate rows, 256 rows (the
-// 4-stage, 256-column kernel, each weight tile read once per 256 rows) from there on.  The tile
-// height only groups rows into items; every row's sums are the same at either height.
+// rows (the 8-stage, 64-column kernel; a gate/up item is 64 gate + 64 up features, a down item
+// 128 outputs) below kExpertLargeFromRows candidate rows, 128 rows from there on (the 4-stage
+// dual kernel: an item is two 128-row weight tiles against one activation tile -- 128 gate and
+// the 128 up features of the same outputs, or 256 down outputs -- so each activation tile is
+// read once per 256 weight rows).  The tile height only groups rows into items; every row's
+// sums are the same at either height.
 constexpr int kExpertTileRows = 64;
-constexpr int kExpertTileRowsLarge = 256;
+constexpr int kExpertTileRowsLarge = 128;
 constexpr int kExpertLargeFromRows = 512;
 
 // ------------------------------------------------------------------------- other kernels

@@ -781,9 +781,10 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       g.n_routed = kE;
       g.grp_cnt = ctx->counts + l * kE;
       g.grp_T = T;
-      g.grp_tiles = 2 * kI / 128;
-      g.grp_b_direct = 1;   // shared experts read the normalised rows directly
       g.grp_rows = (T >= kExpertLargeFromRows) ? kExpertTileRowsLarge : kExpertTileRows;
+      const bool dual = g.grp_rows == kExpertTileRowsLarge;   // gate/up item: 128 gate + 128 up features
+      g.grp_tiles = dual ? kI / 128 : 2 * kI / 128;
+      g.grp_b_direct = 1;   // shared experts read the normalised rows directly
       g.map_stride = ctx->Tcap;
       g.expert_ctr = ctx->d_expert_ctr;
       g.act = ctx->act;
@@ -810,7 +811,7 @@ extern "C" spec_status verify_step(spec_ctx* ctx, int32_t B, int32_t K, const in
       d.n_routed = kE;
       d.grp_cnt = ctx->counts + l * kE;
       d.grp_T = T;
-      d.grp_tiles = kD / 128;
+      d.grp_tiles = dual ? kD / 256 : kD / 128;   // down item: 256 or 128 outputs
       d.grp_rows = g.grp_rows;
       d.rowmap = ctx->rowmap;
       d.map_stride = ctx->Tcap;

@@ -34,7 +34,7 @@ FP8_TOL = 6e-2
 
 @pytest.mark.parametrize("B", [1, 8, 160])
 def test_fp8_experts_exact_on_identical_inputs(B):
-    """T = 4, 32 and 640 rows (the last with 256-row expert tiles)."""
+    """T = 4, 32 and 640 rows (the last with 128-row dual expert items)."""
     shape = S.ModelShape(n_layers=1, vocab=4096)
     seed = 21
     vw = S.verifier_weights(shape, seed, gain_std=0.1)
@@ -78,7 +78,7 @@ def test_fp8_verify_two_layers_ragged_contexts():
 
 
 def test_fp8_verify_batch_256_large_tiles():
-    """T = 1024 candidate rows: the expert launch runs 256-row item tiles on e4m3 operands."""
+    """T = 1024 candidate rows: the expert launch runs 128-row dual items on e4m3 operands."""
     ctx = [int(c) for c in S.integers(9, "ctx", 256, 1, 160)]
     run_verify_case(S.ModelShape(n_layers=1, vocab=4096), 9, ctx, K=3, check=range(3, 256, 16), fp8=True,
                     rel_tol=FP8_TOL)
@@ -127,7 +127,7 @@ def test_fp8_speculative_equals_greedy_and_batch_invariance():
                      ("wrong", lambda b, done: [(t + 1) % shape.vocab for t in greedy[b][len(done):len(done) + K]])):
         reset(B)
         assert _loop(eng, B, K, n, fn) == [g[:n] for g in greedy], name
-    # sequence 0 alone, in a batch of 4 (16 rows) and in a batch of 128 (512 rows: 256-row expert
+    # sequence 0 alone, in a batch of 4 (16 rows) and in a batch of 128 (512 rows: 128-row dual expert
     # tiles): bit-identical b rows and verifier tokens
     dev = torch.device("cuda")
     res = []

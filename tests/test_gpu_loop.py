@@ -197,7 +197,8 @@ def test_rows_identical_across_gemm_schedules():
     """Batch invariance across the GEMM schedules: with few rows every split of a dense K runs
     in its own CTA of a cluster (partials reduced through shared memory), from 128 rows on one
     CTA runs all splits of a tile into separate TMEM accumulators, and from 512 candidate rows
-    the expert launch groups rows in 256-row tiles instead of 64-row ones.  Sequence 0 verified
+    the expert launch groups rows in 128-row dual items (two weight tiles per activation tile)
+    instead of 64-row ones.  Sequence 0 verified
     alone (4 rows), as row 0 of a batch of 40 (160 rows) and of a batch of 128 (512 rows), then
     drafted alone and in each batch: the b rows, verifier tokens, draft states u and draft
     tokens are bit-identical."""

@@ -184,9 +184,8 @@ def test_verify_twelve_layers_b8_ctx768_1024():
 
 
 def test_verify_max_batch_256():
-    """The largest batch of the throughput sweep, B=256 (T=1024 candidate rows, four 256-row
-    GEMM tiles per weight tile): 16 sequences spread over the batch are checked against the
-    oracle."""
+    """The largest batch of the throughput sweep, B=256 (T=1024 candidate rows, 128-row dual
+    expert items): 16 sequences spread over the batch are checked against the oracle."""
     shape = S.ModelShape(n_layers=1, vocab=4096)
     ctx = [int(c) for c in S.integers(9, "ctx", 256, 1, 160)]
     run_verify_case(shape, 9, ctx, K=3, check=range(3, 256, 16))
