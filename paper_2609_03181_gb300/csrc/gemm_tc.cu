@@ -55,10 +55,13 @@ struct Item {
   int phase;  // EPI_MOE: 0 gate/up item, 1 down item
 };
 
-// Per-expert tables of a grouped launch in shared memory, built by every CTA from the counts:
-// grp[e] first item of expert e (grp[66] = items), grp[67 + e] its rows, and for EPI_MOE
-// grp[134 + e] the first down item of expert e counted from the first down item.
+// Per-expert tables of a grouped launch in shared memory, built by every CTA from the counts,
+// indexed by list position p (the shared experts first -- they have the most rows, so their
+// down items are free to start early -- then the routed experts in order): grp[p] first item
+// of the expert at p (grp[66] = items), grp[67 + p] its rows, and for EPI_MOE grp[134 + p] its
+// first down item counted from the first down item.
 constexpr int kGrpItem = 0, kGrpCnt = kE + kShared + 1, kGrpDn = 2 * (kE + kShared + 1);
+__device__ __forceinline__ int grp_expert(int p) { return p < kShared ? kE + p : p - kShared; }
 
 template <int EPI>
 __device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, int i, Item& it, const int* grp) {
@@ -72,19 +75,19 @@ __device__ __forceinline__ void get_item(const GemmArgs& a, const GemmArgs& a2, 
       P = &a2;
       it.phase = 1;
     }
-    int lo = 0, hi = kE + kShared - 1;   // the last expert whose first item is <= i has items
+    int lo = 0, hi = kE + kShared - 1;   // the last position whose first item is <= i has items
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
       if (pre[mid] <= i) lo = mid;
       else hi = mid - 1;
     }
     const int j = i - pre[lo], m = j / P->grp_tiles;
-    it.e = lo;
+    it.e = grp_expert(lo);
     it.n_tile = j - m * P->grp_tiles;
     it.grow = a.grp_rows * m;
     it.rows = min(a.grp_rows, grp[kGrpCnt + lo] - it.grow);
-    it.out_row = lo * a.map_stride + it.grow;
-    it.b_row = (P->grp_b_direct && lo >= a.n_routed) ? it.grow : it.out_row;
+    it.out_row = it.e * a.map_stride + it.grow;
+    it.b_row = (P->grp_b_direct && it.e >= a.n_routed) ? it.grow : it.out_row;
     it.split = 0;
     int bl = 0;
     while ((16 << bl) < it.rows) ++bl;
@@ -564,8 +567,8 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       int c[3], ni[3], nd[3], sc = 0, si = 0, sd = 0, touched = 0;
 #pragma unroll
       for (int k = 0; k < 3; ++k) {
-        const int e = 3 * static_cast<int>(threadIdx.x) + k;
-        c[k] = (e < kE + kShared) ? ((e < a.n_routed) ? a.grp_cnt[e] : a.grp_T) : 0;
+        const int p = 3 * static_cast<int>(threadIdx.x) + k, e = grp_expert(p);
+        c[k] = (p < kE + kShared) ? ((e < a.n_routed) ? a.grp_cnt[e] : a.grp_T) : 0;
         const int mt = (c[k] + a.grp_rows - 1) / a.grp_rows;
         ni[k] = mt * a.grp_tiles;
         nd[k] = (EPI == EPI_MOE) ? mt * a2.grp_tiles : 0;
@@ -588,11 +591,11 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
       int ri = ii - si, rd = id - sd;
 #pragma unroll
       for (int k = 0; k < 3; ++k) {
-        const int e = 3 * static_cast<int>(threadIdx.x) + k;
-        if (e < kE + kShared) {
-          grp[kGrpCnt + e] = c[k];
-          grp[kGrpItem + e] = ri;
-          grp[kGrpDn + e] = rd;
+        const int p = 3 * static_cast<int>(threadIdx.x) + k;
+        if (p < kE + kShared) {
+          grp[kGrpCnt + p] = c[k];
+          grp[kGrpItem + p] = ri;
+          grp[kGrpDn + p] = rd;
         }
         ri += ni[k];
         rd += nd[k];

@@ -182,11 +182,13 @@ constexpr int kSeqSplitRows = 128;
 // 128 outputs) below kExpertLargeFromRows candidate rows, 128 rows from there on (the 4-stage
 // dual kernel: an item is two 128-row weight tiles against one activation tile -- 128 gate and
 // the 128 up features of the same outputs, or 256 down outputs -- so each activation tile is
-// read once per 256 weight rows).  The tile height only groups rows into items; every row's
-// sums are the same at either height.
+// read once per 256 weight rows, and half as many items carry the per-item costs).  Below 16
+// rows (B = 1 at K = 3: about 3.6 of the smaller items per CTA) the coarser items leave a
+// longer tail than they save (measured).  The tile height only groups rows into items; every
+// row's sums are the same at either height.
 constexpr int kExpertTileRows = 64;
 constexpr int kExpertTileRowsLarge = 128;
-constexpr int kExpertLargeFromRows = 512;
+constexpr int kExpertLargeFromRows = 16;
 
 // ------------------------------------------------------------------------- other kernels
 struct AttnArgs {
