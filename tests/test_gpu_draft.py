@@ -1,6 +1,7 @@
 """draft_step through the C ABI against the fp64 oracle's FastMTP head: the shared block
-alone at the paper's widths (B=32, draft-cache context 2048, K=3), with 1..4 rows queued per
-sequence (base states b ~ N(0,1), as a commit of m = 0..3 accepted drafts leaves them).
+alone at the paper's widths (B=32, draft-cache context 2048, K=3; also B=1 and 8), with 1..4
+rows queued per sequence (base states b ~ N(0,1), as a commit of m = 0..3 accepted drafts leaves
+them).
 
 Rules: the committed draft K/V rows and the draft states u^(k) within max relative error
 2e-2; drafted tokens bit-exact at every depth whose oracle top-2 margin exceeds 1e-3 (a depth
@@ -69,6 +70,13 @@ def run_draft_case(B, ctx, K, seed, vocab=129280):
 
 def test_draft_block_b32_ctx2048():
     run_draft_case(B=32, ctx=2048, K=3, seed=2)
+
+
+@pytest.mark.parametrize("B", [1, 8])
+def test_draft_small_batch(B):
+    """The small batches of the latency-bound regime (one 16-row activation box, cluster
+    split-K GEMMs), same rules."""
+    run_draft_case(B=B, ctx=2048, K=3, seed=4 + B)
 
 
 def test_draft_small_context_deep_chain():
