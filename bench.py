@@ -758,14 +758,17 @@ def run_sweep(args):
     grow = (args.warmup + steps_for(1) + 2) * (Kmax + 1)
     clocks = ClockSampler(0)
     clocks.start()
+    fp8 = args.experts == "fp8"
     for router in routers:
         vw, dw, _ = S.successor_weights(shape, 4, ACCEPT_RATIO)
         if router == "zipf":
             for l, lw in enumerate(vw.layers):
                 lw.router_bias = S.zipf_router_bias(4, l, shape.n_experts, 1.2)
+        if fp8:
+            vw = S.quantize_experts_fp8(vw)
         stream = torch.cuda.Stream(dev)
         eng = F.Engine(vw, dw, max_batch=Bmax, K_max=Kmax, max_ctx=max(ctxs) + grow, page_size=64,
-                       device=str(dev), stream=stream)
+                       device=str(dev), stream=stream, expert_fp8=fp8)
         g = torch.Generator(device=dev)
         g.manual_seed(4)
         for l in range(shape.n_layers):
@@ -826,12 +829,12 @@ def run_sweep(args):
                     ctx_mean = float(lens[args.warmup:].mean())
                     tok = float(h[args.warmup:].sum())
                     touched = counted["experts_touched"] / max(1, counted["launches"]["router"])
-                    vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared)
+                    vbytes = algorithmic_bytes(shape, B, K, ctx_mean, touched - shape.n_shared, fp8)
                     load = cnt / cnt.mean(-1, keepdim=True)
                     tok_s = tok / (ms_step * n_steps / 1000.0)
                     if K == 0:
                         ar_tok_s = tok_s
-                    out = {"sweep": True, "router": router, "batch": B, "ctx": ctx, "K": K,
+                    out = {"sweep": True, "router": router, "experts": args.experts, "batch": B, "ctx": ctx, "K": K,
                            "tokens_per_s": tok_s, "ms_step": ms_step,
                            "ms_step_mean": statistics.mean(ev[i][0].elapsed_time(ev[i][3]) for i in timed),
                            "ms_draft": ms_draft, "ms_verify": ms_verify, "ms_commit": ms(2, 3),

@@ -17,8 +17,9 @@ from typing import Iterable
 PACKAGED = os.path.join(os.path.dirname(os.path.abspath(__file__)), "depth_table_gb300.json")
 
 
-def build_table(lines: Iterable[str], router: str = "uniform", source: str = "") -> dict:
-    """The table of one router mode from the JSON lines of a sweep (other lines are skipped)."""
+def build_table(lines: Iterable[str], router: str = "uniform", source: str = "", experts: str = "bf16") -> dict:
+    """The table of one router mode and expert format from the JSON lines of a sweep (other lines
+    are skipped; lines without an `experts` field are bf16)."""
     pts = {}
     meta = {}
     for line in lines:
@@ -28,7 +29,7 @@ def build_table(lines: Iterable[str], router: str = "uniform", source: str = "")
         d = json.loads(line)
         if d.get("sweep_clocks") is not None:
             meta["clocks"] = d["sweep_clocks"]
-        if not d.get("sweep") or d.get("router") != router:
+        if not d.get("sweep") or d.get("router") != router or d.get("experts", "bf16") != experts:
             continue
         key = (int(d["batch"]), int(d["ctx"]))
         p = pts.setdefault(key, {"batch": key[0], "ctx": key[1], "tokens_per_s": {}, "steps": {}})
