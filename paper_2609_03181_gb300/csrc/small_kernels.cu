@@ -68,6 +68,10 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
     tok = 0;
   }
   if (slot_ok && r == 0 && tok != pending[slot] && threadIdx.x == 0) atomicOr(err, ERR_PENDING);
+  if (threadIdx.x == 32) {   // the position, while the embedding row is fetched
+    pos[row] = (slot_ok ? seq_len[slot] : 0) + r;
+    kv_rowoff[row] = static_cast<long long>(b * stage_R + r) * 2 * kH * kHD;
+  }
   const bf16* e = embed + static_cast<size_t>(tok) * kD;
   float x[10];
 #pragma unroll
@@ -77,10 +81,6 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
     h[static_cast<size_t>(row) * kD + i] = x[k];
   }
   norm_row_store(x, gain, eps, xn + static_cast<size_t>(row) * kD, red);
-  if (threadIdx.x == 0) {
-    pos[row] = (slot_ok ? seq_len[slot] : 0) + r;
-    kv_rowoff[row] = static_cast<long long>(b * stage_R + r) * 2 * kH * kHD;
-  }
 }
 
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
@@ -486,20 +486,21 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
     }
     return;
   }
-  int tok = draft_tok[slot * kMaxR + i];
-  if (tok < 0 || tok >= vocab) {
-    if (threadIdx.x == 0) atomicOr(err, ERR_TOKEN_RANGE);
-    tok = 0;
-  }
-  float x[10];
-#pragma unroll
-  for (int k = 0; k < 10; ++k) x[k] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * k]);
-  norm_row_store(x, enorm, eps, out, red);
+  // three independent chains go out together: the token (then its embedding row), the base
+  // state row, and the position (then its page)
+  __shared__ int s_tok;
+  float xb[10];
 #pragma unroll
   for (int k = 0; k < 10; ++k)
-    x[k] = __bfloat162float(draft_b[(static_cast<size_t>(slot) * kMaxR + i) * kD + threadIdx.x + 128 * k]);
-  norm_row_store(x, hnorm, eps, out + kD, red);
+    xb[k] = __bfloat162float(draft_b[(static_cast<size_t>(slot) * kMaxR + i) * kD + threadIdx.x + 128 * k]);
   if (threadIdx.x == 0) {
+    int tok = draft_tok[slot * kMaxR + i];
+    if (tok < 0 || tok >= vocab) {
+      atomicOr(err, ERR_TOKEN_RANGE);
+      tok = 0;
+    }
+    s_tok = tok;
+  } else if (threadIdx.x == 32) {
     const int p = seq_len[slot] - n + i;
     pos[row] = p;
     const int pi = p / page_size;
@@ -511,6 +512,13 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
       kv_rowoff[row] = (static_cast<long long>(page) * 2 * kH * page_size + (p % page_size)) * kHD;
     }
   }
+  __syncthreads();
+  const int tok = s_tok;
+  float x[10];
+#pragma unroll
+  for (int k = 0; k < 10; ++k) x[k] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * k]);
+  norm_row_store(xb, hnorm, eps, out + kD, red);   // while the embedding row is on its way
+  norm_row_store(x, enorm, eps, out, red);
 }
 
 cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len, const int* pending,
@@ -552,6 +560,13 @@ __global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_
   __shared__ float red[4];
   __shared__ int s_tok;
   const int b = blockIdx.x;
+  // the loads that do not depend on the drafted token go out together with the key: the
+  // token's state row u and the sequence's position
+  float xu[10];
+  if (k < K) {
+#pragma unroll
+    for (int q = 0; q < 10; ++q) xu[q] = __bfloat162float(u[static_cast<size_t>(b) * kD + threadIdx.x + 128 * q]);
+  }
   if (threadIdx.x == 0) {
     int tok = argmax_key_index(am_key[b]);
     am_key[b] = 0ull;
@@ -561,6 +576,12 @@ __global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_
     }
     s_tok = tok;
     cand[b * cand_ld + k] = tok;
+  } else if (threadIdx.x == 32 && k < K) {
+    const int slot = slots[b];
+    const bool slot_ok = slot >= 0 && slot < n_slots;
+    if (!slot_ok) atomicOr(err, ERR_SLOT_RANGE);
+    pos[b] = (slot_ok ? seq_len[slot] : 0) + k - 1;
+    kv_rowoff[b] = b * dstage_seq_stride + static_cast<long long>(k - 1) * 2 * kH * kHD;
   }
   __syncthreads();
   if (k >= K) return;
@@ -569,17 +590,8 @@ __global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_
   float x[10];
 #pragma unroll
   for (int q = 0; q < 10; ++q) x[q] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * q]);
+  norm_row_store(xu, hnorm, eps, out + kD, red);   // while the embedding row is on its way
   norm_row_store(x, enorm, eps, out, red);
-#pragma unroll
-  for (int q = 0; q < 10; ++q) x[q] = __bfloat162float(u[static_cast<size_t>(b) * kD + threadIdx.x + 128 * q]);
-  norm_row_store(x, hnorm, eps, out + kD, red);
-  if (threadIdx.x == 0) {
-    const int slot = slots[b];
-    const bool slot_ok = slot >= 0 && slot < n_slots;
-    if (!slot_ok) atomicOr(err, ERR_SLOT_RANGE);
-    pos[b] = (slot_ok ? seq_len[slot] : 0) + k - 1;
-    kv_rowoff[b] = b * dstage_seq_stride + static_cast<long long>(k - 1) * 2 * kH * kHD;
-  }
 }
 
 cudaError_t draft_next_launch(unsigned long long* am_key, int vocab, int* err, int B, int k, int K, const int* slots,
