@@ -422,7 +422,8 @@ __device__ __forceinline__ void loss_chunk(const GemmArgs& a, const Item& it, in
   st.a = acc;
 }
 
-// Cluster split-K reduction, run by the 128 epilogue threads of every CTA of the cluster after
+// Cluster split-K reduction by whole chunks (the epilogues without a quad form below; the dense
+// launches use the quad form), run by the 128 epilogue threads of every CTA of the cluster after
 // the first cluster barrier: CTA `rank` takes chunks rank, rank + S, ..., adds the S partial
 // tiles of each (read from the cluster's shared memory) in split order -- the same sums as the
 // other schedules -- and runs the epilogue on them.  The epilogue operands of its first chunk
@@ -484,6 +485,177 @@ __device__ __forceinline__ void cluster_reduce(const GemmArgs& a, const EpiSmem&
   }
 }
 
+// Cluster split-K reduction in quad units, for the epilogues whose row pairs need no more than
+// one warp (F32, RESID, QKV, SWIGLU).  A unit is 4 activation rows (one float4 column of the
+// partial tiles) x 32 tile rows: row group g of the tile is rows 16g..16g+15 (lanes 0..15) and
+// their rotate-half / gate-up partners 64+16g..64+16g+15 (lanes 16..31), so a pair meets by one
+// shuffle.  Units are dealt over the cluster's CTAs first, then over their 4 epilogue warps:
+// a tile of 4 activation rows is reduced by 4 warps on 4 SMs, each reading the S partials of
+// its unit at once (one round trip through distributed shared memory), instead of by all 128
+// threads of one CTA in two.  The sums and the epilogue arithmetic are those of cluster_reduce.
+template <int EPI>
+__device__ __forceinline__ constexpr bool quad_epi() {
+  return EPI == EPI_F32 || EPI == EPI_RESID || EPI == EPI_QKV || EPI == EPI_SWIGLU;
+}
+__device__ __forceinline__ int quad_row(int g, int lane) { return (lane < 16) ? 16 * g + lane : 48 + 16 * g + lane; }
+// the k-th unit of epilogue warp `slot` of cluster rank `rank`: units go round the cluster's
+// CTAs first, then their warps
+__device__ __forceinline__ int quad_unit(int k, int slot, int rank, int S) { return (k * 4 + slot) * S + rank; }
+
+// Epilogue operands of one unit, read before the reduction: the old residuals (RESID) or the
+// cos/sin of the 4 rows' positions at this lane's feature (QKV q and k tiles).
+struct QuadOps {
+  float old[4];
+  float2 rope[4];
+};
+struct QuadPre {
+  QuadOps u[2];   // the first two units of the warp
+};
+
+template <int EPI>
+__device__ __forceinline__ void quad_ops(const GemmArgs& a, const Item& it, const EpiSmem& sm, int u, int lane,
+                                         QuadOps& o) {
+  const int r = quad_row(u & 3, lane), j0 = 4 * (u >> 2);
+  if constexpr (EPI == EPI_RESID) {
+    const int n = it.n_tile * 128 + r;
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj)
+      o.old[jj] = (n < a.N && j0 + jj < it.rows) ? a.out[static_cast<size_t>(it.out_row + j0 + jj) * a.ldo + n] : 0.f;
+  } else if constexpr (EPI == EPI_QKV) {
+    if (it.n_tile < 2 * kH) {
+      bool bad = false;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        int q = (j0 + jj < it.rows) ? sm.s_pos[j0 + jj] : 0;
+        if (q < 0 || q >= a.max_pos) {
+          bad = true;
+          q = 0;
+        }
+        o.rope[jj] = a.rope[static_cast<size_t>(q) * (kHD / 2) + (r & 63)];
+      }
+      if (bad) atomicOr(a.err, ERR_POSITION);
+    }
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void quad_post(const GemmArgs& a, const Item& it, const EpiSmem& sm, int u, int lane,
+                                          float (&v)[4], const QuadOps& o) {
+  const int r = quad_row(u & 3, lane), j0 = 4 * (u >> 2);
+  if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
+    const int n = it.n_tile * 128 + r;
+    if (n < a.N) {
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj)
+        if (j0 + jj < it.rows)
+          a.out[static_cast<size_t>(it.out_row + j0 + jj) * a.ldo + n] = (EPI == EPI_RESID) ? o.old[jj] + v[jj] : v[jj];
+    }
+  } else if constexpr (EPI == EPI_QKV) {
+    const int which = it.n_tile / kH;   // 0 q, 1 k, 2 v
+    const int head = it.n_tile % kH;
+    if (which < 2) {
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const float partner = __shfl_xor_sync(0xffffffffu, v[jj], 16);
+        v[jj] = (r < 64) ? rope_lo(v[jj], partner, o.rope[jj]) : rope_hi(v[jj], partner, o.rope[jj]);
+      }
+    }
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      const int j = j0 + jj;
+      if (j >= it.rows) continue;
+      const int m = it.out_row + j;
+      if (which == 0) {
+        a.q_out[static_cast<size_t>(m) * (kH * kHD) + head * kHD + r] = __float2bfloat16(v[jj]);
+      } else {
+        const long long off = sm.s_off[j];
+        if (off >= 0) a.kv_base[off + (which == 2 ? a.v_off : 0) + head * a.head_stride + r] = __float2bfloat16(v[jj]);
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    // lanes 0..15 hold gate features, lanes 16..31 the up features of the same outputs; the
+    // gate lane computes rows 0 and 1 of the unit, the up lane rows 2 and 3
+    const int up = lane >> 4;
+    float other[4];
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) other[jj] = __shfl_xor_sync(0xffffffffu, v[jj], 16);
+    const int f = it.n_tile * 64 + (r & 63);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int jj = 2 * up + h, j = j0 + jj;
+      const float g = up ? other[jj] : v[jj];
+      const float uu = up ? v[jj] : other[jj];
+      if (j < it.rows) a.act[static_cast<size_t>(it.out_row + j) * a.ld_act + f] = __float2bfloat16(silu_f(g) * uu);
+    }
+  }
+}
+
+// Epilogue warp `slot` (0..3) of cluster rank `rank` takes units (k * 4 + slot) * S + rank,
+// k = 0, 1, ..., two at a time with every split's loads of both in flight.
+template <int EPI>
+__device__ __forceinline__ void quad_prefetch(const GemmArgs& a, const Item& it, const EpiSmem& sm, int slot, int lane,
+                                              QuadPre& qp) {
+  const int S = a.cluster, rank = static_cast<int>(cluster_ctarank());
+  const int U = 4 * ((it.rows + 3) >> 2);
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int u = quad_unit(k, slot, rank, S);
+    if (u < U) quad_ops<EPI>(a, it, sm, u, lane, qp.u[k]);
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void cluster_reduce_quads(const GemmArgs& a, const EpiSmem& sm, uint32_t part_saddr,
+                                                     int slot, int lane, const QuadPre& qp) {
+  Item it;
+  get_item<EPI>(a, a, blockIdx.x, it, nullptr);
+  const int S = a.cluster, rank = static_cast<int>(cluster_ctarank());
+  const int U = 4 * ((it.rows + 3) >> 2);
+  int n_mine = 0;
+  while (quad_unit(n_mine, slot, rank, S) < U) ++n_mine;
+  if (n_mine == 0) cluster_arrive();
+  for (int k0 = 0; k0 < n_mine; k0 += 2) {
+    float4 p[2][kMaxSplit];
+    QuadOps o[2];
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      if (k0 + kk >= n_mine) break;
+      const int u = quad_unit(k0 + kk, slot, rank, S);
+      const int r = quad_row(u & 3, lane);
+      const uint32_t at = part_saddr + static_cast<uint32_t>(((u >> 2) * 128 + r) * 16);
+#pragma unroll
+      for (int sp = 0; sp < kMaxSplit; ++sp)
+        if (sp < S) p[kk][sp] = ld_dsmem_f4(at, sp);
+      if (k0 == 0) o[kk] = qp.u[kk];
+      else quad_ops<EPI>(a, it, sm, u, lane, o[kk]);
+    }
+    float v[2][4];
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      if (k0 + kk >= n_mine) break;
+      float4 t = p[kk][0];
+#pragma unroll
+      for (int sp = 1; sp < kMaxSplit; ++sp)
+        if (sp < S) {
+          t.x += p[kk][sp].x;
+          t.y += p[kk][sp].y;
+          t.z += p[kk][sp].z;
+          t.w += p[kk][sp].w;
+        }
+      v[kk][0] = t.x;
+      v[kk][1] = t.y;
+      v[kk][2] = t.z;
+      v[kk][3] = t.w;
+    }
+    if (k0 + 2 >= n_mine) cluster_arrive();   // no more reads of the other CTAs' partial tiles
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      if (k0 + kk >= n_mine) break;
+      quad_post<EPI>(a, it, sm, quad_unit(k0 + kk, slot, rank, S), lane, v[kk], o[kk]);
+    }
+  }
+}
+
 // ------------------------------------------------------------------ kernel
 template <int NMAX, int EPI, int ST, bool F8 = false>
 __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a,
@@ -507,6 +679,7 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
   int* s_last = s_vote + 4;
   EpiSmem esm;
   EpiPre first_pre;   // cluster split-K: the epilogue operands of the first chunk this CTA reduces
+  QuadPre quad_pre;   // cluster split-K in quad units: those of the warp's first two units
   esm.xchg = reinterpret_cast<float*>(smem + C::STAGES * (C::A_BYTES + C::B_BYTES) + 256);
   esm.am_val = esm.xchg + C::XCHG_FLOATS;
   esm.am_idx = reinterpret_cast<int*>(esm.am_val + 128);
@@ -818,16 +991,20 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
         stage_meta<EPI>(a, it, esm);
       }
       const bool rope = (EPI == EPI_QKV) && it.n_tile < 2 * kH;
-      const int c_first = (a.cluster > 1) ? static_cast<int>(cluster_ctarank()) : 0;
       RopeRegs rr;
-      if (rope) {
-        rope_load(a, it, c_first * 16, esm, rr);
-        rope_store(esm, 0, rr);
-        named_bar_sync(1, 128);
-      }
       EpiPre cur, nxt;
-      epi_pre<EPI>(a, it, row, c_first * 16, esm, cur);
-      first_pre = cur;
+      if (quad_epi<EPI>() && a.cluster > 1) {
+        quad_prefetch<EPI>(a, it, esm, ew, lane, quad_pre);
+      } else {
+        const int c_first = (a.cluster > 1) ? static_cast<int>(cluster_ctarank()) : 0;
+        if (rope) {
+          rope_load(a, it, c_first * 16, esm, rr);
+          rope_store(esm, 0, rr);
+          named_bar_sync(1, 128);
+        }
+        epi_pre<EPI>(a, it, row, c_first * 16, esm, cur);
+        first_pre = cur;
+      }
       bool ok = mbar_wait(&tfull[acc], acc_ph, s_abort);
       ok = __all_sync(0xffffffffu, ok);
       if (lane == 0) s_vote[ew] = ok ? 1 : 0;
@@ -1099,8 +1276,12 @@ __global__ void __launch_bounds__(192, 1) gemm_tc_kernel(const __grid_constant__
 
   if (a.cluster > 1) {
     cluster_sync_all();   // every split's partial tile is in its CTA's shared memory
-    if (warp >= 2) cluster_reduce<EPI>(a, esm, smem_u32(smA), (warp & 3) * 32 + lane, first_pre);
-    else cluster_arrive();
+    if (warp >= 2) {
+      if (quad_epi<EPI>() && a.cluster > 1) cluster_reduce_quads<EPI>(a, esm, smem_u32(smA), warp - 2, lane, quad_pre);
+      else cluster_reduce<EPI>(a, esm, smem_u32(smA), (warp & 3) * 32 + lane, first_pre);
+    } else {
+      cluster_arrive();
+    }
     cluster_wait();       // no CTA leaves while the others still read its shared memory
   }
   tc_fence_before();
