@@ -129,15 +129,15 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
   __shared__ __align__(16) bf16 xs[kRouteRows * kRouteStride];   // the rounded rows
   __shared__ float lg[kRouteRows][kE];                           // logits, then probabilities
   __shared__ int dst[kRouteRows][kTopK];                         // input row of each selection
+  __shared__ unsigned long long keys[kRouteCtaRows][kE];         // (probability, lower id first) keys
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
-  // The router matrix is never written by earlier kernels: most of this lane's share of its
-  // expert's row (expert 8 warp + g, columns 32 c + 8 t4 .. + 7) is loaded before the wait, the
-  // rest after the norm.
-  constexpr int kSteps = kD / 32, kEarly = 32;
+  // The router matrix is never written by earlier kernels: this lane's share of its expert's
+  // row (expert 8 warp + g, columns 32 c + 8 t4 .. + 7) is loaded before the wait.
+  constexpr int kSteps = kD / 32;
   const uint4* wrow = reinterpret_cast<const uint4*>(a.wr + static_cast<size_t>(warp * 8 + g) * kD) + t4;
   uint4 wq[kSteps];
 #pragma unroll
-  for (int c = 0; c < kEarly; ++c) wq[c] = wrow[4 * c];
+  for (int c = 0; c < kSteps; ++c) wq[c] = wrow[4 * c];
   uint2 gq[kD / 128];   // norm gain (bf16, also a weight), lane's columns 4 (lane + 32 k) .. + 3
 #pragma unroll
   for (int k = 0; k < kD / 128; ++k) gq[k] = *reinterpret_cast<const uint2*>(a.gain + 4 * (lane + 32 * k));
@@ -189,8 +189,6 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
       }
     }
   }
-#pragma unroll
-  for (int c = kEarly; c < kSteps; ++c) wq[c] = wrow[4 * c];
   __syncthreads();
   // logits D[row][expert] = xs W^T: 40 steps of 32 columns, two k16 MMAs each.  Within a step
   // the columns enter the MMA in a fixed permuted order (lane t4's four pairs 32c + 8t4 + 2j,
@@ -220,16 +218,11 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
     lg[g + 8][e + 1] = d[3] + b1;
   }
   __syncthreads();
-  // softmax and top-6 of rows warp and warp + 8.  Lane l holds experts l and l + 32; the six
-  // winners come out in rank order from six warp-wide maxima of (probability, lower id first)
-  // keys -- the order better() defines.  Both rows are ranked before any row of an expert is
-  // claimed, so that their atomic adds are in flight together.
-  int rank[2][2] = {{-1, -1}, {-1, -1}};
-  float pv[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
-#pragma unroll
-  for (int h2 = 0; h2 < 2; ++h2) {
-    const int r = warp + 8 * h2;
-    if (r >= nr) break;
+  // softmax of row `warp` (warp w < nr; lane l holds experts l and l + 32), the probabilities
+  // back into lg
+  static_assert(kRouteCtaRows * kE == 256, "one thread per (row, expert) ranks the experts");
+  if (warp < nr) {
+    const int r = warp;
     const float l0 = lg[r][lane], l1 = lg[r][lane + 32];
     const float m = warp_max(fmaxf(l0, l1));
     const float e0 = expf(l0 - m), e1 = expf(l1 - m);
@@ -242,43 +235,33 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
       if (!(p0 == p0)) p0 = -1.f;
       if (!(p1 == p1)) p1 = -1.f;
     }
-    pv[h2][0] = p0;
-    pv[h2][1] = p1;
-    unsigned long long k0 = argmax_key(p0, lane), k1 = argmax_key(p1, lane + 32);   // 0: taken
+    lg[r][lane] = p0;
+    lg[r][lane + 32] = p1;
+    keys[r][lane] = argmax_key(p0, lane);
+    keys[r][lane + 32] = argmax_key(p1, lane + 32);
+  }
+  __syncthreads();
+  // top-6: thread (r, e) counts the experts whose (probability, lower id first) key beats its
+  // own -- its rank, the place argmax rounds would give it -- and, ranked among the first six,
+  // takes the next row of expert e
+  {
+    const int r = threadIdx.x >> 6, e = threadIdx.x & 63;
+    if (r < nr) {
+      const float pe = lg[r][e];
+      const unsigned long long mine = keys[r][e];
+      int rank = 0;
 #pragma unroll
-    for (int k = 0; k < kTopK; ++k) {
-      unsigned long long best = k0 > k1 ? k0 : k1;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
-        best = other > best ? other : best;
-      }
-      if (best == k0) {
-        rank[h2][0] = k;
-        k0 = 0ull;
-      } else if (best == k1) {
-        rank[h2][1] = k;
-        k1 = 0ull;
+      for (int o = 0; o < kE; ++o) rank += (keys[r][o] > mine) ? 1 : 0;
+      if (rank < kTopK) {
+        const int t = t0 + r;
+        const int pos = atomicAdd(a.counts + e, 1);
+        a.idx[static_cast<size_t>(t) * kTopK + rank] = e;
+        a.gate[static_cast<size_t>(t) * kTopK + rank] = pe;
+        a.rowmap[static_cast<size_t>(e) * a.map_stride + pos] = (t << 3) | rank;
+        dst[r][rank] = e * a.map_stride + pos;
       }
     }
   }
-  int pos[2][2];
-#pragma unroll
-  for (int h2 = 0; h2 < 2; ++h2)
-#pragma unroll
-    for (int j = 0; j < 2; ++j)
-      if (rank[h2][j] >= 0) pos[h2][j] = atomicAdd(a.counts + lane + 32 * j, 1);
-#pragma unroll
-  for (int h2 = 0; h2 < 2; ++h2)
-#pragma unroll
-    for (int j = 0; j < 2; ++j)
-      if (rank[h2][j] >= 0) {
-        const int t = t0 + warp + 8 * h2, e = lane + 32 * j;
-        a.idx[static_cast<size_t>(t) * kTopK + rank[h2][j]] = e;
-        a.gate[static_cast<size_t>(t) * kTopK + rank[h2][j]] = pv[h2][j];
-        a.rowmap[static_cast<size_t>(e) * a.map_stride + pos[h2][j]] = (t << 3) | rank[h2][j];
-        dst[warp + 8 * h2][rank[h2][j]] = e * a.map_stride + pos[h2][j];
-      }
   __syncthreads();
   // the rounded rows into their experts' input rows, 8 elements per thread and step (16 bytes
   // of bf16, or with fp8 experts 8 bytes of e4m3)
