@@ -25,24 +25,28 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 }
 __device__ __forceinline__ float block128_sum(float v, float* red) { return block_sum<128>(v, red); }
 
+// The norm gain of this thread's elements i = tid + NT*k as floats.  A gain is a weight, never
+// written by an earlier kernel, so every kernel below reads it before its wait.
+template <int NT>
+__device__ __forceinline__ void load_gain_t(const bf16* gain, float (&gv)[kD / NT]) {
+#pragma unroll
+  for (int k = 0; k < kD / NT; ++k) gv[k] = __bfloat162float(gain[threadIdx.x + NT * k]);
+}
 // x (kD/NT values per thread, element i = tid + NT*k) -> bf16 x * rsqrt(mean(x^2) + eps) * gain
 template <int NT>
-__device__ __forceinline__ void norm_row_store_t(const float (&x)[kD / NT], const bf16* gain, float eps, bf16* out,
-                                                 float* red) {
+__device__ __forceinline__ void norm_row_store_t(const float (&x)[kD / NT], const float (&gv)[kD / NT], float eps,
+                                                 bf16* out, float* red) {
   float ss = 0.f;
 #pragma unroll
   for (int k = 0; k < kD / NT; ++k) ss += x[k] * x[k];
   ss = block_sum<NT>(ss, red);
   const float inv = rsqrtf(ss / kD + eps);
 #pragma unroll
-  for (int k = 0; k < kD / NT; ++k) {
-    const int i = threadIdx.x + NT * k;
-    out[i] = __float2bfloat16(x[k] * inv * __bfloat162float(gain[i]));
-  }
+  for (int k = 0; k < kD / NT; ++k) out[threadIdx.x + NT * k] = __float2bfloat16(x[k] * inv * gv[k]);
 }
-__device__ __forceinline__ void norm_row_store(const float (&x)[10], const bf16* gain, float eps, bf16* out,
+__device__ __forceinline__ void norm_row_store(const float (&x)[10], const float (&gv)[10], float eps, bf16* out,
                                                float* red) {
-  norm_row_store_t<128>(x, gain, eps, out, red);
+  norm_row_store_t<128>(x, gv, eps, out, red);
 }
 
 // ---------------------------------------------------------------- embedding + norm
@@ -52,6 +56,8 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
                                                          long long* kv_rowoff, int stage_R, int n_slots, int* err,
                                                          int* zero, int n_zero, int* zero2, int n_zero2) {
   pdl_trigger(kTrEmbed);
+  float gv[10];
+  load_gain_t<128>(gain, gv);
   pdl_wait();
   if (blockIdx.x == 0) {   // the step's per-expert row counters and tile counters start from zero
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
@@ -80,7 +86,7 @@ __global__ void __launch_bounds__(128) embed_norm_kernel(const int* cand, int R,
     x[k] = __bfloat162float(e[i]);
     h[static_cast<size_t>(row) * kD + i] = x[k];
   }
-  norm_row_store(x, gain, eps, xn + static_cast<size_t>(row) * kD, red);
+  norm_row_store(x, gv, eps, xn + static_cast<size_t>(row) * kD, red);
 }
 
 cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, const int* pending,
@@ -94,13 +100,15 @@ cudaError_t embed_norm_launch(const int* cand, int B, int R, const int* slots, c
 // ---------------------------------------------------------------- RMSNorm
 __global__ void __launch_bounds__(128) rmsnorm_kernel(const float* x, const bf16* gain, float eps, bf16* out) {
   pdl_trigger(kTrNorm);
+  float gv[10];
+  load_gain_t<128>(gain, gv);
   pdl_wait();
   __shared__ float red[4];
   const size_t row = blockIdx.x;
   float v[10];
 #pragma unroll
   for (int k = 0; k < 10; ++k) v[k] = x[row * kD + threadIdx.x + 128 * k];
-  norm_row_store(v, gain, eps, out + row * kD, red);
+  norm_row_store(v, gv, eps, out + row * kD, red);
 }
 
 cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps, bf16* out, cudaStream_t s) {
@@ -299,8 +307,10 @@ cudaError_t router_launch(const RouteArgs& a, cudaStream_t s) {
 __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, const float* gate, const bf16* gain,
                                                       float eps, bf16* out) {
   pdl_trigger(kTrCombine);
-  pdl_wait();
   constexpr int NT = 256, EPT = kD / NT;
+  float gv[EPT];
+  load_gain_t<NT>(gain, gv);
+  pdl_wait();
   __shared__ float red[NT / 32];
   const size_t t = blockIdx.x;
   float g[kTopK];
@@ -324,7 +334,7 @@ __global__ void __launch_bounds__(256) combine_kernel(float* h, const float* y, 
     x[k] += acc;
     h[t * kD + threadIdx.x + NT * k] = x[k];
   }
-  norm_row_store_t<NT>(x, gain, eps, out + t * kD, red);
+  norm_row_store_t<NT>(x, gv, eps, out + t * kD, red);
   trace_exit();
 }
 
@@ -443,6 +453,9 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
                                                          const int* block_table, int max_pages, int n_pages, int* cand,
                                                          int cand_ld, int n_slots, int* err) {
   pdl_trigger(kTrDraftPrep);
+  float ge[10], gh[10];
+  load_gain_t<128>(enorm, ge);
+  load_gain_t<128>(hnorm, gh);
   pdl_wait();
   __shared__ float red[4];
   const int b = blockIdx.x / R, i = blockIdx.x % R, row = blockIdx.x;
@@ -500,8 +513,8 @@ __global__ void __launch_bounds__(128) draft_prep_kernel(int R, const int* slots
   float x[10];
 #pragma unroll
   for (int k = 0; k < 10; ++k) x[k] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * k]);
-  norm_row_store(xb, hnorm, eps, out + kD, red);   // while the embedding row is on its way
-  norm_row_store(x, enorm, eps, out, red);
+  norm_row_store(xb, gh, eps, out + kD, red);   // while the embedding row is on its way
+  norm_row_store(x, ge, eps, out, red);
 }
 
 cudaError_t draft_prep_launch(int B, int R, const int* slots, const int* seq_len, const int* pending,
@@ -539,6 +552,9 @@ __global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_
                                                          int* pos, long long* kv_rowoff, long long dstage_seq_stride,
                                                          int* cand, int cand_ld) {
   pdl_trigger(kTrDraftNext);
+  float ge[10], gh[10];
+  load_gain_t<128>(enorm, ge);
+  load_gain_t<128>(hnorm, gh);
   pdl_wait();
   __shared__ float red[4];
   __shared__ int s_tok;
@@ -573,8 +589,8 @@ __global__ void __launch_bounds__(128) draft_next_kernel(unsigned long long* am_
   float x[10];
 #pragma unroll
   for (int q = 0; q < 10; ++q) x[q] = __bfloat162float(embed[static_cast<size_t>(tok) * kD + threadIdx.x + 128 * q]);
-  norm_row_store(xu, hnorm, eps, out + kD, red);   // while the embedding row is on its way
-  norm_row_store(x, enorm, eps, out, red);
+  norm_row_store(xu, gh, eps, out + kD, red);   // while the embedding row is on its way
+  norm_row_store(x, ge, eps, out, red);
 }
 
 cudaError_t draft_next_launch(unsigned long long* am_key, int vocab, int* err, int B, int k, int K, const int* slots,
