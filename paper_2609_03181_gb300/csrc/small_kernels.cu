@@ -117,8 +117,9 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
 }
 
 // ---------------------------------------------------------------- router
-// kRouteCtaRows token rows per CTA, in the first rows of a 16-row MMA tile (the router matrix
-// is read from L2 once per CTA; more CTAs spread the copies of the selected rows).  Per row: RMSNorm of the residual row -> xn (bf16, also the experts' input); the 64 logits of the
+// 4 token rows per CTA (8 or 16 when that many CTAs would not fit on the GPU at once), in the
+// first rows of a 16-row MMA tile (the router matrix is read from L2 once per CTA; more CTAs
+// spread the copies of the selected rows).  Per row: RMSNorm of the residual row -> xn (bf16, also the experts' input); the 64 logits of the
 // rounded row on bf16 tensor cores (mma.sync m16n8k16, fp32 accumulation; warp w computes
 // experts 8w..8w+7 of all 16 rows, each lane streaming 16-byte pieces of its expert's row);
 // fp32 softmax; top-6 by probability (lower id on ties).  Each selected (token, rank, expert)
@@ -128,16 +129,15 @@ cudaError_t rmsnorm_launch(const float* x, int rows, const bf16* gain, float eps
 // pass nor a row gather follows.  A row's arithmetic is the same whatever rows share its CTA,
 // and a (token, expert) row's result does not depend on its position among the expert's rows.
 constexpr int kRouteRows = 16;      // rows of the MMA tile
-constexpr int kRouteCtaRows = 4;    // token rows of a CTA
+constexpr int kRouteCtaRows = 4;    // token rows of a CTA while one such CTA per SM covers T
 constexpr int kRouteStride = kD + 32;   // bf16 per staged row: rows 64 bytes apart in the banks
 constexpr int kMaxT = 2048;
 
-__global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ RouteArgs a) {
+__global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ RouteArgs a, int cta_rows) {
   pdl_trigger(kTrRouter);
   __shared__ __align__(16) bf16 xs[kRouteRows * kRouteStride];   // the rounded rows
   __shared__ float lg[kRouteRows][kE];                           // logits, then probabilities
   __shared__ int dst[kRouteRows][kTopK];                         // input row of each selection
-  __shared__ unsigned long long keys[kRouteCtaRows][kE];         // (probability, lower id first) keys
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
   // The router matrix is never written by earlier kernels: this lane's share of its expert's
   // row (expert 8 warp + g, columns 32 c + 8 t4 .. + 7) is loaded before the wait.
@@ -150,8 +150,8 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
 #pragma unroll
   for (int k = 0; k < kD / 128; ++k) gq[k] = *reinterpret_cast<const uint2*>(a.gain + 4 * (lane + 32 * k));
   pdl_wait();
-  const int t0 = blockIdx.x * kRouteCtaRows;
-  const int nr = min(kRouteCtaRows, a.T - t0);
+  const int t0 = blockIdx.x * cta_rows;
+  const int nr = min(cta_rows, a.T - t0);
   // RMSNorm: warp w takes rows w and w + 8 of the 16-row MMA tile, of which the first nr are
   // token rows and the rest zeros; a lane sums its 40 squares of a row in order, then a warp tree
   {
@@ -226,11 +226,13 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
     lg[g + 8][e + 1] = d[3] + b1;
   }
   __syncthreads();
-  // softmax of row `warp` (warp w < nr; lane l holds experts l and l + 32), the probabilities
-  // back into lg
-  static_assert(kRouteCtaRows * kE == 256, "one thread per (row, expert) ranks the experts");
-  if (warp < nr) {
-    const int r = warp;
+  // softmax of rows warp and warp + 8 (lane l holds experts l and l + 32); lg then holds each
+  // probability p as the 32-bit order key of p + 0 (a larger key = a larger p)
+  unsigned* ok = reinterpret_cast<unsigned*>(&lg[0][0]);
+#pragma unroll
+  for (int h2 = 0; h2 < 2; ++h2) {
+    const int r = warp + 8 * h2;
+    if (r >= nr) break;
     const float l0 = lg[r][lane], l1 = lg[r][lane + 32];
     const float m = warp_max(fmaxf(l0, l1));
     const float e0 = expf(l0 - m), e1 = expf(l1 - m);
@@ -243,31 +245,31 @@ __global__ void __launch_bounds__(256) router_kernel(const __grid_constant__ Rou
       if (!(p0 == p0)) p0 = -1.f;
       if (!(p1 == p1)) p1 = -1.f;
     }
-    lg[r][lane] = p0;
-    lg[r][lane + 32] = p1;
-    keys[r][lane] = argmax_key(p0, lane);
-    keys[r][lane + 32] = argmax_key(p1, lane + 32);
+    ok[r * kE + lane] = static_cast<unsigned>(argmax_key(p0, lane) >> 32);
+    ok[r * kE + lane + 32] = static_cast<unsigned>(argmax_key(p1, lane + 32) >> 32);
   }
   __syncthreads();
-  // top-6: thread (r, e) counts the experts whose (probability, lower id first) key beats its
-  // own -- its rank, the place argmax rounds would give it -- and, ranked among the first six,
-  // takes the next row of expert e
-  {
-    const int r = threadIdx.x >> 6, e = threadIdx.x & 63;
-    if (r < nr) {
-      const float pe = lg[r][e];
-      const unsigned long long mine = keys[r][e];
-      int rank = 0;
+  // top-6: the thread of (row r, expert e) counts the experts whose (probability, lower id
+  // first) key beats its own -- its rank, the place six argmax rounds would give it -- and,
+  // ranked among the first six, takes the next row of expert e
+  for (int pr = threadIdx.x; pr < nr * kE; pr += 256) {
+    const int r = pr >> 6, e = pr & 63;
+    // the full keys (order key << 32 | ~id), as argmax_key builds them
+    const unsigned pk = ok[r * kE + e];
+    const unsigned long long mine = (static_cast<unsigned long long>(pk) << 32) | static_cast<unsigned>(~e);
+    int rank = 0;
 #pragma unroll
-      for (int o = 0; o < kE; ++o) rank += (keys[r][o] > mine) ? 1 : 0;
-      if (rank < kTopK) {
-        const int t = t0 + r;
-        const int pos = atomicAdd(a.counts + e, 1);
-        a.idx[static_cast<size_t>(t) * kTopK + rank] = e;
-        a.gate[static_cast<size_t>(t) * kTopK + rank] = pe;
-        a.rowmap[static_cast<size_t>(e) * a.map_stride + pos] = (t << 3) | rank;
-        dst[r][rank] = e * a.map_stride + pos;
-      }
+    for (int o = 0; o < kE; ++o)
+      rank += ((static_cast<unsigned long long>(ok[r * kE + o]) << 32 | static_cast<unsigned>(~o)) > mine) ? 1 : 0;
+    if (rank < kTopK) {
+      // the probability back from its key (the key of p + 0 maps one to one onto p)
+      const float pe = __uint_as_float((pk & 0x80000000u) ? (pk & 0x7fffffffu) : ~pk);
+      const int t = t0 + r;
+      const int pos = atomicAdd(a.counts + e, 1);
+      a.idx[static_cast<size_t>(t) * kTopK + rank] = e;
+      a.gate[static_cast<size_t>(t) * kTopK + rank] = pe;
+      a.rowmap[static_cast<size_t>(e) * a.map_stride + pos] = (t << 3) | rank;
+      dst[r][rank] = e * a.map_stride + pos;
     }
   }
   __syncthreads();
@@ -299,7 +301,11 @@ cudaError_t router_prepare() { return cudaSuccess; }
 
 cudaError_t router_launch(const RouteArgs& a, cudaStream_t s) {
   if (a.T > kMaxT || a.T < 1 || a.T > a.map_stride) return cudaErrorInvalidValue;
-  return launch_pdl(router_kernel, dim3((a.T + kRouteCtaRows - 1) / kRouteCtaRows), dim3(256), 0, s, a);
+  // 4 rows a CTA while that fits one wave of one CTA per SM, else 8 or 16 (the router is one CTA
+  // per SM: 240 registers a thread); a row's arithmetic does not depend on the rows beside it
+  int rows = kRouteCtaRows;
+  while (rows < kRouteRows && (a.T + rows - 1) / rows > num_sms()) rows *= 2;
+  return launch_pdl(router_kernel, dim3((a.T + rows - 1) / rows), dim3(256), 0, s, a, rows);
 }
 
 // ---------------------------------------------------------------- combine
