@@ -55,6 +55,9 @@ constexpr int kQBytes = kMaxR * kHD * 2;         // the queries of one (sequence
 // are then all fetched before the wait for the previous kernel.
 constexpr int kAttnStages = 2;
 constexpr int kAttnStagesSmall = 4;
+// Launches whose items fit two CTAs per SM at once take three stages: three of a super-chunk's
+// four chunks are fetched before the wait.
+constexpr int kAttnStagesMid = 3;
 constexpr int kConsumers = 128;                  // four warps, each owning 32 of the 128 dims
 constexpr int kAttnThreads = kConsumers + 32;    // plus the producer warp
 constexpr int kPartStride = kAttnPartStride;     // floats per (super-chunk, query): O[128], M, L, pad
@@ -227,7 +230,7 @@ __device__ __forceinline__ void merge_seq_head(const AttnArgs& a, int b, int h, 
 }
 
 template <int kStages>
-__global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : 1) attn_kernel(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(kAttnThreads, kStages == 2 ? 3 : (kStages == 3 ? 2 : 1)) attn_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ uint8_t asmem_raw[];
   const uint32_t raw_u32 = smem_u32(asmem_raw);
   uint8_t* stages = asmem_raw + (((raw_u32 + 1023u) & ~1023u) - raw_u32);   // [S][K 16 KB | V 16 KB]
@@ -699,6 +702,9 @@ cudaError_t attention_prepare() {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(attn_kernel<kAttnStagesSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(attn_smem(kAttnStagesSmall, 2048)));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_kernel<kAttnStagesMid>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(attn_smem(kAttnStagesMid, 2048)));
   return e;
 }
 
@@ -722,6 +728,8 @@ cudaError_t attention_launch(const AttnArgs& a_in, int B, cudaStream_t s) {
   AttnArgs a = a_in;
   a.B = B;
   if (B <= 2) return attention_launch_s<kAttnStagesSmall>(a, B, s);
+  const long long items = static_cast<long long>(B) * kH * ((a.n_chunks + kSuper - 1) / kSuper);
+  if (items <= 2LL * num_sms()) return attention_launch_s<kAttnStagesMid>(a, B, s);
   return attention_launch_s<kAttnStages>(a, B, s);
 }
 
